@@ -1,0 +1,171 @@
+/*
+ * af1.h — C ABI of the GB300 (sm_103a) implementation of the AF1
+ * binary-factorized linear layer.
+ *
+ * The layer (AF1, Sec. 3.1, Eq. final_reconstruction; App. "Double-factor
+ * binary representation", Eq. double_factor_equiv and Eq. binary_paths) is
+ *
+ *     W_hat = Diag(a) . U . Diag(s) . V^T . Diag(b)        (d_out x d_in)
+ *     y     = x . W_hat^T
+ *
+ * with U = A_pm1 in {-1,+1}^{m x r}, V = B_pm1^T in {-1,+1}^{n x r}, the row
+ * scale a (m), the merged rank scale s = m1 * m2 (r) and the column scale
+ * b (n); m = d_out, n = d_in. What is stored per matrix is exactly what
+ * App. "Effective Bit-Width" (Eq. app_af1_memory) counts: r(m + n) sign bits
+ * plus three 16-bit scale vectors. Scales are FP16 here (the paper stores
+ * BF16; both cost 16 bits). The dense W_hat is never formed: a forward call
+ * evaluates y = a * (U (s * (V^T (b * x)))) on the GPU.
+ *
+ * Conventions for every entry point
+ *   - Return value: AF1_OK (0) or a negative AF1_ERR_* code; af1_last_error()
+ *     then returns a message for the calling thread. No C++ exception crosses
+ *     this boundary.
+ *   - All data pointers are DEVICE pointers (cudaMalloc, or memory the CUDA
+ *     runtime reports as device or managed). A host pointer is rejected with
+ *     AF1_ERR_BAD_POINTER before any work is queued.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = the legacy default
+ *     stream). Work is queued on it in stream order.
+ *   - FP16 values are passed as their 16-bit patterns (uint16_t).
+ *
+ * Canonical packed format (the paper prescribes no bit layout; this is the
+ * reading this library fixes): each factor is packed along its contraction
+ * axis, least significant bit first, bit = 1 for +1 and bit = 0 for -1,
+ * 32 signs per uint32 word, each row padded with zero bits to a multiple of
+ * 4 words (16 bytes). With W(c) = 4 * ceil(c / 128):
+ *   U words: m rows x W(r) words;  bit (k % 32) of word (k / 32) of row i = U[i][k]
+ *   V words: r rows x W(n) words;  bit (j % 32) of word (j / 32) of row k = V[j][k]
+ * Internally a layer keeps the signs in a tile layout of its own (same bit
+ * count plus tile padding); the canonical words are the exchange format.
+ */
+#ifndef AF1_H
+#define AF1_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define AF1_API __attribute__((visibility("default")))
+#else
+#define AF1_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- status codes -------------------------------------------------------- */
+#define AF1_OK 0
+#define AF1_ERR_INVALID_ARG (-1)   /* bad size, dtype, flag or NULL where required */
+#define AF1_ERR_BAD_POINTER (-2)   /* a pointer that is not device-accessible       */
+#define AF1_ERR_MISALIGNED (-3)    /* pointer or leading dimension misaligned       */
+#define AF1_ERR_OVER_BUDGET (-4)   /* r above the 1.0-BPW rank of (m, n)            */
+#define AF1_ERR_INVALID_SIGN (-5)  /* a sign entry that is not exactly +1 or -1     */
+#define AF1_ERR_CUDA (-6)          /* a CUDA runtime error (message has details)    */
+#define AF1_ERR_TIMEOUT (-7)       /* a bounded device wait gave up                 */
+#define AF1_ERR_WORKSPACE (-8)     /* workspace missing, too small or misaligned    */
+
+/* ---- output dtypes for af1_linear_forward -------------------------------- */
+#define AF1_F16 0
+#define AF1_F32 1
+
+/* ---- layer description flags --------------------------------------------- */
+/* Allow r above the exact 1.0-BPW rank (for other budgets such as the
+   paper's 2.5-BPW setting). Without it r > af1_rank_for_budget(m, n, 1, 1)
+   is rejected with AF1_ERR_OVER_BUDGET. */
+#define AF1_FLAG_ANY_RANK 1
+
+typedef struct af1_layer_desc {
+  int64_t m;       /* d_out: rows of W_hat, length of a, length of y rows */
+  int64_t n;       /* d_in: columns of W_hat, length of b and of x rows   */
+  int64_t r;       /* rank: length of s, inner dimension of U and V       */
+  int32_t flags;   /* AF1_FLAG_* */
+  int32_t reserved;/* must be 0 */
+} af1_layer_desc;
+
+typedef struct af1_layer af1_layer; /* opaque, owns its device buffers */
+
+/* Exact rank for a storage budget of (budget_num / budget_den) bits per
+ * weight: the largest r with r(m+n) + 16(m+r+n) <= budget * m * n
+ * (App. "Effective Bit-Width", Eq. app_af1_memory, read as a hard cap on the
+ * full storage; App. A.3 rounds the sign bits only). Writes 0 when not even
+ * rank 1 fits. Host-only, no GPU needed. Errors: INVALID_ARG for m, n <= 0,
+ * budget_den <= 0, budget_num < 0, r_out NULL, or overflow. */
+AF1_API int af1_rank_for_budget(int64_t m, int64_t n, int64_t budget_num, int64_t budget_den,
+                        int64_t* r_out);
+
+/* Build a layer from sign matrices (the factors NABF produces, Sec. 3.1).
+ *   U:   int8 [m x r] row-major, entries exactly +1 or -1
+ *   V:   int8 [n x r] row-major (V = B_pm1^T), entries exactly +1 or -1
+ *   a:   FP16 bits [m]; s: FP16 bits [r]; b: FP16 bits [n]
+ *   out_U, out_V: optional (may be NULL) device buffers that receive the
+ *        canonical packed words, [m x W(r)] and [r x W(n)] uint32.
+ * All inputs are device pointers read on `stream`; the layer takes its own
+ * copies, so the caller may free them once this call returns (the call
+ * synchronizes `stream` to validate the signs). On success *out owns the
+ * layer (release with af1_free). Errors: INVALID_ARG, BAD_POINTER,
+ * OVER_BUDGET, INVALID_SIGN (nothing is created), CUDA. */
+AF1_API int af1_pack_layer(const af1_layer_desc* desc, const int8_t* U, const int8_t* V,
+                   const uint16_t* a, const uint16_t* s, const uint16_t* b,
+                   uint32_t* out_U, uint32_t* out_V, void* stream, af1_layer** out);
+
+/* Build a layer from canonical packed words (the deployable format), e.g. a
+ * saved checkpoint. U_words [m x W(r)], V_words [r x W(n)] uint32, device.
+ * Padding bits are ignored. Same ownership, synchronization and errors as
+ * af1_pack_layer (no INVALID_SIGN: every bit is a valid sign). */
+AF1_API int af1_load_packed_layer(const af1_layer_desc* desc, const uint32_t* U_words,
+                          const uint32_t* V_words, const uint16_t* a, const uint16_t* s,
+                          const uint16_t* b, void* stream, af1_layer** out);
+
+/* Copy the description of a layer into *desc. */
+AF1_API int af1_layer_get_desc(const af1_layer* layer, af1_layer_desc* desc);
+
+/* Device bytes the layer holds for its signs (tile layout) and its scales. */
+AF1_API int af1_layer_device_bytes(const af1_layer* layer, int64_t* sign_bytes, int64_t* scale_bytes);
+
+/* Bytes of workspace one af1_linear_forward call with `tokens` rows needs
+ * (>= 256). Returns a negative AF1_ERR_* code on bad arguments. */
+AF1_API int64_t af1_workspace_bytes(const af1_layer* layer, int64_t tokens);
+
+/* y = x . W_hat^T for `tokens` rows (AF1 Eq. final_reconstruction applied
+ * right to left).
+ *   x:  FP16 [tokens x n], row stride ldx elements (ldx >= n, ldx % 8 == 0),
+ *       16-byte aligned device pointer.
+ *   y:  [tokens x m], row stride ldy >= m elements, 16-byte aligned; y_dtype
+ *       AF1_F16 (ldy % 8 == 0) or AF1_F32 (ldy % 4 == 0). Only the first m
+ *       entries of each row are written.
+ *   workspace: device scratch of at least af1_workspace_bytes(layer, tokens)
+ *       bytes, 256-byte aligned, owned by the caller. It must be zero-filled
+ *       before its first use; every completed call leaves its bookkeeping
+ *       words at zero again, so one workspace serves any sequence of calls
+ *       on one stream, for any layer. Calls that may overlap on the GPU
+ *       (different streams) need different workspaces.
+ * Asynchronous and stream-ordered: nothing is synchronized. tokens == 0 is a
+ * no-op returning AF1_OK. Launch errors are returned at once; a device-side
+ * wait that gave up is reported by af1_workspace_status. The layer is not
+ * modified, so several streams may use one layer concurrently, each with its
+ * own workspace. Errors: INVALID_ARG, BAD_POINTER, MISALIGNED, WORKSPACE,
+ * CUDA. */
+AF1_API int af1_linear_forward(const af1_layer* layer, const void* x, int64_t ldx, int64_t tokens,
+                       void* y, int64_t ldy, int y_dtype, void* workspace,
+                       int64_t workspace_bytes, void* stream);
+
+/* Synchronize `stream` and report the status word the kernels keep in a
+ * workspace: AF1_OK, or AF1_ERR_TIMEOUT if a bounded device-side wait gave
+ * up since the workspace was last cleared (the word is then reset to 0). */
+AF1_API int af1_workspace_status(void* workspace, void* stream);
+
+/* Release a layer and its device buffers. NULL is a no-op. Synchronizes the
+ * device before freeing, so queued work that reads the layer completes. */
+AF1_API void af1_free(af1_layer* layer);
+
+/* Message for the last error on the calling thread ("" if none). */
+AF1_API const char* af1_last_error(void);
+
+/* Library version string. */
+AF1_API const char* af1_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* AF1_H */

@@ -1,0 +1,233 @@
+"""GB300 (sm_103a) AF1 binary-factorized linear layer.
+
+Thin ctypes binding over libaf1.so, whose C ABI is include/af1.h. The binding
+only marshals arguments: PyTorch supplies device memory and the current
+stream, and every step of the forward pass runs in the library's CUDA
+kernels. There is no CPU or PyTorch fallback: if libaf1.so is missing this
+package fails to import.
+
+The layer (AF1, Sec. 3.1, Eq. final_reconstruction) is
+    W_hat = Diag(a) U Diag(s) V^T Diag(b),     y = x W_hat^T
+with U (m x r) and V (n x r) sign matrices, FP16 scales a (m), s (r), b (n).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+__all__ = [
+    "AF1Error", "Layer", "rank_for_budget", "workspace_status", "last_error", "version", "lib_path",
+    "words_per_row", "AF1_F16", "AF1_F32",
+]
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+lib_path = os.path.join(_HERE, "libaf1.so")
+
+if not os.path.exists(lib_path):
+    raise ImportError(
+        f"{lib_path} is missing: build it with `python paper_2609_06161_gb300/build.py` "
+        "(or __graft_entry__.build()); there is no fallback implementation")
+
+_lib = ctypes.CDLL(lib_path)
+
+AF1_OK = 0
+AF1_F16 = 0
+AF1_F32 = 1
+AF1_FLAG_ANY_RANK = 1
+_ERR_NAMES = {
+    -1: "AF1_ERR_INVALID_ARG", -2: "AF1_ERR_BAD_POINTER", -3: "AF1_ERR_MISALIGNED",
+    -4: "AF1_ERR_OVER_BUDGET", -5: "AF1_ERR_INVALID_SIGN", -6: "AF1_ERR_CUDA",
+    -7: "AF1_ERR_TIMEOUT", -8: "AF1_ERR_WORKSPACE",
+}
+
+
+class _Desc(ctypes.Structure):
+    _fields_ = [("m", ctypes.c_int64), ("n", ctypes.c_int64), ("r", ctypes.c_int64),
+                ("flags", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+
+
+_vp = ctypes.c_void_p
+_i64 = ctypes.c_int64
+_lib.af1_rank_for_budget.argtypes = [_i64, _i64, _i64, _i64, ctypes.POINTER(_i64)]
+_lib.af1_rank_for_budget.restype = ctypes.c_int
+_lib.af1_pack_layer.argtypes = [ctypes.POINTER(_Desc), _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
+                                ctypes.POINTER(_vp)]
+_lib.af1_pack_layer.restype = ctypes.c_int
+_lib.af1_load_packed_layer.argtypes = [ctypes.POINTER(_Desc), _vp, _vp, _vp, _vp, _vp, _vp,
+                                       ctypes.POINTER(_vp)]
+_lib.af1_load_packed_layer.restype = ctypes.c_int
+_lib.af1_layer_get_desc.argtypes = [_vp, ctypes.POINTER(_Desc)]
+_lib.af1_layer_get_desc.restype = ctypes.c_int
+_lib.af1_layer_device_bytes.argtypes = [_vp, ctypes.POINTER(_i64), ctypes.POINTER(_i64)]
+_lib.af1_layer_device_bytes.restype = ctypes.c_int
+_lib.af1_workspace_bytes.argtypes = [_vp, _i64]
+_lib.af1_workspace_bytes.restype = _i64
+_lib.af1_linear_forward.argtypes = [_vp, _vp, _i64, _i64, _vp, _i64, ctypes.c_int, _vp, _i64, _vp]
+_lib.af1_linear_forward.restype = ctypes.c_int
+_lib.af1_workspace_status.argtypes = [_vp, _vp]
+_lib.af1_workspace_status.restype = ctypes.c_int
+_lib.af1_free.argtypes = [_vp]
+_lib.af1_free.restype = None
+_lib.af1_last_error.argtypes = []
+_lib.af1_last_error.restype = ctypes.c_char_p
+_lib.af1_version.argtypes = []
+_lib.af1_version.restype = ctypes.c_char_p
+
+
+class AF1Error(RuntimeError):
+    def __init__(self, code: int, message: str):
+        self.code = code
+        self.name = _ERR_NAMES.get(code, str(code))
+        super().__init__(f"{self.name}: {message}")
+
+
+def last_error() -> str:
+    return _lib.af1_last_error().decode()
+
+
+def version() -> str:
+    return _lib.af1_version().decode()
+
+
+def _check(rc: int):
+    if rc != AF1_OK:
+        raise AF1Error(rc, last_error())
+
+
+def words_per_row(cols: int) -> int:
+    """uint32 words per packed row of `cols` signs (rows padded to 16 bytes)."""
+    return 4 * ((cols + 127) // 128)
+
+
+def rank_for_budget(m: int, n: int, num: int = 1, den: int = 1) -> int:
+    """Largest r whose exact AF1 storage fits num/den bits per weight."""
+    r = _i64(0)
+    _check(_lib.af1_rank_for_budget(m, n, num, den, ctypes.byref(r)))
+    return r.value
+
+
+def _stream_handle(stream) -> int:
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return int(s.cuda_stream)
+
+
+def _ptr(t) -> int:
+    return 0 if t is None else int(t.data_ptr())
+
+
+def workspace_status(workspace: torch.Tensor, stream=None) -> None:
+    """Synchronize and raise AF1Error(AF1_ERR_TIMEOUT) if a bounded device wait gave up."""
+    _check(_lib.af1_workspace_status(_ptr(workspace), _stream_handle(stream)))
+
+
+class Layer:
+    """An AF1 layer resident on the current CUDA device."""
+
+    def __init__(self, handle: int, m: int, n: int, r: int):
+        self._h = handle
+        self.m, self.n, self.r = m, n, r
+
+    # -- construction --------------------------------------------------------
+    @classmethod
+    def from_signs(cls, U: torch.Tensor, V: torch.Tensor, a: torch.Tensor, s: torch.Tensor,
+                   b: torch.Tensor, any_rank: bool = False, return_words: bool = False, stream=None):
+        """U: int8 (m, r), V: int8 (n, r) of +-1; a, s, b: float16 vectors. All on
+        the current CUDA device. With return_words, also returns the canonical
+        packed words (Uw: (m, W(r)), Vw: (r, W(n)) as int32 tensors)."""
+        m, r = U.shape
+        n = V.shape[0]
+        if V.shape[1] != r:
+            raise ValueError("U and V must have the same rank")
+        U, V = U.contiguous(), V.contiguous()
+        a, s, b = a.contiguous(), s.contiguous(), b.contiguous()
+        Uw = Vw = None
+        if return_words:
+            Uw = torch.empty((m, words_per_row(r)), dtype=torch.int32, device=U.device)
+            Vw = torch.empty((r, words_per_row(n)), dtype=torch.int32, device=U.device)
+        d = _Desc(m, n, r, AF1_FLAG_ANY_RANK if any_rank else 0, 0)
+        h = _vp()
+        _check(_lib.af1_pack_layer(ctypes.byref(d), _ptr(U), _ptr(V), _ptr(a), _ptr(s), _ptr(b),
+                                   _ptr(Uw), _ptr(Vw), _stream_handle(stream), ctypes.byref(h)))
+        layer = cls(h.value, m, n, r)
+        return (layer, Uw, Vw) if return_words else layer
+
+    @classmethod
+    def from_words(cls, Uw: torch.Tensor, Vw: torch.Tensor, a: torch.Tensor, s: torch.Tensor,
+                   b: torch.Tensor, m: int, n: int, r: int, any_rank: bool = False, stream=None):
+        """Uw: (m, W(r)), Vw: (r, W(n)) canonical packed words (int32/uint32)."""
+        Uw, Vw = Uw.contiguous(), Vw.contiguous()
+        a, s, b = a.contiguous(), s.contiguous(), b.contiguous()
+        d = _Desc(m, n, r, AF1_FLAG_ANY_RANK if any_rank else 0, 0)
+        h = _vp()
+        _check(_lib.af1_load_packed_layer(ctypes.byref(d), _ptr(Uw), _ptr(Vw), _ptr(a), _ptr(s), _ptr(b),
+                                          _stream_handle(stream), ctypes.byref(h)))
+        return cls(h.value, m, n, r)
+
+    # -- queries ---------------------------------------------------------------
+    def workspace_bytes(self, tokens: int = 1) -> int:
+        v = _lib.af1_workspace_bytes(self._h, tokens)
+        if v < 0:
+            raise AF1Error(int(v), last_error())
+        return int(v)
+
+    def make_workspace(self, tokens: int = 16, device=None) -> torch.Tensor:
+        """A zero-filled workspace tensor usable for any number of tokens."""
+        return torch.zeros(self.workspace_bytes(tokens), dtype=torch.uint8,
+                           device=device or torch.device("cuda", torch.cuda.current_device()))
+
+    def device_bytes(self):
+        sb, cb = _i64(0), _i64(0)
+        _check(_lib.af1_layer_device_bytes(self._h, ctypes.byref(sb), ctypes.byref(cb)))
+        return sb.value, cb.value
+
+    # -- compute -----------------------------------------------------------------
+    def forward_into(self, x: torch.Tensor, y: torch.Tensor, workspace: torch.Tensor, stream=None) -> None:
+        """y[:tokens, :m] = x[:tokens, :n] W_hat^T; x float16 (tokens, ldx),
+        y float16 or float32 (tokens, ldy), both 2-D with unit column stride."""
+        if x.dim() != 2 or y.dim() != 2 or x.stride(1) != 1 or y.stride(1) != 1:
+            raise ValueError("x and y must be 2-D with contiguous rows")
+        if x.dtype != torch.float16:
+            raise ValueError("x must be float16")
+        if y.dtype == torch.float16:
+            yd = AF1_F16
+        elif y.dtype == torch.float32:
+            yd = AF1_F32
+        else:
+            raise ValueError("y must be float16 or float32")
+        tokens = x.shape[0]
+        if y.shape[0] < tokens:
+            raise ValueError("y has fewer rows than x")
+        ldx = x.stride(0) if tokens > 1 else max(x.stride(0), self.n + (-self.n) % 8)
+        ldy = y.stride(0) if tokens > 1 else max(y.stride(0), self.m + (-self.m) % (8 if yd == AF1_F16 else 4))
+        _check(_lib.af1_linear_forward(self._h, _ptr(x), ldx, tokens, _ptr(y), ldy, yd, _ptr(workspace),
+                                       workspace.numel() * workspace.element_size(), _stream_handle(stream)))
+
+    def forward(self, x: torch.Tensor, out_dtype=torch.float16, workspace: torch.Tensor | None = None,
+                stream=None) -> torch.Tensor:
+        if x.dim() == 1:
+            x = x.unsqueeze(0)
+        tokens = x.shape[0]
+        if x.stride(1) != 1 or x.stride(0) % 8 != 0 or x.data_ptr() % 16 != 0:
+            pad = (-self.n) % 8
+            xp = torch.zeros((tokens, self.n + pad), dtype=torch.float16, device=x.device)
+            xp[:, :self.n] = x
+            x = xp
+        align = 8 if out_dtype == torch.float16 else 4
+        ldy = self.m + (-self.m) % align
+        y = torch.empty((tokens, ldy), dtype=out_dtype, device=x.device)
+        ws = workspace if workspace is not None else self.make_workspace(tokens, x.device)
+        self.forward_into(x, y, ws, stream)
+        return y[:, :self.m]
+
+    def free(self) -> None:
+        if getattr(self, "_h", None):
+            _lib.af1_free(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.free()
+        except Exception:
+            pass

@@ -1,0 +1,346 @@
+// af1_api.cu — the C ABI declared in include/af1.h: argument validation,
+// layer ownership and dispatch to the kernels. No C++ exception crosses the
+// boundary; every failure returns an AF1_ERR_* code and sets a thread-local
+// message.
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <cstdio>
+#include <new>
+#include <string>
+
+#include "../../include/af1.h"
+#include "af1_internal.h"
+#include "af1_layout.h"
+
+namespace {
+
+thread_local std::string g_err;
+
+int fail(int code, const std::string& msg) {
+  g_err = msg;
+  return code;
+}
+
+int fail_cuda(cudaError_t e, const char* what) {
+  std::string m = std::string(what) + ": " + cudaGetErrorName(e) + " (" + cudaGetErrorString(e) + ")";
+  return fail(AF1_ERR_CUDA, m);
+}
+
+int64_t words_per_row(int64_t cols) { return 4 * ((cols + 127) / 128); }
+int64_t align256(int64_t v) { return (v + 255) / 256 * 256; }
+
+// Exact floor((B - 16(m+n)) / (m+n+16)) with B = num * m * n / den, in
+// 128-bit integer arithmetic: the largest r with r(m+n) + 16(m+r+n) <= B.
+int rank_rule(int64_t m, int64_t n, int64_t num, int64_t den, int64_t* r) {
+  if (m <= 0 || n <= 0 || den <= 0 || num < 0 || r == nullptr)
+    return fail(AF1_ERR_INVALID_ARG, "af1_rank_for_budget: m, n, den must be > 0, num >= 0, r_out non-NULL");
+  if (m > (int64_t)1 << 31 || n > (int64_t)1 << 31 || num > (int64_t)1 << 20 || den > (int64_t)1 << 20)
+    return fail(AF1_ERR_INVALID_ARG, "af1_rank_for_budget: arguments out of range");
+  // r <= (num*m*n - 16*den*(m+n)) / (den*(m+n+16))
+  __int128 top = (__int128)num * m * n - (__int128)16 * den * (m + n);
+  __int128 bot = (__int128)den * (m + n + 16);
+  if (top < bot) {
+    *r = 0;
+    return AF1_OK;
+  }
+  *r = (int64_t)(top / bot);
+  return AF1_OK;
+}
+
+int check_device_ptr(const void* p, const char* name, int device) {
+  if (p == nullptr) return fail(AF1_ERR_INVALID_ARG, std::string(name) + " is NULL");
+  cudaPointerAttributes at;
+  cudaError_t e = cudaPointerGetAttributes(&at, p);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    return fail(AF1_ERR_BAD_POINTER, std::string(name) + " is not a CUDA pointer");
+  }
+  if (at.type != cudaMemoryTypeDevice && at.type != cudaMemoryTypeManaged)
+    return fail(AF1_ERR_BAD_POINTER, std::string(name) + " is not device memory");
+  if (at.type == cudaMemoryTypeDevice && at.device != device)
+    return fail(AF1_ERR_BAD_POINTER, std::string(name) + " lives on another device");
+  return AF1_OK;
+}
+
+int check_desc(const af1_layer_desc* d) {
+  if (d == nullptr) return fail(AF1_ERR_INVALID_ARG, "desc is NULL");
+  if (d->m <= 0 || d->n <= 0 || d->r <= 0) return fail(AF1_ERR_INVALID_ARG, "m, n and r must be positive");
+  if (d->m > ((int64_t)1 << 30) || d->n > ((int64_t)1 << 30) || d->r > ((int64_t)1 << 30))
+    return fail(AF1_ERR_INVALID_ARG, "m, n or r too large");
+  if (d->reserved != 0 || (d->flags & ~AF1_FLAG_ANY_RANK) != 0)
+    return fail(AF1_ERR_INVALID_ARG, "unknown flags or non-zero reserved field");
+  if (!(d->flags & AF1_FLAG_ANY_RANK)) {
+    int64_t rmax = 0;
+    int rc = rank_rule(d->m, d->n, 1, 1, &rmax);
+    if (rc != AF1_OK) return rc;
+    if (d->r > rmax)
+      return fail(AF1_ERR_OVER_BUDGET, "r = " + std::to_string(d->r) + " exceeds the 1.0-BPW rank " +
+                                           std::to_string(rmax) + " of this shape");
+  }
+  return AF1_OK;
+}
+
+// Allocate a layer with its tile plans; buffers zero-filled on `st`.
+int create_layer(const af1_layer_desc* d, cudaStream_t st, af1_layer** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return fail_cuda(e, "cudaGetDevice");
+  int sms = 0;
+  e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) return fail_cuda(e, "cudaDeviceGetAttribute");
+  af1_layer* L = new (std::nothrow) af1_layer();
+  if (L == nullptr) return fail(AF1_ERR_CUDA, "host allocation failed");
+  L->m = d->m;
+  L->n = d->n;
+  L->r = d->r;
+  L->flags = d->flags;
+  L->device = dev;
+  L->num_sms = sms;
+  af1::plan_tiles(L->p1, d->r, d->n, /*rtc_target=*/64, sms, /*ktc_max=*/4);
+  af1::plan_tiles(L->p2, d->m, d->r, /*rtc_target=*/16, sms, /*ktc_max=*/af1::kMaxKTC);
+  const int64_t t1 = (int64_t)L->p1.RT * L->p1.KT * af1::kTileBytes;
+  const int64_t t2 = (int64_t)L->p2.RT * L->p2.KT * af1::kTileBytes;
+  const int64_t sa = align256(2 * d->m), ss = align256(2 * d->r), sb = align256(2 * d->n);
+  const int64_t total = align256(t1) + align256(t2) + sa + ss + sb;
+  e = cudaMalloc(&L->alloc, (size_t)total);
+  if (e != cudaSuccess) {
+    delete L;
+    return fail_cuda(e, "cudaMalloc(layer)");
+  }
+  uint8_t* base = static_cast<uint8_t*>(L->alloc);
+  L->tiles1 = base;
+  L->tiles2 = base + align256(t1);
+  L->a = reinterpret_cast<uint16_t*>(L->tiles2 + align256(t2));
+  L->s = reinterpret_cast<uint16_t*>(reinterpret_cast<uint8_t*>(L->a) + sa);
+  L->b = reinterpret_cast<uint16_t*>(reinterpret_cast<uint8_t*>(L->s) + ss);
+  L->sign_bytes = t1 + t2;
+  L->scale_bytes = 2 * (d->m + d->r + d->n);
+  e = cudaMemsetAsync(L->alloc, 0, (size_t)total, st);
+  if (e != cudaSuccess) {
+    cudaFree(L->alloc);
+    delete L;
+    return fail_cuda(e, "cudaMemsetAsync(layer)");
+  }
+  *out = L;
+  return AF1_OK;
+}
+
+void destroy_layer(af1_layer* L) {
+  if (L == nullptr) return;
+  cudaDeviceSynchronize();
+  if (L->alloc) cudaFree(L->alloc);
+  delete L;
+}
+
+int copy_scales(af1_layer* L, const uint16_t* a, const uint16_t* s, const uint16_t* b, cudaStream_t st) {
+  cudaError_t e = cudaMemcpyAsync(L->a, a, 2 * L->m, cudaMemcpyDeviceToDevice, st);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(L->s, s, 2 * L->r, cudaMemcpyDeviceToDevice, st);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(L->b, b, 2 * L->n, cudaMemcpyDeviceToDevice, st);
+  if (e != cudaSuccess) return fail_cuda(e, "cudaMemcpyAsync(scales)");
+  return AF1_OK;
+}
+
+int check_scales(const uint16_t* a, const uint16_t* s, const uint16_t* b, int dev) {
+  int rc = check_device_ptr(a, "a", dev);
+  if (rc == AF1_OK) rc = check_device_ptr(s, "s", dev);
+  if (rc == AF1_OK) rc = check_device_ptr(b, "b", dev);
+  return rc;
+}
+
+}  // namespace
+
+extern "C" {
+
+int af1_rank_for_budget(int64_t m, int64_t n, int64_t budget_num, int64_t budget_den, int64_t* r_out) {
+  return rank_rule(m, n, budget_num, budget_den, r_out);
+}
+
+int af1_pack_layer(const af1_layer_desc* desc, const int8_t* U, const int8_t* V, const uint16_t* a,
+                   const uint16_t* s, const uint16_t* b, uint32_t* out_U, uint32_t* out_V, void* stream,
+                   af1_layer** out) {
+  if (out == nullptr) return fail(AF1_ERR_INVALID_ARG, "out is NULL");
+  *out = nullptr;
+  int rc = check_desc(desc);
+  if (rc != AF1_OK) return rc;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return fail_cuda(e, "cudaGetDevice");
+  if ((rc = check_device_ptr(U, "U", dev)) != AF1_OK) return rc;
+  if ((rc = check_device_ptr(V, "V", dev)) != AF1_OK) return rc;
+  if ((rc = check_scales(a, s, b, dev)) != AF1_OK) return rc;
+  if (out_U && (rc = check_device_ptr(out_U, "out_U", dev)) != AF1_OK) return rc;
+  if (out_V && (rc = check_device_ptr(out_V, "out_V", dev)) != AF1_OK) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const int64_t m = desc->m, n = desc->n, r = desc->r;
+  const int64_t wu = words_per_row(r), wv = words_per_row(n);
+
+  // Scratch for canonical words the caller did not ask for, plus a flag.
+  int64_t need = 256 + (out_U ? 0 : align256(4 * m * wu)) + (out_V ? 0 : align256(4 * r * wv));
+  uint8_t* scratch = nullptr;
+  e = cudaMalloc(&scratch, (size_t)need);
+  if (e != cudaSuccess) return fail_cuda(e, "cudaMalloc(pack scratch)");
+  uint32_t* flag = reinterpret_cast<uint32_t*>(scratch);
+  uint8_t* cur = scratch + 256;
+  uint32_t* Uw = out_U;
+  uint32_t* Vw = out_V;
+  if (!Uw) {
+    Uw = reinterpret_cast<uint32_t*>(cur);
+    cur += align256(4 * m * wu);
+  }
+  if (!Vw) Vw = reinterpret_cast<uint32_t*>(cur);
+
+  af1_layer* L = nullptr;
+  rc = create_layer(desc, st, &L);
+  if (rc != AF1_OK) {
+    cudaFree(scratch);
+    return rc;
+  }
+  e = cudaMemsetAsync(flag, 0, 4, st);
+  // U: m rows of r signs, row-major. V^T: r rows of n signs read from the
+  // n x r row-major V (row stride 1, column stride r).
+  if (e == cudaSuccess) e = af1::launch_pack_signs(U, m, r, r, 1, Uw, wu, flag, st);
+  if (e == cudaSuccess) e = af1::launch_pack_signs(V, r, n, 1, r, Vw, wv, flag, st);
+  if (e == cudaSuccess) e = af1::launch_words_to_tiles(Vw, wv, L->p1, L->tiles1, st);
+  if (e == cudaSuccess) e = af1::launch_words_to_tiles(Uw, wu, L->p2, L->tiles2, st);
+  if (e != cudaSuccess) {
+    destroy_layer(L);
+    cudaFree(scratch);
+    return fail_cuda(e, "pack kernels");
+  }
+  rc = copy_scales(L, a, s, b, st);
+  uint32_t hflag = 0;
+  if (rc == AF1_OK) {
+    e = cudaMemcpyAsync(&hflag, flag, 4, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) rc = fail_cuda(e, "pack synchronize");
+  }
+  cudaFree(scratch);
+  if (rc == AF1_OK && hflag != 0) rc = fail(AF1_ERR_INVALID_SIGN, "a sign entry is not exactly +1 or -1");
+  if (rc != AF1_OK) {
+    destroy_layer(L);
+    return rc;
+  }
+  *out = L;
+  g_err.clear();
+  return AF1_OK;
+}
+
+int af1_load_packed_layer(const af1_layer_desc* desc, const uint32_t* U_words, const uint32_t* V_words,
+                          const uint16_t* a, const uint16_t* s, const uint16_t* b, void* stream, af1_layer** out) {
+  if (out == nullptr) return fail(AF1_ERR_INVALID_ARG, "out is NULL");
+  *out = nullptr;
+  int rc = check_desc(desc);
+  if (rc != AF1_OK) return rc;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return fail_cuda(e, "cudaGetDevice");
+  if ((rc = check_device_ptr(U_words, "U_words", dev)) != AF1_OK) return rc;
+  if ((rc = check_device_ptr(V_words, "V_words", dev)) != AF1_OK) return rc;
+  if ((rc = check_scales(a, s, b, dev)) != AF1_OK) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  af1_layer* L = nullptr;
+  rc = create_layer(desc, st, &L);
+  if (rc != AF1_OK) return rc;
+  e = af1::launch_words_to_tiles(V_words, words_per_row(desc->n), L->p1, L->tiles1, st);
+  if (e == cudaSuccess) e = af1::launch_words_to_tiles(U_words, words_per_row(desc->r), L->p2, L->tiles2, st);
+  if (e != cudaSuccess) {
+    destroy_layer(L);
+    return fail_cuda(e, "pack kernels");
+  }
+  rc = copy_scales(L, a, s, b, st);
+  if (rc == AF1_OK) {
+    e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) rc = fail_cuda(e, "load synchronize");
+  }
+  if (rc != AF1_OK) {
+    destroy_layer(L);
+    return rc;
+  }
+  *out = L;
+  g_err.clear();
+  return AF1_OK;
+}
+
+int af1_layer_get_desc(const af1_layer* layer, af1_layer_desc* desc) {
+  if (layer == nullptr || desc == nullptr) return fail(AF1_ERR_INVALID_ARG, "layer or desc is NULL");
+  desc->m = layer->m;
+  desc->n = layer->n;
+  desc->r = layer->r;
+  desc->flags = layer->flags;
+  desc->reserved = 0;
+  return AF1_OK;
+}
+
+int af1_layer_device_bytes(const af1_layer* layer, int64_t* sign_bytes, int64_t* scale_bytes) {
+  if (layer == nullptr) return fail(AF1_ERR_INVALID_ARG, "layer is NULL");
+  if (sign_bytes) *sign_bytes = layer->sign_bytes;
+  if (scale_bytes) *scale_bytes = layer->scale_bytes;
+  return AF1_OK;
+}
+
+int64_t af1_workspace_bytes(const af1_layer* layer, int64_t tokens) {
+  if (layer == nullptr) return fail(AF1_ERR_INVALID_ARG, "layer is NULL");
+  if (tokens < 0) return fail(AF1_ERR_INVALID_ARG, "tokens must be >= 0");
+  return af1::plan_workspace(*layer).total;
+}
+
+int af1_linear_forward(const af1_layer* layer, const void* x, int64_t ldx, int64_t tokens, void* y, int64_t ldy,
+                       int y_dtype, void* workspace, int64_t workspace_bytes, void* stream) {
+  if (layer == nullptr) return fail(AF1_ERR_INVALID_ARG, "layer is NULL");
+  if (tokens < 0) return fail(AF1_ERR_INVALID_ARG, "tokens must be >= 0");
+  if (y_dtype != AF1_F16 && y_dtype != AF1_F32) return fail(AF1_ERR_INVALID_ARG, "y_dtype must be AF1_F16 or AF1_F32");
+  if (tokens == 0) {
+    g_err.clear();
+    return AF1_OK;
+  }
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return fail_cuda(e, "cudaGetDevice");
+  if (dev != layer->device) return fail(AF1_ERR_BAD_POINTER, "the current device is not the layer's device");
+  int rc;
+  if ((rc = check_device_ptr(x, "x", dev)) != AF1_OK) return rc;
+  if ((rc = check_device_ptr(y, "y", dev)) != AF1_OK) return rc;
+  if (workspace == nullptr) return fail(AF1_ERR_WORKSPACE, "workspace is NULL");
+  if ((rc = check_device_ptr(workspace, "workspace", dev)) != AF1_OK) return AF1_ERR_WORKSPACE;
+  if (ldx < layer->n) return fail(AF1_ERR_INVALID_ARG, "ldx < n");
+  if (ldy < layer->m) return fail(AF1_ERR_INVALID_ARG, "ldy < m");
+  if ((reinterpret_cast<uintptr_t>(x) & 15) != 0 || (reinterpret_cast<uintptr_t>(y) & 15) != 0)
+    return fail(AF1_ERR_MISALIGNED, "x and y must be 16-byte aligned");
+  if (ldx % 8 != 0) return fail(AF1_ERR_MISALIGNED, "ldx must be a multiple of 8");
+  if (ldy % (y_dtype == AF1_F16 ? 8 : 4) != 0)
+    return fail(AF1_ERR_MISALIGNED, "ldy * element size must be a multiple of 16 bytes");
+  if ((reinterpret_cast<uintptr_t>(workspace) & 255) != 0)
+    return fail(AF1_ERR_WORKSPACE, "workspace must be 256-byte aligned");
+  const int64_t need = af1::plan_workspace(*layer).total;
+  if (workspace_bytes < need)
+    return fail(AF1_ERR_WORKSPACE, "workspace too small: need " + std::to_string(need) + " bytes");
+  e = af1::launch_forward(*layer, x, ldx, tokens, y, ldy, y_dtype, workspace, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return fail_cuda(e, "forward launch");
+  g_err.clear();
+  return AF1_OK;
+}
+
+int af1_workspace_status(void* workspace, void* stream) {
+  if (workspace == nullptr) return fail(AF1_ERR_WORKSPACE, "workspace is NULL");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  uint32_t h = 0;
+  cudaError_t e = cudaMemcpyAsync(&h, workspace, 4, cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  if (e != cudaSuccess) return fail_cuda(e, "af1_workspace_status");
+  if (h != 0) {
+    cudaMemsetAsync(workspace, 0, 4, st);
+    cudaStreamSynchronize(st);
+    return fail(AF1_ERR_TIMEOUT, "a bounded device-side wait gave up; re-zero the workspace before reuse");
+  }
+  g_err.clear();
+  return AF1_OK;
+}
+
+void af1_free(af1_layer* layer) { destroy_layer(layer); }
+
+const char* af1_last_error(void) { return g_err.c_str(); }
+
+const char* af1_version(void) { return "af1-gb300 0.1.0 (sm_103a)"; }
+
+}  // extern "C"

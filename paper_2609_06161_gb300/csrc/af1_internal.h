@@ -1,0 +1,55 @@
+// af1_internal.h — host-side structures shared by the C-ABI layer and the
+// kernel launchers. Not installed; the public interface is include/af1.h.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <string>
+
+#include "af1_layout.h"
+
+struct af1_layer {
+  int64_t m = 0, n = 0, r = 0;
+  int32_t flags = 0;
+  int device = 0;
+  int num_sms = 0;
+  // Phase 1 contracts V (B = V^T, r x n) with z = b * x; phase 2 contracts
+  // U (m x r) with s' = s * t.
+  af1::TileMatrix p1, p2;
+  uint8_t* tiles1 = nullptr;  // p1.RT * p1.KT * 256 bytes
+  uint8_t* tiles2 = nullptr;
+  uint16_t* a = nullptr;      // FP16 row scale, m entries
+  uint16_t* s = nullptr;      // FP16 rank scale, r entries
+  uint16_t* b = nullptr;      // FP16 column scale, n entries
+  void* alloc = nullptr;      // single device allocation holding all of the above
+  int64_t sign_bytes = 0, scale_bytes = 0;
+};
+
+namespace af1 {
+
+// Workspace carve-up for one layer and a pass of up to kMaxPassTokens tokens.
+struct Workspace {
+  int64_t status = 0;     // uint32 status word
+  int64_t counters1 = 0;  // uint32[p1.RG]
+  int64_t counters2 = 0;  // uint32[p2.RG]
+  int64_t tacc = 0;       // float[kMaxPassTokens][p1.RT*16], zero between calls
+  int64_t sbuf = 0;       // float[kMaxPassTokens][p2.KT*128]
+  int64_t yacc = 0;       // float[kMaxPassTokens][p2.RT*16], zero between calls
+  int64_t total = 0;
+};
+Workspace plan_workspace(const af1_layer& L);
+
+void plan_tiles(TileMatrix& t, int64_t R, int64_t C, int rtc_target, int num_sms, int ktc_max);
+
+// Kernel launchers (stream-ordered, asynchronous). Return cudaSuccess or the
+// launch error.
+cudaError_t launch_pack_signs(const int8_t* src, int64_t rows, int64_t cols, int64_t row_stride,
+                              int64_t col_stride, uint32_t* words, int64_t words_per_row,
+                              uint32_t* bad_flag, cudaStream_t st);
+cudaError_t launch_words_to_tiles(const uint32_t* words, int64_t words_per_row, const TileMatrix& t,
+                                  uint8_t* tiles, cudaStream_t st);
+cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64_t tokens, void* y,
+                           int64_t ldy, int y_dtype, void* ws, cudaStream_t st);
+
+}  // namespace af1

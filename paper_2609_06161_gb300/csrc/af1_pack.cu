@@ -1,0 +1,94 @@
+// af1_pack.cu — sign packing kernels.
+//
+// (1) pack_signs: an int8 matrix of +-1 (the sign factors of AF1 Sec. 3.1,
+//     A_pm1 and B_pm1) -> the canonical words of the packed format declared in
+//     include/af1.h (bit = 1 for +1, LSB first, rows padded to 16 bytes).
+// (2) words_to_tiles: canonical words -> the internal tile layout described in
+//     af1_layout.h. The bit count is unchanged (1 bit per sign); only the
+//     order differs, plus the zero padding of partial tiles.
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "af1_internal.h"
+#include "af1_layout.h"
+
+namespace af1 {
+namespace {
+
+__global__ void pack_signs_kernel(const int8_t* __restrict__ src, int64_t rows, int64_t cols,
+                                  int64_t row_stride, int64_t col_stride, uint32_t* __restrict__ words,
+                                  int64_t wpr, uint32_t* bad_flag) {
+  int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= rows * wpr) return;
+  // Consecutive threads take consecutive rows of one word column, so that a
+  // column-strided source (V read as V^T) is read coalesced.
+  int64_t row = t % rows;
+  int64_t w = t / rows;
+  uint32_t word = 0;
+  bool bad = false;
+#pragma unroll 4
+  for (int b = 0; b < 32; ++b) {
+    int64_t col = w * 32 + b;
+    if (col < cols) {
+      int8_t v = src[row * row_stride + col * col_stride];
+      if (v == 1) {
+        word |= 1u << b;
+      } else if (v != -1) {
+        bad = true;
+      }
+    }
+  }
+  words[row * wpr + w] = word;
+  if (bad) atomicOr(bad_flag, 1u);
+}
+
+__global__ void words_to_tiles_kernel(const uint32_t* __restrict__ words, int64_t wpr, TileMatrix tm,
+                                      uint32_t* __restrict__ tiles) {
+  int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  int64_t total = (int64_t)tm.RT * tm.KT * 64;
+  if (t >= total) return;
+  int which = (int)(t & 1);
+  int lane = (int)((t >> 1) & 31);
+  int64_t rest = t >> 6;
+  int rt = (int)(rest % tm.RT);
+  int kt = (int)(rest / tm.RT);
+  int64_t row = (int64_t)rt * kTileRows + (lane >> 2) + 8 * which;
+  int c = lane & 3;
+  uint32_t out = 0;
+  if (row < tm.R) {
+    const uint32_t* src = words + row * wpr;
+#pragma unroll
+    for (int b = 0; b < 32; ++b) {
+      int64_t col = (int64_t)kt * kTileCols + bit_col(b, c);
+      if (col < tm.C) out |= ((src[col >> 5] >> (col & 31)) & 1u) << b;
+    }
+  }
+  tiles[tile_index(tm, rt, kt) * 64 + lane * 2 + which] = out;
+}
+
+}  // namespace
+
+cudaError_t launch_pack_signs(const int8_t* src, int64_t rows, int64_t cols, int64_t row_stride,
+                              int64_t col_stride, uint32_t* words, int64_t wpr, uint32_t* bad_flag,
+                              cudaStream_t st) {
+  int64_t total = rows * wpr;
+  if (total == 0) return cudaSuccess;
+  int threads = 256;
+  int64_t blocks = (total + threads - 1) / threads;
+  pack_signs_kernel<<<(unsigned)blocks, threads, 0, st>>>(src, rows, cols, row_stride, col_stride, words,
+                                                          wpr, bad_flag);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_words_to_tiles(const uint32_t* words, int64_t wpr, const TileMatrix& tm, uint8_t* tiles,
+                                  cudaStream_t st) {
+  int64_t total = (int64_t)tm.RT * tm.KT * 64;
+  if (total == 0) return cudaSuccess;
+  int threads = 256;
+  int64_t blocks = (total + threads - 1) / threads;
+  words_to_tiles_kernel<<<(unsigned)blocks, threads, 0, st>>>(words, wpr, tm,
+                                                              reinterpret_cast<uint32_t*>(tiles));
+  return cudaGetLastError();
+}
+
+}  // namespace af1
