@@ -1,0 +1,403 @@
+"""Benchmark: AF1 binary-factorized linears on the decode path.
+
+Workload: the seven linears of a LLaMA-3-8B decoder layer (q, k, v, o, gate,
+up, down) at their exact 1.0-BPW ranks, replicated over 32 layers with
+distinct seeded synthetic weights (0.87 GB of packed signs per step, far
+above the 129 MB L2, so no flush is needed). One step is one decode token
+batch (default 1 token) through all 224 linears, issued in model order on one
+stream through af1_linear_forward and replayed as a CUDA graph.
+
+Prints one JSON line. `--impl reference` times the CPU FP64 oracle instead
+(the reference arm of this paper-only build), on a bounded sample per step.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+NCORES = len(os.sched_getaffinity(0))
+for _v in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
+    os.environ.setdefault(_v, str(NCORES))
+
+import numpy as np  # noqa: E402
+
+METRIC = "tokens/s and us/layer for binary-factorized linear (AF1, 1.0 BPW); % of HBM roofline"
+LAYERS = 32
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=50)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--batch", type=int, default=1, help="decode tokens per step (1..16)")
+    p.add_argument("--impl", choices=["af1", "reference"], default="af1")
+    p.add_argument("--layers", type=int, default=LAYERS)
+    p.add_argument("--no-dense", action="store_true", help="skip the dense BF16 baseline")
+    p.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
+    return p.parse_args()
+
+
+def shapes():
+    import synth
+    from oracle import af1_oracle as O  # exact rank rule, host-side bookkeeping only
+    out = []
+    for name, m, n in synth.LLAMA3_8B_LINEARS:
+        out.append((name, m, n, O.rank_for_budget(m, n, 1)))
+    return out
+
+
+def algorithmic_bytes(m, n, r, b):
+    """Logical packed sign bits / 8 + FP16 scales + FP16 x and y."""
+    return r * (m + n) // 8 + 2 * (m + n + r) + 2 * b * n + 2 * b * m
+
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle timing (cpu_baseline and the reference arm)
+# ---------------------------------------------------------------------------
+
+def oracle_layer_sample(batch, seed_base=0):
+    """The 7 linears of one decoder layer, as canonical packed words."""
+    import synth
+    data = []
+    for i, (name, m, n, r) in enumerate(shapes()):
+        d = synth.layer_words(seed_base + i, m, n, r, batch)
+        data.append((name, m, n, r, d))
+    return data
+
+
+def time_oracle_layer(data):
+    from oracle import af1_oracle as O
+    t0 = time.perf_counter()
+    for (_name, m, n, r, d) in data:
+        O.forward_from_packed(d["Uw"], d["Vw"], d["a"], d["s"], d["b"], d["x"], m, n, r)
+    return time.perf_counter() - t0
+
+
+def cpu_baseline(batch, min_seconds=10.0):
+    data = oracle_layer_sample(batch)
+    times = []
+    t_start = time.perf_counter()
+    while True:
+        times.append(time_oracle_layer(data))
+        if time.perf_counter() - t_start >= min_seconds:
+            break
+    per_layer = float(np.median(times))
+    value = batch / (per_layer * LAYERS)
+    return {"value": value, "unit": "tokens/s", "cores": NCORES, "kind": "oracle",
+            "sample": (f"FP64 numpy oracle (unpack + factored forward) on the 7 linears of one decoder layer, "
+                       f"batch {batch}, {len(times)} repetitions ({sum(times):.1f} s), median scaled x{LAYERS} layers; "
+                       f"BLAS threads {NCORES}, unpacking single-threaded")}
+
+
+def run_reference(args):
+    world, rank, _ = dist_env()
+    if rank != 0:
+        return
+    data = oracle_layer_sample(args.batch)
+    for _ in range(max(args.warmup, 0)):
+        time_oracle_layer(data)
+    times = [time_oracle_layer(data) for _ in range(args.steps)]
+    step = float(np.mean(times))
+    value = args.batch / (step * LAYERS)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": step * LAYERS * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (seeded PCG64 signs/scales/activations)",
+        "config": config_dict(args),
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": NCORES, "kind": "oracle",
+                         "sample": (f"each step: FP64 oracle forward of the 7 linears of one decoder layer "
+                                    f"(1/{LAYERS} of the workload), batch {args.batch}; value scaled x{LAYERS}")},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+
+
+def config_dict(args):
+    return {"workload": (f"LLaMA-3-8B-shaped AF1 decoder linears (q,k,v,o 4096x4096 r2028 / k,v 1024x4096 r800 / "
+                         f"gate,up 14336x4096 r3167 / down 4096x14336 r3167) x {args.layers} layers, decode batch "
+                         f"{args.batch}, one stream in model order, CUDA graph"),
+            "batch": args.batch, "layers": args.layers, "linears_per_step": 7 * args.layers,
+            "l2": "inputs larger than L2 (packed weights per step >> 129 MB), no flush"}
+
+
+# ---------------------------------------------------------------------------
+# Clock sampling during the timed region
+# ---------------------------------------------------------------------------
+
+class Clocks:
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = os.path.join("/tmp", f"af1_clocks_{os.getpid()}.csv")
+
+    def start(self):
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.f.close()
+        sm, mx, reasons = [], 0.0, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx = max(mx, float(parts[2]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        os.unlink(self.path)
+        if not sm:
+            return None
+        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# The AF1 arm
+# ---------------------------------------------------------------------------
+
+def build_layers(P, torch, layers, batch, rank):
+    import synth
+    objs = []
+    for li in range(layers):
+        for si, (name, m, n, r) in enumerate(shapes()):
+            d = synth.layer_words(100000 * (rank + 1) + 7 * li + si, m, n, r, batch)
+            f16 = lambda bits: torch.from_numpy(np.ascontiguousarray(bits).view(np.float16)).cuda()
+            Uw = torch.from_numpy(d["Uw"].view(np.int32)).cuda()
+            Vw = torch.from_numpy(d["Vw"].view(np.int32)).cuda()
+            layer = P.Layer.from_words(Uw, Vw, f16(d["a"]), f16(d["s"]), f16(d["b"]), m, n, r)
+            del Uw, Vw
+            x = f16(d["x"]).reshape(batch, n)
+            objs.append((name, m, n, r, layer, x))
+    return objs
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+        return
+    import torch
+    import torch.distributed as dist
+
+    world, rank, local = dist_env()
+    if world > 1:
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    else:
+        torch.cuda.set_device(0)
+    import paper_2609_06161_gb300 as P
+
+    b = args.batch
+    if not 1 <= b <= 16:
+        raise SystemExit("--batch must be in 1..16 for the decode path")
+    dev = torch.device("cuda", torch.cuda.current_device())
+    objs = build_layers(P, torch, args.layers, b, rank)
+    ws = torch.zeros(max(o[4].workspace_bytes(b) for o in objs), dtype=torch.uint8, device=dev)
+    # Inputs and outputs live in one device buffer each so the e2e leg can move
+    # them with a single copy per direction.
+    xs = [o[5] for o in objs]
+    xoff, yoff, xo, yo = [], [], 0, 0
+    for (name, m, n, r, layer, x) in objs:
+        xoff.append(xo)
+        xo += b * n
+        yoff.append(yo)
+        yo += b * m
+    xbuf = torch.empty(xo, dtype=torch.float16, device=dev)
+    ybuf = torch.empty(yo, dtype=torch.float16, device=dev)
+    for i, x in enumerate(xs):
+        xbuf[xoff[i]:xoff[i] + x.numel()].copy_(x.reshape(-1))
+    views = []
+    for i, (name, m, n, r, layer, x) in enumerate(objs):
+        views.append((layer, xbuf[xoff[i]:xoff[i] + b * n].view(b, n), ybuf[yoff[i]:yoff[i] + b * m].view(b, m)))
+
+    stream = torch.cuda.Stream()
+
+    def step():
+        for (layer, xv, yv) in views:
+            layer.forward_into(xv, yv, ws, stream=stream)
+
+    with torch.cuda.stream(stream):
+        step()
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        step()
+    torch.cuda.synchronize()
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    for _ in range(max(args.warmup, 3)):
+        graph.replay()
+    barrier()
+    clocks = Clocks(local)
+    clocks.start()
+    time.sleep(0.3)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier()
+    e0.record(stream)
+    with torch.cuda.stream(stream):
+        for _ in range(args.steps):
+            graph.replay()
+    e1.record(stream)
+    barrier()
+    ms = e0.elapsed_time(e1)
+    clk = clocks.stop()
+    t = torch.tensor([ms], dtype=torch.float64, device=dev)
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    ms_max = float(t.item())
+    ms_step = ms_max / args.steps
+    tokens_per_step = b * world
+    value = tokens_per_step / (ms_step * 1e-3)
+    nlin = len(views)
+    us_layer = ms_step * 1e3 / nlin
+    alg = sum(algorithmic_bytes(m, n, r, b) for (name, m, n, r, layer, x) in objs)
+    achieved_gbs = alg / (ms_step * 1e-3) / 1e9
+
+    # e2e: host buffers in pinned memory, copies inside the timed region.
+    xh = torch.empty(xo, dtype=torch.float16, pin_memory=True)
+    xh.copy_(xbuf.cpu())
+    yh = torch.empty(yo, dtype=torch.float16, pin_memory=True)
+    for _ in range(3):
+        with torch.cuda.stream(stream):
+            xbuf.copy_(xh, non_blocking=True)
+            graph.replay()
+            yh.copy_(ybuf, non_blocking=True)
+        stream.synchronize()
+    barrier()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        with torch.cuda.stream(stream):
+            xbuf.copy_(xh, non_blocking=True)
+            graph.replay()
+            yh.copy_(ybuf, non_blocking=True)
+        stream.synchronize()
+    e2e_s = time.perf_counter() - t0
+    te = torch.tensor([e2e_s], dtype=torch.float64, device=dev)
+    if world > 1:
+        dist.all_reduce(te, op=dist.ReduceOp.MAX)
+    e2e_value = tokens_per_step * args.steps / float(te.item())
+
+    dense = None
+    if not args.no_dense and rank == 0:
+        dense = dense_bf16(torch, objs, b, args, stream)
+
+    if rank == 0:
+        peaks = load_peaks()
+        hbm = peaks.get("hbm_gbs")
+        line = {
+            "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+            "warmup": max(args.warmup, 3), "ms_per_step": ms_step, "us_per_layer": us_layer,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "e4m3 MMA / f32 accumulate (1-bit signs, f16 scales and activations)",
+            "data": "synthetic (seeded PCG64 packed signs, |N(0,0.02)|+1e-3 scales, N(0,1) activations)",
+            "config": config_dict(args),
+            "roofline": {"bound": "hbm", "kernel": "af1_linear_forward (phase-1 + phase-2 kernels, per call)",
+                         "achieved": achieved_gbs, "peak": hbm, "unit": "GB/s",
+                         "frac": (achieved_gbs / hbm) if hbm else None, "peak_source": "MEASURED_PEAKS.json hbm_gbs"
+                         if "hbm_gbs" in peaks else "fallback 6800 GB/s",
+                         "algorithmic_bytes_per_step": alg, "traffic": None},
+            "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": xo * 2,
+                    "d2h_bytes_per_step": yo * 2},
+            "gpu_launches": 2 * nlin * args.steps,
+            "clocks": clk,
+        }
+        if dense is not None:
+            line["dense_bf16_baseline"] = dense
+        if not args.no_cpu and world == 1:
+            line["cpu_baseline"] = cpu_baseline(b)
+        print(json.dumps(line))
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def load_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return json.load(f)
+    except Exception:
+        return {"hbm_gbs": 6800.0}
+
+
+def dense_bf16(torch, objs, b, args, stream):
+    """Same step with dense BF16 weights and torch.matmul (cuBLAS): a reported
+    baseline, not part of the AF1 path."""
+    g = torch.Generator(device="cuda")
+    g.manual_seed(1234)
+    ws, xs = [], []
+    for (name, m, n, r, layer, x) in objs:
+        ws.append(torch.randn((m, n), generator=g, device="cuda", dtype=torch.bfloat16) * 0.02)
+        xs.append(x.to(torch.bfloat16))
+    ys = [None] * len(ws)
+
+    def step():
+        for i in range(len(ws)):
+            ys[i] = torch.matmul(xs[i], ws[i].t())
+
+    with torch.cuda.stream(stream):
+        step()
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        step()
+    for _ in range(3):
+        graph.replay()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    steps = max(5, min(args.steps, 20))
+    e0.record(stream)
+    with torch.cuda.stream(stream):
+        for _ in range(steps):
+            graph.replay()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / steps
+    nbytes = sum(w.numel() * 2 for w in ws)
+    del ws, xs, ys, graph
+    torch.cuda.empty_cache()
+    return {"ms_per_step": ms, "tokens_per_s": b / (ms * 1e-3), "weight_bytes": nbytes,
+            "achieved_gbs": nbytes / (ms * 1e-3) / 1e9}
+
+
+if __name__ == "__main__":
+    main()

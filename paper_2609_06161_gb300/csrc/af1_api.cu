@@ -9,7 +9,7 @@
 #include <new>
 #include <string>
 
-#include "../../include/af1.h"
+#include "af1.h"
 #include "af1_internal.h"
 #include "af1_layout.h"
 
@@ -66,8 +66,8 @@ int check_device_ptr(const void* p, const char* name, int device) {
 int check_desc(const af1_layer_desc* d) {
   if (d == nullptr) return fail(AF1_ERR_INVALID_ARG, "desc is NULL");
   if (d->m <= 0 || d->n <= 0 || d->r <= 0) return fail(AF1_ERR_INVALID_ARG, "m, n and r must be positive");
-  if (d->m > ((int64_t)1 << 30) || d->n > ((int64_t)1 << 30) || d->r > ((int64_t)1 << 30))
-    return fail(AF1_ERR_INVALID_ARG, "m, n or r too large");
+  if (d->m > ((int64_t)1 << 30) || d->n > af1::kMaxCols || d->r > af1::kMaxCols)
+    return fail(AF1_ERR_INVALID_ARG, "m must be <= 2^30 and n, r <= " + std::to_string(af1::kMaxCols));
   if (d->reserved != 0 || (d->flags & ~AF1_FLAG_ANY_RANK) != 0)
     return fail(AF1_ERR_INVALID_ARG, "unknown flags or non-zero reserved field");
   if (!(d->flags & AF1_FLAG_ANY_RANK)) {
@@ -97,8 +97,14 @@ int create_layer(const af1_layer_desc* d, cudaStream_t st, af1_layer** out) {
   L->flags = d->flags;
   L->device = dev;
   L->num_sms = sms;
-  af1::plan_tiles(L->p1, d->r, d->n, /*rtc_target=*/64, sms, /*ktc_max=*/4);
-  af1::plan_tiles(L->p2, d->m, d->r, /*rtc_target=*/16, sms, /*ktc_max=*/af1::kMaxKTC);
+  int max_smem = 0;
+  e = cudaDeviceGetAttribute(&max_smem, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+  if (e != cudaSuccess) {
+    delete L;
+    return fail_cuda(e, "cudaDeviceGetAttribute");
+  }
+  af1::plan_tiles(L->p1, d->r, d->n, sms, max_smem);
+  af1::plan_tiles(L->p2, d->m, d->r, sms, max_smem);
   const int64_t t1 = (int64_t)L->p1.RT * L->p1.KT * af1::kTileBytes;
   const int64_t t2 = (int64_t)L->p2.RT * L->p2.KT * af1::kTileBytes;
   const int64_t sa = align256(2 * d->m), ss = align256(2 * d->r), sb = align256(2 * d->n);

@@ -5,13 +5,18 @@
 //
 // Two kernels per pass of up to 16 tokens, chained with programmatic
 // dependent launch (PDL):
-//   phase 1: t = B z with B = V^T (r x n) and z = b * x; the last CTA of each
-//            row block applies the rank scale, s' = s * t (fp32, workspace).
-//   phase 2: u = U s' (m x r); the last CTA of each row block applies the
-//            row scale, y = a * u, and stores FP16 or FP32.
-// Each CTA owns a block of sign tiles (af1_layout.h). It issues bulk copies
-// (TMA, cp.async.bulk) of its whole block into shared memory before it waits
-// on the previous kernel, so weight streaming overlaps the dependency.
+//   phase 1: t = B z with B = V^T (r x n) and z = b * x; then s' = s * t
+//            (the rank scale), written as FP32 to the workspace.
+//   phase 2: u = U s' (m x r); then y = a * u, stored as FP16 or FP32.
+// Each phase is a sign-matrix product over an R x C tile matrix
+// (af1_layout.h). A CTA owns a block of RTC row tiles x KTC column tiles; the
+// KS CTAs that share a row block form one thread-block cluster and reduce
+// their split-K partial sums through distributed shared memory (each CTA
+// finalises 1/KS of the rows, summing the KS partials in a fixed order), so
+// there are no global atomics and the result is deterministic. Every CTA
+// issues bulk copies (cp.async.bulk) of its whole weight block and loads its
+// scales before it waits on the previous kernel, so weight streaming overlaps
+// the dependency.
 //
 // Sign contraction on FP8 tensor cores. A sign bit is expanded into an e4m3
 // A-fragment byte with one LOP3 per 4 signs: (word & mask_p) | base_p puts
@@ -21,7 +26,7 @@
 // and since sign = 2 bit - 1,
 //     sum_k sign_k z_k = 2 D - Q,   Q = sum_k (L_k + H_k) z'_k   (H = L + d).
 // Each activation z'_k is scaled by a per-(CTA, token) power of two so that
-// its magnitude sits in [128, 256), and is split into 4 e4m3 terms
+// the largest magnitude sits in [128, 256), and is split into 4 e4m3 terms
 // (z' ~ t1 + t2 + t3 + t4, ~16 significant bits) that occupy the 8 columns of
 // an m16n8k32 MMA (2 tokens x 4 terms). Products are exact and the MMA
 // accumulates in FP32, so the only rounding is the term split and FP32
@@ -38,9 +43,10 @@ namespace {
 
 constexpr long long kWaitCycles = 2000000000ll;  // ~1 s at 2 GHz
 constexpr unsigned kStatusTimeout = 1u;
+constexpr int kMaxWarps = 8;
 
 // ---------------------------------------------------------------------------
-// PTX helpers (hand-written; mbarrier, bulk copy, PDL, MMA, FP8 conversion)
+// PTX helpers (hand-written: mbarrier, bulk copy, PDL, cluster, MMA, FP8)
 // ---------------------------------------------------------------------------
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
@@ -94,6 +100,25 @@ __device__ __forceinline__ void griddep_launch_dependents() {
 }
 __device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
+// Split cluster barrier used only to know that every CTA of the cluster has
+// started (required before its shared memory may be written remotely).
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.aligned;" ::: "memory"); }
+
+// Cluster-wide barrier with release/acquire semantics for shared memory.
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// Store a float into the shared memory of CTA `rank` of this cluster, at the
+// offset that `local` has in this CTA.
+__device__ __forceinline__ void st_cluster_f32(float* local, uint32_t rank, float v) {
+  uint32_t remote;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(local)), "r"(rank));
+  asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(remote), "f"(v) : "memory");
+}
+
 __device__ __forceinline__ void mma_e4m3(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
                                          uint32_t b0, uint32_t b1) {
   asm volatile(
@@ -103,18 +128,19 @@ __device__ __forceinline__ void mma_e4m3(float (&d)[4], uint32_t a0, uint32_t a1
       : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
-// Round a float to e4m3 (nearest even, saturating); returns the byte.
-__device__ __forceinline__ uint32_t to_e4m3(float v) {
+// Two floats -> two e4m3 bytes (round to nearest even, saturating); `lo`
+// lands in bits 0..7.
+__device__ __forceinline__ uint32_t e4m3x2(float lo, float hi) {
   uint16_t r;
-  asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(r) : "f"(0.0f), "f"(v));
-  return r & 0xFFu;
+  asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(r) : "f"(hi), "f"(lo));
+  return r;
 }
-// Exact value of an e4m3 byte.
-__device__ __forceinline__ float from_e4m3(uint32_t byte) {
+// Exact values of two e4m3 bytes (bits 0..7 and 8..15).
+__device__ __forceinline__ float2 e4m3x2_value(uint32_t two) {
   uint32_t h2;
-  uint16_t in = static_cast<uint16_t>(byte);
+  uint16_t in = static_cast<uint16_t>(two);
   asm("cvt.rn.f16x2.e4m3x2 %0, %1;" : "=r"(h2) : "h"(in));
-  return __half2float(__ushort_as_half(static_cast<unsigned short>(h2 & 0xFFFFu)));
+  return __half22float2(*reinterpret_cast<__half2*>(&h2));
 }
 
 // Slot p of a word (see af1_layout.h): 1 / d_p and L_p + H_p.
@@ -123,8 +149,6 @@ __device__ __forceinline__ float from_e4m3(uint32_t byte) {
 //   L_p:      1     1     1   1/2     1     1   1/2     1
 __constant__ float c_inv_delta[8] = {8.f, 4.f, 2.f, 2.f, 4.f, 2.f, 2.f, -0.5f};
 __constant__ float c_lph[8] = {2.125f, 2.25f, 2.5f, 1.5f, 2.25f, 2.5f, 1.5f, 0.f};
-__device__ __forceinline__ float slot_inv_delta(int p) { return c_inv_delta[p]; }
-__device__ __forceinline__ float slot_lph(int p) { return c_lph[p]; }
 
 // Expand one lane word into its 8 e4m3 A-fragment registers.
 __device__ __forceinline__ void expand_word(uint32_t w, uint32_t (&s)[8]) {
@@ -140,28 +164,24 @@ __device__ __forceinline__ void expand_word(uint32_t w, uint32_t (&s)[8]) {
 }
 
 // ---------------------------------------------------------------------------
-// Kernel arguments
+// Kernel arguments and shared-memory plan
 // ---------------------------------------------------------------------------
 
 struct PhaseArgs {
   const uint8_t* tiles;
   TileMatrix tm;
   int tokens;
-  // phase 1 input: z = colscale * x
+  // phase 1 input: z = colscale * x (FP16)
   const __half* x;
   int64_t ldx;
   const __half* colscale;
-  // phase 2 input: z = zin
+  // phase 2 input: z = zin (FP32)
   const float* zin;
   int64_t ldz;
-  // cross-CTA accumulation (zero on entry, left zero)
-  float* acc;
-  int64_t ldacc;
-  unsigned* counters;
   unsigned* status;
-  // finalisation
+  // finalisation: out = rowscale * (sum over the row)
   const __half* rowscale;
-  float* sout;  // phase 1: s' = s * t
+  float* sout;  // phase 1
   int64_t lds;
   void* y;  // phase 2
   int64_t ldy;
@@ -170,115 +190,150 @@ struct PhaseArgs {
 
 struct SmemHeader {
   uint64_t mbar[kMaxKTC];
-  float scale[kMaxPassTokens];   // 2^sigma per token
-  float iscale[kMaxPassTokens];  // 2^-sigma
-  float q[kMaxPassTokens];
-  float red[32 * kMaxPassTokens];
-  unsigned flag;
+  float maxv[kMaxPassTokens * kMaxWarps];  // per-warp max |z / d| per token
+  float qpart[kMaxPassTokens * kMaxWarps]; // per-warp partial Q per token
 };
 constexpr int kHeaderBytes = ((int)sizeof(SmemHeader) + 127) / 128 * 128;
 
-template <int PHASE>
-__device__ __forceinline__ float fetch_z(const PhaseArgs& a, int tok, int64_t k) {
-  if (PHASE == 1) {
-    return __half2float(a.colscale[k]) * __half2float(a.x[(int64_t)tok * a.ldx + k]);
-  } else {
-    return a.zin[(int64_t)tok * a.ldz + k];
-  }
+// Rows of a block that each of the KS CTAs of a cluster finalises.
+__host__ __device__ inline int slice_rows(int rtc, int ks_count) {
+  return (rtc * kTileRows + ks_count - 1) / ks_count;
 }
 
-// Block-wide reduction of NV values per thread (max or sum), result in hdr.red[0..NV).
-template <int NV, bool MAX, int WARPS>
-__device__ __forceinline__ void block_reduce(float (&v)[NV], float* red) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-#pragma unroll
-  for (int i = 0; i < NV; ++i) {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      float other = __shfl_xor_sync(0xffffffffu, v[i], o);
-      v[i] = MAX ? fmaxf(v[i], other) : v[i] + other;
+struct SmemPlan {
+  int frag, wts, recv, rs, bi, total;
+};
+
+__host__ __device__ inline int align128(int v) { return (v + 127) / 128 * 128; }
+
+// Shared-memory regions of one CTA; every region starts on a 128-byte
+// boundary (bulk-copy destinations and vector accesses need >= 16 bytes).
+__host__ __device__ inline SmemPlan smem_plan(const TileMatrix& tm, int ng) {
+  SmemPlan p;
+  const int slice = slice_rows(tm.RTC, tm.KS);
+  int off = kHeaderBytes;
+  p.frag = off;
+  off = align128(off + tm.KTC * 4 * ng * 256);
+  p.wts = off;
+  off = align128(off + tm.RTC * tm.KTC * kTileBytes);
+  p.recv = off;  // [KS][2 * ng][slice] partial sums pushed by the cluster
+  off = align128(off + tm.KS * 2 * ng * slice * 4);
+  p.rs = off;
+  off = align128(off + slice * 4);
+  p.bi = off;
+  off = align128(off + tm.KTC * kTileCols * 4);
+  p.total = off;
+  return p;
+}
+
+// Four consecutive activations of one token (zero beyond column C). The
+// inputs may have been written by the kernel this one overlaps with through
+// programmatic dependent launch, so they are read through L2 (ld.global.cg),
+// never through the non-coherent L1/texture path.
+template <int PHASE>
+__device__ __forceinline__ float4 load_z4(const PhaseArgs& a, int tok, int64_t k) {
+  const int64_t C = a.tm.C;
+  float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (PHASE == 1) {
+    const __half* p = a.x + (int64_t)tok * a.ldx + k;
+    if (k + 3 < C) {
+      const uint2 raw = __ldcg(reinterpret_cast<const uint2*>(p));
+      const float2 f0 = __half22float2(*reinterpret_cast<const __half2*>(&raw.x));
+      const float2 f1 = __half22float2(*reinterpret_cast<const __half2*>(&raw.y));
+      z = make_float4(f0.x, f0.y, f1.x, f1.y);
+    } else {
+      if (k < C) z.x = __half2float(__ldcg(p));
+      if (k + 1 < C) z.y = __half2float(__ldcg(p + 1));
+      if (k + 2 < C) z.z = __half2float(__ldcg(p + 2));
+    }
+  } else {
+    const float* p = a.zin + (int64_t)tok * a.ldz + k;
+    if (k + 3 < C) {
+      z = __ldcg(reinterpret_cast<const float4*>(p));
+    } else {
+      if (k < C) z.x = __ldcg(p);
+      if (k + 1 < C) z.y = __ldcg(p + 1);
+      if (k + 2 < C) z.z = __ldcg(p + 2);
     }
   }
-  __syncthreads();
-  if (lane == 0) {
+  return z;
+}
+
+__device__ __forceinline__ float warp_max(float v) {
 #pragma unroll
-    for (int i = 0; i < NV; ++i) red[warp * NV + i] = v[i];
-  }
-  __syncthreads();
-  if (threadIdx.x < NV) {
-    float r = red[threadIdx.x];
-    for (int w = 1; w < WARPS; ++w) {
-      float o = red[w * NV + threadIdx.x];
-      r = MAX ? fmaxf(r, o) : r + o;
-    }
-    red[WARPS * NV + threadIdx.x] = r;
-  }
-  __syncthreads();
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// sigma for a token from the per-warp maxima: 2^sigma * max in [128, 256).
+template <int WARPS>
+__device__ __forceinline__ int token_sigma(const SmemHeader& h, int tok) {
+  float m = 0.f;
+#pragma unroll
+  for (int w = 0; w < WARPS; ++w) m = fmaxf(m, h.maxv[tok * WARPS + w]);
+  int e = 0;
+  if (m > 0.f) frexpf(m, &e);  // m = f * 2^e, f in [0.5, 1)
+  return m > 0.f ? 8 - e : 0;
 }
 
 // Build the e4m3 B fragments of this CTA's column range for all token slots
-// (2 * NG), plus the per-token scale 2^sigma and the constant Q.
+// (2 * NG). bi[kl] holds colscale * (1 / d) (phase 1) or 1 / d (phase 2), and
+// 0 beyond column C (staged and published by the caller). Two CTA barriers:
+// one after the maxima, one after the fragments.
 template <int PHASE, int NG, int WARPS>
-__device__ void build_fragments(const PhaseArgs& a, SmemHeader& h, uint8_t* frag, int64_t k0, int ncols) {
+__device__ void build_fragments(const PhaseArgs& a, SmemHeader& h, uint32_t* frag32, const float* bi, int64_t k0,
+                                int ncols) {
   constexpr int NT = 2 * NG;
+  constexpr int NTH = WARPS * 32;
   const int T = a.tokens;
-  const int64_t C = a.tm.C;
-  // pass A: max |z / d| per token
-  float mx[NT];
-#pragma unroll
-  for (int t = 0; t < NT; ++t) mx[t] = 0.f;
-  for (int kl = threadIdx.x; kl < ncols; kl += WARPS * 32) {
-    const int64_t k = k0 + kl;
-    if (k < C) {
-      const float invd = fabsf(slot_inv_delta((kl & 127) >> 4));
-#pragma unroll
-      for (int t = 0; t < NT; ++t) {
-        if (t < T) mx[t] = fmaxf(mx[t], fabsf(fetch_z<PHASE>(a, t, k)) * invd);
-      }
+  const int n4 = ncols >> 2;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  for (int tok = 0; tok < T; ++tok) {
+    float mx = 0.f;
+    for (int c4 = threadIdx.x; c4 < n4; c4 += NTH) {
+      const float4 z = load_z4<PHASE>(a, tok, k0 + 4 * c4);
+      const float4 w = *reinterpret_cast<const float4*>(bi + 4 * c4);
+      mx = fmaxf(mx, fmaxf(fmaxf(fabsf(z.x * w.x), fabsf(z.y * w.y)), fmaxf(fabsf(z.z * w.z), fabsf(z.w * w.w))));
     }
-  }
-  block_reduce<NT, true, WARPS>(mx, h.red);
-  if (threadIdx.x < NT) {
-    const float m = h.red[WARPS * NT + threadIdx.x];
-    int e = 0;
-    if (m > 0.f) frexpf(m, &e);  // m = f * 2^e, f in [0.5, 1)
-    const int sigma = (m > 0.f) ? 8 - e : 0;  // 2^sigma * m in [128, 256)
-    h.scale[threadIdx.x] = ldexpf(1.f, sigma);
-    h.iscale[threadIdx.x] = ldexpf(1.f, -sigma);
+    mx = warp_max(mx);
+    if (lane == 0) h.maxv[tok * WARPS + warp] = mx;
   }
   __syncthreads();
-  // pass B: split into 4 e4m3 terms, scatter into fragment order, sum Q
-  float q[NT];
-#pragma unroll
-  for (int t = 0; t < NT; ++t) q[t] = 0.f;
-  for (int kl = threadIdx.x; kl < ncols; kl += WARPS * 32) {
-    const int64_t k = k0 + kl;
-    const int p = (kl & 127) >> 4;
-    const float invd = slot_inv_delta(p);
-    const float lph = slot_lph(p);
-    const int kt_l = kl >> 7, kk = kl & 127, mu = kk >> 5, r32 = kk & 31;
-    const int breg = r32 >> 4, c = (r32 & 15) >> 2, e = r32 & 3;
-#pragma unroll
-    for (int t = 0; t < NT; ++t) {
-      float rem = 0.f;
-      if (t < T && k < C) rem = fetch_z<PHASE>(a, t, k) * invd * h.scale[t];
-      const int gamma = t >> 1;
-      float tsum = 0.f;
+#pragma unroll 1
+  for (int tok = 0; tok < NT; ++tok) {
+    const float sc = tok < T ? ldexpf(1.f, token_sigma<WARPS>(h, tok)) : 0.f;
+    const int gam = tok >> 1, tb = (tok & 1) * 4;
+    float q = 0.f;
+    for (int c4 = threadIdx.x; c4 < n4; c4 += NTH) {
+      float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (tok < T) {
+        const float4 z = load_z4<PHASE>(a, tok, k0 + 4 * c4);
+        const float4 w = *reinterpret_cast<const float4*>(bi + 4 * c4);
+        v = make_float4(z.x * w.x * sc, z.y * w.y * sc, z.z * w.z * sc, z.w * w.w * sc);
+      }
+      const float4 v0 = v;
+      const int kt_l = c4 >> 5, mu = (c4 >> 3) & 3, breg = (c4 >> 2) & 1, c = c4 & 3;
+      uint32_t* dst = frag32 + ((((kt_l * 4 + mu) * NG + gam) * 32 + 4 * tb + c) * 2 + breg);
 #pragma unroll
       for (int term = 0; term < kTerms; ++term) {
-        const uint32_t byte = to_e4m3(rem);
-        const float back = from_e4m3(byte);
-        rem -= back;
-        tsum += back;
-        const int g = 4 * (t & 1) + term;
-        const int lane_f = 4 * g + c;
-        frag[((((kt_l * 4 + mu) * NG + gamma) * 32 + lane_f) * 8) + breg * 4 + e] = (uint8_t)byte;
+        const uint32_t lo = e4m3x2(v.x, v.y), hi = e4m3x2(v.z, v.w);
+        const float2 blo = e4m3x2_value(lo), bhi = e4m3x2_value(hi);
+        v.x -= blo.x;
+        v.y -= blo.y;
+        v.z -= bhi.x;
+        v.w -= bhi.y;
+        dst[term * 4 * 2] = lo | (hi << 16);  // column g = tb + term: 4 lanes per g
       }
-      q[t] += lph * tsum;
+      q += c_lph[(c4 >> 2) & 7] * (((v0.x - v.x) + (v0.y - v.y)) + ((v0.z - v.z) + (v0.w - v.w)));
     }
+    q = warp_sum(q);
+    if (lane == 0) h.qpart[tok * WARPS + warp] = q;
   }
-  block_reduce<NT, false, WARPS>(q, h.red);
-  if (threadIdx.x < NT) h.q[threadIdx.x] = h.red[WARPS * NT + threadIdx.x];
   __syncthreads();
 }
 
@@ -287,34 +342,71 @@ __global__ void __launch_bounds__(WARPS * 32) phase_kernel(const PhaseArgs a) {
   extern __shared__ __align__(128) uint8_t smem[];
   SmemHeader& h = *reinterpret_cast<SmemHeader*>(smem);
   const TileMatrix& tm = a.tm;
-  uint8_t* frag = smem + kHeaderBytes;
-  uint8_t* wts = frag + tm.KTC * 4 * NG * 256;
+  const SmemPlan sp = smem_plan(tm, NG);
+  uint32_t* frag32 = reinterpret_cast<uint32_t*>(smem + sp.frag);
+  uint8_t* wts = smem + sp.wts;
+  float* recv = reinterpret_cast<float*>(smem + sp.recv);
+  float* rs = reinterpret_cast<float*>(smem + sp.rs);
+  float* bi = reinterpret_cast<float*>(smem + sp.bi);
 
-  const int rg = blockIdx.x, ks = blockIdx.y;
+  const int rg = blockIdx.x, ks = blockIdx.y, KS = gridDim.y;
   const int rtc = blk_rows(tm, rg), ktc = blk_cols(tm, ks);
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const uint32_t chunk = (uint32_t)rtc * kTileBytes;
-  const uint8_t* gblk = a.tiles + blk_base(tm, rg, ks) * kTileBytes;
+  const int64_t row0 = (int64_t)rg * tm.RTC * kTileRows;
+  const int64_t k0 = (int64_t)ks * tm.KTC * kTileCols;
+  const int slice = slice_rows(rtc, KS);   // rows finalised per CTA
+  const int my0 = ks * slice;              // first block row this CTA finalises
 
+  cluster_arrive_relaxed();  // this CTA has started (matched by cluster_wait)
   if (tid == 0) {
+    // Barriers and weight copies; the first CTA barrier in build_fragments
+    // publishes the initialised barriers to the other warps.
+    const uint32_t chunk = (uint32_t)rtc * kTileBytes;
+    const uint8_t* gblk = a.tiles + blk_base(tm, rg, ks) * kTileBytes;
     for (int i = 0; i < ktc; ++i) mbar_init(&h.mbar[i], 1);
     fence_barrier_init();
-  }
-  __syncthreads();
-  if (tid == 0) {
     for (int i = 0; i < ktc; ++i) {
       mbar_expect_tx(&h.mbar[i], chunk);
       bulk_g2s(wts + (size_t)i * chunk, gblk + (size_t)i * chunk, chunk, &h.mbar[i]);
     }
   }
-  // The weights do not depend on earlier kernels; everything below does.
+  // Layer constants: row scales of the rows this CTA finalises, column
+  // factors of its column slice.
+  for (int i = tid; i < slice; i += WARPS * 32) {
+    const int64_t row = row0 + my0 + i;
+    rs[i] = (my0 + i < rtc * kTileRows && row < tm.R) ? __half2float(a.rowscale[row]) : 0.f;
+  }
+  for (int i = tid; i < ktc * kTileCols; i += WARPS * 32) {
+    const int64_t k = k0 + i;
+    float v = 0.f;
+    if (k < tm.C) v = c_inv_delta[(i & 127) >> 4] * (PHASE == 1 ? __half2float(a.colscale[k]) : 1.f);
+    bi[i] = v;
+  }
+  // Everything above is independent of earlier kernels; everything below
+  // may read their outputs.
   griddep_launch_dependents();
   griddep_wait();
+  __syncthreads();  // rs / bi staged by all warps are read by every warp below
 
-  build_fragments<PHASE, NG, WARPS>(a, h, frag, (int64_t)ks * tm.KTC * kTileCols, ktc * kTileCols);
+  build_fragments<PHASE, NG, WARPS>(a, h, frag32, bi, k0, ktc * kTileCols);
+  // Every CTA of the cluster has started, so partials may be pushed into
+  // peers' shared memory from here on.
+  cluster_wait();
 
   const int g = lane >> 2, c = lane & 3;
   const int T = a.tokens;
+  // Per-thread constants of the tokens this lane finalises: 2 * gg + (c >> 1).
+  float qv[NG], is[NG];
+#pragma unroll
+  for (int gg = 0; gg < NG; ++gg) {
+    const int tok = 2 * gg + (c >> 1);
+    float q = 0.f;
+#pragma unroll
+    for (int w = 0; w < WARPS; ++w) q += h.qpart[tok * WARPS + w];
+    qv[gg] = q;
+    is[gg] = tok < T ? ldexpf(1.f, -token_sigma<WARPS>(h, tok)) : 0.f;
+  }
+
   bool ok = true;
   const int rt_per_warp = (rtc + WARPS - 1) / WARPS;
   for (int j0 = 0; j0 < rt_per_warp && ok; j0 += TPP) {
@@ -334,7 +426,7 @@ __global__ void __launch_bounds__(WARPS * 32) phase_kernel(const PhaseArgs a) {
       for (int mu = 0; mu < 4; ++mu)
 #pragma unroll
         for (int gg = 0; gg < NG; ++gg) {
-          const uint2 v = *reinterpret_cast<const uint2*>(frag + ((((kt_l * 4 + mu) * NG + gg) * 32 + lane) * 8));
+          const uint2 v = *reinterpret_cast<const uint2*>(frag32 + (((kt_l * 4 + mu) * NG + gg) * 32 + lane) * 2);
           bf[mu][gg][0] = v.x;
           bf[mu][gg][1] = v.y;
         }
@@ -356,12 +448,12 @@ __global__ void __launch_bounds__(WARPS * 32) phase_kernel(const PhaseArgs a) {
       }
     }
     if (!ok) break;
-    // Partial sums of these row tiles -> cross-CTA accumulation buffer.
+    // (2 D - Q) 2^-sigma of these row tiles, pushed into the shared memory of
+    // the cluster CTA that finalises each row (slot ks of its buffer).
 #pragma unroll
     for (int j = 0; j < TPP; ++j) {
       const int rt_l = warp + WARPS * (j0 + j);
       if (rt_l < rtc) {
-        const int64_t row0 = (int64_t)(rg * tm.RTC + rt_l) * kTileRows + g;
 #pragma unroll
         for (int gg = 0; gg < NG; ++gg) {
           float vlo = acc[j][gg][0] + acc[j][gg][1];
@@ -370,51 +462,46 @@ __global__ void __launch_bounds__(WARPS * 32) phase_kernel(const PhaseArgs a) {
           vhi += __shfl_xor_sync(0xffffffffu, vhi, 1);
           const int tok = 2 * gg + (c >> 1);
           if ((c & 1) == 0 && tok < T) {
-            const float qv = h.q[tok], is = h.iscale[tok];
-            if (row0 < tm.R) atomicAdd(a.acc + (int64_t)tok * a.ldacc + row0, (2.f * vlo - qv) * is);
-            if (row0 + 8 < tm.R) atomicAdd(a.acc + (int64_t)tok * a.ldacc + row0 + 8, (2.f * vhi - qv) * is);
+#pragma unroll
+            for (int half = 0; half < 2; ++half) {
+              const int rl = rt_l * kTileRows + g + 8 * half;
+              const int owner = rl / slice;
+              float* dst = recv + ((ks * 2 * NG + tok) * slice + (rl - owner * slice));
+              st_cluster_f32(dst, (uint32_t)owner, (2.f * (half ? vhi : vlo) - qv[gg]) * is[gg]);
+            }
           }
         }
       }
     }
   }
 
-  if (!__syncthreads_and(ok ? 1 : 0)) {
-    // A bulk copy never completed: flag it, let the copies drain (bounded),
-    // and leave without touching the shared bookkeeping.
-    if (tid == 0) {
-      atomicOr(a.status, kStatusTimeout);
-      for (int i = 0; i < ktc; ++i) mbar_wait_bounded(&h.mbar[i], 0);
-    }
-    return;
+  const bool all_ok = __syncthreads_and(ok ? 1 : 0) != 0;
+  if (!all_ok && tid == 0) {
+    // A bulk copy never completed: flag it and let the copies drain
+    // (bounded). The cluster barrier is still honoured so that no CTA of the
+    // cluster waits on this one.
+    atomicOr(a.status, kStatusTimeout);
+    for (int i = 0; i < ktc; ++i) mbar_wait_bounded(&h.mbar[i], 0);
   }
-
-  if (tid == 0) {
-    __threadfence();
-    const unsigned old = atomicAdd(a.counters + rg, 1u);
-    const unsigned last = (old == gridDim.y - 1) ? 1u : 0u;
-    if (last) a.counters[rg] = 0u;
-    h.flag = last;
-  }
-  __syncthreads();
-  if (!h.flag) return;
-  __threadfence();
-  const int nrows = rtc * kTileRows;
-  const int64_t r0 = (int64_t)rg * tm.RTC * kTileRows;
-  for (int idx = tid; idx < T * nrows; idx += WARPS * 32) {
-    const int tok = idx / nrows;
-    const int64_t row = r0 + (idx - tok * nrows);
-    if (row >= tm.R) continue;
-    float* p = a.acc + (int64_t)tok * a.ldacc + row;
-    const float v = __ldcg(p);
-    __stcg(p, 0.f);
-    const float sc = __half2float(a.rowscale[row]);
-    if (PHASE == 1) {
-      a.sout[(int64_t)tok * a.lds + row] = v * sc;
-    } else if (a.ydtype == 0) {
-      reinterpret_cast<__half*>(a.y)[(int64_t)tok * a.ldy + row] = __float2half_rn(v * sc);
-    } else {
-      reinterpret_cast<float*>(a.y)[(int64_t)tok * a.ldy + row] = v * sc;
+  // All partials of the cluster have landed in their owners' buffers.
+  cluster_sync();
+  const int cnt = min(slice, rtc * kTileRows - my0);
+  if (all_ok && cnt > 0) {
+    for (int idx = tid; idx < T * cnt; idx += WARPS * 32) {
+      const int tok = idx / cnt;
+      const int i = idx - tok * cnt;
+      const int64_t row = row0 + my0 + i;
+      if (row >= tm.R) continue;
+      float v = 0.f;
+      for (int q = 0; q < KS; ++q) v += recv[(q * 2 * NG + tok) * slice + i];
+      const float out = v * rs[i];
+      if (PHASE == 1) {
+        a.sout[(int64_t)tok * a.lds + row] = out;
+      } else if (a.ydtype == 0) {
+        reinterpret_cast<__half*>(a.y)[(int64_t)tok * a.ldy + row] = __float2half_rn(out);
+      } else {
+        reinterpret_cast<float*>(a.y)[(int64_t)tok * a.ldy + row] = out;
+      }
     }
   }
 }
@@ -423,34 +510,37 @@ __global__ void __launch_bounds__(WARPS * 32) phase_kernel(const PhaseArgs a) {
 // Host side
 // ---------------------------------------------------------------------------
 
-constexpr int kWarps1 = 8, kWarps2 = 4;
+constexpr int kWarps = 8;
 
 template <int NG>
 constexpr int tpp_for() {
-  return NG == 1 ? 8 : NG == 2 ? 4 : NG == 4 ? 2 : 1;
-}
-
-int64_t smem_bytes(const TileMatrix& tm, int ng) {
-  return kHeaderBytes + (int64_t)tm.KTC * 4 * ng * 256 + (int64_t)tm.RTC * tm.KTC * kTileBytes;
+  return NG == 1 ? 4 : NG == 2 ? 2 : 1;
 }
 
 template <int PHASE, int NG>
 cudaError_t launch_phase(const PhaseArgs& a, cudaStream_t st) {
-  constexpr int W = PHASE == 1 ? kWarps1 : kWarps2;
-  auto kern = phase_kernel<PHASE, NG, W, tpp_for<NG>()>;
-  const int64_t smem = smem_bytes(a.tm, NG);
-  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  auto kern = phase_kernel<PHASE, NG, kWarps, tpp_for<NG>()>;
+  const int smem = smem_plan(a.tm, NG).total;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
+  if (a.tm.KS > 8) {
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    if (e != cudaSuccess) return e;
+  }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)a.tm.RG, (unsigned)a.tm.KS, 1);
-  cfg.blockDim = dim3(W * 32, 1, 1);
+  cfg.blockDim = dim3(kWarps * 32, 1, 1);
   cfg.dynamicSmemBytes = (size_t)smem;
   cfg.stream = st;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = 1;
+  attr[1].val.clusterDim.y = (unsigned)a.tm.KS;
+  attr[1].val.clusterDim.z = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   return cudaLaunchKernelEx(&cfg, kern, a);
 }
 
@@ -468,20 +558,38 @@ int64_t align256(int64_t v) { return (v + 255) / 256 * 256; }
 
 }  // namespace
 
-void plan_tiles(TileMatrix& t, int64_t R, int64_t C, int rtc_target, int num_sms, int ktc_max) {
+int forward_smem_bytes(const TileMatrix& t, int ng) { return smem_plan(t, ng).total; }
+
+void plan_tiles(TileMatrix& t, int64_t R, int64_t C, int num_sms, int max_smem) {
   t.R = R;
   t.C = C;
   t.RT = (int)((R + kTileRows - 1) / kTileRows);
   t.KT = (int)((C + kTileCols - 1) / kTileCols);
-  t.RTC = t.RT < rtc_target ? t.RT : rtc_target;
-  t.RG = (t.RT + t.RTC - 1) / t.RTC;
+  // Split K over a cluster of KS CTAs, each holding KTC column tiles.
+  if (t.KT <= 8) {
+    t.KS = t.KT;
+    t.KTC = 1;
+  } else {
+    // Portable clusters of up to 8 CTAs with at most 8 column tiles each;
+    // beyond 64 column tiles, clusters of up to 16 (at most kMaxKTC tiles).
+    t.KTC = (t.KT + 7) / 8;
+    if (t.KTC > 8) t.KTC = (t.KT + 15) / 16;
+    t.KS = (t.KT + t.KTC - 1) / t.KTC;
+  }
+  // Row tiles per block: aim for about two CTAs per SM, at least 8 row tiles
+  // so that the per-CTA activation split is amortised, at most 32.
   const int sms = num_sms > 0 ? num_sms : 148;
-  int ktc = (int)((double)t.RG * t.KT / (2.0 * sms) + 0.5);
-  if (ktc < 1) ktc = 1;
-  if (ktc > ktc_max) ktc = ktc_max;
-  if (ktc > t.KT) ktc = t.KT;
-  t.KTC = ktc;
-  t.KS = (t.KT + t.KTC - 1) / t.KTC;
+  int rtc = (int)(((int64_t)t.RT * t.KS + sms) / (2 * sms));
+  if (rtc < 8) rtc = 8;
+  if (rtc > 32) rtc = 32;
+  if (rtc > t.RT) rtc = t.RT;
+  t.RTC = rtc;
+  while (t.RTC > 1) {
+    t.RG = (t.RT + t.RTC - 1) / t.RTC;
+    if (smem_plan(t, 8).total <= max_smem) break;
+    t.RTC = (t.RTC + 1) / 2;
+  }
+  t.RG = (t.RT + t.RTC - 1) / t.RTC;
 }
 
 Workspace plan_workspace(const af1_layer& L) {
@@ -489,16 +597,8 @@ Workspace plan_workspace(const af1_layer& L) {
   int64_t off = 0;
   w.status = off;
   off += 256;
-  w.counters1 = off;
-  off += align256((int64_t)L.p1.RG * 4);
-  w.counters2 = off;
-  off += align256((int64_t)L.p2.RG * 4);
-  w.tacc = off;
-  off += align256((int64_t)kMaxPassTokens * L.p1.RT * kTileRows * 4);
   w.sbuf = off;
   off += align256((int64_t)kMaxPassTokens * L.p2.KT * kTileCols * 4);
-  w.yacc = off;
-  off += align256((int64_t)kMaxPassTokens * L.p2.RT * kTileRows * 4);
   w.total = off;
   return w;
 }
@@ -519,9 +619,6 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
     p1.x = static_cast<const __half*>(x) + t0 * ldx;
     p1.ldx = ldx;
     p1.colscale = reinterpret_cast<const __half*>(L.b);
-    p1.acc = reinterpret_cast<float*>(wsb + W.tacc);
-    p1.ldacc = (int64_t)L.p1.RT * kTileRows;
-    p1.counters = reinterpret_cast<unsigned*>(wsb + W.counters1);
     p1.status = reinterpret_cast<unsigned*>(wsb + W.status);
     p1.rowscale = reinterpret_cast<const __half*>(L.s);
     p1.sout = reinterpret_cast<float*>(wsb + W.sbuf);
@@ -535,9 +632,6 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
     p2.tokens = T;
     p2.zin = p1.sout;
     p2.ldz = p1.lds;
-    p2.acc = reinterpret_cast<float*>(wsb + W.yacc);
-    p2.ldacc = (int64_t)L.p2.RT * kTileRows;
-    p2.counters = reinterpret_cast<unsigned*>(wsb + W.counters2);
     p2.status = p1.status;
     p2.rowscale = reinterpret_cast<const __half*>(L.a);
     p2.y = static_cast<uint8_t*>(y) + t0 * ldy * ysize;

@@ -30,17 +30,15 @@ namespace af1 {
 
 // Workspace carve-up for one layer and a pass of up to kMaxPassTokens tokens.
 struct Workspace {
-  int64_t status = 0;     // uint32 status word
-  int64_t counters1 = 0;  // uint32[p1.RG]
-  int64_t counters2 = 0;  // uint32[p2.RG]
-  int64_t tacc = 0;       // float[kMaxPassTokens][p1.RT*16], zero between calls
-  int64_t sbuf = 0;       // float[kMaxPassTokens][p2.KT*128]
-  int64_t yacc = 0;       // float[kMaxPassTokens][p2.RT*16], zero between calls
+  int64_t status = 0;  // uint32 status word
+  int64_t sbuf = 0;    // float[kMaxPassTokens][p2.KT*128]: s' = s * t from phase 1
   int64_t total = 0;
 };
 Workspace plan_workspace(const af1_layer& L);
 
-void plan_tiles(TileMatrix& t, int64_t R, int64_t C, int rtc_target, int num_sms, int ktc_max);
+// Choose the tile blocks and the split-K cluster of one sign matrix.
+void plan_tiles(TileMatrix& t, int64_t R, int64_t C, int num_sms, int max_smem);
+int forward_smem_bytes(const TileMatrix& t, int ng);
 
 // Kernel launchers (stream-ordered, asynchronous). Return cudaSuccess or the
 // launch error.

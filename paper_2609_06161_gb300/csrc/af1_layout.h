@@ -37,7 +37,8 @@ constexpr int kTileBytes = 256;
 constexpr int kTerms = 4;             // e4m3 terms per activation value
 constexpr int kTokensPerGroup = 2;    // MMA n = 8 columns = 2 tokens x 4 terms
 constexpr int kMaxPassTokens = 16;    // tokens per kernel pass
-constexpr int kMaxKTC = 8;            // column tiles per CTA block
+constexpr int kMaxKTC = 16;           // column tiles per CTA block (one mbarrier each)
+constexpr int kMaxCols = kMaxKTC * 16 * 128;  // longest contraction: 16 CTAs x 16 tiles
 
 struct TileMatrix {
   int64_t R = 0, C = 0;  // valid rows / columns

@@ -257,3 +257,20 @@ def test_error_codes(P):
     assert e.value.code == -4
     P.workspace_status(ws)
     layer.free()
+
+
+def test_first_calls_interleaved_with_other_layers(P):
+    """Each layer's first forward call, with a fresh workspace that the
+    allocator may place where another layer's workspace just was. Inputs a
+    preceding kernel may have written must never be served stale."""
+    shapes = [(520, 2000, 600), (1024, 4096, 800), (256, 384, 200), (1024, 4096, 800), (1000, 700, 321)]
+    for rep in range(3):
+        for i, (m, n, r) in enumerate(shapes):
+            tokens = (1, 3, 5, 9, 2)[(i + rep) % 5]
+            d = synth.layer_signs(900 + 10 * rep + i, m, n, r, tokens)
+            layer = signs_layer(P, d)
+            y = run_gpu(layer, d["x"], n, torch.float32)
+            ref = oracle_from_signs(d, n)
+            for t in range(tokens):
+                assert O.rowwise_rel_err(y[t:t + 1], ref[t:t + 1]) <= TOL, (m, n, r, tokens, t)
+            layer.free()
