@@ -149,6 +149,24 @@ AF1_API int af1_linear_forward(const af1_layer* layer, const void* x, int64_t ld
                        void* y, int64_t ldy, int y_dtype, void* workspace,
                        int64_t workspace_bytes, void* stream);
 
+/* af1_linear_forward for callers that cannot allocate device memory when
+ * they run a layer: for example a runtime that reserves all GPU memory at
+ * start-up and forbids later cudaMalloc calls, or a plugin whose host owns
+ * the allocator and hands it no scratch buffer. The paper has no counterpart;
+ * this is a deployment convenience.
+ * Same arguments as af1_linear_forward minus the workspace: the scratch is a
+ * 1 MiB array compiled into the library, present on every GPU that loads it
+ * until the process exits. Nothing is allocated by this call. Layers whose
+ * scratch need (af1_workspace_bytes) exceeds 1 MiB are rejected with
+ * AF1_ERR_WORKSPACE; every shape with r <= 16256 fits.
+ * The first call on a device looks up the array's device address (once per
+ * device); make that first call before any stream capture. All calls share
+ * the array and leave their intermediate results in it, so calls that may
+ * overlap on the GPU (different streams or devices' contexts racing on one
+ * device) corrupt each other: issue them in one stream. */
+AF1_API int af1_linear_forward_static(const af1_layer* layer, const void* x, int64_t ldx, int64_t tokens,
+                                      void* y, int64_t ldy, int y_dtype, void* stream);
+
 /* Synchronize `stream` and report the status word the kernels keep in a
  * workspace: AF1_OK, or AF1_ERR_TIMEOUT if a bounded device-side wait gave
  * up since the workspace was last cleared (the word is then reset to 0). */

@@ -156,6 +156,11 @@ int check_scales(const uint16_t* a, const uint16_t* s, const uint16_t* b, int de
 
 }  // namespace
 
+namespace af1 {
+// Record a failure in the calling thread's af1_last_error() message.
+int set_error(int code, const std::string& msg) { return fail(code, msg); }
+}  // namespace af1
+
 extern "C" {
 
 int af1_rank_for_budget(int64_t m, int64_t n, int64_t budget_num, int64_t budget_den, int64_t* r_out) {

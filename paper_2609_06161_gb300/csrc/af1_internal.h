@@ -47,6 +47,9 @@ cudaError_t launch_pack_signs(const int8_t* src, int64_t rows, int64_t cols, int
                               uint32_t* bad_flag, cudaStream_t st);
 cudaError_t launch_words_to_tiles(const uint32_t* words, int64_t words_per_row, const TileMatrix& t,
                                   uint8_t* tiles, cudaStream_t st);
+// Set the calling thread's af1_last_error() message; returns `code`.
+int set_error(int code, const std::string& msg);
+
 cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64_t tokens, void* y,
                            int64_t ldy, int y_dtype, void* ws, cudaStream_t st);
 
