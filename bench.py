@@ -1,4 +1,4 @@
-"""Benchmark: AF1 binary-factorized linears on the decode path.
+"""Benchmark: AF1 binary-factorized linears (decode path by default).
 
 Workload: the seven linears of a LLaMA-3-8B decoder layer (q, k, v, o, gate,
 up, down) at their exact 1.0-BPW ranks, replicated over 32 layers with
@@ -6,6 +6,10 @@ distinct seeded synthetic weights (0.87 GB of packed signs per step, far
 above the 129 MB L2, so no flush is needed). One step is one decode token
 batch (default 1 token) through all 224 linears, issued in model order on one
 stream through af1_linear_forward and replayed as a CUDA graph.
+
+`--workload prefill` times the tensor-core prefill path instead: the same
+seven linears over 4 layers at 2048 tokens per call (1 % outlier channels),
+reported against the tensor roofline.
 
 Prints one JSON line. `--impl reference` times the CPU FP64 oracle instead
 (the reference arm of this paper-only build), on a bounded sample per step.
@@ -42,6 +46,10 @@ def parse():
     p.add_argument("--layers", type=int, default=LAYERS)
     p.add_argument("--no-dense", action="store_true", help="skip the dense BF16 baseline")
     p.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
+    p.add_argument("--workload", choices=["decode", "prefill"], default="decode",
+                   help="decode: config 1 (1-16 tokens); prefill: config 2 (2048 tokens, tensor cores)")
+    p.add_argument("--tokens", type=int, default=2048, help="prefill tokens per call")
+    p.add_argument("--no-graph", action="store_true", help="eager launches instead of a CUDA graph (for profilers)")
     return p.parse_args()
 
 
@@ -129,6 +137,12 @@ def run_reference(args):
 
 
 def config_dict(args):
+    if args.workload == "prefill":
+        return {"workload": (f"LLaMA-3-8B-shaped AF1 linears (q,k,v,o,gate,up,down at 1.0-BPW ranks) x {args.layers} "
+                             f"layers, prefill {args.tokens} tokens per call, FP16 N(0,1) activations with 1% outlier "
+                             f"channels x20, one stream in model order" + ("" if args.no_graph else ", CUDA graph")),
+                "tokens": args.tokens, "layers": args.layers, "linears_per_step": 7 * args.layers,
+                "l2": "inputs larger than L2 (weights + activations per step >> 129 MB), no flush"}
     return {"workload": (f"LLaMA-3-8B-shaped AF1 decoder linears (q,k,v,o 4096x4096 r2028 / k,v 1024x4096 r800 / "
                          f"gate,up 14336x4096 r3167 / down 4096x14336 r3167) x {args.layers} layers, decode batch "
                          f"{args.batch}, one stream in model order, CUDA graph"),
@@ -192,12 +206,12 @@ class Clocks:
 # The AF1 arm
 # ---------------------------------------------------------------------------
 
-def build_layers(P, torch, layers, batch, rank):
+def build_layers(P, torch, layers, batch, rank, outlier_frac=0.0):
     import synth
     objs = []
     for li in range(layers):
         for si, (name, m, n, r) in enumerate(shapes()):
-            d = synth.layer_words(100000 * (rank + 1) + 7 * li + si, m, n, r, batch)
+            d = synth.layer_words(100000 * (rank + 1) + 7 * li + si, m, n, r, batch, outlier_frac=outlier_frac)
             f16 = lambda bits: torch.from_numpy(np.ascontiguousarray(bits).view(np.float16)).cuda()
             Uw = torch.from_numpy(d["Uw"].view(np.int32)).cuda()
             Vw = torch.from_numpy(d["Vw"].view(np.int32)).cuda()
@@ -224,11 +238,18 @@ def main():
         torch.cuda.set_device(0)
     import paper_2609_06161_gb300 as P
 
-    b = args.batch
-    if not 1 <= b <= 16:
-        raise SystemExit("--batch must be in 1..16 for the decode path")
+    if args.workload == "prefill":
+        b = args.tokens
+        if b <= 16:
+            raise SystemExit("--tokens must be > 16 for the prefill path")
+        if args.layers == LAYERS:
+            args.layers = 4
+    else:
+        b = args.batch
+        if not 1 <= b <= 16:
+            raise SystemExit("--batch must be in 1..16 for the decode path")
     dev = torch.device("cuda", torch.cuda.current_device())
-    objs = build_layers(P, torch, args.layers, b, rank)
+    objs = build_layers(P, torch, args.layers, b, rank, outlier_frac=0.01 if args.workload == "prefill" else 0.0)
     ws = torch.zeros(max(o[4].workspace_bytes(b) for o in objs), dtype=torch.uint8, device=dev)
     # Inputs and outputs live in one device buffer each so the e2e leg can move
     # them with a single copy per direction.
@@ -256,9 +277,15 @@ def main():
     with torch.cuda.stream(stream):
         step()
     torch.cuda.synchronize()
-    graph = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(graph, stream=stream):
-        step()
+    if args.no_graph:
+        class _Eager:
+            def replay(self):
+                step()
+        graph = _Eager()
+    else:
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=stream):
+            step()
     torch.cuda.synchronize()
 
     def barrier():
@@ -325,6 +352,20 @@ def main():
     if rank == 0:
         peaks = load_peaks()
         hbm = peaks.get("hbm_gbs")
+        if args.workload == "prefill":
+            flops = sum(2 * b * r * (m + n) for (name, m, n, r, layer, x) in objs)
+            tflops = flops / (ms_step * 1e-3) / 1e12
+            tpeak = peaks.get("bf16_tflops_sustained", 1700.0)
+            roof = {"bound": "tensor", "kernel": "af1_linear_forward prefill (two tcgen05 kind::f16 GEMM kernels per call)",
+                    "achieved": tflops, "peak": tpeak, "unit": "TFLOP/s", "frac": tflops / tpeak,
+                    "peak_source": "MEASURED_PEAKS.json bf16_tflops_sustained (FP16 dense rate = BF16 rate)",
+                    "algorithmic_flops_per_step": flops, "traffic": None}
+        else:
+            roof = {"bound": "hbm", "kernel": "af1_linear_forward (phase-1 + phase-2 kernels, per call)",
+                    "achieved": achieved_gbs, "peak": hbm, "unit": "GB/s",
+                    "frac": (achieved_gbs / hbm) if hbm else None, "peak_source": "MEASURED_PEAKS.json hbm_gbs"
+                    if "hbm_gbs" in peaks else "fallback 6800 GB/s",
+                    "algorithmic_bytes_per_step": alg, "traffic": None}
         line = {
             "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
             "warmup": max(args.warmup, 3), "ms_per_step": ms_step, "us_per_layer": us_layer,
@@ -332,11 +373,7 @@ def main():
             "dtype": "e4m3 MMA / f32 accumulate (1-bit signs, f16 scales and activations)",
             "data": "synthetic (seeded PCG64 packed signs, |N(0,0.02)|+1e-3 scales, N(0,1) activations)",
             "config": config_dict(args),
-            "roofline": {"bound": "hbm", "kernel": "af1_linear_forward (phase-1 + phase-2 kernels, per call)",
-                         "achieved": achieved_gbs, "peak": hbm, "unit": "GB/s",
-                         "frac": (achieved_gbs / hbm) if hbm else None, "peak_source": "MEASURED_PEAKS.json hbm_gbs"
-                         if "hbm_gbs" in peaks else "fallback 6800 GB/s",
-                         "algorithmic_bytes_per_step": alg, "traffic": None},
+            "roofline": roof,
             "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": xo * 2,
                     "d2h_bytes_per_step": yo * 2},
             "gpu_launches": 2 * nlin * args.steps,
@@ -344,8 +381,11 @@ def main():
         }
         if dense is not None:
             line["dense_bf16_baseline"] = dense
-        if not args.no_cpu and world == 1:
+        if not args.no_cpu and world == 1 and args.workload == "decode":
             line["cpu_baseline"] = cpu_baseline(b)
+        if args.workload == "prefill":
+            line["dtype"] = "f16 tcgen05 MMA / f32 accumulate (1-bit signs expanded to +-b, f16 activations)"
+            line["us_per_layer"] = ms_step * 1e3 / nlin
         print(json.dumps(line))
     if world > 1:
         dist.destroy_process_group()

@@ -293,7 +293,7 @@ int af1_layer_device_bytes(const af1_layer* layer, int64_t* sign_bytes, int64_t*
 int64_t af1_workspace_bytes(const af1_layer* layer, int64_t tokens) {
   if (layer == nullptr) return fail(AF1_ERR_INVALID_ARG, "layer is NULL");
   if (tokens < 0) return fail(AF1_ERR_INVALID_ARG, "tokens must be >= 0");
-  return af1::plan_workspace(*layer).total;
+  return af1::plan_workspace(*layer, tokens).total;
 }
 
 int af1_linear_forward(const af1_layer* layer, const void* x, int64_t ldx, int64_t tokens, void* y, int64_t ldy,
@@ -323,7 +323,7 @@ int af1_linear_forward(const af1_layer* layer, const void* x, int64_t ldx, int64
     return fail(AF1_ERR_MISALIGNED, "ldy * element size must be a multiple of 16 bytes");
   if ((reinterpret_cast<uintptr_t>(workspace) & 255) != 0)
     return fail(AF1_ERR_WORKSPACE, "workspace must be 256-byte aligned");
-  const int64_t need = af1::plan_workspace(*layer).total;
+  const int64_t need = af1::plan_workspace(*layer, tokens).total;
   if (workspace_bytes < need)
     return fail(AF1_ERR_WORKSPACE, "workspace too small: need " + std::to_string(need) + " bytes");
   e = af1::launch_forward(*layer, x, ldx, tokens, y, ldy, y_dtype, workspace, static_cast<cudaStream_t>(stream));

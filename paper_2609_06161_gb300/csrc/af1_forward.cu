@@ -592,21 +592,31 @@ void plan_tiles(TileMatrix& t, int64_t R, int64_t C, int num_sms, int max_smem) 
   t.RG = (t.RT + t.RTC - 1) / t.RTC;
 }
 
-Workspace plan_workspace(const af1_layer& L) {
+Workspace plan_workspace(const af1_layer& L, int64_t tokens) {
   Workspace w;
   int64_t off = 0;
   w.status = off;
   off += 256;
   w.sbuf = off;
   off += align256((int64_t)kMaxPassTokens * L.p2.KT * kTileCols * 4);
+  w.hbuf = off;
+  if (tokens > kMaxPassTokens) {
+    const int64_t t = tokens < kPrefillPassTokens ? tokens : kPrefillPassTokens;
+    off += align256(t * prefill_h_ld(L) * 2);
+  }
   w.total = off;
   return w;
 }
 
 cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64_t tokens, void* y,
                            int64_t ldy, int y_dtype, void* ws, cudaStream_t st) {
-  const Workspace W = plan_workspace(L);
+  const Workspace W = plan_workspace(L, tokens);
   uint8_t* wsb = static_cast<uint8_t*>(ws);
+  if (tokens > kMaxPassTokens) {
+    // Prefill: two tensor-core GEMMs per pass (af1_prefill.cu).
+    return launch_prefill(L, x, ldx, tokens, y, ldy, y_dtype, wsb + W.hbuf, reinterpret_cast<unsigned*>(wsb + W.status),
+                          st);
+  }
   const int ysize = y_dtype == 0 ? 2 : 4;
   for (int64_t t0 = 0; t0 < tokens; t0 += kMaxPassTokens) {
     const int T = (int)((tokens - t0) < kMaxPassTokens ? (tokens - t0) : kMaxPassTokens);

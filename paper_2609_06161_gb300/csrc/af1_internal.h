@@ -28,13 +28,18 @@ struct af1_layer {
 
 namespace af1 {
 
-// Workspace carve-up for one layer and a pass of up to kMaxPassTokens tokens.
+// Tokens per prefill pass (calls with more than kMaxPassTokens tokens).
+constexpr int64_t kPrefillPassTokens = 2048;
+
+// Workspace carve-up for one layer and one forward call of `tokens` tokens.
 struct Workspace {
   int64_t status = 0;  // uint32 status word
-  int64_t sbuf = 0;    // float[kMaxPassTokens][p2.KT*128]: s' = s * t from phase 1
+  int64_t sbuf = 0;    // float[kMaxPassTokens][p2.KT*128]: s' = s * t (decode)
+  int64_t hbuf = 0;    // FP16 [min(tokens, kPrefillPassTokens)][prefill_h_ld]: H (prefill)
   int64_t total = 0;
 };
-Workspace plan_workspace(const af1_layer& L);
+Workspace plan_workspace(const af1_layer& L, int64_t tokens);
+int64_t prefill_h_ld(const af1_layer& L);
 
 // Choose the tile blocks and the split-K cluster of one sign matrix.
 void plan_tiles(TileMatrix& t, int64_t R, int64_t C, int num_sms, int max_smem);
@@ -50,6 +55,8 @@ cudaError_t launch_words_to_tiles(const uint32_t* words, int64_t words_per_row, 
 // Set the calling thread's af1_last_error() message; returns `code`.
 int set_error(int code, const std::string& msg);
 
+cudaError_t launch_prefill(const af1_layer& L, const void* x, int64_t ldx, int64_t tokens, void* y, int64_t ldy,
+                           int y_dtype, uint8_t* h_buf, unsigned* status, cudaStream_t st);
 cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64_t tokens, void* y,
                            int64_t ldy, int y_dtype, void* ws, cudaStream_t st);
 

@@ -54,7 +54,7 @@ int af1_linear_forward_static(const af1_layer* layer, const void* x, int64_t ldx
   if (tokens < 0) return fail(AF1_ERR_INVALID_ARG, "tokens must be >= 0");
   if (y_dtype != AF1_F16 && y_dtype != AF1_F32) return fail(AF1_ERR_INVALID_ARG, "y_dtype must be AF1_F16 or AF1_F32");
   if (tokens == 0) return AF1_OK;
-  const int64_t need = af1::plan_workspace(*layer).total;
+  const int64_t need = af1::plan_workspace(*layer, tokens).total;
   if (need > kStaticScratchBytes)
     return fail(AF1_ERR_WORKSPACE, "layer needs " + std::to_string(need) + " bytes of scratch; the built-in array holds " +
                                        std::to_string(kStaticScratchBytes));

@@ -274,3 +274,59 @@ def test_first_calls_interleaved_with_other_layers(P):
             for t in range(tokens):
                 assert O.rowwise_rel_err(y[t:t + 1], ref[t:t + 1]) <= TOL, (m, n, r, tokens, t)
             layer.free()
+
+
+# ---------------------------------------------------------------------------
+# Prefill path (more than 16 tokens): tcgen05 GEMMs
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("m,n,r", [(16, 16, 8), (100, 130, 77), (256, 384, 200), (1000, 700, 321),
+                                   (1024, 4096, 800)])
+@pytest.mark.parametrize("tokens", [17, 128, 129, 300])
+def test_prefill_matches_oracle(P, m, n, r, tokens):
+    d = synth.layer_signs(31 * m + n + tokens, m, n, r, tokens, outlier_frac=0.01)
+    layer = signs_layer(P, d)
+    for out_dtype in (torch.float32, torch.float16):
+        y = run_gpu(layer, d["x"], n, out_dtype)
+        ref = oracle_from_signs(d, n)
+        assert O.rowwise_rel_err(y, ref) <= TOL, out_dtype
+    layer.free()
+
+
+@pytest.mark.parametrize("m,n,r", [(64, 96, 40), (130, 200, 100), (256, 256, 120)])
+@pytest.mark.parametrize("tokens", [40, 200])
+def test_prefill_integer_inputs_bit_exact(P, m, n, r, tokens):
+    d = synth.integer_layer(77 + m + tokens, m, n, r, tokens)
+    layer = signs_layer(P, d)
+    y = run_gpu(layer, d["x"], n, torch.float32)
+    np.testing.assert_array_equal(y, oracle_from_signs(d, n))
+    layer.free()
+
+
+@pytest.mark.parametrize("m,n", [(4096, 4096), (1024, 4096), (14336, 4096), (4096, 14336)])
+def test_prefill_full_size_sampled_rows(P, m, n):
+    """The prefill workload: LLaMA-3-8B-shaped linears, 2048 tokens, 1 % outlier channels x20."""
+    tokens = 2048
+    r = O.rank_for_budget(m, n, 1)
+    d = synth.layer_words(7000 + m // 1024 + n // 1024, m, n, r, tokens, outlier_frac=0.01)
+    layer = words_layer(P, d, m, n, r)
+    y = run_gpu(layer, d["x"], n)
+    rows = np.sort(synth.rng(5).choice(m, size=128, replace=False))
+    ref = O.forward_from_packed(d["Uw"], d["Vw"], d["a"], d["s"], d["b"], d["x"], m, n, r, rows=rows)
+    assert O.rowwise_rel_err(y[:, rows], ref) <= TOL
+    layer.free()
+
+
+def test_prefill_hadamard_identity(P):
+    N = 256
+    H = sylvester(8)
+    g = synth.rng(99)
+    a = synth.scales_f16(g, N)
+    b = synth.scales_f16(g, N)
+    s = np.full(N, np.float16(1.0 / N)).view(np.uint16)
+    x = synth.activations_f16(g, 64, N)
+    layer = signs_layer(P, dict(U=H, V=H, a=a, s=s, b=b, x=x), any_rank=True)
+    y = run_gpu(layer, x, N)
+    af, bf, xf = (O.f16_bits_to_f64(v) for v in (a, b, x))
+    assert O.rowwise_rel_err(y, xf.reshape(64, N) * (af * bf)[None, :]) <= TOL
+    layer.free()

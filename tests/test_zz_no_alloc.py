@@ -36,7 +36,7 @@ def test_static_scratch_entry_matches_workspace_entry():
             xp[:, :n] = x
             x = xp
         ldy = m + (-m) % 4
-        ws = layer.make_workspace()
+        ws = layer.make_workspace(tokens)
         y_ref = torch.empty((tokens, ldy), dtype=torch.float32, device="cuda")
         rc = fwd(layer._h, x.data_ptr(), ldx, tokens, y_ref.data_ptr(), ldy, 1, ws.data_ptr(),
                  ws.numel(), stream)
