@@ -50,6 +50,9 @@ def parse():
                    help="decode: config 1 (1-16 tokens); prefill: config 2 (2048 tokens, tensor cores)")
     p.add_argument("--tokens", type=int, default=2048, help="prefill tokens per call")
     p.add_argument("--no-graph", action="store_true", help="eager launches instead of a CUDA graph (for profilers)")
+    p.add_argument("--schedule", choices=["dag", "serial"], default="dag",
+                   help="dag: a decoder layer's independent linears (q/k/v, gate/up) on parallel streams; "
+                        "serial: all 7 linears chained on one stream")
     return p.parse_args()
 
 
@@ -145,7 +148,9 @@ def config_dict(args):
                 "l2": "inputs larger than L2 (weights + activations per step >> 129 MB), no flush"}
     return {"workload": (f"LLaMA-3-8B-shaped AF1 decoder linears (q,k,v,o 4096x4096 r2028 / k,v 1024x4096 r800 / "
                          f"gate,up 14336x4096 r3167 / down 4096x14336 r3167) x {args.layers} layers, decode batch "
-                         f"{args.batch}, one stream in model order, CUDA graph"),
+                         f"{args.batch}, " + ("q|k|v and gate|up on parallel streams (decoder dependency DAG)"
+                                               if args.schedule == "dag" else "one stream in model order")
+                         + ("" if args.no_graph else ", CUDA graph")),
             "batch": args.batch, "layers": args.layers, "linears_per_step": 7 * args.layers,
             "l2": "inputs larger than L2 (packed weights per step >> 129 MB), no flush"}
 
@@ -269,24 +274,59 @@ def main():
         views.append((layer, xbuf[xoff[i]:xoff[i] + b * n].view(b, n), ybuf[yoff[i]:yoff[i] + b * m].view(b, m)))
 
     stream = torch.cuda.Stream()
+    side = [torch.cuda.Stream(), torch.cuda.Stream()]
+    ws_side = [torch.zeros_like(ws), torch.zeros_like(ws)]
 
-    def step():
+    def step_serial():
         for (layer, xv, yv) in views:
             layer.forward_into(xv, yv, ws, stream=stream)
 
-    with torch.cuda.stream(stream):
-        step()
-    torch.cuda.synchronize()
-    if args.no_graph:
-        class _Eager:
-            def replay(self):
-                step()
-        graph = _Eager()
-    else:
-        graph = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(graph, stream=stream):
-            step()
-    torch.cuda.synchronize()
+    def step_dag():
+        # Per decoder layer: q | k | v in parallel, then o, then gate | up in
+        # parallel, then down (attention and activations are not part of this
+        # workload). Each parallel branch has its own workspace.
+        for li in range(len(views) // 7):
+            q, k, v, o, gate, up, down = views[7 * li:7 * li + 7]
+            ev = torch.cuda.Event()
+            ev.record(stream)
+            for st in side:
+                st.wait_event(ev)
+            q[0].forward_into(q[1], q[2], ws, stream=stream)
+            k[0].forward_into(k[1], k[2], ws_side[0], stream=side[0])
+            v[0].forward_into(v[1], v[2], ws_side[1], stream=side[1])
+            for st in side:
+                e = torch.cuda.Event()
+                e.record(st)
+                stream.wait_event(e)
+            o[0].forward_into(o[1], o[2], ws, stream=stream)
+            ev = torch.cuda.Event()
+            ev.record(stream)
+            side[0].wait_event(ev)
+            gate[0].forward_into(gate[1], gate[2], ws, stream=stream)
+            up[0].forward_into(up[1], up[2], ws_side[0], stream=side[0])
+            e = torch.cuda.Event()
+            e.record(side[0])
+            stream.wait_event(e)
+            down[0].forward_into(down[1], down[2], ws, stream=stream)
+
+    def make_graph(fn):
+        with torch.cuda.stream(stream):
+            fn()
+        torch.cuda.synchronize()
+        if args.no_graph:
+            class _Eager:
+                def replay(self):
+                    with torch.cuda.stream(stream):
+                        fn()
+            return _Eager()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            fn()
+        torch.cuda.synchronize()
+        return g
+
+    step = step_dag if (args.schedule == "dag" and len(views) % 7 == 0) else step_serial
+    graph = make_graph(step)
 
     def barrier():
         if world > 1:
@@ -320,6 +360,23 @@ def main():
     us_layer = ms_step * 1e3 / nlin
     alg = sum(algorithmic_bytes(m, n, r, b) for (name, m, n, r, layer, x) in objs)
     achieved_gbs = alg / (ms_step * 1e-3) / 1e9
+
+    serial = None
+    if step is step_dag:
+        g2 = make_graph(step_serial)
+        for _ in range(3):
+            g2.replay()
+        torch.cuda.synchronize()
+        f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        f0.record(stream)
+        with torch.cuda.stream(stream):
+            for _ in range(args.steps):
+                g2.replay()
+        f1.record(stream)
+        torch.cuda.synchronize()
+        sms = f0.elapsed_time(f1) / args.steps
+        serial = {"ms_per_step": sms, "us_per_layer": sms * 1e3 / len(views), "tokens_per_s": b / (sms * 1e-3)}
+        del g2
 
     # e2e: host buffers in pinned memory, copies inside the timed region.
     xh = torch.empty(xo, dtype=torch.float16, pin_memory=True)
@@ -381,6 +438,8 @@ def main():
         }
         if dense is not None:
             line["dense_bf16_baseline"] = dense
+        if serial is not None:
+            line["serial_chain"] = serial
         if not args.no_cpu and world == 1 and args.workload == "decode":
             line["cpu_baseline"] = cpu_baseline(b)
         if args.workload == "prefill":

@@ -103,6 +103,7 @@ int create_layer(const af1_layer_desc* d, cudaStream_t st, af1_layer** out) {
     delete L;
     return fail_cuda(e, "cudaDeviceGetAttribute");
   }
+  L->max_smem = max_smem;
   af1::plan_tiles(L->p1, d->r, d->n, sms, max_smem);
   af1::plan_tiles(L->p2, d->m, d->r, sms, max_smem);
   const int64_t t1 = (int64_t)L->p1.RT * L->p1.KT * af1::kTileBytes;

@@ -43,7 +43,7 @@ namespace {
 
 constexpr long long kWaitCycles = 2000000000ll;  // ~1 s at 2 GHz
 constexpr unsigned kStatusTimeout = 1u;
-constexpr int kMaxWarps = 8;
+constexpr int kMaxWarps = 16;
 
 // ---------------------------------------------------------------------------
 // PTX helpers (hand-written: mbarrier, bulk copy, PDL, cluster, MMA, FP8)
@@ -192,6 +192,9 @@ struct SmemHeader {
   uint64_t mbar[kMaxKTC];
   float maxv[kMaxPassTokens * kMaxWarps];  // per-warp max |z / d| per token
   float qpart[kMaxPassTokens * kMaxWarps]; // per-warp partial Q per token
+  float sc[kMaxPassTokens];                // 2^sigma per token (0 for padding slots)
+  float qis[kMaxPassTokens];               // Q * 2^-sigma per token
+  float is[kMaxPassTokens];                // 2^-sigma per token
 };
 constexpr int kHeaderBytes = ((int)sizeof(SmemHeader) + 127) / 128 * 128;
 
@@ -201,7 +204,7 @@ __host__ __device__ inline int slice_rows(int rtc, int ks_count) {
 }
 
 struct SmemPlan {
-  int frag, wts, recv, rs, bi, total;
+  int frag, wts, recv, rs, bi, red, total;
 };
 
 __host__ __device__ inline int align128(int v) { return (v + 127) / 128 * 128; }
@@ -222,6 +225,8 @@ __host__ __device__ inline SmemPlan smem_plan(const TileMatrix& tm, int ng) {
   off = align128(off + slice * 4);
   p.bi = off;
   off = align128(off + tm.KTC * kTileCols * 4);
+  p.red = off;  // [WK][2 * ng][rows of the block], WK * rows <= 16 warps x 16 rows
+  off = align128(off + kMaxWarps * 2 * ng * kTileRows * 4);
   p.total = off;
   return p;
 }
@@ -270,52 +275,85 @@ __device__ __forceinline__ float warp_sum(float v) {
   return v;
 }
 
-// sigma for a token from the per-warp maxima: 2^sigma * max in [128, 256).
-template <int WARPS>
-__device__ __forceinline__ int token_sigma(const SmemHeader& h, int tok) {
-  float m = 0.f;
-#pragma unroll
-  for (int w = 0; w < WARPS; ++w) m = fmaxf(m, h.maxv[tok * WARPS + w]);
-  int e = 0;
-  if (m > 0.f) frexpf(m, &e);  // m = f * 2^e, f in [0.5, 1)
-  return m > 0.f ? 8 - e : 0;
+// The power of two 2^sigma that brings a positive maximum m into [128, 256),
+// read from m's exponent field (m = f 2^e with f in [0.5, 1), sigma = 8 - e).
+// m comes from products of FP16 values, so 127 +- sigma stays a normal
+// exponent. Returns 2^sigma in *sc and 2^-sigma in *is; m == 0 gives 1, 1.
+__device__ __forceinline__ void pow2_scale(float m, float* sc, float* is) {
+  if (!(m > 0.f)) {
+    *sc = 1.f;
+    *is = 1.f;
+    return;
+  }
+  const int e = (int)((__float_as_uint(m) >> 23) & 0xFFu) - 126;
+  const int sigma = min(8 - e, 120);  // FP32-subnormal maxima (not produced by FP16 inputs) stay in range
+  *sc = __uint_as_float((uint32_t)(127 + sigma) << 23);
+  *is = __uint_as_float((uint32_t)(127 - sigma) << 23);
 }
 
 // Build the e4m3 B fragments of this CTA's column range for all token slots
 // (2 * NG). bi[kl] holds colscale * (1 / d) (phase 1) or 1 / d (phase 2), and
-// 0 beyond column C (staged and published by the caller). Two CTA barriers:
-// one after the maxima, one after the fragments.
+// 0 beyond column C (staged and published by the caller). Each thread owns
+// one group of 4 columns (the block has at most 16 x 128 columns, i.e. 512
+// groups, and the CTA has WARPS * 32 >= 512 threads when NG <= 2; with
+// 8 warps a thread owns up to two groups). Two CTA barriers: after the
+// maxima and after the fragments.
 template <int PHASE, int NG, int WARPS>
 __device__ void build_fragments(const PhaseArgs& a, SmemHeader& h, uint32_t* frag32, const float* bi, int64_t k0,
                                 int ncols) {
   constexpr int NT = 2 * NG;
   constexpr int NTH = WARPS * 32;
+  constexpr bool STASH = NT <= 4;  // keep z * bi in registers between the passes
   const int T = a.tokens;
   const int n4 = ncols >> 2;
+  const bool one = n4 <= NTH;      // each thread owns at most one group of 4 columns
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  for (int tok = 0; tok < T; ++tok) {
-    float mx = 0.f;
-    for (int c4 = threadIdx.x; c4 < n4; c4 += NTH) {
-      const float4 z = load_z4<PHASE>(a, tok, k0 + 4 * c4);
-      const float4 w = *reinterpret_cast<const float4*>(bi + 4 * c4);
-      mx = fmaxf(mx, fmaxf(fmaxf(fabsf(z.x * w.x), fabsf(z.y * w.y)), fmaxf(fabsf(z.z * w.z), fabsf(z.w * w.w))));
+  float4 zs[STASH ? NT : 1];
+#pragma unroll
+  for (int tok = 0; tok < NT; ++tok) {
+    if (STASH) zs[tok] = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (tok < T) {
+      float mx = 0.f;
+      for (int c4 = threadIdx.x; c4 < n4; c4 += NTH) {
+        const float4 z = load_z4<PHASE>(a, tok, k0 + 4 * c4);
+        const float4 w = *reinterpret_cast<const float4*>(bi + 4 * c4);
+        const float4 zb = make_float4(z.x * w.x, z.y * w.y, z.z * w.z, z.w * w.w);
+        if (STASH) zs[tok] = zb;
+        mx = fmaxf(mx, fmaxf(fmaxf(fabsf(zb.x), fabsf(zb.y)), fmaxf(fabsf(zb.z), fabsf(zb.w))));
+      }
+      mx = warp_max(mx);
+      if (lane == 0) h.maxv[tok * WARPS + warp] = mx;
     }
-    mx = warp_max(mx);
-    if (lane == 0) h.maxv[tok * WARPS + warp] = mx;
   }
   __syncthreads();
-#pragma unroll 1
+  if (threadIdx.x < NT) {
+    // One thread per token slot: block maximum -> 2^sigma, 2^-sigma.
+    float m = 0.f;
+    if ((int)threadIdx.x < T)
+      for (int w = 0; w < WARPS; ++w) m = fmaxf(m, h.maxv[threadIdx.x * WARPS + w]);
+    float sc, is;
+    pow2_scale(m, &sc, &is);
+    h.sc[threadIdx.x] = (int)threadIdx.x < T ? sc : 0.f;
+    h.is[threadIdx.x] = (int)threadIdx.x < T ? is : 0.f;
+  }
+  __syncthreads();
+#pragma unroll
   for (int tok = 0; tok < NT; ++tok) {
-    const float sc = tok < T ? ldexpf(1.f, token_sigma<WARPS>(h, tok)) : 0.f;
+    const float sc = h.sc[tok];
     const int gam = tok >> 1, tb = (tok & 1) * 4;
     float q = 0.f;
     for (int c4 = threadIdx.x; c4 < n4; c4 += NTH) {
-      float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+      float4 zb = make_float4(0.f, 0.f, 0.f, 0.f);
       if (tok < T) {
-        const float4 z = load_z4<PHASE>(a, tok, k0 + 4 * c4);
-        const float4 w = *reinterpret_cast<const float4*>(bi + 4 * c4);
-        v = make_float4(z.x * w.x * sc, z.y * w.y * sc, z.z * w.z * sc, z.w * w.w * sc);
+        if (STASH && one) {
+          zb = zs[tok];
+        } else {
+          const float4 z = load_z4<PHASE>(a, tok, k0 + 4 * c4);
+          const float4 w = *reinterpret_cast<const float4*>(bi + 4 * c4);
+          zb = make_float4(z.x * w.x, z.y * w.y, z.z * w.z, z.w * w.w);
+        }
       }
+      float4 v = make_float4(zb.x * sc, zb.y * sc, zb.z * sc, zb.w * sc);
       const float4 v0 = v;
       const int kt_l = c4 >> 5, mu = (c4 >> 3) & 3, breg = (c4 >> 2) & 1, c = c4 & 3;
       uint32_t* dst = frag32 + ((((kt_l * 4 + mu) * NG + gam) * 32 + 4 * tb + c) * 2 + breg);
@@ -335,6 +373,12 @@ __device__ void build_fragments(const PhaseArgs& a, SmemHeader& h, uint32_t* fra
     if (lane == 0) h.qpart[tok * WARPS + warp] = q;
   }
   __syncthreads();
+  if (threadIdx.x < NT) {
+    float q = 0.f;
+    for (int w = 0; w < WARPS; ++w) q += h.qpart[threadIdx.x * WARPS + w];
+    h.qis[threadIdx.x] = q * h.is[threadIdx.x];
+  }
+  __syncthreads();
 }
 
 template <int PHASE, int NG, int WARPS, int TPP>
@@ -348,33 +392,41 @@ __global__ void __launch_bounds__(WARPS * 32) phase_kernel(const PhaseArgs a) {
   float* recv = reinterpret_cast<float*>(smem + sp.recv);
   float* rs = reinterpret_cast<float*>(smem + sp.rs);
   float* bi = reinterpret_cast<float*>(smem + sp.bi);
+  float* red = reinterpret_cast<float*>(smem + sp.red);
 
   const int rg = blockIdx.x, ks = blockIdx.y, KS = gridDim.y;
   const int rtc = blk_rows(tm, rg), ktc = blk_cols(tm, ks);
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int64_t row0 = (int64_t)rg * tm.RTC * kTileRows;
   const int64_t k0 = (int64_t)ks * tm.KTC * kTileCols;
+  const int nrows = rtc * kTileRows;       // rows of this block
   const int slice = slice_rows(rtc, KS);   // rows finalised per CTA
   const int my0 = ks * slice;              // first block row this CTA finalises
 
   cluster_arrive_relaxed();  // this CTA has started (matched by cluster_wait)
+  // The block's column tiles arrive in at most kMaxKTC bulk copies (one
+  // mbarrier each) of `cpt` column tiles.
+  const int cpt = (ktc + kMaxKTC - 1) / kMaxKTC;
+  const int nchunks = (ktc + cpt - 1) / cpt;
   if (tid == 0) {
-    // Barriers and weight copies; the first CTA barrier in build_fragments
-    // publishes the initialised barriers to the other warps.
-    const uint32_t chunk = (uint32_t)rtc * kTileBytes;
+    // Barriers and weight copies; the CTA barrier below publishes the
+    // initialised barriers to the other warps.
+    const uint32_t per_kt = (uint32_t)rtc * kTileBytes;
     const uint8_t* gblk = a.tiles + blk_base(tm, rg, ks) * kTileBytes;
-    for (int i = 0; i < ktc; ++i) mbar_init(&h.mbar[i], 1);
+    for (int i = 0; i < nchunks; ++i) mbar_init(&h.mbar[i], 1);
     fence_barrier_init();
-    for (int i = 0; i < ktc; ++i) {
-      mbar_expect_tx(&h.mbar[i], chunk);
-      bulk_g2s(wts + (size_t)i * chunk, gblk + (size_t)i * chunk, chunk, &h.mbar[i]);
+    for (int i = 0; i < nchunks; ++i) {
+      const int kts = min(cpt, ktc - i * cpt);
+      const uint32_t bytes = per_kt * (uint32_t)kts;
+      mbar_expect_tx(&h.mbar[i], bytes);
+      bulk_g2s(wts + (size_t)i * cpt * per_kt, gblk + (size_t)i * cpt * per_kt, bytes, &h.mbar[i]);
     }
   }
   // Layer constants: row scales of the rows this CTA finalises, column
   // factors of its column slice.
   for (int i = tid; i < slice; i += WARPS * 32) {
     const int64_t row = row0 + my0 + i;
-    rs[i] = (my0 + i < rtc * kTileRows && row < tm.R) ? __half2float(a.rowscale[row]) : 0.f;
+    rs[i] = (my0 + i < nrows && row < tm.R) ? __half2float(a.rowscale[row]) : 0.f;
   }
   for (int i = tid; i < ktc * kTileCols; i += WARPS * 32) {
     const int64_t k = k0 + i;
@@ -395,20 +447,24 @@ __global__ void __launch_bounds__(WARPS * 32) phase_kernel(const PhaseArgs a) {
 
   const int g = lane >> 2, c = lane & 3;
   const int T = a.tokens;
-  // Per-thread constants of the tokens this lane finalises: 2 * gg + (c >> 1).
-  float qv[NG], is[NG];
+  // Warps split the block into WR row-tile classes x WK column-tile classes.
+  int WK = WARPS / rtc;
+  if (WK < 1) WK = 1;
+  if (WK > ktc) WK = ktc;
+  const int WR = WARPS / WK;
+  const int wr = warp / WK, wk = warp - wr * WK;
+  const bool wactive = warp < WR * WK;
+  // 2^-sigma and Q 2^-sigma of the tokens this lane finalises: 2 gg + (c >> 1).
+  float isv[NG], qisv[NG];
 #pragma unroll
   for (int gg = 0; gg < NG; ++gg) {
     const int tok = 2 * gg + (c >> 1);
-    float q = 0.f;
-#pragma unroll
-    for (int w = 0; w < WARPS; ++w) q += h.qpart[tok * WARPS + w];
-    qv[gg] = q;
-    is[gg] = tok < T ? ldexpf(1.f, -token_sigma<WARPS>(h, tok)) : 0.f;
+    isv[gg] = h.is[tok];
+    qisv[gg] = h.qis[tok];
   }
 
   bool ok = true;
-  const int rt_per_warp = (rtc + WARPS - 1) / WARPS;
+  const int rt_per_warp = wactive ? (rtc - wr + WR - 1) / WR : 0;
   for (int j0 = 0; j0 < rt_per_warp && ok; j0 += TPP) {
     float acc[TPP][NG][4];
 #pragma unroll
@@ -416,8 +472,8 @@ __global__ void __launch_bounds__(WARPS * 32) phase_kernel(const PhaseArgs a) {
 #pragma unroll
       for (int gg = 0; gg < NG; ++gg) acc[j][gg][0] = acc[j][gg][1] = acc[j][gg][2] = acc[j][gg][3] = 0.f;
 
-    for (int kt_l = 0; kt_l < ktc; ++kt_l) {
-      if (!mbar_wait_bounded(&h.mbar[kt_l], 0)) {
+    for (int kt_l = wk; kt_l < ktc; kt_l += WK) {
+      if (!mbar_wait_bounded(&h.mbar[kt_l / cpt], 0)) {
         ok = false;
         break;
       }
@@ -432,7 +488,7 @@ __global__ void __launch_bounds__(WARPS * 32) phase_kernel(const PhaseArgs a) {
         }
 #pragma unroll
       for (int j = 0; j < TPP; ++j) {
-        const int rt_l = warp + WARPS * (j0 + j);
+        const int rt_l = wr + WR * (j0 + j);
         if (rt_l < rtc) {
           const uint2 w = *reinterpret_cast<const uint2*>(wts + ((size_t)(kt_l * rtc + rt_l) * kTileBytes) + lane * 8);
           uint32_t lo[8], hi[8];
@@ -448,11 +504,12 @@ __global__ void __launch_bounds__(WARPS * 32) phase_kernel(const PhaseArgs a) {
       }
     }
     if (!ok) break;
-    // (2 D - Q) 2^-sigma of these row tiles, pushed into the shared memory of
-    // the cluster CTA that finalises each row (slot ks of its buffer).
+    // 2 D 2^-sigma of these row tiles over this warp's column tiles: to the
+    // in-CTA reduction buffer (WK > 1) or, minus Q 2^-sigma, straight into
+    // the shared memory of the cluster CTA that finalises the row.
 #pragma unroll
     for (int j = 0; j < TPP; ++j) {
-      const int rt_l = warp + WARPS * (j0 + j);
+      const int rt_l = wr + WR * (j0 + j);
       if (rt_l < rtc) {
 #pragma unroll
         for (int gg = 0; gg < NG; ++gg) {
@@ -465,9 +522,14 @@ __global__ void __launch_bounds__(WARPS * 32) phase_kernel(const PhaseArgs a) {
 #pragma unroll
             for (int half = 0; half < 2; ++half) {
               const int rl = rt_l * kTileRows + g + 8 * half;
-              const int owner = rl / slice;
-              float* dst = recv + ((ks * 2 * NG + tok) * slice + (rl - owner * slice));
-              st_cluster_f32(dst, (uint32_t)owner, (2.f * (half ? vhi : vlo) - qv[gg]) * is[gg]);
+              const float p = 2.f * (half ? vhi : vlo) * isv[gg];
+              if (WK > 1) {
+                red[(wk * 2 * NG + tok) * nrows + rl] = p;
+              } else {
+                const int owner = rl / slice;
+                st_cluster_f32(recv + ((ks * 2 * NG + tok) * slice + (rl - owner * slice)), (uint32_t)owner,
+                               p - qisv[gg]);
+              }
             }
           }
         }
@@ -481,11 +543,22 @@ __global__ void __launch_bounds__(WARPS * 32) phase_kernel(const PhaseArgs a) {
     // (bounded). The cluster barrier is still honoured so that no CTA of the
     // cluster waits on this one.
     atomicOr(a.status, kStatusTimeout);
-    for (int i = 0; i < ktc; ++i) mbar_wait_bounded(&h.mbar[i], 0);
+    for (int i = 0; i < nchunks; ++i) mbar_wait_bounded(&h.mbar[i], 0);
+  }
+  if (WK > 1 && all_ok) {
+    // Sum the WK column-class partials of each row in a fixed order and push.
+    for (int idx = tid; idx < T * nrows; idx += WARPS * 32) {
+      const int tok = idx / nrows;
+      const int rl = idx - tok * nrows;
+      float v = 0.f;
+      for (int q = 0; q < WK; ++q) v += red[(q * 2 * NG + tok) * nrows + rl];
+      const int owner = rl / slice;
+      st_cluster_f32(recv + ((ks * 2 * NG + tok) * slice + (rl - owner * slice)), (uint32_t)owner, v - h.qis[tok]);
+    }
   }
   // All partials of the cluster have landed in their owners' buffers.
   cluster_sync();
-  const int cnt = min(slice, rtc * kTileRows - my0);
+  const int cnt = min(slice, nrows - my0);
   if (all_ok && cnt > 0) {
     for (int idx = tid; idx < T * cnt; idx += WARPS * 32) {
       const int tok = idx / cnt;
@@ -510,16 +583,21 @@ __global__ void __launch_bounds__(WARPS * 32) phase_kernel(const PhaseArgs a) {
 // Host side
 // ---------------------------------------------------------------------------
 
-constexpr int kWarps = 8;
-
+// 16 warps per CTA for up to 4 tokens (shorter serial MMA chains per warp);
+// 8 warps for 5-16 tokens (register budget of the wider fragments).
+template <int NG>
+constexpr int warps_for() {
+  return NG <= 2 ? 16 : 8;
+}
 template <int NG>
 constexpr int tpp_for() {
-  return NG == 1 ? 4 : NG == 2 ? 2 : 1;
+  return NG == 1 ? 2 : NG == 2 ? 2 : NG == 4 ? 2 : 1;
 }
 
 template <int PHASE, int NG>
 cudaError_t launch_phase(const PhaseArgs& a, cudaStream_t st) {
-  auto kern = phase_kernel<PHASE, NG, kWarps, tpp_for<NG>()>;
+  constexpr int W = warps_for<NG>();
+  auto kern = phase_kernel<PHASE, NG, W, tpp_for<NG>()>;
   const int smem = smem_plan(a.tm, NG).total;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
@@ -529,7 +607,7 @@ cudaError_t launch_phase(const PhaseArgs& a, cudaStream_t st) {
   }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)a.tm.RG, (unsigned)a.tm.KS, 1);
-  cfg.blockDim = dim3(kWarps * 32, 1, 1);
+  cfg.blockDim = dim3(W * 32, 1, 1);
   cfg.dynamicSmemBytes = (size_t)smem;
   cfg.stream = st;
   cudaLaunchAttribute attr[2];
@@ -560,36 +638,61 @@ int64_t align256(int64_t v) { return (v + 255) / 256 * 256; }
 
 int forward_smem_bytes(const TileMatrix& t, int ng) { return smem_plan(t, ng).total; }
 
+// Column tiles per CTA of the decode split of K: one tile per CTA up to 8
+// tiles, then clusters of 8 CTAs, beyond 64 tiles clusters of up to 16.
+int decode_ktc(int KT) {
+  if (KT <= 8) return 1;
+  int ktc = (KT + 7) / 8;
+  if (ktc > 8) ktc = (KT + 15) / 16;
+  return ktc;
+}
+
+// Launch-time split of K: a cluster of KS CTAs per row group (decode_ktc),
+// with a finer split (up to 16 CTAs) when the shared-memory plan of a wide
+// pass needs it.
+TileMatrix launch_plan(const TileMatrix& layout, int ng, int max_smem) {
+  TileMatrix t = layout;
+  t.KTC = decode_ktc(layout.KT);
+  t.KS = (layout.KT + t.KTC - 1) / t.KTC;
+  while (smem_plan(t, ng).total > max_smem && t.KS < 16 && t.KTC > 1) {
+    const int ks = t.KS + 1;
+    t.KTC = (layout.KT + ks - 1) / ks;
+    t.KS = (layout.KT + t.KTC - 1) / t.KTC;
+  }
+  return t;
+}
+
 void plan_tiles(TileMatrix& t, int64_t R, int64_t C, int num_sms, int max_smem) {
+  // Pack-time layout: one block per group of RTC row tiles holding all KT
+  // column tiles, column-tile major, so that any split of K chosen at launch
+  // (launch_plan) gives every CTA one contiguous range of its block.
   t.R = R;
   t.C = C;
   t.RT = (int)((R + kTileRows - 1) / kTileRows);
   t.KT = (int)((C + kTileCols - 1) / kTileCols);
-  // Split K over a cluster of KS CTAs, each holding KTC column tiles.
-  if (t.KT <= 8) {
-    t.KS = t.KT;
-    t.KTC = 1;
-  } else {
-    // Portable clusters of up to 8 CTAs with at most 8 column tiles each;
-    // beyond 64 column tiles, clusters of up to 16 (at most kMaxKTC tiles).
-    t.KTC = (t.KT + 7) / 8;
-    if (t.KTC > 8) t.KTC = (t.KT + 15) / 16;
-    t.KS = (t.KT + t.KTC - 1) / t.KTC;
-  }
-  // Row tiles per block: aim for about two CTAs per SM, at least 8 row tiles
-  // so that the per-CTA activation split is amortised, at most 32.
+  t.KTC = t.KT;
+  t.KS = 1;
+  // Row tiles per group: about two CTAs per SM with the decode split of K
+  // (decode_ktc), at least 8 (the activation split is amortised over the
+  // group's rows), at most 32.
   const int sms = num_sms > 0 ? num_sms : 148;
-  int rtc = (int)(((int64_t)t.RT * t.KS + sms) / (2 * sms));
+  const int dk = decode_ktc(t.KT);
+  const int ks = (t.KT + dk - 1) / dk;
+  int rtc = (int)(((int64_t)t.RT * ks + sms) / (2 * sms));
   if (rtc < 8) rtc = 8;
   if (rtc > 32) rtc = 32;
   if (rtc > t.RT) rtc = t.RT;
   t.RTC = rtc;
-  while (t.RTC > 1) {
-    t.RG = (t.RT + t.RTC - 1) / t.RTC;
-    if (smem_plan(t, 8).total <= max_smem) break;
-    t.RTC = (t.RTC + 1) / 2;
-  }
   t.RG = (t.RT + t.RTC - 1) / t.RTC;
+  // The widest pass (16 tokens) must fit with a split of at most 16 CTAs.
+  for (;;) {
+    TileMatrix probe = t;
+    probe.KTC = (t.KT + 15) / 16;
+    probe.KS = (t.KT + probe.KTC - 1) / probe.KTC;
+    if (t.RTC <= 1 || smem_plan(probe, 8).total <= max_smem) break;
+    t.RTC = (t.RTC + 1) / 2;
+    t.RG = (t.RT + t.RTC - 1) / t.RTC;
+  }
 }
 
 Workspace plan_workspace(const af1_layer& L, int64_t tokens) {
@@ -624,7 +727,7 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
 
     PhaseArgs p1 = {};
     p1.tiles = L.tiles1;
-    p1.tm = L.p1;
+    p1.tm = launch_plan(L.p1, ng, L.max_smem);
     p1.tokens = T;
     p1.x = static_cast<const __half*>(x) + t0 * ldx;
     p1.ldx = ldx;
@@ -638,7 +741,7 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
 
     PhaseArgs p2 = {};
     p2.tiles = L.tiles2;
-    p2.tm = L.p2;
+    p2.tm = launch_plan(L.p2, ng, L.max_smem);
     p2.tokens = T;
     p2.zin = p1.sout;
     p2.ldz = p1.lds;

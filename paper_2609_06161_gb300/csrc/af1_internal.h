@@ -14,6 +14,7 @@ struct af1_layer {
   int32_t flags = 0;
   int device = 0;
   int num_sms = 0;
+  int max_smem = 0;  // opt-in shared memory per block on this device
   // Phase 1 contracts V (B = V^T, r x n) with z = b * x; phase 2 contracts
   // U (m x r) with s' = s * t.
   af1::TileMatrix p1, p2;
