@@ -81,7 +81,7 @@ int check_desc(const af1_layer_desc* d) {
   return AF1_OK;
 }
 
-// Allocate a layer with its tile plans; buffers zero-filled on `st`.
+// Allocate a layer in the row-block layout; buffers zero-filled on `st`.
 int create_layer(const af1_layer_desc* d, cudaStream_t st, af1_layer** out) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
@@ -104,10 +104,10 @@ int create_layer(const af1_layer_desc* d, cudaStream_t st, af1_layer** out) {
     return fail_cuda(e, "cudaDeviceGetAttribute");
   }
   L->max_smem = max_smem;
-  af1::plan_tiles(L->p1, d->r, d->n, sms, max_smem);
-  af1::plan_tiles(L->p2, d->m, d->r, sms, max_smem);
-  const int64_t t1 = (int64_t)L->p1.RT * L->p1.KT * af1::kTileBytes;
-  const int64_t t2 = (int64_t)L->p2.RT * L->p2.KT * af1::kTileBytes;
+  L->p1 = af1::make_sign_matrix(d->r, d->n);
+  L->p2 = af1::make_sign_matrix(d->m, d->r);
+  const int64_t t1 = af1::sign_matrix_bytes(L->p1);
+  const int64_t t2 = af1::sign_matrix_bytes(L->p2);
   const int64_t sa = align256(2 * d->m), ss = align256(2 * d->r), sb = align256(2 * d->n);
   const int64_t total = align256(t1) + align256(t2) + sa + ss + sb;
   e = cudaMalloc(&L->alloc, (size_t)total);
@@ -116,9 +116,9 @@ int create_layer(const af1_layer_desc* d, cudaStream_t st, af1_layer** out) {
     return fail_cuda(e, "cudaMalloc(layer)");
   }
   uint8_t* base = static_cast<uint8_t*>(L->alloc);
-  L->tiles1 = base;
-  L->tiles2 = base + align256(t1);
-  L->a = reinterpret_cast<uint16_t*>(L->tiles2 + align256(t2));
+  L->signs1 = base;
+  L->signs2 = base + align256(t1);
+  L->a = reinterpret_cast<uint16_t*>(L->signs2 + align256(t2));
   L->s = reinterpret_cast<uint16_t*>(reinterpret_cast<uint8_t*>(L->a) + sa);
   L->b = reinterpret_cast<uint16_t*>(reinterpret_cast<uint8_t*>(L->s) + ss);
   L->sign_bytes = t1 + t2;
@@ -213,8 +213,8 @@ int af1_pack_layer(const af1_layer_desc* desc, const int8_t* U, const int8_t* V,
   // n x r row-major V (row stride 1, column stride r).
   if (e == cudaSuccess) e = af1::launch_pack_signs(U, m, r, r, 1, Uw, wu, flag, st);
   if (e == cudaSuccess) e = af1::launch_pack_signs(V, r, n, 1, r, Vw, wv, flag, st);
-  if (e == cudaSuccess) e = af1::launch_words_to_tiles(Vw, wv, L->p1, L->tiles1, st);
-  if (e == cudaSuccess) e = af1::launch_words_to_tiles(Uw, wu, L->p2, L->tiles2, st);
+  if (e == cudaSuccess) e = af1::launch_words_to_blocks(Vw, wv, L->p1, L->signs1, st);
+  if (e == cudaSuccess) e = af1::launch_words_to_blocks(Uw, wu, L->p2, L->signs2, st);
   if (e != cudaSuccess) {
     destroy_layer(L);
     cudaFree(scratch);
@@ -254,8 +254,8 @@ int af1_load_packed_layer(const af1_layer_desc* desc, const uint32_t* U_words, c
   af1_layer* L = nullptr;
   rc = create_layer(desc, st, &L);
   if (rc != AF1_OK) return rc;
-  e = af1::launch_words_to_tiles(V_words, words_per_row(desc->n), L->p1, L->tiles1, st);
-  if (e == cudaSuccess) e = af1::launch_words_to_tiles(U_words, words_per_row(desc->r), L->p2, L->tiles2, st);
+  e = af1::launch_words_to_blocks(V_words, words_per_row(desc->n), L->p1, L->signs1, st);
+  if (e == cudaSuccess) e = af1::launch_words_to_blocks(U_words, words_per_row(desc->r), L->p2, L->signs2, st);
   if (e != cudaSuccess) {
     destroy_layer(L);
     return fail_cuda(e, "pack kernels");

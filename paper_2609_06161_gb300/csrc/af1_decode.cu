@@ -1,0 +1,787 @@
+// af1_decode.cu — decode path (1..16 tokens per pass) of the forward pass of
+// an AF1 binary-factorized linear layer on sm_103a:
+//     y = a * (U (s * (V^T (b * x)))),
+// the right-to-left evaluation of AF1 Eq. final_reconstruction /
+// Eq. double_factor_equiv that never forms the dense W_hat.
+//
+// Two kernels per pass, chained with programmatic dependent launch (PDL):
+//   phase 1: t = B z with B = V^T (r x n) and z = b * x; s' = s * t is
+//            written as FP32 to the workspace;
+//   phase 2: u = U s' (m x r); y = a * u, stored as FP16 or FP32.
+// A phase is an R x C sign matrix (af1_layout.h) times T <= 16 vectors.
+// CTA (rb, ks) owns row block rb (128 rows: the M of one tcgen05 MMA) and
+// the ks-th slice of CPC column chunks; the KS CTAs of a row block form one
+// thread-block cluster and reduce their partial sums through distributed
+// shared memory, each CTA finalising 1/KS of the rows by summing the KS
+// partials in a fixed order (deterministic, no global atomics).
+//
+// Inside a CTA (256 threads):
+//   * one thread starts bulk copies (cp.async.bulk) of the CTA's packed
+//     chunks, 2 KB each, before anything else;
+//   * warps 0-3 (thread i = matrix row i = tensor-memory lane i) expand every
+//     chunk into e4m3 A values in tensor memory (tcgen05.st) through a ring
+//     of A buffers. The signs do not depend on the previous kernel, so this
+//     runs while it is still finishing;
+//   * warps 4-7 wait for the previous kernel (griddepcontrol.wait), read the
+//     CTA's activations and write the B operand (e4m3, N = 16/32/64 rows =
+//     4 terms x tokens) to shared memory in the 128-byte-swizzled K-major
+//     layout of the MMA descriptor;
+//   * lane 0 of warps 4..4+NACC-1 issue the MMAs (tcgen05.mma kind::f8f6f4,
+//     A from tensor memory, B from shared memory), each into its own
+//     accumulator: one issuing thread sustains about one MMA per 93 cycles
+//     whatever N is, so NACC independent issuers multiply the rate;
+//   * warps 0-3 read the accumulators back (tcgen05.ld), add terms and
+//     accumulators, apply the sign correction and the activation scale and
+//     push the partial sums to the cluster CTA that owns each row.
+//
+// Sign arithmetic. A sign bit becomes an e4m3 byte with one LOP3 per 4 signs:
+// (word & mask_p) | base_p puts the bit at a fixed position p of a constant
+// byte, giving A = L_p + d_p * bit with L_p, d_p powers of two (mantissa bits,
+// exponent bit 0 or the sign bit). With z'_k = z_k / d_k the MMA yields
+// D = sum_k L_k z'_k + sum_k bit_k z_k, and since sign = 2 bit - 1,
+//     sum_k sign_k z_k = 2 D - Q,   Q = sum_k (L_k + H_k) z'_k  (H = L + d).
+// Each z'_k is scaled by a per-(CTA, token) power of two 2^sigma that puts
+// the largest magnitude in [128, 256), and split into 4 e4m3 terms
+// (z' ~ t1 + t2 + t3 + t4, about 16 significant bits) that occupy 4 of the N
+// rows of B. Products are exact and the MMA accumulates in FP32.
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "af1_internal.h"
+#include "af1_layout.h"
+
+namespace af1 {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kTmemCols = 256;        // per CTA: two CTAs fit on one SM
+constexpr int kMaxCPC = 64;           // column chunks per CTA (one mbarrier each)
+constexpr int kMaxKS = 16;            // CTAs per cluster
+constexpr int kMinSmem = 80 * 1024;   // at most two CTAs per SM: their tensor memory always fits
+constexpr long long kWaitCycles = 2000000000ll;  // ~1 s at 2 GHz
+constexpr unsigned kStatusTimeout = 1u;
+
+// ---------------------------------------------------------------------------
+// PTX helpers (hand-written: mbarrier, bulk copy, PDL, cluster, tcgen05, FP8)
+// ---------------------------------------------------------------------------
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t done;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+      : "=r"(done)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return done != 0;
+}
+// Bounded wait: false (and the CTA error flag set) if the phase did not
+// complete within kWaitCycles.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint32_t* err) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const long long t0 = clock64();
+  while (!mbar_try_wait(bar, parity)) {
+    if (clock64() - t0 > kWaitCycles) {
+      atomicOr(err, 1u);
+      return false;
+    }
+  }
+  return true;
+}
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          smem_u32(dst)),
+      "l"(src), "r"(bytes), "r"(smem_u32(bar))
+      : "memory");
+}
+__device__ __forceinline__ void griddep_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+// Split cluster barrier: arrive (relaxed) at start, wait before the first
+// write into a peer's shared memory (the peer must have started).
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.aligned;" ::: "memory"); }
+// Cluster-wide barrier with release/acquire semantics for shared memory.
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void st_cluster_f32(float* local, uint32_t rank, float v) {
+  uint32_t remote;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(local)), "r"(rank));
+  asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(remote), "f"(v) : "memory");
+}
+// Named barrier of the four builder warps (4..7).
+__device__ __forceinline__ void builders_sync() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row groups
+// 1024 bytes apart (stride byte offset), descriptor version 1.
+__device__ __forceinline__ uint64_t smem_desc(uint32_t addr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((addr >> 4) & 0x3FFFu);  // start address
+  d |= (uint64_t)1u << 16;                 // leading byte offset (unused for this layout)
+  d |= (uint64_t)(1024u >> 4) << 32;       // stride byte offset
+  d |= (uint64_t)1u << 46;                 // version
+  d |= (uint64_t)2u << 61;                 // 128-byte swizzle
+  return d;
+}
+// D (FP32, tensor memory) [+]= A (e4m3, tensor memory) x B (e4m3, shared
+// memory)^T, M = 128, K = 32, N = the template argument.
+template <int N>
+__device__ __forceinline__ void mma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, bool accumulate) {
+  constexpr uint32_t idesc = (1u << 4) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(kBlockRows >> 4) << 24);
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], [%1], %2, %3, p;\n}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate ? 1u : 0u)
+      : "memory");
+}
+__device__ __forceinline__ void mma_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+               : "memory");
+}
+__device__ __forceinline__ void tmem_st16(uint32_t addr, const uint32_t (&r)[32], int o) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(
+          addr),
+      "r"(r[o + 0]), "r"(r[o + 1]), "r"(r[o + 2]), "r"(r[o + 3]), "r"(r[o + 4]), "r"(r[o + 5]), "r"(r[o + 6]),
+      "r"(r[o + 7]), "r"(r[o + 8]), "r"(r[o + 9]), "r"(r[o + 10]), "r"(r[o + 11]), "r"(r[o + 12]), "r"(r[o + 13]),
+      "r"(r[o + 14]), "r"(r[o + 15])
+      : "memory");
+}
+__device__ __forceinline__ void tmem_ld16(uint32_t addr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+        "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(addr));
+}
+
+// Two floats -> two e4m3 bytes (round to nearest even, saturating); `lo`
+// lands in bits 0..7.
+__device__ __forceinline__ uint32_t e4m3x2(float lo, float hi) {
+  uint16_t r;
+  asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+// Exact values of two e4m3 bytes (bits 0..7 and 8..15).
+__device__ __forceinline__ float2 e4m3x2_value(uint32_t two) {
+  uint32_t h2;
+  uint16_t in = static_cast<uint16_t>(two);
+  asm("cvt.rn.f16x2.e4m3x2 %0, %1;" : "=r"(h2) : "h"(in));
+  return __half22float2(*reinterpret_cast<__half2*>(&h2));
+}
+
+// Bit position p of a byte (column 4p + e of a word, af1_layout.h): 1 / d_p
+// and L_p + H_p.
+//   p:        0     1     2     3     4     5     6     7
+//   d_p:    1/8   1/4   1/2   1/2   1/4   1/2   1/2    -2
+//   L_p:      1     1     1   1/2     1     1   1/2     1
+__constant__ float c_inv_delta[8] = {8.f, 4.f, 2.f, 2.f, 4.f, 2.f, 2.f, -0.5f};
+__constant__ float c_lph[8] = {2.125f, 2.25f, 2.5f, 1.5f, 2.25f, 2.5f, 1.5f, 0.f};
+
+// One word (32 columns) -> 8 tensor-memory columns of e4m3 A values:
+// column p holds columns 4p .. 4p+3 of the word (bit p of each byte).
+__device__ __forceinline__ void expand_word(uint32_t w, uint32_t* s) {
+  const uint32_t v = w >> 3;
+  s[0] = (w & 0x01010101u) | 0x38383838u;  // mantissa bit 0: {1, 1.125}
+  s[1] = (w & 0x02020202u) | 0x38383838u;  // mantissa bit 1: {1, 1.25}
+  s[2] = (w & 0x04040404u) | 0x38383838u;  // mantissa bit 2: {1, 1.5}
+  s[3] = (w & 0x08080808u) | 0x30303030u;  // exponent bit 0: {0.5, 1}
+  s[4] = (v & 0x02020202u) | 0x38383838u;  // byte bit 4 -> mantissa bit 1
+  s[5] = (v & 0x04040404u) | 0x38383838u;  // byte bit 5 -> mantissa bit 2
+  s[6] = (v & 0x08080808u) | 0x30303030u;  // byte bit 6 -> exponent bit 0
+  s[7] = (w & 0x80808080u) | 0x38383838u;  // sign bit: {1, -1}
+}
+
+// The power of two 2^sigma that brings a positive maximum m into [128, 256),
+// read from m's exponent field (m = f 2^e with f in [0.5, 1), sigma = 8 - e).
+// Returns 2^sigma in *sc and 2^-sigma in *is; m == 0 gives 1, 1.
+__device__ __forceinline__ void pow2_scale(float m, float* sc, float* is) {
+  if (!(m > 0.f)) {
+    *sc = 1.f;
+    *is = 1.f;
+    return;
+  }
+  const int e = (int)((__float_as_uint(m) >> 23) & 0xFFu) - 126;
+  const int sigma = max(min(8 - e, 120), -120);
+  *sc = __uint_as_float((uint32_t)(127 + sigma) << 23);
+  *is = __uint_as_float((uint32_t)(127 - sigma) << 23);
+}
+
+// ---------------------------------------------------------------------------
+// Kernel arguments and shared-memory plan
+// ---------------------------------------------------------------------------
+
+struct DecodeArgs {
+  const uint8_t* signs;  // af1_layout.h row-block layout
+  SignMatrix sm;
+  int KS, CPC;           // cluster size along K, chunks per CTA
+  int tokens;            // T (1..N/4)
+  const __half* x;       // phase 1 input [T][ldx] (FP16)
+  int64_t ldx;
+  const float* zin;      // phase 2 input [T][ldz] (FP32)
+  int64_t ldz;
+  const __half* colscale;  // phase 1: b (C entries)
+  const __half* rowscale;  // phase 1: s; phase 2: a (R entries)
+  float* sout;             // phase 1 output [T][lds]
+  int64_t lds;
+  void* y;                 // phase 2 output [T][ldy], FP16 (ydtype 0) or FP32
+  int64_t ldy;
+  int ydtype;
+  unsigned* status;
+};
+
+struct __align__(8) DecodeHeader {
+  uint64_t wfull[kMaxCPC];  // packed chunk c has landed (bulk copy)
+  uint64_t afull[8];        // A buffer holds its chunk (128 expander arrivals)
+  uint64_t aempty[8];       // the MMAs that read an A buffer are done (NACC commits)
+  uint64_t ddone;           // all MMAs done (NACC commits)
+  uint64_t stats;           // per-token 2^-sigma and Q 2^-sigma are published
+  uint32_t tmem_base, err;
+  uint32_t maxbits[kMaxPassTokens];  // max |z'| per token, as FP32 bits
+  float sc[kMaxPassTokens], is[kMaxPassTokens], qis[kMaxPassTokens];
+};
+
+struct DecodeSmem {
+  int bt, w, recv, qpart, rs, hdr, total;  // byte offsets from the 1024-aligned base
+};
+
+__host__ __device__ inline int align128(int v) { return (v + 127) & ~127; }
+__host__ __device__ inline int slice_rows(int KS) { return (kBlockRows + KS - 1) / KS; }
+
+__host__ __device__ inline DecodeSmem decode_smem(int N, int CPC, int KS, int T) {
+  DecodeSmem p;
+  int off = 0;
+  p.bt = off;
+  off += N * 128 * CPC;  // B: chunk c at c N 128, 1024-aligned
+  p.w = off;
+  off += kChunkBytes * CPC;
+  p.recv = off;
+  off = align128(off + KS * T * slice_rows(KS) * 4);
+  p.qpart = off;
+  off = align128(off + T * 128 * 4);
+  p.rs = off;
+  off = align128(off + slice_rows(KS) * 4);
+  p.hdr = off;
+  off = align128(off + (int)sizeof(DecodeHeader));
+  p.total = off + 1024;  // slack for aligning the base to 1024 bytes
+  return p;
+}
+
+__host__ __device__ constexpr int nacc_for(int N) { return N <= 32 ? 4 : 2; }
+__host__ __device__ constexpr int nbuf_for(int N) { return (kTmemCols - nacc_for(N) * N) / 32; }
+
+// ---------------------------------------------------------------------------
+// Kernel
+// ---------------------------------------------------------------------------
+
+template <int PHASE>
+__device__ __forceinline__ float4 load4(const DecodeArgs& a, int t, int64_t k) {
+  // Four consecutive activations of token t from column k (zero beyond C).
+  // Written by the kernel this one overlaps through PDL, so read through L2
+  // (ld.global.cg), never through the non-coherent L1 path.
+  const int64_t C = a.sm.C;
+  float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (PHASE == 1) {
+    const __half* p = a.x + (int64_t)t * a.ldx + k;
+    if (k + 3 < C) {
+      const uint2 raw = __ldcg(reinterpret_cast<const uint2*>(p));
+      const float2 f0 = __half22float2(*reinterpret_cast<const __half2*>(&raw.x));
+      const float2 f1 = __half22float2(*reinterpret_cast<const __half2*>(&raw.y));
+      z = make_float4(f0.x, f0.y, f1.x, f1.y);
+    } else {
+      if (k < C) z.x = __half2float(__ldcg(p));
+      if (k + 1 < C) z.y = __half2float(__ldcg(p + 1));
+      if (k + 2 < C) z.z = __half2float(__ldcg(p + 2));
+    }
+  } else {
+    const float* p = a.zin + (int64_t)t * a.ldz + k;
+    if (k + 3 < C) {
+      z = __ldcg(reinterpret_cast<const float4*>(p));
+    } else {
+      if (k < C) z.x = __ldcg(p);
+      if (k + 1 < C) z.y = __ldcg(p + 1);
+      if (k + 2 < C) z.z = __ldcg(p + 2);
+    }
+  }
+  return z;
+}
+
+// z'_k = z_k * colscale_k / d_p for the 4 columns k..k+3 (one bit position p).
+template <int PHASE>
+__device__ __forceinline__ float4 load_scaled4(const DecodeArgs& a, int t, int64_t k) {
+  float4 z = load4<PHASE>(a, t, k);
+  const float id = c_inv_delta[(k >> 2) & 7];
+  if (PHASE == 1) {
+    const int64_t C = a.sm.C;
+    float b0 = 0.f, b1 = 0.f, b2 = 0.f, b3 = 0.f;
+    if (k + 3 < C) {
+      const uint2 raw = __ldg(reinterpret_cast<const uint2*>(a.colscale + k));
+      const float2 f0 = __half22float2(*reinterpret_cast<const __half2*>(&raw.x));
+      const float2 f1 = __half22float2(*reinterpret_cast<const __half2*>(&raw.y));
+      b0 = f0.x;
+      b1 = f0.y;
+      b2 = f1.x;
+      b3 = f1.y;
+    } else {
+      if (k < C) b0 = __half2float(a.colscale[k]);
+      if (k + 1 < C) b1 = __half2float(a.colscale[k + 1]);
+      if (k + 2 < C) b2 = __half2float(a.colscale[k + 2]);
+    }
+    z = make_float4(z.x * b0, z.y * b1, z.z * b2, z.w * b3);
+  }
+  return make_float4(z.x * id, z.y * id, z.z * id, z.w * id);
+}
+
+template <int PHASE, int N>
+__global__ void __launch_bounds__(kThreads, 1) decode_kernel(const DecodeArgs a) {
+  constexpr int NACC = nacc_for(N);
+  constexpr int NBUF = nbuf_for(N);
+  constexpr int DCOL = NBUF * 32;  // first accumulator column
+  constexpr int STASH = 4;         // activation groups a builder thread keeps in registers
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  const int T = a.tokens;
+  const int KS = a.KS;
+  const DecodeSmem sp = decode_smem(N, a.CPC, KS, T);
+  uint8_t* Bt = smem + sp.bt;
+  const uint32_t* W = reinterpret_cast<const uint32_t*>(smem + sp.w);
+  float* recv = reinterpret_cast<float*>(smem + sp.recv);
+  float* qpart = reinterpret_cast<float*>(smem + sp.qpart);
+  float* rs = reinterpret_cast<float*>(smem + sp.rs);
+  DecodeHeader& h = *reinterpret_cast<DecodeHeader*>(smem + sp.hdr);
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int rb = blockIdx.x, ks = blockIdx.y;
+  const int nch_total = a.sm.NCH;
+  const int c0 = ks * a.CPC;
+  const int nch = min(a.CPC, nch_total - c0);  // >= 1 by construction of KS
+  const int64_t row0 = (int64_t)rb * kBlockRows;
+  const int64_t k0 = (int64_t)c0 * kChunkCols;
+  const int slice = slice_rows(KS);
+  const int my0 = ks * slice;  // first block row this CTA finalises
+
+  cluster_arrive_relaxed();  // matched by cluster_wait before the first remote store
+
+  if (tid == 128) {
+    for (int c = 0; c < nch; ++c) mbar_init(&h.wfull[c], 1);
+    for (int b = 0; b < NBUF; ++b) {
+      mbar_init(&h.afull[b], 128);
+      mbar_init(&h.aempty[b], NACC);
+    }
+    mbar_init(&h.ddone, NACC);
+    mbar_init(&h.stats, 16);
+    h.err = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    // Packed chunks of this CTA: contiguous 2 KB blocks of row block rb.
+    const uint8_t* src = a.signs + ((int64_t)rb * nch_total + c0) * kChunkBytes;
+    for (int c = 0; c < nch; ++c) {
+      mbar_expect_tx(&h.wfull[c], kChunkBytes);
+      bulk_g2s(smem + sp.w + c * kChunkBytes, src + (int64_t)c * kChunkBytes, kChunkBytes, &h.wfull[c]);
+    }
+  }
+  if (tid < kMaxPassTokens) h.maxbits[tid] = 0u;  // published by the CTA barrier below
+  __syncwarp();
+  if (warp == 4) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&h.tmem_base)),
+                 "r"((uint32_t)kTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  // Row scales of the rows this CTA finalises (layer constants).
+  for (int i = tid; i < slice; i += kThreads) {
+    const int64_t row = row0 + my0 + i;
+    rs[i] = (my0 + i < kBlockRows && row < a.sm.R) ? __half2float(a.rowscale[row]) : 0.f;
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = h.tmem_base;
+  griddep_launch_dependents();
+
+  if (warp < 4) {
+    // ---- A: expand packed chunks into the tensor-memory ring --------------
+    const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+    bool ok = true;
+    for (int c = 0; c < nch && ok; ++c) {
+      const int b = c % NBUF, use = c / NBUF;
+      if (use >= 1) {
+        ok = mbar_wait(&h.aempty[b], (use - 1) & 1, &h.err);
+        tc_fence_after();
+      }
+      if (ok) ok = mbar_wait(&h.wfull[c], 0, &h.err);
+      if (!ok) break;
+      uint32_t r[32];
+      const uint32_t* wc = W + c * (kChunkBytes / 4);
+#pragma unroll
+      for (int kw = 0; kw < kChunkWords; ++kw) expand_word(wc[kw * kBlockRows + tid], r + 8 * kw);
+      const uint32_t addr = tmem + lane_base + (uint32_t)(b * 32);
+      tmem_st16(addr, r, 0);
+      tmem_st16(addr + 16, r, 16);
+      asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+      tc_fence_before();
+      mbar_arrive(&h.afull[b]);
+    }
+  } else {
+    // ---- B: activations -> e4m3 terms in the swizzled B tile --------------
+    const int bt = tid - 128;
+    const int g4 = nch * (kChunkCols / 4);  // groups of 4 columns per token
+    const int ngroups = T * g4;
+    for (int t = 0; t < T; ++t) qpart[t * 128 + bt] = 0.f;  // own column only
+    griddep_wait();  // activations are written by the previous kernel
+    float4 stash[STASH];
+    // Pass 1: maxima of |z'| per token.
+    {
+      int cur_t = -1;
+      float mx = 0.f;
+#pragma unroll
+      for (int i = 0; i < STASH; ++i) stash[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+      for (int i = 0, g = bt; g < ngroups; ++i, g += 128) {
+        const int t = g / g4, c4 = g - t * g4;
+        const float4 u = load_scaled4<PHASE>(a, t, k0 + 4 * c4);
+        if (i < STASH) {
+#pragma unroll
+          for (int j = 0; j < STASH; ++j)
+            if (j == i) stash[j] = u;
+        }
+        if (t != cur_t) {
+          if (cur_t >= 0 && mx > 0.f) atomicMax(&h.maxbits[cur_t], __float_as_uint(mx));
+          cur_t = t;
+          mx = 0.f;
+        }
+        mx = fmaxf(mx, fmaxf(fmaxf(fabsf(u.x), fabsf(u.y)), fmaxf(fabsf(u.z), fabsf(u.w))));
+      }
+      if (cur_t >= 0 && mx > 0.f) atomicMax(&h.maxbits[cur_t], __float_as_uint(mx));
+    }
+    builders_sync();
+    // Pass 2: split into 4 e4m3 terms, write B rows 4t + q, and Q partials.
+    {
+      int cur_t = -1;
+      float sc = 0.f, q = 0.f;
+      for (int i = 0, g = bt; g < ngroups; ++i, g += 128) {
+        const int t = g / g4, c4 = g - t * g4;
+        if (t != cur_t) {
+          if (cur_t >= 0) qpart[cur_t * 128 + bt] = q;
+          cur_t = t;
+          q = 0.f;
+          float is_unused;
+          pow2_scale(__uint_as_float(h.maxbits[t]), &sc, &is_unused);
+        }
+        float4 u;
+        if (i < STASH) {
+          u = stash[0];
+#pragma unroll
+          for (int j = 1; j < STASH; ++j)
+            if (j == i) u = stash[j];
+        } else {
+          u = load_scaled4<PHASE>(a, t, k0 + 4 * c4);
+        }
+        float4 v = make_float4(u.x * sc, u.y * sc, u.z * sc, u.w * sc);
+        const float4 v0 = v;
+        const int kl = 4 * c4;  // column within the CTA's range
+        const int c = kl >> 7, kin = kl & 127;
+        uint8_t* base = Bt + c * (N * 128) + (kin & 15);
+        const int j16 = kin >> 4;
+#pragma unroll
+        for (int term = 0; term < kTerms; ++term) {
+          const uint32_t lo = e4m3x2(v.x, v.y), hi = e4m3x2(v.z, v.w);
+          const float2 flo = e4m3x2_value(lo), fhi = e4m3x2_value(hi);
+          v.x -= flo.x;
+          v.y -= flo.y;
+          v.z -= fhi.x;
+          v.w -= fhi.y;
+          const int n = 4 * t + term;
+          *reinterpret_cast<uint32_t*>(base + n * 128 + ((j16 ^ (n & 7)) << 4)) = lo | (hi << 16);
+        }
+        q += c_lph[c4 & 7] * (((v0.x - v.x) + (v0.y - v.y)) + ((v0.z - v.z) + (v0.w - v.w)));
+      }
+      if (cur_t >= 0) qpart[cur_t * 128 + bt] = q;
+    }
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // B is read by the tensor cores
+    builders_sync();
+    const int ia = warp - 4;
+    if (lane == 0 && ia < NACC) {
+      // ---- MMA issue: chunk c, K step kk (32 columns) by issuer kk % NACC --
+      const uint32_t b0 = smem_u32(Bt);
+      bool ok = true;
+      for (int c = 0; c < nch && ok; ++c) {
+        const int b = c % NBUF, use = c / NBUF;
+        ok = mbar_wait(&h.afull[b], use & 1, &h.err);
+        if (!ok) break;
+        tc_fence_after();
+#pragma unroll
+        for (int kk = ia; kk < 4; kk += NACC) {
+          mma_ts<N>(tmem + (uint32_t)(DCOL + ia * N), tmem + (uint32_t)(b * 32 + kk * 8),
+                    smem_desc(b0 + (uint32_t)(c * N * 128 + kk * 32)), c > 0 || kk >= NACC);
+        }
+        mma_commit(&h.aempty[b]);
+      }
+      mma_commit(&h.ddone);
+    }
+    if (bt >= 112) {
+      // ---- per-token 2^-sigma and Q 2^-sigma, summed in a fixed order ------
+      const int t = bt - 112;
+      if (t < T) {
+        float qs = 0.f;
+        for (int j = 0; j < 128; ++j) qs += qpart[t * 128 + j];
+        float sc, is;
+        pow2_scale(__uint_as_float(h.maxbits[t]), &sc, &is);
+        h.is[t] = is;
+        h.qis[t] = qs * is;
+      }
+      mbar_arrive(&h.stats);
+    }
+    __syncwarp();
+  }
+
+  // ---- epilogue: accumulators -> per-row partial sums -> owner CTA ----------
+  griddep_wait();  // outputs may still be read by the previous kernel until it completes
+  cluster_wait();  // every CTA of the cluster has started
+  if (warp < 4) {
+    const bool ok = mbar_wait(&h.ddone, 0, &h.err) && mbar_wait(&h.stats, 0, &h.err);
+    tc_fence_after();
+    const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+    const int i = tid;  // block row
+    const int owner = i / slice;
+#pragma unroll
+    for (int cb = 0; cb < N / 16; ++cb) {
+      float acc[16];
+#pragma unroll
+      for (int j = 0; j < 16; ++j) acc[j] = 0.f;
+#pragma unroll
+      for (int d = 0; d < NACC; ++d) {
+        uint32_t r[16];
+        tmem_ld16(tmem + lane_base + (uint32_t)(DCOL + d * N + cb * 16), r);
+        asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+        for (int j = 0; j < 16; ++j) acc[j] += __uint_as_float(r[j]);
+      }
+#pragma unroll
+      for (int tt = 0; tt < 4; ++tt) {
+        const int t = cb * 4 + tt;
+        if (ok && t < T) {
+          const float dsum = (acc[4 * tt] + acc[4 * tt + 1]) + (acc[4 * tt + 2] + acc[4 * tt + 3]);
+          const float p = 2.f * dsum * h.is[t] - h.qis[t];
+          st_cluster_f32(recv + ((ks * T + t) * slice + (i - owner * slice)), (uint32_t)owner, p);
+        }
+      }
+    }
+  }
+  // All partials of the cluster have landed in their owners' buffers.
+  cluster_sync();
+  const int cnt = min(slice, kBlockRows - my0);
+  for (int idx = tid; idx < T * cnt; idx += kThreads) {
+    const int t = idx / cnt;
+    const int i = idx - t * cnt;
+    const int64_t row = row0 + my0 + i;
+    if (row >= a.sm.R) continue;
+    float v = 0.f;
+    for (int q = 0; q < KS; ++q) v += recv[(q * T + t) * slice + i];
+    const float out = v * rs[i];
+    if (PHASE == 1) {
+      a.sout[(int64_t)t * a.lds + row] = out;
+    } else if (a.ydtype == 0) {
+      reinterpret_cast<__half*>(a.y)[(int64_t)t * a.ldy + row] = __float2half_rn(out);
+    } else {
+      reinterpret_cast<float*>(a.y)[(int64_t)t * a.ldy + row] = out;
+    }
+  }
+
+  // ---- teardown ---------------------------------------------------------------
+  tc_fence_before();
+  __syncthreads();
+  if (tid == 128 && h.err != 0) {
+    // Something timed out: let the bulk copies drain (bounded) so that none
+    // lands after the CTA has exited, and report it.
+    for (int c = 0; c < nch; ++c) mbar_wait(&h.wfull[c], 0, &h.err);
+    atomicOr(a.status, kStatusTimeout);
+  }
+  if (warp == 4) {
+    tc_fence_after();
+    if (lane == 0) mbar_wait(&h.ddone, 0, &h.err);  // no MMA may still read tensor memory
+    __syncwarp();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"((uint32_t)kTmemCols)
+                 : "memory");
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Host side
+// ---------------------------------------------------------------------------
+
+struct DecodePlan {
+  int N = 0, KS = 0, CPC = 0, smem = 0;
+  bool ok = false;
+};
+
+int n_for_tokens(int T) { return T <= 4 ? 16 : T <= 8 ? 32 : 64; }
+
+// Split of one sign matrix for a pass of T tokens: about one CTA per SM
+// (row blocks x KS <= SMs), KS <= 16 CTAs per cluster, and the CTA's chunks
+// within the shared-memory budget.
+DecodePlan plan_decode(const SignMatrix& sm, int T, int num_sms, int max_smem) {
+  DecodePlan p;
+  p.N = n_for_tokens(T);
+  const int sms = num_sms > 0 ? num_sms : 148;
+  int ks = sms / (sm.RB > 0 ? sm.RB : 1);
+  if (ks < 1) ks = 1;
+  if (ks > kMaxKS) ks = kMaxKS;
+  if (ks > sm.NCH) ks = sm.NCH;
+  for (; ks <= kMaxKS; ++ks) {
+    const int cpc = (sm.NCH + ks - 1) / ks;
+    if (cpc > kMaxCPC) continue;
+    const int KS = (sm.NCH + cpc - 1) / cpc;
+    const int need = decode_smem(p.N, cpc, KS, T).total;
+    if (need <= max_smem) {
+      p.KS = KS;
+      p.CPC = cpc;
+      p.smem = need < kMinSmem ? kMinSmem : need;
+      p.ok = true;
+      return p;
+    }
+  }
+  return p;
+}
+
+template <int PHASE, int N>
+cudaError_t launch_decode_n(const DecodeArgs& a, const DecodePlan& p, cudaStream_t st) {
+  auto kern = decode_kernel<PHASE, N>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, p.smem);
+  if (e != cudaSuccess) return e;
+  if (p.KS > 8) {
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    if (e != cudaSuccess) return e;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)a.sm.RB, (unsigned)p.KS, 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = (size_t)p.smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = 1;
+  attr[1].val.clusterDim.y = (unsigned)p.KS;
+  attr[1].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  return cudaLaunchKernelEx(&cfg, kern, a);
+}
+
+template <int PHASE>
+cudaError_t launch_decode(DecodeArgs a, const DecodePlan& p, cudaStream_t st) {
+  a.KS = p.KS;
+  a.CPC = p.CPC;
+  switch (p.N) {
+    case 16: return launch_decode_n<PHASE, 16>(a, p, st);
+    case 32: return launch_decode_n<PHASE, 32>(a, p, st);
+    default: return launch_decode_n<PHASE, 64>(a, p, st);
+  }
+}
+
+int64_t align256(int64_t v) { return (v + 255) / 256 * 256; }
+
+}  // namespace
+
+int64_t decode_ldz(const af1_layer& L) { return (int64_t)L.p2.NCH * kChunkCols; }
+
+Workspace plan_workspace(const af1_layer& L, int64_t tokens) {
+  Workspace w;
+  int64_t off = 0;
+  w.status = off;
+  off += 256;
+  w.sbuf = off;
+  off += align256((int64_t)kMaxPassTokens * decode_ldz(L) * 4);
+  w.hbuf = off;
+  if (tokens > kMaxPassTokens) {
+    const int64_t t = tokens < kPrefillPassTokens ? tokens : kPrefillPassTokens;
+    off += align256(t * prefill_h_ld(L) * 2);
+  }
+  w.total = off;
+  return w;
+}
+
+cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64_t tokens, void* y,
+                           int64_t ldy, int y_dtype, void* ws, cudaStream_t st) {
+  const Workspace W = plan_workspace(L, tokens);
+  uint8_t* wsb = static_cast<uint8_t*>(ws);
+  if (tokens > kMaxPassTokens) {
+    // Prefill: two tensor-core GEMMs per pass (af1_prefill.cu).
+    return launch_prefill(L, x, ldx, tokens, y, ldy, y_dtype, wsb + W.hbuf, reinterpret_cast<unsigned*>(wsb + W.status),
+                          st);
+  }
+  // Widest pass whose plans fit (16 tokens normally; fewer only for very
+  // long contractions).
+  int pass = kMaxPassTokens;
+  DecodePlan p1, p2;
+  for (;;) {
+    const int T = (int)(tokens < pass ? tokens : pass);
+    p1 = plan_decode(L.p1, T, L.num_sms, L.max_smem);
+    p2 = plan_decode(L.p2, T, L.num_sms, L.max_smem);
+    if ((p1.ok && p2.ok) || pass <= 4) break;
+    pass /= 2;
+  }
+  if (!p1.ok || !p2.ok) return cudaErrorInvalidConfiguration;
+  const int ysize = y_dtype == 0 ? 2 : 4;
+  for (int64_t t0 = 0; t0 < tokens; t0 += pass) {
+    const int T = (int)((tokens - t0) < pass ? (tokens - t0) : pass);
+    const DecodePlan q1 = plan_decode(L.p1, T, L.num_sms, L.max_smem);
+    const DecodePlan q2 = plan_decode(L.p2, T, L.num_sms, L.max_smem);
+    if (!q1.ok || !q2.ok) return cudaErrorInvalidConfiguration;
+
+    DecodeArgs a1 = {};
+    a1.signs = L.signs1;
+    a1.sm = L.p1;
+    a1.tokens = T;
+    a1.x = static_cast<const __half*>(x) + t0 * ldx;
+    a1.ldx = ldx;
+    a1.colscale = reinterpret_cast<const __half*>(L.b);
+    a1.rowscale = reinterpret_cast<const __half*>(L.s);
+    a1.sout = reinterpret_cast<float*>(wsb + W.sbuf);
+    a1.lds = decode_ldz(L);
+    a1.status = reinterpret_cast<unsigned*>(wsb + W.status);
+    cudaError_t e = launch_decode<1>(a1, q1, st);
+    if (e != cudaSuccess) return e;
+
+    DecodeArgs a2 = {};
+    a2.signs = L.signs2;
+    a2.sm = L.p2;
+    a2.tokens = T;
+    a2.zin = a1.sout;
+    a2.ldz = a1.lds;
+    a2.rowscale = reinterpret_cast<const __half*>(L.a);
+    a2.y = static_cast<uint8_t*>(y) + t0 * ldy * ysize;
+    a2.ldy = ldy;
+    a2.ydtype = y_dtype;
+    a2.status = a1.status;
+    e = launch_decode<2>(a2, q2, st);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+}  // namespace af1

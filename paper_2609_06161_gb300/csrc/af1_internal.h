@@ -17,9 +17,9 @@ struct af1_layer {
   int max_smem = 0;  // opt-in shared memory per block on this device
   // Phase 1 contracts V (B = V^T, r x n) with z = b * x; phase 2 contracts
   // U (m x r) with s' = s * t.
-  af1::TileMatrix p1, p2;
-  uint8_t* tiles1 = nullptr;  // p1.RT * p1.KT * 256 bytes
-  uint8_t* tiles2 = nullptr;
+  af1::SignMatrix p1, p2;
+  uint8_t* signs1 = nullptr;  // sign_matrix_bytes(p1)
+  uint8_t* signs2 = nullptr;  // sign_matrix_bytes(p2)
   uint16_t* a = nullptr;      // FP16 row scale, m entries
   uint16_t* s = nullptr;      // FP16 rank scale, r entries
   uint16_t* b = nullptr;      // FP16 column scale, n entries
@@ -35,24 +35,21 @@ constexpr int64_t kPrefillPassTokens = 2048;
 // Workspace carve-up for one layer and one forward call of `tokens` tokens.
 struct Workspace {
   int64_t status = 0;  // uint32 status word
-  int64_t sbuf = 0;    // float[kMaxPassTokens][p2.KT*128]: s' = s * t (decode)
+  int64_t sbuf = 0;    // float[kMaxPassTokens][decode_ldz]: s' = s * t (decode)
   int64_t hbuf = 0;    // FP16 [min(tokens, kPrefillPassTokens)][prefill_h_ld]: H (prefill)
   int64_t total = 0;
 };
 Workspace plan_workspace(const af1_layer& L, int64_t tokens);
 int64_t prefill_h_ld(const af1_layer& L);
-
-// Choose the tile blocks and the split-K cluster of one sign matrix.
-void plan_tiles(TileMatrix& t, int64_t R, int64_t C, int num_sms, int max_smem);
-int forward_smem_bytes(const TileMatrix& t, int ng);
+int64_t decode_ldz(const af1_layer& L);
 
 // Kernel launchers (stream-ordered, asynchronous). Return cudaSuccess or the
 // launch error.
 cudaError_t launch_pack_signs(const int8_t* src, int64_t rows, int64_t cols, int64_t row_stride,
                               int64_t col_stride, uint32_t* words, int64_t words_per_row,
                               uint32_t* bad_flag, cudaStream_t st);
-cudaError_t launch_words_to_tiles(const uint32_t* words, int64_t words_per_row, const TileMatrix& t,
-                                  uint8_t* tiles, cudaStream_t st);
+cudaError_t launch_words_to_blocks(const uint32_t* words, int64_t words_per_row, const SignMatrix& sm,
+                                   uint8_t* out, cudaStream_t st);
 // Set the calling thread's af1_last_error() message; returns `code`.
 int set_error(int code, const std::string& msg);
 

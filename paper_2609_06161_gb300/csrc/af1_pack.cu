@@ -3,9 +3,9 @@
 // (1) pack_signs: an int8 matrix of +-1 (the sign factors of AF1 Sec. 3.1,
 //     A_pm1 and B_pm1) -> the canonical words of the packed format declared in
 //     include/af1.h (bit = 1 for +1, LSB first, rows padded to 16 bytes).
-// (2) words_to_tiles: canonical words -> the internal tile layout described in
-//     af1_layout.h. The bit count is unchanged (1 bit per sign); only the
-//     order differs, plus the zero padding of partial tiles.
+// (2) words_to_blocks: canonical words -> the internal row-block layout
+//     described in af1_layout.h. The bit count is unchanged (1 bit per sign);
+//     only the order differs, plus the zero rows of a partial row block.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -42,28 +42,25 @@ __global__ void pack_signs_kernel(const int8_t* __restrict__ src, int64_t rows, 
   if (bad) atomicOr(bad_flag, 1u);
 }
 
-__global__ void words_to_tiles_kernel(const uint32_t* __restrict__ words, int64_t wpr, TileMatrix tm,
-                                      uint32_t* __restrict__ tiles) {
-  int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  int64_t total = (int64_t)tm.RT * tm.KT * 64;
+// One thread per device word: gather the 32 bits of word kw of row `row`
+// from the canonical word of the same row and word index (same 32 columns,
+// bit b of the device word = canonical bit bit_col(b)).
+__global__ void words_to_blocks_kernel(const uint32_t* __restrict__ words, int64_t wpr, SignMatrix sm,
+                                       uint32_t* __restrict__ out) {
+  const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t total = (int64_t)sm.RB * sm.NCH * kChunkWords * kBlockRows;
   if (t >= total) return;
-  int which = (int)(t & 1);
-  int lane = (int)((t >> 1) & 31);
-  int64_t rest = t >> 6;
-  int rt = (int)(rest % tm.RT);
-  int kt = (int)(rest / tm.RT);
-  int64_t row = (int64_t)rt * kTileRows + (lane >> 2) + 8 * which;
-  int c = lane & 3;
-  uint32_t out = 0;
-  if (row < tm.R) {
-    const uint32_t* src = words + row * wpr;
+  const int64_t i = t % kBlockRows;               // row within the block
+  const int64_t kw = (t / kBlockRows) % ((int64_t)sm.NCH * kChunkWords);
+  const int64_t rb = t / ((int64_t)kBlockRows * sm.NCH * kChunkWords);
+  const int64_t row = rb * kBlockRows + i;
+  uint32_t v = 0;
+  if (row < sm.R) {
+    const uint32_t src = words[row * wpr + kw];
 #pragma unroll
-    for (int b = 0; b < 32; ++b) {
-      int64_t col = (int64_t)kt * kTileCols + bit_col(b, c);
-      if (col < tm.C) out |= ((src[col >> 5] >> (col & 31)) & 1u) << b;
-    }
+    for (int b = 0; b < 32; ++b) v |= ((src >> bit_col(b)) & 1u) << b;
   }
-  tiles[tile_index(tm, rt, kt) * 64 + lane * 2 + which] = out;
+  out[t] = v;
 }
 
 }  // namespace
@@ -80,14 +77,13 @@ cudaError_t launch_pack_signs(const int8_t* src, int64_t rows, int64_t cols, int
   return cudaGetLastError();
 }
 
-cudaError_t launch_words_to_tiles(const uint32_t* words, int64_t wpr, const TileMatrix& tm, uint8_t* tiles,
-                                  cudaStream_t st) {
-  int64_t total = (int64_t)tm.RT * tm.KT * 64;
+cudaError_t launch_words_to_blocks(const uint32_t* words, int64_t wpr, const SignMatrix& sm, uint8_t* out,
+                                   cudaStream_t st) {
+  const int64_t total = (int64_t)sm.RB * sm.NCH * kChunkWords * kBlockRows;
   if (total == 0) return cudaSuccess;
-  int threads = 256;
-  int64_t blocks = (total + threads - 1) / threads;
-  words_to_tiles_kernel<<<(unsigned)blocks, threads, 0, st>>>(words, wpr, tm,
-                                                              reinterpret_cast<uint32_t*>(tiles));
+  const int threads = 256;
+  const int64_t blocks = (total + threads - 1) / threads;
+  words_to_blocks_kernel<<<(unsigned)blocks, threads, 0, st>>>(words, wpr, sm, reinterpret_cast<uint32_t*>(out));
   return cudaGetLastError();
 }
 

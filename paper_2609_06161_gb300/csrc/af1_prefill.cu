@@ -38,8 +38,8 @@ constexpr long long kWaitCycles = 2000000000ll;
 constexpr unsigned kStatusTimeout = 1u;
 
 struct PrefillArgs {
-  const uint32_t* tiles;  // packed signs, af1_layout.h tile order
-  TileMatrix tm;          // R = features, C = K
+  const uint32_t* signs;  // packed signs, af1_layout.h row-block layout
+  SignMatrix sm;          // R = features, C = K
   const __half* act;      // B operand source: [tokens][ld_act] FP16
   int64_t ld_act;
   int tokens;
@@ -158,7 +158,7 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_kernel(const PrefillArgs 
   PrefillBarriers& bar = *reinterpret_cast<PrefillBarriers*>(smem + STAGES * (kTileA + kTileB));
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const TileMatrix& tm = a.tm;
+  const SignMatrix& tm = a.sm;
   const int f0 = blockIdx.x * BM;  // first feature (row of the sign matrix)
   const int t0 = blockIdx.y * BN;  // first token
   const int nk = (int)((tm.C + BK - 1) / BK);
@@ -245,51 +245,49 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_kernel(const PrefillArgs 
     const int R = threadIdx.x - 128;  // 0..127 = TMEM lane of this thread
     const int64_t frow = f0 + R;
     const bool row_ok = frow < tm.R;
-    const int rt = (int)(frow >> 4), ri = (int)(frow & 15);
-    const int g = ri & 7, which = ri >> 3;
+    // Words of this row: index (rb * 4 NCH + kw) * 128 + R (rows past R are
+    // zero words of the padded block).
+    const uint32_t* rowp = a.signs + (int64_t)blockIdx.x * tm.NCH * kChunkWords * kBlockRows + R;
     for (int it = 0; it < nk; ++it) {
       const int s = it % STAGES;
       if (it >= STAGES) mbar_wait(&bar.empty[s], ((it / STAGES) & 1) ^ 1, &bar.err);
-      const int kt = it >> 1, half = it & 1;  // two K-stages per 128-column tile
-      uint32_t w[4] = {0u, 0u, 0u, 0u};
-      if (row_ok) {
-        const uint32_t* base = a.tiles + tile_index(tm, rt, kt) * 64 + which;
-#pragma unroll
-        for (int c = 0; c < 4; ++c) w[c] = __ldg(base + (4 * g + c) * 2);
-      }
+      // Stage columns 64 it .. 64 it + 63 = words 2 it and 2 it + 1.
+      const uint32_t w0 = __ldg(rowp + (int64_t)(2 * it) * kBlockRows);
+      const uint32_t w1 = __ldg(rowp + (int64_t)(2 * it + 1) * kBlockRows);
       uint8_t* dst = tileA + s * kTileA;
       const int64_t k0 = (int64_t)it * BK;
 #pragma unroll
       for (int j = 0; j < 8; ++j) {
-        // chunk j = columns 8j .. 8j+7 of the stage = slot p, lanes c0, c0+1
-        const int p = half * 4 + (j >> 1);
-        const int c0 = (j & 1) * 2;
-        uint4 v;
-        uint32_t* vv = reinterpret_cast<uint32_t*>(&v);
+        // 16-byte chunk j = stage columns 8j .. 8j+7 = columns 4p + e of word
+        // j / 4 with p = 2 (j % 4) (first 4) and p + 1 (last 4).
+        const uint32_t wd = (j < 4) ? w0 : w1;
+        const int p = 2 * (j & 3);
+        const uint32_t b01 = __byte_perm(wd, 0u, 0x1404);  // bytes 0,1 -> bytes 1,3 (e = 0, 1)
+        const uint32_t b23 = __byte_perm(wd, 0u, 0x3424);  // bytes 2,3 -> bytes 1,3 (e = 2, 3)
+        uint32_t sv[4] = {0x3C003C00u, 0x3C003C00u, 0x3C003C00u, 0x3C003C00u};  // +-1 for GEMM2
+        if (GEMM1) {
+          const int64_t kc = k0 + j * 8;
+          if (kc + 7 < tm.C) {
+            const uint4 bb = __ldg(reinterpret_cast<const uint4*>(a.colscale + kc));
+            sv[0] = bb.x;
+            sv[1] = bb.y;
+            sv[2] = bb.z;
+            sv[3] = bb.w;
+          } else {
+            const uint16_t* cs = reinterpret_cast<const uint16_t*>(a.colscale);
 #pragma unroll
-        for (int cc = 0; cc < 2; ++cc) {
-          const uint32_t wd = w[c0 + cc];
-          // bytes 0,1 -> halves of pair 0; bytes 2,3 -> pair 1 (columns e = 0..3)
-          const uint32_t b01 = __byte_perm(wd, 0u, 0x1404);  // byte0 -> byte1, byte1 -> byte3
-          const uint32_t b23 = __byte_perm(wd, 0u, 0x3424);  // byte2 -> byte1, byte3 -> byte3
-          uint32_t s01 = 0x3C003C00u, s23 = 0x3C003C00u;    // +-1 for GEMM2
-          if (GEMM1) {
-            const int64_t kc = k0 + j * 8 + cc * 4;
-            if (kc + 3 < tm.C) {
-              const uint2 bb = __ldg(reinterpret_cast<const uint2*>(a.colscale + kc));
-              s01 = bb.x;
-              s23 = bb.y;
-            } else {
-              const uint16_t* cs = reinterpret_cast<const uint16_t*>(a.colscale);
-              uint32_t e0 = kc < tm.C ? cs[kc] : 0u, e1 = kc + 1 < tm.C ? cs[kc + 1] : 0u;
-              uint32_t e2 = kc + 2 < tm.C ? cs[kc + 2] : 0u, e3 = kc + 3 < tm.C ? cs[kc + 3] : 0u;
-              s01 = e0 | (e1 << 16);
-              s23 = e2 | (e3 << 16);
+            for (int q = 0; q < 4; ++q) {
+              const uint32_t e0 = kc + 2 * q < tm.C ? cs[kc + 2 * q] : 0u;
+              const uint32_t e1 = kc + 2 * q + 1 < tm.C ? cs[kc + 2 * q + 1] : 0u;
+              sv[q] = e0 | (e1 << 16);
             }
           }
-          vv[cc * 2 + 0] = signed_pair(b01, p, s01);
-          vv[cc * 2 + 1] = signed_pair(b23, p, s23);
         }
+        uint4 v;
+        v.x = signed_pair(b01, p, sv[0]);
+        v.y = signed_pair(b23, p, sv[1]);
+        v.z = signed_pair(b01, p + 1, sv[2]);
+        v.w = signed_pair(b23, p + 1, sv[3]);
         *reinterpret_cast<uint4*>(dst + swz(R, j)) = v;
       }
       fence_proxy_async();
@@ -343,7 +341,7 @@ cudaError_t launch_gemm(const PrefillArgs& a, cudaStream_t st) {
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((unsigned)((a.tm.R + BM - 1) / BM), (unsigned)((a.tokens + BN - 1) / BN), 1);
+  cfg.gridDim = dim3((unsigned)a.sm.RB, (unsigned)((a.tokens + BN - 1) / BN), 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.dynamicSmemBytes = kSmemBytes;
   cfg.stream = st;
@@ -366,8 +364,8 @@ cudaError_t launch_prefill(const af1_layer& L, const void* x, int64_t ldx, int64
   for (int64_t t0 = 0; t0 < tokens; t0 += kPrefillPassTokens) {
     const int T = (int)((tokens - t0) < kPrefillPassTokens ? (tokens - t0) : kPrefillPassTokens);
     PrefillArgs g1 = {};
-    g1.tiles = reinterpret_cast<const uint32_t*>(L.tiles1);
-    g1.tm = L.p1;
+    g1.signs = reinterpret_cast<const uint32_t*>(L.signs1);
+    g1.sm = L.p1;
     g1.act = static_cast<const __half*>(x) + t0 * ldx;
     g1.ld_act = ldx;
     g1.tokens = T;
@@ -380,8 +378,8 @@ cudaError_t launch_prefill(const af1_layer& L, const void* x, int64_t ldx, int64
     cudaError_t e = launch_gemm<true>(g1, st);
     if (e != cudaSuccess) return e;
     PrefillArgs g2 = {};
-    g2.tiles = reinterpret_cast<const uint32_t*>(L.tiles2);
-    g2.tm = L.p2;
+    g2.signs = reinterpret_cast<const uint32_t*>(L.signs2);
+    g2.sm = L.p2;
     g2.act = reinterpret_cast<const __half*>(h_buf);
     g2.ld_act = ldh;
     g2.tokens = T;
