@@ -119,7 +119,7 @@ AF1_API int af1_load_packed_layer(const af1_layer_desc* desc, const uint32_t* U_
 /* Copy the description of a layer into *desc. */
 AF1_API int af1_layer_get_desc(const af1_layer* layer, af1_layer_desc* desc);
 
-/* Device bytes the layer holds for its signs (tile layout) and its scales. */
+/* Device bytes the layer holds for its signs (row-block layout) and its scales. */
 AF1_API int af1_layer_device_bytes(const af1_layer* layer, int64_t* sign_bytes, int64_t* scale_bytes);
 
 /* Bytes of workspace one af1_linear_forward call with `tokens` rows needs
