@@ -53,16 +53,60 @@ def parse():
     p.add_argument("--schedule", choices=["dag", "serial"], default="dag",
                    help="dag: a decoder layer's independent linears (q/k/v, gate/up) on parallel streams; "
                         "serial: all 7 linears chained on one stream")
+    p.add_argument("--no-sweep", action="store_true",
+                   help="skip the per-shape sweep (LLaMA-3-8B at 1/4/16 tokens, 70B shapes at 1/8/64/512)")
+    p.add_argument("--no-stack", action="store_true", help="skip the 32-layer stack with HiSA-like ranks")
     return p.parse_args()
 
 
-def shapes():
+def shapes(rank_fn=None):
+    """The seven LLaMA-3-8B decoder linears at their exact 1.0-BPW ranks.
+    rank_fn defaults to the library's rank rule; the oracle legs pass the
+    oracle's."""
     import synth
-    from oracle import af1_oracle as O  # exact rank rule, host-side bookkeeping only
-    out = []
-    for name, m, n in synth.LLAMA3_8B_LINEARS:
-        out.append((name, m, n, O.rank_for_budget(m, n, 1)))
-    return out
+    if rank_fn is None:
+        import paper_2609_06161_gb300 as P
+        rank_fn = P.rank_for_budget
+    return [(name, m, n, int(rank_fn(m, n))) for name, m, n in synth.LLAMA3_8B_LINEARS]
+
+
+def oracle_shapes():
+    from oracle import af1_oracle as O
+    return shapes(lambda m, n: O.rank_for_budget(m, n, 1))
+
+
+def hisa_ranks(mn, seed=3):
+    """HiSA-like rank allocation over the matrices `mn` = [(m, n), ...]: each
+    1.0-BPW rank scaled by a seeded factor in [0.7, 1.3], then renormalised
+    so that the total storage stays within 1.0 bit per weight: one common
+    factor, floor, then +1 steps in a seeded order while the budget holds
+    (slack below one rank step)."""
+    import math
+    import synth
+    import paper_2609_06161_gb300 as P
+    base = [P.rank_for_budget(m, n) for (m, n) in mn]
+    f, order = synth.hisa_rank_factors(seed, len(mn))
+    drawn = [max(1, int(round(b * fi))) for b, fi in zip(base, f)]
+    budget = sum(m * n for (m, n) in mn)
+    fixed = sum(P.storage_bits(m, n, 1) - (m + n + 16) for (m, n) in mn)  # 16 (m + n) per matrix
+    per = sum(r * (m + n + 16) for r, (m, n) in zip(drawn, mn))
+    c = (budget - fixed) / per
+    ranks = [max(1, math.floor(c * r)) for r in drawn]
+    total = sum(P.storage_bits(m, n, r) for r, (m, n) in zip(ranks, mn))
+    while total > budget:  # floor of a positive factor cannot overshoot; kept as a guard
+        i = max(range(len(ranks)), key=lambda j: ranks[j])
+        total -= mn[i][0] + mn[i][1] + 16
+        ranks[i] -= 1
+    grew = True
+    while grew:
+        grew = False
+        for i in order:
+            step = mn[i][0] + mn[i][1] + 16
+            if total + step <= budget:
+                ranks[i] += 1
+                total += step
+                grew = True
+    return ranks
 
 
 def algorithmic_bytes(m, n, r, b):
@@ -85,7 +129,7 @@ def oracle_layer_sample(batch, seed_base=0):
     """The 7 linears of one decoder layer, as canonical packed words."""
     import synth
     data = []
-    for i, (name, m, n, r) in enumerate(shapes()):
+    for i, (name, m, n, r) in enumerate(oracle_shapes()):
         d = synth.layer_words(seed_base + i, m, n, r, batch)
         data.append((name, m, n, r, d))
     return data
@@ -225,6 +269,147 @@ def build_layers(P, torch, layers, batch, rank, outlier_frac=0.0):
             x = f16(d["x"]).reshape(batch, n)
             objs.append((name, m, n, r, layer, x))
     return objs
+
+
+L2_BYTES = 129e6  # GB300 L2; per-shape timings rotate over copies totalling >= 2x this
+
+
+def device_layer(P, torch, m, n, r, seed, any_rank=False):
+    """A layer with seeded random sign words drawn on the device (fast at
+    full size; padding bits are cleared by the library's re-layout) and the
+    synthetic FP16 scales of synth."""
+    import synth
+    g = torch.Generator(device="cuda")
+    g.manual_seed(seed)
+    wu, wv = P.words_per_row(r), P.words_per_row(n)
+    Uw = torch.randint(-2**31, 2**31 - 1, (m, wu), generator=g, device="cuda", dtype=torch.int64).to(torch.int32)
+    Vw = torch.randint(-2**31, 2**31 - 1, (r, wv), generator=g, device="cuda", dtype=torch.int64).to(torch.int32)
+    rs = synth.rng(seed)
+    f16 = lambda bits: torch.from_numpy(np.ascontiguousarray(bits).view(np.float16)).cuda()
+    a, s_, b = f16(synth.scales_f16(rs, m)), f16(synth.scales_f16(rs, r)), f16(synth.scales_f16(rs, n))
+    layer = P.Layer.from_words(Uw, Vw, a, s_, b, m, n, r, any_rank=any_rank)
+    del Uw, Vw
+    return layer
+
+
+def time_graph(torch, fn, stream, reps):
+    """ms per call of fn() replayed as a CUDA graph (3 warm-up replays)."""
+    with torch.cuda.stream(stream):
+        fn()
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        fn()
+    for _ in range(3):
+        g.replay()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    with torch.cuda.stream(stream):
+        for _ in range(reps):
+            g.replay()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    del g
+    return e0.elapsed_time(e1) / reps
+
+
+def sweep(P, torch, peaks, stream):
+    """Per-shape timings: every LLaMA-3-8B shape at 1, 4 and 16 tokens and the
+    70B-class shapes at 1 and 8 tokens (decode path, HBM roofline) and at 64
+    and 512 tokens (prefill path, tensor roofline); each against dense BF16
+    torch.matmul of the same shape. Calls rotate over copies of the layer
+    totalling at least twice the L2, so every call streams its weights from
+    HBM."""
+    import math
+    import synth
+    hbm = peaks.get("hbm_gbs", 6800.0)
+    tpk = peaks.get("bf16_tflops_sustained", 1700.0)
+    plan = [("q/o", 4096, 4096, (1, 4, 16)), ("k/v", 1024, 4096, (1, 4, 16)),
+            ("gate/up", 14336, 4096, (1, 4, 16)), ("down", 4096, 14336, (1, 4, 16))]
+    plan += [(f"70b {m}x{n}", m, n, (1, 8, 64, 512)) for (m, n) in synth.LLAMA_70B_SHAPES]
+    out = []
+    for si, (name, m, n, batches) in enumerate(plan):
+        r = P.rank_for_budget(m, n)
+        packed = r * (m + n) // 8 + 2 * (m + n + r)
+        copies = max(2, min(128, math.ceil(2 * L2_BYTES / packed)))
+        layers = [device_layer(P, torch, m, n, r, 7000 + 100 * si + c) for c in range(copies)]
+        dense_copies = max(2, math.ceil(2 * L2_BYTES / (2 * m * n)))
+        gd = torch.Generator(device="cuda")
+        gd.manual_seed(8000 + si)
+        dense = [torch.randn((m, n), generator=gd, device="cuda", dtype=torch.bfloat16) * 0.02
+                 for _ in range(dense_copies)]
+        for b in batches:
+            gx = torch.Generator(device="cuda")
+            gx.manual_seed(9000 + b)
+            x = torch.randn((b, n), generator=gx, device="cuda", dtype=torch.float16)
+            y = torch.empty((b, m), device="cuda", dtype=torch.float16)
+            ws = torch.zeros(layers[0].workspace_bytes(b), dtype=torch.uint8, device="cuda")
+
+            def run():
+                for L in layers:
+                    L.forward_into(x, y, ws, stream=stream)
+            reps = 5 if b <= 16 else 2
+            us = time_graph(torch, run, stream, reps) * 1e3 / copies
+            xb = x.to(torch.bfloat16)
+
+            def run_dense():
+                for W in dense:
+                    torch.matmul(xb, W.t())
+            us_dense = time_graph(torch, run_dense, stream, reps) * 1e3 / dense_copies
+            e = {"shape": name, "m": m, "n": n, "r": r, "tokens": b, "us_per_call": us,
+                 "tokens_per_s": b / (us * 1e-6), "copies": copies, "dense_bf16_us": us_dense,
+                 "speedup_vs_dense_bf16": us_dense / us}
+            if b <= 16:
+                alg = algorithmic_bytes(m, n, r, b)
+                e.update({"path": "decode", "bound": "hbm", "algorithmic_bytes": alg,
+                          "achieved_gbs": alg / (us * 1e-6) / 1e9, "frac": alg / (us * 1e-6) / 1e9 / hbm})
+            else:
+                fl = 2 * b * r * (m + n)
+                e.update({"path": "prefill", "bound": "tensor", "flops": fl,
+                          "achieved_tflops": fl / (us * 1e-6) / 1e12, "frac": fl / (us * 1e-6) / 1e12 / tpk})
+            out.append(e)
+            del ws, x, y, xb
+        for L in layers:
+            L.free()
+        del layers, dense
+        torch.cuda.empty_cache()
+    return out
+
+
+def stack_hisa(P, torch, peaks, stream, steps, dense_ms=None):
+    """32-layer LLaMA-3-8B stack with HiSA-like per-matrix ranks (+-30 %
+    around the 1.0-BPW rank, renormalised to 1.0 BPW over the stack), one
+    decode token per step, all 224 linears chained on one stream as a CUDA
+    graph."""
+    import synth
+    mn = [(m, n) for _ in range(LAYERS) for (_nm, m, n) in synth.LLAMA3_8B_LINEARS]
+    ranks = hisa_ranks(mn)
+    layers = [device_layer(P, torch, m, n, r, 20000 + i, any_rank=True) for i, ((m, n), r) in enumerate(zip(mn, ranks))]
+    gx = torch.Generator(device="cuda")
+    gx.manual_seed(31)
+    xs = [torch.randn((1, n), generator=gx, device="cuda", dtype=torch.float16) for (m, n) in mn]
+    ys = [torch.empty((1, m), device="cuda", dtype=torch.float16) for (m, n) in mn]
+    ws = torch.zeros(max(L.workspace_bytes(1) for L in layers), dtype=torch.uint8, device="cuda")
+
+    def run():
+        for L, x, y in zip(layers, xs, ys):
+            L.forward_into(x, y, ws, stream=stream)
+    ms = time_graph(torch, run, stream, max(5, min(steps, 20)))
+    alg = sum(algorithmic_bytes(m, n, r, 1) for (m, n), r in zip(mn, ranks))
+    bits = sum(P.storage_bits(m, n, r) for (m, n), r in zip(mn, ranks))
+    out = {"workload": "32 x 7 LLaMA-3-8B linears, HiSA-like ranks (+-30 %, renormalised), 1 token, one stream",
+           "ms_per_token": ms, "tokens_per_s": 1e3 / ms, "us_per_linear": ms * 1e3 / len(mn),
+           "bpw": bits / sum(m * n for (m, n) in mn), "rank_min": min(ranks), "rank_max": max(ranks),
+           "achieved_gbs": alg / (ms * 1e-3) / 1e9, "frac": alg / (ms * 1e-3) / 1e9 / peaks.get("hbm_gbs", 6800.0)}
+    if dense_ms is not None:
+        out["dense_bf16_ms_per_token"] = dense_ms
+        out["speedup_vs_dense_bf16"] = dense_ms / ms
+    for L in layers:
+        L.free()
+    del layers, xs, ys, ws
+    torch.cuda.empty_cache()
+    return out
 
 
 def main():
@@ -405,9 +590,17 @@ def main():
     dense = None
     if not args.no_dense and rank == 0:
         dense = dense_bf16(torch, objs, b, args, stream)
+    peaks = load_peaks()
+    sweep_rows = stack = None
+    if args.workload == "decode" and rank == 0:
+        # Extra measurements, outside the timed region of the headline number.
+        if not args.no_stack:
+            stack = stack_hisa(P, torch, peaks, stream, args.steps,
+                               dense_ms=dense["ms_per_step"] if dense and b == 1 else None)
+        if not args.no_sweep:
+            sweep_rows = sweep(P, torch, peaks, stream)
 
     if rank == 0:
-        peaks = load_peaks()
         hbm = peaks.get("hbm_gbs")
         if args.workload == "prefill":
             flops = sum(2 * b * r * (m + n) for (name, m, n, r, layer, x) in objs)
@@ -440,6 +633,10 @@ def main():
             line["dense_bf16_baseline"] = dense
         if serial is not None:
             line["serial_chain"] = serial
+        if stack is not None:
+            line["stack_hisa"] = stack
+        if sweep_rows is not None:
+            line["sweep"] = sweep_rows
         if not args.no_cpu and world == 1 and args.workload == "decode":
             line["cpu_baseline"] = cpu_baseline(b)
         if args.workload == "prefill":

@@ -93,6 +93,13 @@ typedef struct af1_layer af1_layer; /* opaque, owns its device buffers */
 AF1_API int af1_rank_for_budget(int64_t m, int64_t n, int64_t budget_num, int64_t budget_den,
                         int64_t* r_out);
 
+/* Bits one layer stores (App. "Effective Bit-Width", Eq. app_af1_memory):
+ * r(m + n) sign bits plus 16 bits per FP16 scale, m + r + n of them. This is
+ * the count the 1.0-BPW budget caps; a rank allocation over several layers
+ * (HiSA) sums it. Host-only. Errors: INVALID_ARG for m, n, r <= 0, m or n
+ * above 2^31, r above 2^31, or bits_out NULL. */
+AF1_API int af1_storage_bits(int64_t m, int64_t n, int64_t r, int64_t* bits_out);
+
 /* Build a layer from sign matrices (the factors NABF produces, Sec. 3.1).
  *   U:   int8 [m x r] row-major, entries exactly +1 or -1
  *   V:   int8 [n x r] row-major (V = B_pm1^T), entries exactly +1 or -1

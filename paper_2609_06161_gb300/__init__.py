@@ -52,6 +52,8 @@ _vp = ctypes.c_void_p
 _i64 = ctypes.c_int64
 _lib.af1_rank_for_budget.argtypes = [_i64, _i64, _i64, _i64, ctypes.POINTER(_i64)]
 _lib.af1_rank_for_budget.restype = ctypes.c_int
+_lib.af1_storage_bits.argtypes = [_i64, _i64, _i64, ctypes.POINTER(_i64)]
+_lib.af1_storage_bits.restype = ctypes.c_int
 _lib.af1_pack_layer.argtypes = [ctypes.POINTER(_Desc), _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
                                 ctypes.POINTER(_vp)]
 _lib.af1_pack_layer.restype = ctypes.c_int
@@ -106,6 +108,13 @@ def rank_for_budget(m: int, n: int, num: int = 1, den: int = 1) -> int:
     r = _i64(0)
     _check(_lib.af1_rank_for_budget(m, n, num, den, ctypes.byref(r)))
     return r.value
+
+
+def storage_bits(m: int, n: int, r: int) -> int:
+    """Bits one layer stores: r(m+n) signs plus m + r + n FP16 scales."""
+    b = _i64(0)
+    _check(_lib.af1_storage_bits(m, n, r, ctypes.byref(b)))
+    return b.value
 
 
 def _stream_handle(stream) -> int:

@@ -168,6 +168,15 @@ int af1_rank_for_budget(int64_t m, int64_t n, int64_t budget_num, int64_t budget
   return rank_rule(m, n, budget_num, budget_den, r_out);
 }
 
+int af1_storage_bits(int64_t m, int64_t n, int64_t r, int64_t* bits_out) {
+  if (m <= 0 || n <= 0 || r <= 0 || bits_out == nullptr)
+    return fail(AF1_ERR_INVALID_ARG, "af1_storage_bits: m, n, r must be > 0 and bits_out non-NULL");
+  if (m > (int64_t)1 << 31 || n > (int64_t)1 << 31 || r > (int64_t)1 << 31)
+    return fail(AF1_ERR_INVALID_ARG, "af1_storage_bits: arguments out of range");
+  *bits_out = r * (m + n) + 16 * (m + r + n);
+  return AF1_OK;
+}
+
 int af1_pack_layer(const af1_layer_desc* desc, const int8_t* U, const int8_t* V, const uint16_t* a,
                    const uint16_t* s, const uint16_t* b, uint32_t* out_U, uint32_t* out_V, void* stream,
                    af1_layer** out) {

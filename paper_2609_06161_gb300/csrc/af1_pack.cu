@@ -58,7 +58,10 @@ __global__ void words_to_blocks_kernel(const uint32_t* __restrict__ words, int64
   if (row < sm.R) {
     const uint32_t src = words[row * wpr + kw];
 #pragma unroll
-    for (int b = 0; b < 32; ++b) v |= ((src >> bit_col(b)) & 1u) << b;
+    for (int b = 0; b < 32; ++b) {
+      const int col = bit_col(b);
+      if (32 * kw + col < sm.C) v |= ((src >> col) & 1u) << b;  // padding columns stay 0
+    }
   }
   out[t] = v;
 }

@@ -111,3 +111,13 @@ def integer_layer(seed: int, d_out: int, d_in: int, r: int, tokens: int, xmax: i
     b = np.full(d_in, one, dtype=np.uint16)
     x = g.integers(-xmax, xmax + 1, size=(tokens, d_in)).astype(np.float16).view(np.uint16)
     return dict(U=U, V=V, a=a, s=s, b=b, x=x)
+
+
+def hisa_rank_factors(seed: int, count: int) -> np.ndarray:
+    """Per-matrix rank factors for a HiSA-like allocation over `count`
+    matrices: i.i.d. uniform in [0.7, 1.3] (the +-30 % spread around the
+    1.0-BPW rank), plus a seeded visiting order for the final +1 steps of the
+    renormalisation. Random numbers only; the budget arithmetic is the
+    caller's."""
+    g = rng(seed)
+    return g.uniform(0.7, 1.3, size=count), g.permutation(count)

@@ -52,6 +52,35 @@ def test_rank_rule_matches_oracle():
             assert P.rank_for_budget(m, n, num, den) == O.rank_for_budget(m, n, Fraction(num, den)), (m, n, num, den)
 
 
+def test_storage_bits_matches_oracle():
+    _ensure_built()
+    import paper_2609_06161_gb300 as P
+    from oracle import af1_oracle as O
+    for (m, n, r) in [(4096, 4096, 2028), (1024, 4096, 800), (28672, 8192, 6352), (7, 9, 3), (1, 1, 1)]:
+        assert P.storage_bits(m, n, r) == O.storage_bits(m, n, r), (m, n, r)
+    with pytest.raises(P.AF1Error):
+        P.storage_bits(4, 4, 0)
+
+
+def test_hisa_allocation_respects_budget():
+    # bench.hisa_ranks: +-30 % draws renormalised so that the stack stays at
+    # (not above) 1.0 BPW, with less than one rank step of slack.
+    _ensure_built()
+    import bench
+    from oracle import af1_oracle as O
+    import synth
+    shapes = [(m, n) for (_nm, m, n) in synth.LLAMA3_8B_LINEARS] * 4
+    ranks = bench.hisa_ranks(shapes, seed=3)
+    mats = [(m, n, r) for (m, n), r in zip(shapes, ranks)]
+    budget = sum(m * n for (m, n) in shapes)
+    total = sum(O.storage_bits(m, n, r) for (m, n, r) in mats)
+    assert total <= budget
+    assert all(total + (m + n + 16) > budget for (m, n, _r) in mats)
+    base = [O.rank_for_budget(m, n, 1) for (m, n) in shapes]
+    assert any(r != b for r, b in zip(ranks, base))
+    assert all(0.6 * b <= r <= 1.4 * b for r, b in zip(ranks, base))
+
+
 def test_host_validation_errors():
     _ensure_built()
     import paper_2609_06161_gb300 as P
