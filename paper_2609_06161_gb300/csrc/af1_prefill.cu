@@ -5,18 +5,22 @@
 //   GEMM1: H[t][k] = s_k * sum_j B[k][j] * (b_j x[t][j])    (B = V^T, r x n)
 //   GEMM2: y[t][i] = a_i * sum_k U[i][k] * H[t][k]          (U, m x r)
 //
-// A CTA computes D = A . B^T for 128 features x 128 tokens, D in tensor
-// memory (128 lanes x 128 FP32 columns). Per K-stage of 64:
-//   * warp 0 copies the 128 x 64 FP16 activation tile with cp.async into the
-//     128-byte-swizzled K-major layout the MMA descriptor describes;
+// A CTA computes D = A . B^T for 128 features x BN tokens (BN = 64, 128 or
+// 256), D in tensor memory (128 lanes x BN FP32 columns). Per K-stage of 64:
+//   * one thread of warp 0 loads the BN x 64 FP16 activation tile with one
+//     TMA copy (cp.async.bulk.tensor, 128-byte swizzle, zero fill past the
+//     tokens / columns): the K-major layout the MMA descriptor describes;
 //   * warps 4-7 (one feature row per thread) expand the packed signs of the
 //     128 x 64 weight tile into FP16 (+-b_j for GEMM1, +-1 for GEMM2: exact)
-//     in the same layout;
-//   * warp 1 (one lane) issues four tcgen05.mma.kind::f16 (K = 16 each) and
-//     commits them to the stage's "empty" mbarrier.
+//     in the same layout; each thread loads the next stage's sign words (and
+//     column scales) while it expands the current one;
+//   * one thread of warp 1 issues four tcgen05.mma.kind::f16 (K = 16 each,
+//     N = BN) and commits them to the stage's "empty" mbarrier.
 // Warps 4-7 then read D back with tcgen05.ld (warp w owns TMEM lanes
 // 32 (w % 4) .. +31), apply the per-feature scale and store FP16 / FP32.
 // All mbarrier waits are bounded; a wait that gives up sets the status word.
+#include <cuda.h>
+#include <cudaTypedefs.h>
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -28,20 +32,25 @@ namespace af1 {
 namespace {
 
 constexpr int BM = 128;  // features per CTA (MMA M, TMEM lanes)
-constexpr int BN = 128;  // tokens per CTA (MMA N, TMEM columns)
 constexpr int BK = 64;   // K per stage: one 128-byte swizzle row of FP16
 constexpr int STAGES = 4;
 constexpr int kThreads = 256;
 constexpr int kTileA = BM * BK * 2;  // 16 KB
-constexpr int kTileB = BN * BK * 2;  // 16 KB
 constexpr long long kWaitCycles = 2000000000ll;
 constexpr unsigned kStatusTimeout = 1u;
+
+template <int BN>
+__host__ __device__ constexpr int tile_b_bytes() {
+  return BN * BK * 2;
+}
+template <int BN>
+__host__ __device__ constexpr int smem_bytes() {
+  return STAGES * (kTileA + tile_b_bytes<BN>()) + 1024 /* barriers */ + 1024 /* base alignment */;
+}
 
 struct PrefillArgs {
   const uint32_t* signs;  // packed signs, af1_layout.h row-block layout
   SignMatrix sm;          // R = features, C = K
-  const __half* act;      // B operand source: [tokens][ld_act] FP16
-  int64_t ld_act;
   int tokens;
   const __half* colscale;  // GEMM1: b (length C); GEMM2: nullptr (+-1)
   const __half* rowscale;  // GEMM1: s (length R); GEMM2: a
@@ -52,9 +61,9 @@ struct PrefillArgs {
 };
 
 struct __align__(8) PrefillBarriers {
-  uint64_t full_a[STAGES];
-  uint64_t full_b[STAGES];
-  uint64_t empty[STAGES];
+  uint64_t full_a[STAGES];  // the 4 expander warps have written the stage
+  uint64_t full_b[STAGES];  // the TMA tile has landed
+  uint64_t empty[STAGES];   // the stage's MMAs are done
   uint64_t done;
   uint32_t tmem_addr;
   uint32_t err;
@@ -69,6 +78,10 @@ __device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
 }
 __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+               : "memory");
 }
 __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   uint32_t done;
@@ -98,38 +111,36 @@ __device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wa
 
 __device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
 
-// 16-byte cp.async with zero fill beyond `src_bytes`.
-__device__ __forceinline__ void cp_async16(void* dst, const void* src, uint32_t src_bytes) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_u32(dst)), "l"(src), "r"(src_bytes)
-               : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() {
-  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+// 2-D TMA load of the box at (x = column, y = token) into shared memory,
+// completing on `bar` with the box's byte count.
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, int x, int y, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+          smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar))
+      : "memory");
 }
 
 // Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row groups
 // 1024 bytes apart (stride byte offset), descriptor version 1.
 __device__ __forceinline__ uint64_t smem_desc(uint32_t addr) {
   uint64_t d = 0;
-  d |= (uint64_t)((addr >> 4) & 0x3FFFu);        // start address
-  d |= (uint64_t)1u << 16;                      // leading byte offset (unused for this layout)
-  d |= (uint64_t)(1024u >> 4) << 32;            // stride byte offset
-  d |= (uint64_t)1u << 46;                      // version
-  d |= (uint64_t)2u << 61;                      // 128-byte swizzle
+  d |= (uint64_t)((addr >> 4) & 0x3FFFu);  // start address
+  d |= (uint64_t)1u << 16;                 // leading byte offset (unused for this layout)
+  d |= (uint64_t)(1024u >> 4) << 32;       // stride byte offset
+  d |= (uint64_t)1u << 46;                 // version
+  d |= (uint64_t)2u << 61;                 // 128-byte swizzle
   return d;
 }
 
-// Instruction descriptor, kind::f16: D F32, A and B F16, both K-major,
-// N = BN, M = BM.
-constexpr uint32_t kIdesc = (1u << 4) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
-
+// kind::f16: D F32, A and B F16, both K-major, M = 128, N = BN.
+template <int BN>
 __device__ __forceinline__ void mma_f16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, bool accumulate) {
+  constexpr uint32_t idesc = (1u << 4) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
   asm volatile(
       "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
       " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(d_tmem),
-      "l"(adesc), "l"(bdesc), "r"(kIdesc), "r"(accumulate ? 1u : 0u)
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate ? 1u : 0u)
       : "memory");
 }
 __device__ __forceinline__ void mma_commit(uint64_t* bar) {
@@ -148,8 +159,28 @@ __device__ __forceinline__ uint32_t signed_pair(uint32_t pair_bytes, int p, uint
   return v ^ (~sh & 0x80008000u);
 }
 
-template <bool GEMM1>
-__global__ void __launch_bounds__(kThreads, 1) prefill_kernel(const PrefillArgs a) {
+// Column scales of stage columns kc .. kc + 63 as 8 groups of 8 FP16
+// values, 0 beyond C.
+__device__ __forceinline__ void load_colscale(const __half* cs, int64_t kc, int64_t C, uint4 (&out)[8]) {
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    const int64_t k = kc + 8 * j;
+    if (k + 7 < C) {
+      out[j] = __ldg(reinterpret_cast<const uint4*>(cs + k));
+    } else {
+      const uint16_t* c16 = reinterpret_cast<const uint16_t*>(cs);
+      uint32_t e[8];
+#pragma unroll
+      for (int q = 0; q < 8; ++q) e[q] = k + q < C ? c16[k + q] : 0u;
+      out[j] = make_uint4(e[0] | (e[1] << 16), e[2] | (e[3] << 16), e[4] | (e[5] << 16), e[6] | (e[7] << 16));
+    }
+  }
+}
+
+template <bool GEMM1, int BN>
+__global__ void __launch_bounds__(kThreads, 1)
+    prefill_kernel(const __grid_constant__ CUtensorMap act_map, const PrefillArgs a) {
+  constexpr int kTileB = tile_b_bytes<BN>();
   extern __shared__ uint8_t smem_raw[];
   // 1024-byte alignment for the swizzled operand tiles.
   uint8_t* smem = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -172,6 +203,7 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_kernel(const PrefillArgs 
     mbar_init(&bar.done, 1);
     bar.err = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&act_map)) : "memory");
   }
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&bar.tmem_addr)),
@@ -185,42 +217,19 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_kernel(const PrefillArgs 
   const uint32_t tmem = bar.tmem_addr;
 
   griddep_launch_dependents();
-  griddep_wait();
 
   if (warp == 0) {
-    // ---- activation producer: cp.async into the swizzled B tiles -------
-    constexpr int LAG = 2;
-    for (int it = 0; it < nk; ++it) {
-      const int s = it % STAGES;
-      if (it >= STAGES) mbar_wait(&bar.empty[s], ((it / STAGES) & 1) ^ 1, &bar.err);
-      uint8_t* dst = tileB + s * kTileB;
-      const int64_t k0 = (int64_t)it * BK;
-      for (int q = lane; q < BN * 8; q += 32) {
-        const int r = q >> 3, j = q & 7;
-        const int64_t tok = t0 + r;
-        const int64_t k = k0 + j * 8;
-        uint32_t bytes = 0;
-        const __half* src = a.act;
-        if (tok < a.tokens && k < tm.C) {
-          const int64_t left = tm.C - k;
-          bytes = left >= 8 ? 16u : (uint32_t)(left * 2);
-          src = a.act + tok * a.ld_act + k;
-        }
-        cp_async16(dst + swz(r, j), src, bytes);
-      }
-      cp_async_commit();
-      if (it >= LAG) {
-        cp_async_wait<LAG>();
-        fence_proxy_async();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&bar.full_b[(it - LAG) % STAGES]);
+    // ---- activation producer: one TMA copy per stage ---------------------
+    griddep_wait();  // the activations are written by the previous kernel
+    if (lane == 0) {
+      for (int it = 0; it < nk; ++it) {
+        const int s = it % STAGES;
+        if (it >= STAGES) mbar_wait(&bar.empty[s], ((it / STAGES) & 1) ^ 1, &bar.err);
+        mbar_expect_tx(&bar.full_b[s], (uint32_t)kTileB);
+        tma_load_2d(tileB + s * kTileB, &act_map, it * BK, t0, &bar.full_b[s]);
       }
     }
-    cp_async_wait<0>();
-    fence_proxy_async();
     __syncwarp();
-    if (lane == 0)
-      for (int it = nk - LAG < 0 ? 0 : nk - LAG; it < nk; ++it) mbar_arrive(&bar.full_b[it % STAGES]);
   } else if (warp == 1) {
     // ---- MMA issuer ---------------------------------------------------------
     if (lane == 0) {
@@ -233,7 +242,8 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_kernel(const PrefillArgs 
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 #pragma unroll
         for (int kk = 0; kk < BK / 16; ++kk) {
-          mma_f16(tmem, smem_desc(a0 + s * kTileA + kk * 32), smem_desc(b0 + s * kTileB + kk * 32), it > 0 || kk > 0);
+          mma_f16<BN>(tmem, smem_desc(a0 + s * kTileA + kk * 32), smem_desc(b0 + s * kTileB + kk * 32),
+                      it > 0 || kk > 0);
         }
         mma_commit(&bar.empty[s]);
       }
@@ -246,16 +256,27 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_kernel(const PrefillArgs 
     const int64_t frow = f0 + R;
     const bool row_ok = frow < tm.R;
     // Words of this row: index (rb * 4 NCH + kw) * 128 + R (rows past R are
-    // zero words of the padded block).
+    // zero words of the padded block). Stage `it` uses words 2 it and
+    // 2 it + 1; the next stage's words are loaded while the current stage is
+    // expanded.
     const uint32_t* rowp = a.signs + (int64_t)blockIdx.x * tm.NCH * kChunkWords * kBlockRows + R;
+    uint32_t w0 = __ldg(rowp), w1 = __ldg(rowp + kBlockRows);
+    uint4 cs[8];
+    if (GEMM1) load_colscale(a.colscale, 0, tm.C, cs);
     for (int it = 0; it < nk; ++it) {
       const int s = it % STAGES;
-      if (it >= STAGES) mbar_wait(&bar.empty[s], ((it / STAGES) & 1) ^ 1, &bar.err);
-      // Stage columns 64 it .. 64 it + 63 = words 2 it and 2 it + 1.
-      const uint32_t w0 = __ldg(rowp + (int64_t)(2 * it) * kBlockRows);
-      const uint32_t w1 = __ldg(rowp + (int64_t)(2 * it + 1) * kBlockRows);
+      uint32_t n0 = 0u, n1 = 0u;
+      uint4 ncs[8];
+      if (it + 1 < nk) {
+        n0 = __ldg(rowp + (int64_t)(2 * it + 2) * kBlockRows);
+        n1 = __ldg(rowp + (int64_t)(2 * it + 3) * kBlockRows);
+        if (GEMM1) load_colscale(a.colscale, (int64_t)(it + 1) * BK, tm.C, ncs);
+      }
+      if (it >= STAGES) {
+        if (lane == 0) mbar_wait(&bar.empty[s], ((it / STAGES) & 1) ^ 1, &bar.err);
+        __syncwarp();
+      }
       uint8_t* dst = tileA + s * kTileA;
-      const int64_t k0 = (int64_t)it * BK;
 #pragma unroll
       for (int j = 0; j < 8; ++j) {
         // 16-byte chunk j = stage columns 8j .. 8j+7 = columns 4p + e of word
@@ -264,39 +285,30 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_kernel(const PrefillArgs 
         const int p = 2 * (j & 3);
         const uint32_t b01 = __byte_perm(wd, 0u, 0x1404);  // bytes 0,1 -> bytes 1,3 (e = 0, 1)
         const uint32_t b23 = __byte_perm(wd, 0u, 0x3424);  // bytes 2,3 -> bytes 1,3 (e = 2, 3)
-        uint32_t sv[4] = {0x3C003C00u, 0x3C003C00u, 0x3C003C00u, 0x3C003C00u};  // +-1 for GEMM2
-        if (GEMM1) {
-          const int64_t kc = k0 + j * 8;
-          if (kc + 7 < tm.C) {
-            const uint4 bb = __ldg(reinterpret_cast<const uint4*>(a.colscale + kc));
-            sv[0] = bb.x;
-            sv[1] = bb.y;
-            sv[2] = bb.z;
-            sv[3] = bb.w;
-          } else {
-            const uint16_t* cs = reinterpret_cast<const uint16_t*>(a.colscale);
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-              const uint32_t e0 = kc + 2 * q < tm.C ? cs[kc + 2 * q] : 0u;
-              const uint32_t e1 = kc + 2 * q + 1 < tm.C ? cs[kc + 2 * q + 1] : 0u;
-              sv[q] = e0 | (e1 << 16);
-            }
-          }
-        }
+        uint4 sv = make_uint4(0x3C003C00u, 0x3C003C00u, 0x3C003C00u, 0x3C003C00u);  // +-1 for GEMM2
+        if (GEMM1) sv = cs[j];
         uint4 v;
-        v.x = signed_pair(b01, p, sv[0]);
-        v.y = signed_pair(b23, p, sv[1]);
-        v.z = signed_pair(b01, p + 1, sv[2]);
-        v.w = signed_pair(b23, p + 1, sv[3]);
+        v.x = signed_pair(b01, p, sv.x);
+        v.y = signed_pair(b23, p, sv.y);
+        v.z = signed_pair(b01, p + 1, sv.z);
+        v.w = signed_pair(b23, p + 1, sv.w);
         *reinterpret_cast<uint4*>(dst + swz(R, j)) = v;
       }
       fence_proxy_async();
       __syncwarp();
       if (lane == 0) mbar_arrive(&bar.full_a[s]);
+      w0 = n0;
+      w1 = n1;
+      if (GEMM1) {
+#pragma unroll
+        for (int j = 0; j < 8; ++j) cs[j] = ncs[j];
+      }
     }
     // ---- epilogue: TMEM -> registers -> global ---------------------------
-    mbar_wait(&bar.done, 0, &bar.err);
+    if (lane == 0) mbar_wait(&bar.done, 0, &bar.err);
+    __syncwarp();
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    griddep_wait();  // the output may still be read by the previous kernel until it completes
     const float rsc = row_ok ? __half2float(a.rowscale[frow]) : 0.f;
     const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
 #pragma unroll 1
@@ -326,31 +338,81 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_kernel(const PrefillArgs 
 
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
   __syncthreads();
-  if (bar.err != 0 && threadIdx.x == 0) atomicOr(a.status, kStatusTimeout);
+  if (bar.err != 0 && threadIdx.x == 0) {
+    // A wait gave up: let TMA copies that may still be in flight land
+    // (bounded) before the CTA exits, and report it.
+    for (int s = 0; s < STAGES; ++s) mbar_wait(&bar.full_b[s], 0, &bar.err);
+    atomicOr(a.status, kStatusTimeout);
+  }
   if (warp == 1) {
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"((uint32_t)BN) : "memory");
   }
 }
 
-constexpr int kSmemBytes = STAGES * (kTileA + kTileB) + (int)sizeof(PrefillBarriers) + 1024;
+// cuTensorMapEncodeTiled, looked up once through the runtime (no link
+// dependency on the driver library).
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static bool tried = false;
+  if (!tried) {
+    tried = true;
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
 
-template <bool GEMM1>
-cudaError_t launch_gemm(const PrefillArgs& a, cudaStream_t st) {
-  auto kern = prefill_kernel<GEMM1>;
-  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+// Tensor map of an FP16 [rows][ld] activation matrix with `cols` valid
+// columns: boxes of 64 columns x bn rows, 128-byte swizzle, zero fill
+// outside the matrix.
+cudaError_t make_act_map(CUtensorMap* map, const __half* base, int64_t rows, int64_t cols, int64_t ld, int bn) {
+  PFN_cuTensorMapEncodeTiled_v12000 fn = encode_fn();
+  if (fn == nullptr) return cudaErrorNotSupported;
+  cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)(ld * 2)};
+  cuuint32_t box[2] = {(cuuint32_t)BK, (cuuint32_t)bn};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<__half*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+template <bool GEMM1, int BN>
+cudaError_t launch_gemm_bn(const PrefillArgs& a, const __half* act, int64_t ld_act, cudaStream_t st) {
+  CUtensorMap map;
+  cudaError_t e = make_act_map(&map, act, a.tokens, a.sm.C, ld_act, BN);
+  if (e != cudaSuccess) return e;
+  auto kern = prefill_kernel<GEMM1, BN>;
+  constexpr int smem = smem_bytes<BN>();
+  e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)a.sm.RB, (unsigned)((a.tokens + BN - 1) / BN), 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
-  cfg.dynamicSmemBytes = kSmemBytes;
+  cfg.dynamicSmemBytes = smem;
   cfg.stream = st;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, kern, a);
+  return cudaLaunchKernelEx(&cfg, kern, map, a);
+}
+
+// Token tile: 256 when the pass has enough tokens to keep the GPU busy with
+// it, otherwise smaller tiles (more CTAs).
+template <bool GEMM1>
+cudaError_t launch_gemm(const PrefillArgs& a, const __half* act, int64_t ld_act, int num_sms, cudaStream_t st) {
+  const int64_t ctas256 = (int64_t)a.sm.RB * ((a.tokens + 255) / 256);
+  if (ctas256 >= num_sms / 2) return launch_gemm_bn<GEMM1, 256>(a, act, ld_act, st);
+  const int64_t ctas128 = (int64_t)a.sm.RB * ((a.tokens + 127) / 128);
+  if (ctas128 >= num_sms / 2) return launch_gemm_bn<GEMM1, 128>(a, act, ld_act, st);
+  return launch_gemm_bn<GEMM1, 64>(a, act, ld_act, st);
 }
 
 }  // namespace
@@ -366,8 +428,6 @@ cudaError_t launch_prefill(const af1_layer& L, const void* x, int64_t ldx, int64
     PrefillArgs g1 = {};
     g1.signs = reinterpret_cast<const uint32_t*>(L.signs1);
     g1.sm = L.p1;
-    g1.act = static_cast<const __half*>(x) + t0 * ldx;
-    g1.ld_act = ldx;
     g1.tokens = T;
     g1.colscale = reinterpret_cast<const __half*>(L.b);
     g1.rowscale = reinterpret_cast<const __half*>(L.s);
@@ -375,13 +435,11 @@ cudaError_t launch_prefill(const af1_layer& L, const void* x, int64_t ldx, int64
     g1.ld_out = ldh;
     g1.out_f32 = 0;
     g1.status = status;
-    cudaError_t e = launch_gemm<true>(g1, st);
+    cudaError_t e = launch_gemm<true>(g1, static_cast<const __half*>(x) + t0 * ldx, ldx, L.num_sms, st);
     if (e != cudaSuccess) return e;
     PrefillArgs g2 = {};
     g2.signs = reinterpret_cast<const uint32_t*>(L.signs2);
     g2.sm = L.p2;
-    g2.act = reinterpret_cast<const __half*>(h_buf);
-    g2.ld_act = ldh;
     g2.tokens = T;
     g2.colscale = nullptr;
     g2.rowscale = reinterpret_cast<const __half*>(L.a);
@@ -389,7 +447,7 @@ cudaError_t launch_prefill(const af1_layer& L, const void* x, int64_t ldx, int64
     g2.ld_out = ldy;
     g2.out_f32 = y_dtype == 0 ? 0 : 1;
     g2.status = status;
-    e = launch_gemm<false>(g2, st);
+    e = launch_gemm<false>(g2, reinterpret_cast<const __half*>(h_buf), ldh, L.num_sms, st);
     if (e != cudaSuccess) return e;
   }
   return cudaSuccess;
