@@ -1,0 +1,82 @@
+"""Rank-split over two processes (gloo, CPU): the host-side slicing of the
+packed factors and the all-reduce reproduce the unsplit layer. Each process
+evaluates its slice with the FP64 oracle, so the test needs no GPU."""
+import os
+import socket
+
+import numpy as np
+import pytest
+import torch
+import torch.distributed as dist
+import torch.multiprocessing as mp
+
+from oracle import af1_oracle as O
+import synth
+
+
+def _free_port():
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _load_rank_split():
+    # The module holds no compiled code; load it without the package's
+    # extension so the test also runs where the library is not built.
+    import importlib.util
+    here = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    spec = importlib.util.spec_from_file_location("rank_split", os.path.join(here, "paper_2609_06161_gb300", "rank_split.py"))
+    mod = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(mod)
+    return mod
+
+
+def test_rank_slices_cover_and_align():
+    rs = _load_rank_split()
+    for r in (1, 127, 128, 129, 800, 2028, 3167, 6352):
+        for world in (1, 2, 3, 4, 8):
+            sl = rs.rank_slices(r, world)
+            assert len(sl) == world
+            assert sl[0][0] == 0 and sl[-1][1] == r
+            for (a0, a1), (b0, b1) in zip(sl, sl[1:]):
+                assert a1 == b0
+            for r0, r1 in sl:
+                assert r0 <= r1 and (r0 == r1 or r0 % 128 == 0)
+
+
+def _worker(rank, world, port, shape, seed, result):
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    rs = _load_rank_split()
+    m, n, r, T = shape
+    d = synth.layer_words(seed, m, n, r, T)
+    Uw, Vw = torch.from_numpy(d["Uw"].view(np.int32)), torch.from_numpy(d["Vw"].view(np.int32))
+    s = torch.from_numpy(d["s"].view(np.int16))
+    r0, r1 = rs.rank_slices(r, world)[rank]
+    y = torch.zeros((T, m), dtype=torch.float64)
+    if r1 > r0:
+        Uw_g, Vw_g, s_g = rs.slice_packed(Uw, Vw, s, r0, r1)
+        y = torch.from_numpy(O.forward_from_packed(Uw_g.numpy().view(np.uint32), Vw_g.numpy().view(np.uint32),
+                                                   d["a"], s_g.numpy().view(np.uint16), d["b"], d["x"],
+                                                   m, n, r1 - r0))
+    dist.all_reduce(y, op=dist.ReduceOp.SUM)
+    if rank == 0:
+        ref = O.forward_from_packed(d["Uw"], d["Vw"], d["a"], d["s"], d["b"], d["x"], m, n, r)
+        result.put(float(np.max(np.abs(y.numpy() - ref)) / max(1e-300, float(np.max(np.abs(ref))))))
+    dist.destroy_process_group()
+
+
+@pytest.mark.parametrize("shape,world", [((96, 160, 300, 3), 2), ((64, 200, 129, 2), 2), ((40, 72, 100, 1), 2)])
+def test_rank_split_sum_matches_unsplit(shape, world):
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_worker, args=(g, world, port, shape, 11, q)) for g in range(world)]
+    for p in procs:
+        p.start()
+    for p in procs:
+        p.join(120)
+        assert p.exitcode == 0
+    err = q.get(timeout=10)
+    assert err < 1e-12, err
