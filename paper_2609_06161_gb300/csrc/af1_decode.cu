@@ -256,6 +256,7 @@ struct __align__(8) DecodeHeader {
   uint64_t wfull[kMaxCPC];  // packed chunk c has landed (bulk copy)
   uint64_t afull[8];        // A buffer holds its chunk (128 expander arrivals)
   uint64_t aempty[8];       // the MMAs that read an A buffer are done (NACC commits)
+  uint64_t xfull;           // staged activations have landed (bulk copies)
   uint64_t ddone;           // all MMAs done (NACC commits)
   uint64_t stats;           // per-token 2^-sigma and Q 2^-sigma are published
   uint32_t tmem_base, err;
@@ -264,19 +265,25 @@ struct __align__(8) DecodeHeader {
 };
 
 struct DecodeSmem {
-  int bt, w, recv, qpart, rs, hdr, total;  // byte offsets from the 1024-aligned base
+  int bt, w, act, recv, qpart, rs, hdr, total;  // byte offsets from the 1024-aligned base
 };
 
 __host__ __device__ inline int align128(int v) { return (v + 127) & ~127; }
 __host__ __device__ inline int slice_rows(int KS) { return (kBlockRows + KS - 1) / KS; }
 
-__host__ __device__ inline DecodeSmem decode_smem(int N, int CPC, int KS, int T) {
+// Passes of more than 4 tokens stage the CTA's activations in shared memory
+// with bulk copies (one per token row) before splitting them.
+__host__ __device__ inline bool staged_acts(int N) { return N > 16; }
+
+__host__ __device__ inline DecodeSmem decode_smem(int phase, int N, int CPC, int KS, int T) {
   DecodeSmem p;
   int off = 0;
   p.bt = off;
   off += N * 128 * CPC;  // B: chunk c at c N 128, 1024-aligned
   p.w = off;
   off += kChunkBytes * CPC;
+  p.act = off;  // T rows of CPC * 128 activations (FP16 phase 1, FP32 phase 2)
+  if (staged_acts(N)) off += T * CPC * kChunkCols * (phase == 1 ? 2 : 4);
   p.recv = off;
   off = align128(off + KS * T * slice_rows(KS) * 4);
   p.qpart = off;
@@ -330,8 +337,7 @@ __device__ __forceinline__ float4 load4(const DecodeArgs& a, int t, int64_t k) {
 
 // z'_k = z_k * colscale_k / d_p for the 4 columns k..k+3 (one bit position p).
 template <int PHASE>
-__device__ __forceinline__ float4 load_scaled4(const DecodeArgs& a, int t, int64_t k) {
-  float4 z = load4<PHASE>(a, t, k);
+__device__ __forceinline__ float4 scale4(const DecodeArgs& a, float4 z, int64_t k) {
   const float id = c_inv_delta[(k >> 2) & 7];
   if (PHASE == 1) {
     const int64_t C = a.sm.C;
@@ -354,6 +360,36 @@ __device__ __forceinline__ float4 load_scaled4(const DecodeArgs& a, int t, int64
   return make_float4(z.x * id, z.y * id, z.z * id, z.w * id);
 }
 
+// Four consecutive staged activations of token t at CTA column kl (zero at
+// and beyond kv, the CTA's valid columns).
+template <int PHASE>
+__device__ __forceinline__ float4 act4(const uint8_t* act, int rowlen, int t, int kl, int kv) {
+  float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (PHASE == 1) {
+    const __half* p = reinterpret_cast<const __half*>(act) + (size_t)t * rowlen + kl;
+    if (kl + 3 < kv) {
+      const uint2 raw = *reinterpret_cast<const uint2*>(p);
+      const float2 f0 = __half22float2(*reinterpret_cast<const __half2*>(&raw.x));
+      const float2 f1 = __half22float2(*reinterpret_cast<const __half2*>(&raw.y));
+      z = make_float4(f0.x, f0.y, f1.x, f1.y);
+    } else {
+      if (kl < kv) z.x = __half2float(p[0]);
+      if (kl + 1 < kv) z.y = __half2float(p[1]);
+      if (kl + 2 < kv) z.z = __half2float(p[2]);
+    }
+  } else {
+    const float* p = reinterpret_cast<const float*>(act) + (size_t)t * rowlen + kl;
+    if (kl + 3 < kv) {
+      z = *reinterpret_cast<const float4*>(p);
+    } else {
+      if (kl < kv) z.x = p[0];
+      if (kl + 1 < kv) z.y = p[1];
+      if (kl + 2 < kv) z.z = p[2];
+    }
+  }
+  return z;
+}
+
 template <int PHASE, int N>
 __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const DecodeArgs a) {
   constexpr int NACC = nacc_for(N);
@@ -365,7 +401,9 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const DecodeArgs a)
   uint8_t* smem = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   const int T = a.tokens;
   const int KS = a.KS;
-  const DecodeSmem sp = decode_smem(N, a.CPC, KS, T);
+  const DecodeSmem sp = decode_smem(PHASE, N, a.CPC, KS, T);
+  constexpr bool STAGED = N > 16;  // staged_acts(N)
+  uint8_t* act = smem + sp.act;
   uint8_t* Bt = smem + sp.bt;
   const uint32_t* W = reinterpret_cast<const uint32_t*>(smem + sp.w);
   float* recv = reinterpret_cast<float*>(smem + sp.recv);
@@ -391,6 +429,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const DecodeArgs a)
       mbar_init(&h.afull[b], 128);
       mbar_init(&h.aempty[b], NACC);
     }
+    mbar_init(&h.xfull, 1);
     mbar_init(&h.ddone, NACC);
     mbar_init(&h.stats, 16);
     h.err = 0;
@@ -452,6 +491,44 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const DecodeArgs a)
     const int ngroups = T * g4;
     for (int t = 0; t < T; ++t) qpart[t * 128 + bt] = 0.f;  // own column only
     griddep_wait();  // activations are written by the previous kernel
+    const int rowlen = a.CPC * kChunkCols;
+    const int kv = (int)min((int64_t)nch * kChunkCols, a.sm.C - k0);  // valid columns of this CTA
+    if (STAGED) {
+      // One bulk copy per token row of its 16-byte-multiple valid prefix; the
+      // few remaining columns with plain loads.
+      constexpr int ESZ = PHASE == 1 ? 2 : 4;
+      const int bulk_cols = ((kv * ESZ) & ~15) / ESZ;
+      if (bt == 0) {
+        const uint32_t bytes = (uint32_t)(bulk_cols * ESZ);
+        if (bytes > 0) {
+          mbar_expect_tx(&h.xfull, bytes * (uint32_t)T);
+          for (int t = 0; t < T; ++t) {
+            const uint8_t* src = PHASE == 1 ? reinterpret_cast<const uint8_t*>(a.x + (int64_t)t * a.ldx + k0)
+                                            : reinterpret_cast<const uint8_t*>(a.zin + (int64_t)t * a.ldz + k0);
+            bulk_g2s(act + (size_t)t * rowlen * ESZ, src, bytes, &h.xfull);
+          }
+        } else {
+          mbar_arrive(&h.xfull);
+        }
+      }
+      for (int i = bt; i < T * 8; i += 128) {
+        const int t = i >> 3, k = bulk_cols + (i & 7);
+        if (k < kv) {
+          if (PHASE == 1)
+            reinterpret_cast<__half*>(act)[(size_t)t * rowlen + k] = __ldcg(a.x + (int64_t)t * a.ldx + k0 + k);
+          else
+            reinterpret_cast<float*>(act)[(size_t)t * rowlen + k] = __ldcg(a.zin + (int64_t)t * a.ldz + k0 + k);
+        }
+      }
+      mbar_wait(&h.xfull, 0, &h.err);
+      builders_sync();  // tail values visible
+    }
+    // z' of group (t, c4): from the staged activations or straight from L2.
+    auto zq = [&](int t, int c4) -> float4 {
+      const int64_t k = k0 + 4 * c4;
+      const float4 z = STAGED ? act4<PHASE>(act, rowlen, t, 4 * c4, kv) : load4<PHASE>(a, t, k);
+      return scale4<PHASE>(a, z, k);
+    };
     float4 stash[STASH];
     // Pass 1: maxima of |z'| per token.
     {
@@ -461,7 +538,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const DecodeArgs a)
       for (int i = 0; i < STASH; ++i) stash[i] = make_float4(0.f, 0.f, 0.f, 0.f);
       for (int i = 0, g = bt; g < ngroups; ++i, g += 128) {
         const int t = g / g4, c4 = g - t * g4;
-        const float4 u = load_scaled4<PHASE>(a, t, k0 + 4 * c4);
+        const float4 u = zq(t, c4);
         if (i < STASH) {
 #pragma unroll
           for (int j = 0; j < STASH; ++j)
@@ -497,7 +574,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const DecodeArgs a)
           for (int j = 1; j < STASH; ++j)
             if (j == i) u = stash[j];
         } else {
-          u = load_scaled4<PHASE>(a, t, k0 + 4 * c4);
+          u = zq(t, c4);
         }
         float4 v = make_float4(u.x * sc, u.y * sc, u.z * sc, u.w * sc);
         const float4 v0 = v;
@@ -617,6 +694,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const DecodeArgs a)
     // Something timed out: let the bulk copies drain (bounded) so that none
     // lands after the CTA has exited, and report it.
     for (int c = 0; c < nch; ++c) mbar_wait(&h.wfull[c], 0, &h.err);
+    if (STAGED) mbar_wait(&h.xfull, 0, &h.err);
     atomicOr(a.status, kStatusTimeout);
   }
   if (warp == 4) {
@@ -642,7 +720,7 @@ int n_for_tokens(int T) { return T <= 4 ? 16 : T <= 8 ? 32 : 64; }
 // Split of one sign matrix for a pass of T tokens: about one CTA per SM
 // (row blocks x KS <= SMs), KS <= 16 CTAs per cluster, and the CTA's chunks
 // within the shared-memory budget.
-DecodePlan plan_decode(const SignMatrix& sm, int T, int num_sms, int max_smem) {
+DecodePlan plan_decode(int phase, const SignMatrix& sm, int T, int num_sms, int max_smem) {
   DecodePlan p;
   p.N = n_for_tokens(T);
   const int sms = num_sms > 0 ? num_sms : 148;
@@ -654,7 +732,7 @@ DecodePlan plan_decode(const SignMatrix& sm, int T, int num_sms, int max_smem) {
     const int cpc = (sm.NCH + ks - 1) / ks;
     if (cpc > kMaxCPC) continue;
     const int KS = (sm.NCH + cpc - 1) / cpc;
-    const int need = decode_smem(p.N, cpc, KS, T).total;
+    const int need = decode_smem(phase, p.N, cpc, KS, T).total;
     if (need <= max_smem) {
       p.KS = KS;
       p.CPC = cpc;
@@ -740,8 +818,8 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
   DecodePlan p1, p2;
   for (;;) {
     const int T = (int)(tokens < pass ? tokens : pass);
-    p1 = plan_decode(L.p1, T, L.num_sms, L.max_smem);
-    p2 = plan_decode(L.p2, T, L.num_sms, L.max_smem);
+    p1 = plan_decode(1, L.p1, T, L.num_sms, L.max_smem);
+    p2 = plan_decode(2, L.p2, T, L.num_sms, L.max_smem);
     if ((p1.ok && p2.ok) || pass <= 4) break;
     pass /= 2;
   }
@@ -749,8 +827,8 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
   const int ysize = y_dtype == 0 ? 2 : 4;
   for (int64_t t0 = 0; t0 < tokens; t0 += pass) {
     const int T = (int)((tokens - t0) < pass ? (tokens - t0) : pass);
-    const DecodePlan q1 = plan_decode(L.p1, T, L.num_sms, L.max_smem);
-    const DecodePlan q2 = plan_decode(L.p2, T, L.num_sms, L.max_smem);
+    const DecodePlan q1 = plan_decode(1, L.p1, T, L.num_sms, L.max_smem);
+    const DecodePlan q2 = plan_decode(2, L.p2, T, L.num_sms, L.max_smem);
     if (!q1.ok || !q2.ok) return cudaErrorInvalidConfiguration;
 
     DecodeArgs a1 = {};
