@@ -112,6 +112,25 @@ __device__ __forceinline__ void griddep_launch_dependents() {
 }
 __device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
+__device__ __forceinline__ void tmem_ld16(uint32_t addr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+        "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(addr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// Cluster helpers for the split-K reduction.
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void st_cluster_f32(float* local, uint32_t rank, float v) {
+  uint32_t remote;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(local)), "r"(rank));
+  asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(remote), "f"(v) : "memory");
+}
+
 // 2-D TMA load of the box at (x = column, y = token) into shared memory,
 // completing on `bar` with the box's byte count.
 __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, int x, int y, uint64_t* bar) {
@@ -180,7 +199,12 @@ __device__ __forceinline__ void load_colscale(const __half* cs, int64_t kc, int6
   }
 }
 
-template <bool GEMM1, int BN>
+// KS > 1: split-K over a cluster of KS CTAs along z. CTA ks runs the stages
+// [ks spk, (ks + 1) spk) and the partial tiles are summed through
+// distributed shared memory (each CTA finalises 128 / KS rows, summing the
+// KS partials in a fixed order), reusing the activation stages as the
+// receive buffer once every MMA of the cluster is done.
+template <bool GEMM1, int BN, int KS>
 __global__ void __launch_bounds__(kThreads, 1)
     prefill_kernel(const __grid_constant__ CUtensorMap act_map, const PrefillArgs a) {
   constexpr int kTileB = tile_b_bytes<BN>();
@@ -194,7 +218,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   const SignMatrix& tm = a.sm;
   const int f0 = blockIdx.x * BM;  // first feature (row of the sign matrix)
   const int t0 = blockIdx.y * BN;  // first token
-  const int nk = (int)((tm.C + BK - 1) / BK);
+  const int nk_all = (int)((tm.C + BK - 1) / BK);
+  const int ks = KS > 1 ? (int)blockIdx.z : 0;
+  const int spk = (nk_all + KS - 1) / KS;  // stages per CTA (>= 1 for every ks, by the host plan)
+  const int it0 = ks * spk;
+  const int nk = min(nk_all, it0 + spk) - it0;  // this CTA's stages: it0 .. it0 + nk - 1
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -228,7 +256,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int s = it % STAGES;
         if (it >= STAGES) mbar_wait(&bar.empty[s], ((it / STAGES) & 1) ^ 1, &bar.err);
         mbar_expect_tx(&bar.full_b[s], (uint32_t)kTileB);
-        tma_load_2d(tileB + s * kTileB, &act_map, it * BK, t0, &bar.full_b[s]);
+        tma_load_2d(tileB + s * kTileB, &act_map, (it0 + it) * BK, t0, &bar.full_b[s]);
       }
     }
     __syncwarp();
@@ -261,10 +289,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     // zero words of the padded block). Stage `it` uses words 2 it and
     // 2 it + 1; the next stage's words are loaded while the current stage is
     // expanded.
-    const uint32_t* rowp = a.signs + (int64_t)blockIdx.x * tm.NCH * kChunkWords * kBlockRows + R;
+    const uint32_t* rowp =
+        a.signs + (int64_t)blockIdx.x * tm.NCH * kChunkWords * kBlockRows + R + (int64_t)(2 * it0) * kBlockRows;
     uint32_t w0 = __ldg(rowp), w1 = __ldg(rowp + kBlockRows);
     uint4 cs[8];
-    if (GEMM1) load_colscale(a.colscale, 0, tm.C, cs);
+    if (GEMM1) load_colscale(a.colscale, (int64_t)it0 * BK, tm.C, cs);
     for (int it = 0; it < nk; ++it) {
       const int s = it % STAGES;
       uint32_t n0 = 0u, n1 = 0u;
@@ -272,7 +301,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (it + 1 < nk) {
         n0 = __ldg(rowp + (int64_t)(2 * it + 2) * kBlockRows);
         n1 = __ldg(rowp + (int64_t)(2 * it + 3) * kBlockRows);
-        if (GEMM1) load_colscale(a.colscale, (int64_t)(it + 1) * BK, tm.C, ncs);
+        if (GEMM1) load_colscale(a.colscale, (int64_t)(it0 + it + 1) * BK, tm.C, ncs);
       }
       if (it >= STAGES) {
         if (lane == 0) mbar_wait(&bar.empty[s], ((it / STAGES) & 1) ^ 1, &bar.err);
@@ -322,31 +351,68 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) mbar_wait(&bar.done, 0, &bar.err);
     __syncwarp();
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-    griddep_wait();  // the output may still be read by the previous kernel until it completes
-    const float rsc = row_ok ? __half2float(a.rowscale[frow]) : 0.f;
-    const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
+    if (KS == 1) {
+      griddep_wait();  // the output may still be read by the previous kernel until it completes
+      const float rsc = row_ok ? __half2float(a.rowscale[frow]) : 0.f;
+      const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
 #pragma unroll 1
-    for (int c0 = 0; c0 < BN; c0 += 16) {
-      uint32_t r[16];
-      asm volatile(
-          "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
-          : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-            "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-          : "r"(tmem + lane_base + (uint32_t)c0));
-      asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-      if (row_ok) {
+      for (int c0 = 0; c0 < BN; c0 += 16) {
+        uint32_t r[16];
+        tmem_ld16(tmem + lane_base + (uint32_t)c0, r);
+        if (row_ok) {
 #pragma unroll
-        for (int q = 0; q < 16; ++q) {
-          const int64_t tok = t0 + c0 + q;
-          if (tok < a.tokens) {
-            const float v = __uint_as_float(r[q]) * rsc;
-            if (a.out_f32)
-              reinterpret_cast<float*>(a.out)[tok * a.ld_out + frow] = v;
-            else
-              reinterpret_cast<__half*>(a.out)[tok * a.ld_out + frow] = __float2half_rn(v);
+          for (int q = 0; q < 16; ++q) {
+            const int64_t tok = t0 + c0 + q;
+            if (tok < a.tokens) {
+              const float v = __uint_as_float(r[q]) * rsc;
+              if (a.out_f32)
+                reinterpret_cast<float*>(a.out)[tok * a.ld_out + frow] = v;
+              else
+                reinterpret_cast<__half*>(a.out)[tok * a.ld_out + frow] = __float2half_rn(v);
+            }
           }
         }
       }
+    }
+  }
+
+  if (KS > 1) {
+    // ---- split-K: partial tiles -> owning CTA through distributed shared
+    //      memory. recv[q][i][c ^ (i & 31)] holds CTA q's partial of row i
+    //      of this CTA's slice (XOR on the column keeps the row-wise reads of
+    //      the final sum free of bank conflicts).
+    constexpr int SLICE = BM / KS;
+    float* recv = reinterpret_cast<float*>(tileB);  // KS * SLICE * BN floats = STAGES * kTileB bytes
+    __syncwarp();
+    cluster_sync();  // every MMA of the cluster is done: the activation stages are free
+    if (warp >= 4) {
+      const int R = threadIdx.x - 128;
+      const int owner = R / SLICE, i = R - owner * SLICE;
+      const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
+      float* row = recv + (size_t)(ks * SLICE + i) * BN;
+#pragma unroll 1
+      for (int c0 = 0; c0 < BN; c0 += 16) {
+        uint32_t r[16];
+        tmem_ld16(tmem + lane_base + (uint32_t)c0, r);
+#pragma unroll
+        for (int q = 0; q < 16; ++q) st_cluster_f32(row + ((c0 + q) ^ (i & 31)), (uint32_t)owner, __uint_as_float(r[q]));
+      }
+    }
+    cluster_sync();  // all partials have landed
+    griddep_wait();  // the output may still be read by the previous kernel until it completes
+    for (int idx = threadIdx.x; idx < SLICE * BN; idx += kThreads) {
+      const int c = idx / SLICE, i = idx - c * SLICE;  // token column c, slice row i
+      const int64_t frow = f0 + ks * SLICE + i;
+      const int64_t tok = t0 + c;
+      if (frow >= tm.R || tok >= a.tokens) continue;
+      float v = 0.f;
+#pragma unroll
+      for (int q = 0; q < KS; ++q) v += recv[(size_t)(q * SLICE + i) * BN + (c ^ (i & 31))];
+      v *= __half2float(a.rowscale[frow]);
+      if (a.out_f32)
+        reinterpret_cast<float*>(a.out)[tok * a.ld_out + frow] = v;
+      else
+        reinterpret_cast<__half*>(a.out)[tok * a.ld_out + frow] = __float2half_rn(v);
     }
   }
 
@@ -396,37 +462,60 @@ cudaError_t make_act_map(CUtensorMap* map, const __half* base, int64_t rows, int
   return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
-template <bool GEMM1, int BN>
+template <bool GEMM1, int BN, int KS>
 cudaError_t launch_gemm_bn(const PrefillArgs& a, const __half* act, int64_t ld_act, cudaStream_t st) {
   CUtensorMap map;
   cudaError_t e = make_act_map(&map, act, a.tokens, a.sm.C, ld_act, BN);
   if (e != cudaSuccess) return e;
-  auto kern = prefill_kernel<GEMM1, BN>;
-  constexpr int smem = smem_bytes<BN>();
+  auto kern = prefill_kernel<GEMM1, BN, KS>;
+  // A cluster's CTAs wait for each other while holding tensor memory, so no
+  // third CTA may share an SM with two of them (one that blocks in
+  // tcgen05.alloc would wait for a CTA that waits for it): with at least
+  // 80 KB of shared memory per CTA, at most two CTAs fit on an SM and their
+  // tensor memory (<= 256 columns each) always fits.
+  constexpr int smem = (KS > 1 && smem_bytes<BN>() < 80 * 1024) ? 80 * 1024 : smem_bytes<BN>();
   e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((unsigned)a.sm.RB, (unsigned)((a.tokens + BN - 1) / BN), 1);
+  cfg.gridDim = dim3((unsigned)a.sm.RB, (unsigned)((a.tokens + BN - 1) / BN), (unsigned)KS);
   cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = st;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = 1;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = (unsigned)KS;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = KS > 1 ? 2 : 1;
   return cudaLaunchKernelEx(&cfg, kern, map, a);
 }
 
-// Token tile: 256 when the pass has enough tokens to keep the GPU busy with
-// it, otherwise smaller tiles (more CTAs).
+// Tiling of one GEMM: the smallest token tile of 64 / 128 / 256 that covers
+// the pass, made smaller while the grid would leave half the SMs idle; with
+// tiles of 64, short passes (few row blocks x token tiles) split K over a
+// cluster of 2, 4 or 8 CTAs (every CTA keeps at least two K-stages).
 template <bool GEMM1>
 cudaError_t launch_gemm(const PrefillArgs& a, const __half* act, int64_t ld_act, int num_sms, cudaStream_t st) {
-  const int64_t ctas256 = (int64_t)a.sm.RB * ((a.tokens + 255) / 256);
-  if (ctas256 >= num_sms / 2) return launch_gemm_bn<GEMM1, 256>(a, act, ld_act, st);
-  const int64_t ctas128 = (int64_t)a.sm.RB * ((a.tokens + 127) / 128);
-  if (ctas128 >= num_sms / 2) return launch_gemm_bn<GEMM1, 128>(a, act, ld_act, st);
-  return launch_gemm_bn<GEMM1, 64>(a, act, ld_act, st);
+  const int64_t rb = a.sm.RB;
+  int bn = a.tokens > 128 ? 256 : a.tokens > 64 ? 128 : 64;
+  while (bn > 64 && rb * ((a.tokens + bn - 1) / bn) < num_sms / 2) bn /= 2;
+  if (bn == 256) return launch_gemm_bn<GEMM1, 256, 1>(a, act, ld_act, st);
+  if (bn == 128) return launch_gemm_bn<GEMM1, 128, 1>(a, act, ld_act, st);
+  const int64_t base = rb * ((a.tokens + 63) / 64);
+  const int nk = (int)((a.sm.C + BK - 1) / BK);
+  int ks = 1;
+  while (ks < 8 && base * ks * 2 <= num_sms && nk >= 4 * ks) ks *= 2;
+  // every CTA of the split needs at least one stage
+  while (ks > 1 && (ks - 1) * ((nk + ks - 1) / ks) >= nk) ks /= 2;
+  switch (ks) {
+    case 8: return launch_gemm_bn<GEMM1, 64, 8>(a, act, ld_act, st);
+    case 4: return launch_gemm_bn<GEMM1, 64, 4>(a, act, ld_act, st);
+    case 2: return launch_gemm_bn<GEMM1, 64, 2>(a, act, ld_act, st);
+    default: return launch_gemm_bn<GEMM1, 64, 1>(a, act, ld_act, st);
+  }
 }
 
 }  // namespace
