@@ -34,8 +34,8 @@
  * 4 words (16 bytes). With W(c) = 4 * ceil(c / 128):
  *   U words: m rows x W(r) words;  bit (k % 32) of word (k / 32) of row i = U[i][k]
  *   V words: r rows x W(n) words;  bit (j % 32) of word (j / 32) of row k = V[j][k]
- * Internally a layer keeps the signs in a tile layout of its own (same bit
- * count plus tile padding); the canonical words are the exchange format.
+ * Internally a layer keeps the signs in a row-block layout of its own (same
+ * bit count plus block padding); the canonical words are the exchange format.
  */
 #ifndef AF1_H
 #define AF1_H
@@ -163,9 +163,11 @@ AF1_API int af1_linear_forward(const af1_layer* layer, const void* x, int64_t ld
  * this is a deployment convenience.
  * Same arguments as af1_linear_forward minus the workspace: the scratch is a
  * 1 MiB array compiled into the library, present on every GPU that loads it
- * until the process exits. Nothing is allocated by this call. Layers whose
- * scratch need (af1_workspace_bytes) exceeds 1 MiB are rejected with
- * AF1_ERR_WORKSPACE; every shape with r <= 16256 fits.
+ * until the process exits. Nothing is allocated by this call. Calls whose
+ * scratch need (af1_workspace_bytes(layer, tokens)) exceeds 1 MiB are
+ * rejected with AF1_ERR_WORKSPACE: with up to 16 tokens every shape with
+ * r <= 16256 fits; longer calls also hold min(tokens, 2048) x r FP16 rank
+ * intermediates, so they fit only for short passes of small-rank layers.
  * The first call on a device looks up the array's device address (once per
  * device); make that first call before any stream capture. All calls share
  * the array and leave their intermediate results in it, so calls that may
