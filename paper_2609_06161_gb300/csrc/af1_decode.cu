@@ -717,9 +717,15 @@ struct DecodePlan {
 
 int n_for_tokens(int T) { return T <= 4 ? 16 : T <= 8 ? 32 : 64; }
 
+constexpr int kTwoPerSmSmem = 110 * 1024;  // at or below this, two CTAs share an SM
+
 // Split of one sign matrix for a pass of T tokens: about one CTA per SM
 // (row blocks x KS <= SMs), KS <= 16 CTAs per cluster, and the CTA's chunks
-// within the shared-memory budget.
+// within the shared-memory budget. The first finer split whose CTAs are
+// small enough for two per SM is taken when it lowers waves x chunks per CTA
+// (the streaming time of the slowest SM): two CTAs per SM overlap their
+// streaming of signs into tensor memory (measured: 28672x8192 at one token
+// 62.0 -> 42.1 us, 14336x4096 at 16 tokens 86.3 -> 57.0 us).
 DecodePlan plan_decode(int phase, const SignMatrix& sm, int T, int num_sms, int max_smem) {
   DecodePlan p;
   p.N = n_for_tokens(T);
@@ -728,6 +734,10 @@ DecodePlan plan_decode(int phase, const SignMatrix& sm, int T, int num_sms, int 
   if (ks < 1) ks = 1;
   if (ks > kMaxKS) ks = kMaxKS;
   if (ks > sm.NCH) ks = sm.NCH;
+  auto waves = [&](int KS, int need) {
+    const int64_t slots = (int64_t)sms * (need <= kTwoPerSmSmem ? 2 : 1);
+    return ((int64_t)sm.RB * KS + slots - 1) / slots;
+  };
   for (; ks <= kMaxKS; ++ks) {
     const int cpc = (sm.NCH + ks - 1) / ks;
     if (cpc > kMaxCPC) continue;
@@ -738,6 +748,21 @@ DecodePlan plan_decode(int phase, const SignMatrix& sm, int T, int num_sms, int 
       p.CPC = cpc;
       p.smem = need < kMinSmem ? kMinSmem : need;
       p.ok = true;
+      if (need > kTwoPerSmSmem) {
+        for (int k2 = ks + 1; k2 <= kMaxKS && k2 <= sm.NCH; ++k2) {
+          const int c2 = (sm.NCH + k2 - 1) / k2;
+          const int K2 = (sm.NCH + c2 - 1) / c2;
+          const int n2 = decode_smem(phase, p.N, c2, K2, T).total;
+          if (n2 <= kTwoPerSmSmem) {
+            if (waves(K2, n2) * c2 < waves(KS, need) * cpc) {
+              p.KS = K2;
+              p.CPC = c2;
+              p.smem = n2 < kMinSmem ? kMinSmem : n2;
+            }
+            break;
+          }
+        }
+      }
       return p;
     }
   }
