@@ -725,7 +725,10 @@ constexpr int kTwoPerSmSmem = 110 * 1024;  // at or below this, two CTAs share a
 // small enough for two per SM is taken when it lowers waves x chunks per CTA
 // (the streaming time of the slowest SM): two CTAs per SM overlap their
 // streaming of signs into tensor memory (measured: 28672x8192 at one token
-// 62.0 -> 42.1 us, 14336x4096 at 16 tokens 86.3 -> 57.0 us).
+// 62.0 -> 42.1 us, 14336x4096 at 16 tokens 86.3 -> 57.0 us). Then, while a
+// CTA streams more chunks than its A ring holds, K is split twice as finely
+// (portable clusters, at most two CTAs per SM; 14336x4096 at one token
+// 20.9 -> 15.2 us).
 DecodePlan plan_decode(int phase, const SignMatrix& sm, int T, int num_sms, int max_smem) {
   DecodePlan p;
   p.N = n_for_tokens(T);
@@ -762,6 +765,19 @@ DecodePlan plan_decode(int phase, const SignMatrix& sm, int T, int num_sms, int 
             break;
           }
         }
+      }
+      // CTAs that stream more chunks than their tensor-memory ring holds:
+      // split K further (portable clusters) while the CTA count stays within
+      // two per SM.
+      while (p.CPC > nbuf_for(p.N) && p.KS * 2 <= 8 && (int64_t)sm.RB * p.KS * 2 <= 2 * sms) {
+        const int k2 = p.KS * 2;
+        const int c2 = (sm.NCH + k2 - 1) / k2;
+        const int K2 = (sm.NCH + c2 - 1) / c2;
+        const int n2 = decode_smem(phase, p.N, c2, K2, T).total;
+        if (n2 > max_smem) break;
+        p.KS = K2;
+        p.CPC = c2;
+        p.smem = n2 < kMinSmem ? kMinSmem : n2;
       }
       return p;
     }
