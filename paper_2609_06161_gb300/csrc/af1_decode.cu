@@ -736,6 +736,12 @@ DecodePlan plan_decode(int phase, const SignMatrix& sm, int T, int num_sms, int 
   int ks = sms / (sm.RB > 0 ? sm.RB : 1);
   if (ks < 1) ks = 1;
   if (ks > kMaxKS) ks = kMaxKS;
+  // One-token calls are latency-bound and usually run beside their sibling
+  // linears (q | k | v): portable clusters of at most 8 leave SMs to them
+  // (config-1 stack on the DAG schedule 10.88 -> 10.37 us per linear; the
+  // k/v shape alone 8.49 -> 8.63 us), unless the CTAs would then stream more
+  // chunks than their A ring holds.
+  if (T == 1 && ks > 8 && (sm.NCH + 7) / 8 <= nbuf_for(p.N)) ks = 8;
   if (ks > sm.NCH) ks = sm.NCH;
   auto waves = [&](int KS, int need) {
     const int64_t slots = (int64_t)sms * (need <= kTwoPerSmSmem ? 2 : 1);
