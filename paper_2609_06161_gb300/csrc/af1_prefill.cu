@@ -37,7 +37,7 @@ namespace {
 
 constexpr int BM = 128;  // features per CTA (MMA M, TMEM lanes)
 constexpr int BK = 64;   // K per stage: one 128-byte swizzle row of FP16
-constexpr int STAGES = 4;
+constexpr int kMaxStages = 6;
 constexpr int kThreads = 256;
 constexpr long long kWaitCycles = 2000000000ll;
 constexpr unsigned kStatusTimeout = 1u;
@@ -46,9 +46,16 @@ template <int BN>
 __host__ __device__ constexpr int tile_b_bytes() {
   return BN * BK * 2;
 }
+// Pipeline depth: 6 stages for tiles of 256 tokens (192 KB of activation
+// tiles; tensor memory holds D in 256 columns plus an A ring of 6 x 32), 4
+// for the smaller tiles.
+template <int BN>
+__host__ __device__ constexpr int stages() {
+  return BN == 256 ? 6 : 4;
+}
 template <int BN>
 __host__ __device__ constexpr int smem_bytes() {
-  return STAGES * tile_b_bytes<BN>() + 1024 /* barriers */ + 1024 /* base alignment */;
+  return stages<BN>() * tile_b_bytes<BN>() + 1024 /* barriers */ + 1024 /* base alignment */;
 }
 
 struct PrefillArgs {
@@ -64,9 +71,9 @@ struct PrefillArgs {
 };
 
 struct __align__(8) PrefillBarriers {
-  uint64_t full_a[STAGES];  // the 4 expander warps have stored the stage's A
-  uint64_t full_b[STAGES];  // the TMA tile has landed
-  uint64_t empty[STAGES];   // the stage's MMAs are done
+  uint64_t full_a[kMaxStages];  // the 4 expander warps have stored the stage's A
+  uint64_t full_b[kMaxStages];  // the TMA tile has landed
+  uint64_t empty[kMaxStages];   // the stage's MMAs are done
   uint64_t done;
   uint32_t tmem_addr;
   uint32_t err;
@@ -163,11 +170,11 @@ __device__ __forceinline__ void mma_f16_ts(uint32_t d_tmem, uint32_t a_tmem, uin
       "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate ? 1u : 0u)
       : "memory");
 }
-// Tensor-memory columns: D (BN) then the A ring (STAGES x 32), rounded up
+// Tensor-memory columns: D (BN) then the A ring (stages x 32), rounded up
 // to a power of two.
 template <int BN>
 __host__ __device__ constexpr uint32_t tmem_cols() {
-  return (BN + STAGES * 32) <= 256 ? 256u : 512u;
+  return (BN + stages<BN>() * 32) <= 256 ? 256u : 512u;
 }
 __device__ __forceinline__ void mma_commit(uint64_t* bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
@@ -208,6 +215,7 @@ template <bool GEMM1, int BN, int KS>
 __global__ void __launch_bounds__(kThreads, 1)
     prefill_kernel(const __grid_constant__ CUtensorMap act_map, const PrefillArgs a) {
   constexpr int kTileB = tile_b_bytes<BN>();
+  constexpr int STAGES = stages<BN>();
   extern __shared__ uint8_t smem_raw[];
   // 1024-byte alignment for the swizzled operand tiles.
   uint8_t* smem = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -303,10 +311,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         n1 = __ldg(rowp + (int64_t)(2 * it + 3) * kBlockRows);
         if (GEMM1) load_colscale(a.colscale, (int64_t)(it0 + it + 1) * BK, tm.C, ncs);
       }
-      if (it >= STAGES) {
-        if (lane == 0) mbar_wait(&bar.empty[s], ((it / STAGES) & 1) ^ 1, &bar.err);
-        __syncwarp();
-      }
       uint32_t av[32];
 #pragma unroll
       for (int j = 0; j < 8; ++j) {
@@ -324,7 +328,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         av[4 * j + 2] = signed_pair(b01, p + 1, sv.z);
         av[4 * j + 3] = signed_pair(b23, p + 1, sv.w);
       }
-      if (it >= STAGES) asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+      // The previous stage's store was left in flight while this stage was
+      // expanded: complete it and hand that stage to the MMA issuer.
+      if (it > 0) {
+        asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+        asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bar.full_a[(it - 1) % STAGES]);
+      }
+      if (it >= STAGES) {
+        if (lane == 0) mbar_wait(&bar.empty[s], ((it / STAGES) & 1) ^ 1, &bar.err);
+        __syncwarp();
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+      }
       {
         const uint32_t addr = tmem + ((uint32_t)((warp & 3) * 32) << 16) + (uint32_t)(BN + s * 32);
         asm volatile(
@@ -335,17 +351,19 @@ __global__ void __launch_bounds__(kThreads, 1)
             "r"(av[16]), "r"(av[17]), "r"(av[18]), "r"(av[19]), "r"(av[20]), "r"(av[21]), "r"(av[22]), "r"(av[23]),
             "r"(av[24]), "r"(av[25]), "r"(av[26]), "r"(av[27]), "r"(av[28]), "r"(av[29]), "r"(av[30]), "r"(av[31])
             : "memory");
-        asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
       }
-      asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&bar.full_a[s]);
       w0 = n0;
       w1 = n1;
       if (GEMM1) {
 #pragma unroll
         for (int j = 0; j < 8; ++j) cs[j] = ncs[j];
       }
+    }
+    if (nk > 0) {
+      asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+      asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bar.full_a[(nk - 1) % STAGES]);
     }
     // ---- epilogue: TMEM -> registers -> global ---------------------------
     if (lane == 0) mbar_wait(&bar.done, 0, &bar.err);
