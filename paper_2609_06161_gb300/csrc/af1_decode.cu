@@ -830,6 +830,26 @@ cudaError_t launch_decode(DecodeArgs a, const DecodePlan& p, cudaStream_t st) {
 
 int64_t align256(int64_t v) { return (v + 255) / 256 * 256; }
 
+LutArgs lut_args(const DecodeArgs& d) {
+  LutArgs a = {};
+  a.signs = d.signs;
+  a.sm = d.sm;
+  a.tokens = d.tokens;
+  a.x = d.x;
+  a.ldx = d.ldx;
+  a.zin = d.zin;
+  a.ldz = d.ldz;
+  a.colscale = d.colscale;
+  a.rowscale = d.rowscale;
+  a.sout = d.sout;
+  a.lds = d.lds;
+  a.y = d.y;
+  a.ldy = d.ldy;
+  a.ydtype = d.ydtype;
+  a.status = d.status;
+  return a;
+}
+
 }  // namespace
 
 int64_t decode_ldz(const af1_layer& L) { return (int64_t)L.p2.NCH * kChunkCols; }
@@ -874,9 +894,14 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
   const int ysize = y_dtype == 0 ? 2 : 4;
   for (int64_t t0 = 0; t0 < tokens; t0 += pass) {
     const int T = (int)((tokens - t0) < pass ? (tokens - t0) : pass);
-    const DecodePlan q1 = plan_decode(1, L.p1, T, L.num_sms, L.max_smem);
-    const DecodePlan q2 = plan_decode(2, L.p2, T, L.num_sms, L.max_smem);
-    if (!q1.ok || !q2.ok) return cudaErrorInvalidConfiguration;
+    // Passes of up to 4 tokens run on the CUDA cores (af1_lut.cu): measured
+    // faster than the tensor-core kernel at every layer shape.
+    const LutPlan l1 = plan_lut(L.p1, T, L.num_sms, L.max_smem);
+    const LutPlan l2 = plan_lut(L.p2, T, L.num_sms, L.max_smem);
+    DecodePlan q1, q2;
+    if (!l1.ok) q1 = plan_decode(1, L.p1, T, L.num_sms, L.max_smem);
+    if (!l2.ok) q2 = plan_decode(2, L.p2, T, L.num_sms, L.max_smem);
+    if ((!l1.ok && !q1.ok) || (!l2.ok && !q2.ok)) return cudaErrorInvalidConfiguration;
 
     DecodeArgs a1 = {};
     a1.signs = L.signs1;
@@ -889,7 +914,7 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
     a1.sout = reinterpret_cast<float*>(wsb + W.sbuf);
     a1.lds = decode_ldz(L);
     a1.status = reinterpret_cast<unsigned*>(wsb + W.status);
-    cudaError_t e = launch_decode<1>(a1, q1, st);
+    cudaError_t e = l1.ok ? launch_lut(1, lut_args(a1), l1, st) : launch_decode<1>(a1, q1, st);
     if (e != cudaSuccess) return e;
 
     DecodeArgs a2 = {};
@@ -903,7 +928,7 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
     a2.ldy = ldy;
     a2.ydtype = y_dtype;
     a2.status = a1.status;
-    e = launch_decode<2>(a2, q2, st);
+    e = l2.ok ? launch_lut(2, lut_args(a2), l2, st) : launch_decode<2>(a2, q2, st);
     if (e != cudaSuccess) return e;
   }
   return cudaSuccess;

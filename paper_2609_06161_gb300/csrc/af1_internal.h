@@ -2,6 +2,7 @@
 // kernel launchers. Not installed; the public interface is include/af1.h.
 #pragma once
 
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -52,6 +53,33 @@ cudaError_t launch_words_to_blocks(const uint32_t* words, int64_t words_per_row,
                                    uint8_t* out, cudaStream_t st);
 // Set the calling thread's af1_last_error() message; returns `code`.
 int set_error(int code, const std::string& msg);
+
+// Decode on the CUDA cores (af1_lut.cu): one sign-matrix product of a pass
+// of 1..4 tokens through lookup tables of signed sums.
+struct LutArgs {
+  const uint8_t* signs;  // af1_layout.h row-block layout
+  SignMatrix sm;
+  int KS, CPC;           // set by the launcher from the plan
+  int tokens;            // T (1..4)
+  const __half* x;       // phase 1 input [T][ldx] (FP16)
+  int64_t ldx;
+  const float* zin;      // phase 2 input [T][ldz] (FP32)
+  int64_t ldz;
+  const __half* colscale;  // phase 1: b (C entries)
+  const __half* rowscale;  // phase 1: s; phase 2: a (R entries)
+  float* sout;             // phase 1 output [T][lds]
+  int64_t lds;
+  void* y;                 // phase 2 output [T][ldy], FP16 (ydtype 0) or FP32
+  int64_t ldy;
+  int ydtype;
+  unsigned* status;
+};
+struct LutPlan {
+  int KS = 0, CPC = 0, smem = 0;
+  bool ok = false;
+};
+LutPlan plan_lut(const SignMatrix& sm, int T, int num_sms, int max_smem);
+cudaError_t launch_lut(int phase, const LutArgs& a, const LutPlan& p, cudaStream_t st);
 
 cudaError_t launch_prefill(const af1_layer& L, const void* x, int64_t ldx, int64_t tokens, void* y, int64_t ldy,
                            int y_dtype, uint8_t* h_buf, unsigned* status, cudaStream_t st);

@@ -1,0 +1,453 @@
+// af1_lut.cu — decode path (1..4 tokens per pass) on the CUDA cores: each
+// sign-matrix x vector product of the forward pass
+//     y = a * (U (s * (V^T (b * x))))      (AF1 Eq. final_reconstruction /
+//                                          Eq. double_factor_equiv)
+// is evaluated with lookup tables of signed sums instead of tensor-core MMAs.
+//
+// For every group of 4 columns {k_0..k_3} and every token, the 16 sums
+//     T[i] = sum_q (bit q of i ? +z_{k_q} : -z_{k_q}),   i = 0..15,
+// are built once per CTA in shared memory (FP32). A matrix row then needs one
+// table read and one FP32 add per 4 signs: the 4 sign bits of the group are
+// the table index. All 32 lanes of a warp (32 rows) read the same 16-entry
+// table at the same time, so every read is a conflict-free broadcast. A
+// probe of this inner loop on GB300 sustained about 160 signs per ns per SM
+// at one token, twice the rate at which signs can be expanded into tensor
+// memory and multiplied there.
+//
+// Groups. In the row-block layout (af1_layout.h) bit 8e + p of word kw is
+// column 32 kw + 4p + e, so nibble j = 2e + h of a word (bits 8e + 4h .. +3)
+// holds the signs of columns 32 kw + 16h + 4q + e, q = 0..3: the group of
+// nibble j. Table index bit q <-> column 32 kw + 16h + 4q + e.
+//
+// Table addresses. The tables of one 128-column chunk occupy 2 KB per token
+// (one token) or 4 KB per token pair (entries are float2 {token 2p, 2p+1}):
+// group g = 4j + w (word w of the chunk, nibble j) at g * 64 (one token) or
+// g * 128 (pairs). The byte offset of an entry inside its 256-byte window is
+// built from the sign word with one shift and one LOP3 for four nibbles at a
+// time, and PRMT splices it under the window's upper address bytes, so a
+// lookup costs PRMT + LDS + FADD.
+//
+// Work split (as the tensor-core decode kernel): CTA (rb, ks) owns row block
+// rb (128 rows) and the ks-th slice of CPC chunks; the KS CTAs of a row block
+// form a cluster and reduce their partial sums through distributed shared
+// memory in a fixed order (deterministic). Two threads per row each take two
+// of the four words of every chunk. The packed chunks are fetched with bulk
+// copies before the kernel waits for the previous one (programmatic
+// dependent launch); the activations of the CTA's columns are staged in
+// shared memory, then the tables are built.
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "af1_internal.h"
+#include "af1_layout.h"
+
+namespace af1 {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kMaxCPC = 32;       // chunks per CTA (one mbarrier each)
+constexpr int kMaxKS = 16;        // CTAs per cluster
+constexpr int kMaxTokens = 4;     // tokens per pass on this path
+constexpr long long kWaitCycles = 2000000000ll;  // ~1 s at 2 GHz
+constexpr unsigned kStatusTimeout = 1u;
+
+// ---------------------------------------------------------------------------
+// PTX helpers (mbarrier, bulk copy, PDL, cluster)
+// ---------------------------------------------------------------------------
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t done;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+      : "=r"(done)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return done != 0;
+}
+// Bounded wait: false (and the CTA error flag set) if the phase did not
+// complete within kWaitCycles.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint32_t* err) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const long long t0 = clock64();
+  while (!mbar_try_wait(bar, parity)) {
+    if (clock64() - t0 > kWaitCycles) {
+      atomicOr(err, 1u);
+      return false;
+    }
+  }
+  return true;
+}
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          smem_u32(dst)),
+      "l"(src), "r"(bytes), "r"(smem_u32(bar))
+      : "memory");
+}
+__device__ __forceinline__ void griddep_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.aligned;" ::: "memory"); }
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void st_cluster_f32(float* local, uint32_t rank, float v) {
+  uint32_t remote;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(local)), "r"(rank));
+  asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(remote), "f"(v) : "memory");
+}
+__device__ __forceinline__ float lds_f32(uint32_t addr) {
+  float v;
+  asm volatile("ld.shared.f32 %0, [%1];" : "=f"(v) : "r"(addr));
+  return v;
+}
+template <int OFF>
+__device__ __forceinline__ float2 lds_f32x2(uint32_t addr) {
+  float2 v;
+  asm volatile("ld.shared.v2.f32 {%0,%1}, [%2+%3];" : "=f"(v.x), "=f"(v.y) : "r"(addr), "n"(OFF));
+  return v;
+}
+
+// ---------------------------------------------------------------------------
+// Shared-memory plan
+// ---------------------------------------------------------------------------
+
+// Token pairs of a pass: 0 stands for a single token (FP32 entries).
+__host__ __device__ constexpr int pairs_for(int T) { return T == 1 ? 0 : (T + 1) / 2; }
+// Table bytes of one chunk.
+__host__ __device__ constexpr int table_chunk_bytes(int np) { return np == 0 ? 2048 : 4096 * np; }
+// Staged activations: column k of the CTA at k + k / 32 (the skew keeps the
+// table builders' stride-32 reads on distinct banks).
+__host__ __device__ constexpr int zrow_floats(int CPC) { return CPC * kChunkCols + CPC * (kChunkCols / 32); }
+__host__ __device__ inline int slice_rows(int KS) { return (kBlockRows + KS - 1) / KS; }
+__host__ __device__ inline int align128(int v) { return (v + 127) & ~127; }
+
+struct __align__(8) LutHeader {
+  uint64_t wfull[kMaxCPC];  // packed chunk c has landed
+  uint32_t err;
+};
+
+struct LutSmem {
+  int tbl, w, z, recv, rs, hdr, total;  // byte offsets from the 1024-aligned base
+};
+
+__host__ __device__ inline LutSmem lut_smem(int CPC, int KS, int T) {
+  LutSmem p;
+  int off = 0;
+  p.tbl = off;
+  off += table_chunk_bytes(pairs_for(T)) * CPC;
+  p.w = off;
+  off += kChunkBytes * CPC;
+  p.z = off;
+  off = align128(off + T * zrow_floats(CPC) * 4);
+  p.recv = off;  // [2 KS][T][slice]: partials of the two word halves of each CTA
+  off = align128(off + 2 * KS * T * slice_rows(KS) * 4);
+  p.rs = off;
+  off = align128(off + slice_rows(KS) * 4);
+  p.hdr = off;
+  off = align128(off + (int)sizeof(LutHeader));
+  p.total = off + 1024;  // slack for aligning the base to 1024 bytes
+  return p;
+}
+
+// ---------------------------------------------------------------------------
+// Kernel
+// ---------------------------------------------------------------------------
+
+// Lookups of one word w (word wi of chunk, thread-constant) for one token:
+// tables of the chunk at tb (one token, 64 bytes per group).
+__device__ __forceinline__ void lookup_word1(uint32_t w, uint32_t pat, const uint32_t (&base)[8], float& acc) {
+  const uint32_t lo = ((w << 2) & 0x3C3C3C3Cu) | pat;  // nibbles 0, 2, 4, 6 -> entry offsets
+  const uint32_t hi = ((w >> 2) & 0x3C3C3C3Cu) | pat;  // nibbles 1, 3, 5, 7
+#pragma unroll
+  for (int j = 0; j < 8; ++j) acc += lds_f32(__byte_perm((j & 1) ? hi : lo, base[j], 0x7650 | (j >> 1)));
+}
+
+template <int NP>
+__device__ __forceinline__ void lookup_word2(uint32_t w, uint32_t pat, const uint32_t (&base)[8], float (&acc)[2 * NP]) {
+  const uint32_t lo = ((w << 3) & 0x78787878u) | pat;
+  const uint32_t hi = ((w >> 1) & 0x78787878u) | pat;
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    const uint32_t addr = __byte_perm((j & 1) ? hi : lo, base[j], 0x7650 | (j >> 1));
+    const float2 v0 = lds_f32x2<0>(addr);
+    acc[0] += v0.x;
+    acc[1] += v0.y;
+    if (NP > 1) {
+      const float2 v1 = lds_f32x2<4096>(addr);
+      acc[2] += v1.x;
+      acc[3] += v1.y;
+    }
+  }
+}
+
+template <int PHASE, int NP>
+__global__ void __launch_bounds__(kThreads, 3) lut_kernel(const LutArgs a) {
+  constexpr int NACC = NP == 0 ? 1 : 2 * NP;
+  constexpr int TCB = table_chunk_bytes(NP);
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  const int T = a.tokens;
+  const int KS = a.KS, CPC = a.CPC;
+  const LutSmem sp = lut_smem(CPC, KS, T);
+  const uint32_t* W = reinterpret_cast<const uint32_t*>(smem + sp.w);
+  float* zs = reinterpret_cast<float*>(smem + sp.z);
+  float* recv = reinterpret_cast<float*>(smem + sp.recv);
+  float* rs = reinterpret_cast<float*>(smem + sp.rs);
+  LutHeader& h = *reinterpret_cast<LutHeader*>(smem + sp.hdr);
+
+  const int tid = threadIdx.x;
+  const int rb = blockIdx.x, ks = blockIdx.y;
+  const int nch_total = a.sm.NCH;
+  const int c0 = ks * CPC;
+  const int nch = min(CPC, nch_total - c0);  // >= 1 by construction of KS
+  const int64_t row0 = (int64_t)rb * kBlockRows;
+  const int64_t k0 = (int64_t)c0 * kChunkCols;
+  const int slice = slice_rows(KS);
+  const int my0 = ks * slice;  // first block row this CTA finalises
+  const int zrow = zrow_floats(CPC);
+
+  cluster_arrive_relaxed();  // matched by cluster_wait before the first remote store
+
+  if (tid == 0) {
+    for (int c = 0; c < nch; ++c) mbar_init(&h.wfull[c], 1);
+    h.err = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    const uint8_t* src = a.signs + ((int64_t)rb * nch_total + c0) * kChunkBytes;
+    for (int c = 0; c < nch; ++c) {
+      mbar_expect_tx(&h.wfull[c], kChunkBytes);
+      bulk_g2s(smem + sp.w + c * kChunkBytes, src + (int64_t)c * kChunkBytes, kChunkBytes, &h.wfull[c]);
+    }
+  }
+  // Row scales of the rows this CTA finalises (layer constants).
+  for (int i = tid; i < slice; i += kThreads) {
+    const int64_t row = row0 + my0 + i;
+    rs[i] = (my0 + i < kBlockRows && row < a.sm.R) ? __half2float(a.rowscale[row]) : 0.f;
+  }
+  __syncthreads();
+  griddep_launch_dependents();
+
+  // ---- activations of the CTA's columns -> zs[t][k + k / 32] (FP32) -------
+  // Written by the previous kernel: read through L2 (ld.global.cg).
+  griddep_wait();
+  {
+    const int ncols = nch * kChunkCols;
+    for (int i = tid; i < T * ncols; i += kThreads) {
+      const int t = i / ncols, k = i - t * ncols;
+      const int64_t col = k0 + k;
+      float z = 0.f;
+      if (col < a.sm.C) {
+        if (PHASE == 1)
+          z = __half2float(__ldcg(a.x + (int64_t)t * a.ldx + col)) * __half2float(a.colscale[col]);
+        else
+          z = __ldcg(a.zin + (int64_t)t * a.ldz + col);
+      }
+      zs[t * zrow + k + (k >> 5)] = z;
+    }
+  }
+  __syncthreads();
+
+  // ---- tables: task (c, j, w, q) writes entries 4q .. 4q + 3 of group 4j + w
+  {
+    const int npair = NP == 0 ? 1 : NP;
+    const int ntask = nch * 128 * npair;
+    for (int task = tid; task < ntask; task += kThreads) {
+      const int q = task & 3, w = (task >> 2) & 3, j = (task >> 4) & 7;
+      const int rest = task >> 7;
+      const int p = rest % npair, c = rest / npair;
+      const int e = j >> 1, hh = j & 1;
+      // columns of index bits 0..3 (CTA-local): c 128 + 32 w + 16 hh + 4 qq + e
+      const int kb = c * kChunkCols + 32 * w + 16 * hh + e;
+      const int zb = kb + (kb >> 5);  // same 32-column block for all four
+      uint8_t* dst = smem + sp.tbl + c * TCB + (NP == 0 ? (4 * j + w) * 64 + q * 16 : p * 4096 + (4 * j + w) * 128 + q * 32);
+      float ent[2][4];
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        const int t = NP == 0 ? 0 : 2 * p + u;
+        if (NP == 0 && u == 1) break;
+        float z0 = 0.f, z1 = 0.f, z2 = 0.f, z3 = 0.f;
+        if (t < T) {
+          const float* zr = zs + t * zrow + zb;
+          z0 = zr[0];
+          z1 = zr[4];
+          z2 = zr[8];
+          z3 = zr[12];
+        }
+        const float c23 = ((q & 1) ? z2 : -z2) + ((q & 2) ? z3 : -z3);
+        const float d = z0 + z1, f = z0 - z1;
+        ent[u][0] = c23 - d;  // -z0 - z1
+        ent[u][1] = c23 + f;  // +z0 - z1
+        ent[u][2] = c23 - f;  // -z0 + z1
+        ent[u][3] = c23 + d;  // +z0 + z1
+      }
+      if (NP == 0) {
+        *reinterpret_cast<float4*>(dst) = make_float4(ent[0][0], ent[0][1], ent[0][2], ent[0][3]);
+      } else {
+        *reinterpret_cast<float4*>(dst) = make_float4(ent[0][0], ent[1][0], ent[0][1], ent[1][1]);
+        *reinterpret_cast<float4*>(dst + 16) = make_float4(ent[0][2], ent[1][2], ent[0][3], ent[1][3]);
+      }
+    }
+  }
+  __syncthreads();
+
+  // ---- lookups: thread (r, g) = row r, words 2g and 2g + 1 of every chunk ---
+  const int r = tid & 127, g = tid >> 7;
+  float acc[NACC];
+#pragma unroll
+  for (int i = 0; i < NACC; ++i) acc[i] = 0.f;
+  {
+    const uint32_t tbl0 = smem_u32(smem + sp.tbl);
+    // Entry-offset byte patterns of words 2g and 2g + 1 (their groups'
+    // offsets below the 256-byte window).
+    const uint32_t pat0 = NP == 0 ? (uint32_t)(2 * g * 64) * 0x01010101u : 0u;
+    const uint32_t pat1 = NP == 0 ? (uint32_t)((2 * g + 1) * 64) * 0x01010101u : 0x80808080u;
+    bool ok = true;
+    for (int c = 0; c < nch; ++c) {
+      if (ok) ok = mbar_wait(&h.wfull[c], 0, &h.err);
+      const uint32_t tb = tbl0 + (uint32_t)(c * TCB);
+      uint32_t base[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) base[j] = tb + (uint32_t)(NP == 0 ? j * 256 : j * 512 + g * 256);
+      const uint32_t* wc = W + c * (kChunkBytes / 4) + r;
+      const uint32_t w0 = wc[(2 * g) * kBlockRows], w1 = wc[(2 * g + 1) * kBlockRows];
+      if constexpr (NP == 0) {
+        lookup_word1(w0, pat0, base, acc[0]);
+        lookup_word1(w1, pat1, base, acc[0]);
+      } else {
+        lookup_word2<NP>(w0, pat0, base, acc);
+        lookup_word2<NP>(w1, pat1, base, acc);
+      }
+    }
+  }
+
+  // ---- partial sums -> owner CTA of each row -> final sums -------------------
+  cluster_wait();  // every CTA of the cluster has started
+  {
+    const int owner = r / slice;
+    const int src = ks * 2 + g;
+#pragma unroll
+    for (int t = 0; t < NACC; ++t)
+      if (t < T) st_cluster_f32(recv + ((src * T + t) * slice + (r - owner * slice)), (uint32_t)owner, acc[t]);
+  }
+  cluster_sync();  // all partials of the cluster have landed in their owners' buffers
+  const int cnt = min(slice, kBlockRows - my0);
+  for (int idx = tid; idx < T * cnt; idx += kThreads) {
+    const int t = idx / cnt;
+    const int i = idx - t * cnt;
+    const int64_t row = row0 + my0 + i;
+    if (row >= a.sm.R) continue;
+    float v = 0.f;
+    for (int q = 0; q < 2 * KS; ++q) v += recv[(q * T + t) * slice + i];
+    const float out = v * rs[i];
+    if (PHASE == 1) {
+      a.sout[(int64_t)t * a.lds + row] = out;
+    } else if (a.ydtype == 0) {
+      reinterpret_cast<__half*>(a.y)[(int64_t)t * a.ldy + row] = __float2half_rn(out);
+    } else {
+      reinterpret_cast<float*>(a.y)[(int64_t)t * a.ldy + row] = out;
+    }
+  }
+
+  // ---- teardown ---------------------------------------------------------------
+  __syncthreads();
+  if (tid == 0 && h.err != 0) {
+    // A wait gave up: let the bulk copies drain (bounded) so that none lands
+    // after the CTA has exited, and report it.
+    for (int c = 0; c < nch; ++c) mbar_wait(&h.wfull[c], 0, &h.err);
+    atomicOr(a.status, kStatusTimeout);
+  }
+}
+
+template <int PHASE, int NP>
+cudaError_t launch_np(const LutArgs& a, const LutPlan& p, cudaStream_t st) {
+  auto kern = lut_kernel<PHASE, NP>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, p.smem);
+  if (e != cudaSuccess) return e;
+  if (p.KS > 8) {
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    if (e != cudaSuccess) return e;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)a.sm.RB, (unsigned)p.KS, 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = (size_t)p.smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = 1;
+  attr[1].val.clusterDim.y = (unsigned)p.KS;
+  attr[1].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  LutArgs b = a;
+  b.KS = p.KS;
+  b.CPC = p.CPC;
+  return cudaLaunchKernelEx(&cfg, kern, b);
+}
+
+}  // namespace
+
+// Split of one sign matrix for a pass of T <= 4 tokens: about two CTAs per SM
+// (row blocks x KS ~ 2 SMs, KS <= 16 CTAs per cluster), CTAs small enough
+// that three fit on an SM, and at most kMaxCPC chunks each.
+LutPlan plan_lut(const SignMatrix& sm, int T, int num_sms, int max_smem) {
+  LutPlan p;
+  if (T < 1 || T > kMaxTokens || sm.RB < 1 || sm.NCH < 1) return p;
+  const int sms = num_sms > 0 ? num_sms : 148;
+  const int cap = max_smem / 3 < 72 * 1024 ? max_smem / 3 : 72 * 1024;
+  int ks = (2 * sms + sm.RB - 1) / sm.RB;
+  if (ks > kMaxKS) ks = kMaxKS;
+  if (ks > sm.NCH) ks = sm.NCH;
+  if (ks < 1) ks = 1;
+  for (; ks <= kMaxKS && ks <= sm.NCH; ++ks) {
+    const int cpc = (sm.NCH + ks - 1) / ks;
+    if (cpc > kMaxCPC) continue;
+    const int KS = (sm.NCH + cpc - 1) / cpc;
+    const int need = lut_smem(cpc, KS, T).total;
+    if (need <= cap || (ks == kMaxKS || ks == sm.NCH)) {
+      if (need > max_smem) return p;
+      p.KS = KS;
+      p.CPC = cpc;
+      p.smem = need;
+      p.ok = true;
+      return p;
+    }
+  }
+  return p;
+}
+
+cudaError_t launch_lut(int phase, const LutArgs& a, const LutPlan& p, cudaStream_t st) {
+  const int np = pairs_for(a.tokens);
+  if (phase == 1) {
+    switch (np) {
+      case 0: return launch_np<1, 0>(a, p, st);
+      case 1: return launch_np<1, 1>(a, p, st);
+      default: return launch_np<1, 2>(a, p, st);
+    }
+  }
+  switch (np) {
+    case 0: return launch_np<2, 0>(a, p, st);
+    case 1: return launch_np<2, 1>(a, p, st);
+    default: return launch_np<2, 2>(a, p, st);
+  }
+}
+
+}  // namespace af1
