@@ -178,26 +178,27 @@ __device__ __forceinline__ void lookup_word1(uint32_t w, uint32_t pat, const uin
   for (int j = 0; j < 8; ++j) acc += lds_f32(__byte_perm((j & 1) ? hi : lo, base[j], 0x7650 | (j >> 1)));
 }
 
+// Entry `addr` of the tables of token pairs P .. NP - 1 (4 KB apart).
+template <int P, int NP>
+__device__ __forceinline__ void lookup_pairs(uint32_t addr, float (&acc)[2 * NP]) {
+  if constexpr (P < NP) {
+    const float2 v = lds_f32x2<P * 4096>(addr);
+    acc[2 * P] += v.x;
+    acc[2 * P + 1] += v.y;
+    lookup_pairs<P + 1, NP>(addr, acc);
+  }
+}
+
 template <int NP>
 __device__ __forceinline__ void lookup_word2(uint32_t w, uint32_t pat, const uint32_t (&base)[8], float (&acc)[2 * NP]) {
   const uint32_t lo = ((w << 3) & 0x78787878u) | pat;
   const uint32_t hi = ((w >> 1) & 0x78787878u) | pat;
 #pragma unroll
-  for (int j = 0; j < 8; ++j) {
-    const uint32_t addr = __byte_perm((j & 1) ? hi : lo, base[j], 0x7650 | (j >> 1));
-    const float2 v0 = lds_f32x2<0>(addr);
-    acc[0] += v0.x;
-    acc[1] += v0.y;
-    if (NP > 1) {
-      const float2 v1 = lds_f32x2<4096>(addr);
-      acc[2] += v1.x;
-      acc[3] += v1.y;
-    }
-  }
+  for (int j = 0; j < 8; ++j) lookup_pairs<0, NP>(__byte_perm((j & 1) ? hi : lo, base[j], 0x7650 | (j >> 1)), acc);
 }
 
 template <int PHASE, int NP>
-__global__ void __launch_bounds__(kThreads, 3) lut_kernel(const LutArgs a) {
+__global__ void __launch_bounds__(kThreads, 4) lut_kernel(const LutArgs a) {
   constexpr int NACC = NP == 0 ? 1 : 2 * NP;
   constexpr int TCB = table_chunk_bytes(NP);
   extern __shared__ uint8_t smem_raw[];
@@ -244,21 +245,68 @@ __global__ void __launch_bounds__(kThreads, 3) lut_kernel(const LutArgs a) {
   griddep_launch_dependents();
 
   // ---- activations of the CTA's columns -> zs[t][k + k / 32] (FP32) -------
-  // Written by the previous kernel: read through L2 (ld.global.cg).
+  // Written by the previous kernel: read through L2 (ld.global.cg), 8
+  // columns per load, a batch of loads per thread in flight at once.
   griddep_wait();
   {
-    const int ncols = nch * kChunkCols;
-    for (int i = tid; i < T * ncols; i += kThreads) {
-      const int t = i / ncols, k = i - t * ncols;
-      const int64_t col = k0 + k;
-      float z = 0.f;
-      if (col < a.sm.C) {
-        if (PHASE == 1)
-          z = __half2float(__ldcg(a.x + (int64_t)t * a.ldx + col)) * __half2float(a.colscale[col]);
-        else
-          z = __ldcg(a.zin + (int64_t)t * a.ldz + col);
+    const int g8 = nch * (kChunkCols / 8);  // 8-column groups per token
+    const int ng = T * g8;
+    constexpr int kBatch = 2;
+    for (int i0 = tid; i0 < ng; i0 += kBatch * kThreads) {
+      float v[kBatch][8];
+#pragma unroll
+      for (int u = 0; u < kBatch; ++u) {
+        const int i = i0 + u * kThreads;
+        const int t = i / g8, k = (i - t * g8) * 8;
+        const int64_t col = k0 + k;
+        if (i < ng && col + 7 < a.sm.C) {
+          if (PHASE == 1) {
+            const uint4 xr = __ldcg(reinterpret_cast<const uint4*>(a.x + (int64_t)t * a.ldx + col));
+            const uint4 br = __ldg(reinterpret_cast<const uint4*>(a.colscale + col));
+            const uint32_t xw[4] = {xr.x, xr.y, xr.z, xr.w}, bw[4] = {br.x, br.y, br.z, br.w};
+#pragma unroll
+            for (int h2 = 0; h2 < 4; ++h2) {
+              const float2 xf = __half22float2(*reinterpret_cast<const __half2*>(&xw[h2]));
+              const float2 bf = __half22float2(*reinterpret_cast<const __half2*>(&bw[h2]));
+              v[u][2 * h2] = xf.x * bf.x;
+              v[u][2 * h2 + 1] = xf.y * bf.y;
+            }
+          } else {
+            const float4 z0 = __ldcg(reinterpret_cast<const float4*>(a.zin + (int64_t)t * a.ldz + col));
+            const float4 z1 = __ldcg(reinterpret_cast<const float4*>(a.zin + (int64_t)t * a.ldz + col + 4));
+            v[u][0] = z0.x;
+            v[u][1] = z0.y;
+            v[u][2] = z0.z;
+            v[u][3] = z0.w;
+            v[u][4] = z1.x;
+            v[u][5] = z1.y;
+            v[u][6] = z1.z;
+            v[u][7] = z1.w;
+          }
+        } else {
+#pragma unroll
+          for (int q = 0; q < 8; ++q) {
+            float z = 0.f;
+            if (i < ng && col + q < a.sm.C) {
+              if (PHASE == 1)
+                z = __half2float(__ldcg(a.x + (int64_t)t * a.ldx + col + q)) * __half2float(a.colscale[col + q]);
+              else
+                z = __ldcg(a.zin + (int64_t)t * a.ldz + col + q);
+            }
+            v[u][q] = z;
+          }
+        }
       }
-      zs[t * zrow + k + (k >> 5)] = z;
+#pragma unroll
+      for (int u = 0; u < kBatch; ++u) {
+        const int i = i0 + u * kThreads;
+        if (i < ng) {
+          const int t = i / g8, k = (i - t * g8) * 8;
+          float* dst = zs + t * zrow + k + (k >> 5);  // 8 columns within one 32-column block
+#pragma unroll
+          for (int q = 0; q < 8; ++q) dst[q] = v[u][q];
+        }
+      }
     }
   }
   __syncthreads();
@@ -434,20 +482,17 @@ LutPlan plan_lut(const SignMatrix& sm, int T, int num_sms, int max_smem) {
   return p;
 }
 
+template <int PHASE>
+cudaError_t launch_phase(const LutArgs& a, const LutPlan& p, cudaStream_t st) {
+  switch (pairs_for(a.tokens)) {
+    case 0: return launch_np<PHASE, 0>(a, p, st);
+    case 1: return launch_np<PHASE, 1>(a, p, st);
+    default: return launch_np<PHASE, 2>(a, p, st);
+  }
+}
+
 cudaError_t launch_lut(int phase, const LutArgs& a, const LutPlan& p, cudaStream_t st) {
-  const int np = pairs_for(a.tokens);
-  if (phase == 1) {
-    switch (np) {
-      case 0: return launch_np<1, 0>(a, p, st);
-      case 1: return launch_np<1, 1>(a, p, st);
-      default: return launch_np<1, 2>(a, p, st);
-    }
-  }
-  switch (np) {
-    case 0: return launch_np<2, 0>(a, p, st);
-    case 1: return launch_np<2, 1>(a, p, st);
-    default: return launch_np<2, 2>(a, p, st);
-  }
+  return phase == 1 ? launch_phase<1>(a, p, st) : launch_phase<2>(a, p, st);
 }
 
 }  // namespace af1
