@@ -178,23 +178,22 @@ __device__ __forceinline__ void lookup_word1(uint32_t w, uint32_t pat, const uin
   for (int j = 0; j < 8; ++j) acc += lds_f32(__byte_perm((j & 1) ? hi : lo, base[j], 0x7650 | (j >> 1)));
 }
 
-// Entry `addr` of the tables of token pairs P .. NP - 1 (4 KB apart).
-template <int P, int NP>
-__device__ __forceinline__ void lookup_pairs(uint32_t addr, float (&acc)[2 * NP]) {
-  if constexpr (P < NP) {
-    const float2 v = lds_f32x2<P * 4096>(addr);
-    acc[2 * P] += v.x;
-    acc[2 * P + 1] += v.y;
-    lookup_pairs<P + 1, NP>(addr, acc);
-  }
-}
-
 template <int NP>
 __device__ __forceinline__ void lookup_word2(uint32_t w, uint32_t pat, const uint32_t (&base)[8], float (&acc)[2 * NP]) {
   const uint32_t lo = ((w << 3) & 0x78787878u) | pat;
   const uint32_t hi = ((w >> 1) & 0x78787878u) | pat;
 #pragma unroll
-  for (int j = 0; j < 8; ++j) lookup_pairs<0, NP>(__byte_perm((j & 1) ? hi : lo, base[j], 0x7650 | (j >> 1)), acc);
+  for (int j = 0; j < 8; ++j) {
+    const uint32_t addr = __byte_perm((j & 1) ? hi : lo, base[j], 0x7650 | (j >> 1));
+    const float2 v0 = lds_f32x2<0>(addr);
+    acc[0] += v0.x;
+    acc[1] += v0.y;
+    if (NP > 1) {
+      const float2 v1 = lds_f32x2<4096>(addr);
+      acc[2] += v1.x;
+      acc[3] += v1.y;
+    }
+  }
 }
 
 template <int PHASE, int NP>
@@ -236,11 +235,11 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const LutArgs a) {
       bulk_g2s(smem + sp.w + c * kChunkBytes, src + (int64_t)c * kChunkBytes, kChunkBytes, &h.wfull[c]);
     }
   }
-  // Row scales of the rows this CTA finalises (layer constants).
-  for (int i = tid; i < slice; i += kThreads) {
-    const int64_t row = row0 + my0 + i;
-    rs[i] = (my0 + i < kBlockRows && row < a.sm.R) ? __half2float(a.rowscale[row]) : 0.f;
-  }
+  // Row scale of row my0 + tid of the block (a layer constant): loaded now,
+  // stored to shared memory once the activations are staged.
+  const float rs_own = (tid < slice && my0 + tid < kBlockRows && row0 + my0 + tid < a.sm.R)
+                           ? __half2float(a.rowscale[row0 + my0 + tid])
+                           : 0.f;
   __syncthreads();
   griddep_launch_dependents();
 
@@ -309,6 +308,7 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const LutArgs a) {
       }
     }
   }
+  if (tid < slice) rs[tid] = rs_own;
   __syncthreads();
 
   // ---- tables: task (c, j, w, q) writes entries 4q .. 4q + 3 of group 4j + w
@@ -400,9 +400,21 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const LutArgs a) {
     const int i = idx - t * cnt;
     const int64_t row = row0 + my0 + i;
     if (row >= a.sm.R) continue;
-    float v = 0.f;
-    for (int q = 0; q < 2 * KS; ++q) v += recv[(q * T + t) * slice + i];
-    const float out = v * rs[i];
+    // The 2 KS partials in four interleaved chains (fixed order:
+    // deterministic), so their reads overlap.
+    const float* pr = recv + t * slice + i;
+    const int qstride = T * slice;
+    float v0 = 0.f, v1 = 0.f, v2 = 0.f, v3 = 0.f;
+    int q = 0;
+#pragma unroll 2
+    for (; q + 4 <= 2 * KS; q += 4) {
+      v0 += pr[q * qstride];
+      v1 += pr[(q + 1) * qstride];
+      v2 += pr[(q + 2) * qstride];
+      v3 += pr[(q + 3) * qstride];
+    }
+    for (; q < 2 * KS; ++q) v0 += pr[q * qstride];
+    const float out = ((v0 + v1) + (v2 + v3)) * rs[i];
     if (PHASE == 1) {
       a.sout[(int64_t)t * a.lds + row] = out;
     } else if (a.ydtype == 0) {
