@@ -241,7 +241,6 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const LutArgs a) {
                            ? __half2float(a.rowscale[row0 + my0 + tid])
                            : 0.f;
   __syncthreads();
-  griddep_launch_dependents();
 
   // ---- activations of the CTA's columns -> zs[t][k + k / 32] (FP32) -------
   // Written by the previous kernel: read through L2 (ld.global.cg), 8
@@ -384,6 +383,12 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const LutArgs a) {
     }
   }
 
+  // Let the next kernel launch only now: its CTAs would otherwise hold SM
+  // slots (waiting for this kernel) that sibling kernels on other streams
+  // need, and its sign copies still get the reduction's time as a head start
+  // (measured: config-1 stack 7.40 -> 6.53 us per linear on the DAG schedule,
+  // trigger at the start vs here).
+  griddep_launch_dependents();
   // ---- partial sums -> owner CTA of each row -> final sums -------------------
   cluster_wait();  // every CTA of the cluster has started
   {
