@@ -459,7 +459,6 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const DecodeArgs a)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = h.tmem_base;
-  griddep_launch_dependents();
 
   if (warp < 4) {
     // ---- A: expand packed chunks into the tensor-memory ring --------------
@@ -634,6 +633,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const DecodeArgs a)
     __syncwarp();
   }
 
+  griddep_launch_dependents();
   // ---- epilogue: accumulators -> per-row partial sums -> owner CTA ----------
   griddep_wait();  // outputs may still be read by the previous kernel until it completes
   cluster_wait();  // every CTA of the cluster has started
