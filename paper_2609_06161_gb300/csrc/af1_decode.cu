@@ -894,8 +894,8 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
   const int ysize = y_dtype == 0 ? 2 : 4;
   for (int64_t t0 = 0; t0 < tokens; t0 += pass) {
     const int T = (int)((tokens - t0) < pass ? (tokens - t0) : pass);
-    // Passes of up to 4 tokens run on the CUDA cores (af1_lut.cu): measured
-    // faster than the tensor-core kernel at every layer shape.
+    // Passes run on the CUDA cores (af1_lut.cu) whenever that kernel has a
+    // plan; the tensor-core kernel is the fallback.
     const LutPlan l1 = plan_lut(L.p1, T, L.num_sms, L.max_smem);
     const LutPlan l2 = plan_lut(L.p2, T, L.num_sms, L.max_smem);
     DecodePlan q1, q2;

@@ -55,12 +55,12 @@ cudaError_t launch_words_to_blocks(const uint32_t* words, int64_t words_per_row,
 int set_error(int code, const std::string& msg);
 
 // Decode on the CUDA cores (af1_lut.cu): one sign-matrix product of a pass
-// of 1..4 tokens through lookup tables of signed sums.
+// of 1..16 tokens through lookup tables of signed sums.
 struct LutArgs {
   const uint8_t* signs;  // af1_layout.h row-block layout
   SignMatrix sm;
   int KS, CPC;           // set by the launcher from the plan
-  int tokens;            // T (1..4)
+  int tokens;            // T (1..16)
   const __half* x;       // phase 1 input [T][ldx] (FP16)
   int64_t ldx;
   const float* zin;      // phase 2 input [T][ldz] (FP32)

@@ -1,4 +1,4 @@
-// af1_lut.cu — decode path (1..4 tokens per pass) on the CUDA cores: each
+// af1_lut.cu — decode path (1..16 tokens per pass) on the CUDA cores: each
 // sign-matrix x vector product of the forward pass
 //     y = a * (U (s * (V^T (b * x))))      (AF1 Eq. final_reconstruction /
 //                                          Eq. double_factor_equiv)
@@ -27,14 +27,15 @@
 // time, and PRMT splices it under the window's upper address bytes, so a
 // lookup costs PRMT + LDS + FADD.
 //
-// Work split (as the tensor-core decode kernel): CTA (rb, ks) owns row block
-// rb (128 rows) and the ks-th slice of CPC chunks; the KS CTAs of a row block
-// form a cluster and reduce their partial sums through distributed shared
-// memory in a fixed order (deterministic). Two threads per row each take two
-// of the four words of every chunk. The packed chunks are fetched with bulk
-// copies before the kernel waits for the previous one (programmatic
-// dependent launch); the activations of the CTA's columns are staged in
-// shared memory, then the tables are built.
+// Work split (as the tensor-core decode kernel): CTA (rb, ks, tg) owns row
+// block rb (128 rows), the ks-th slice of CPC chunks and token group tg (up
+// to 4 tokens of the pass); the KS CTAs of a row block and token group form
+// a cluster and reduce their partial sums through distributed shared memory
+// in a fixed order (deterministic). Two threads per row each take two of the
+// four words of every chunk. The packed chunks are fetched with bulk copies
+// before the kernel waits for the previous one (programmatic dependent
+// launch); the activations of the CTA's columns are staged in shared memory,
+// then the tables are built.
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -48,7 +49,7 @@ namespace {
 constexpr int kThreads = 256;
 constexpr int kMaxCPC = 32;       // chunks per CTA (one mbarrier each)
 constexpr int kMaxKS = 16;        // CTAs per cluster
-constexpr int kMaxTokens = 4;     // tokens per pass on this path
+constexpr int kGroupTokens = 4;   // tokens per CTA: a pass of T tokens runs ceil(T / 4) CTAs per tile
 constexpr long long kWaitCycles = 2000000000ll;  // ~1 s at 2 GHz
 constexpr unsigned kStatusTimeout = 1u;
 
@@ -146,11 +147,13 @@ struct LutSmem {
   int tbl, w, z, recv, rs, hdr, total;  // byte offsets from the 1024-aligned base
 };
 
-__host__ __device__ inline LutSmem lut_smem(int CPC, int KS, int T) {
+// T tokens of a CTA, tables laid out for np token pairs (pairs_for of the
+// pass's first group; a smaller last group leaves its missing tokens zero).
+__host__ __device__ inline LutSmem lut_smem(int CPC, int KS, int T, int np) {
   LutSmem p;
   int off = 0;
   p.tbl = off;
-  off += table_chunk_bytes(pairs_for(T)) * CPC;
+  off += table_chunk_bytes(np) * CPC;
   p.w = off;
   off += kChunkBytes * CPC;
   p.z = off;
@@ -202,9 +205,13 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const LutArgs a) {
   constexpr int TCB = table_chunk_bytes(NP);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-  const int T = a.tokens;
+  // Token group blockIdx.z: tokens tg0 .. tg0 + T - 1 of the pass.
+  const int tg0 = (int)blockIdx.z * kGroupTokens;
+  const int T = min(kGroupTokens, a.tokens - tg0);
+  const __half* xg = PHASE == 1 ? a.x + (int64_t)tg0 * a.ldx : nullptr;
+  const float* zg = PHASE == 2 ? a.zin + (int64_t)tg0 * a.ldz : nullptr;
   const int KS = a.KS, CPC = a.CPC;
-  const LutSmem sp = lut_smem(CPC, KS, T);
+  const LutSmem sp = lut_smem(CPC, KS, T, NP);
   const uint32_t* W = reinterpret_cast<const uint32_t*>(smem + sp.w);
   float* zs = reinterpret_cast<float*>(smem + sp.z);
   float* recv = reinterpret_cast<float*>(smem + sp.recv);
@@ -259,7 +266,7 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const LutArgs a) {
         const int64_t col = k0 + k;
         if (i < ng && col + 7 < a.sm.C) {
           if (PHASE == 1) {
-            const uint4 xr = __ldcg(reinterpret_cast<const uint4*>(a.x + (int64_t)t * a.ldx + col));
+            const uint4 xr = __ldcg(reinterpret_cast<const uint4*>(xg + (int64_t)t * a.ldx + col));
             const uint4 br = __ldg(reinterpret_cast<const uint4*>(a.colscale + col));
             const uint32_t xw[4] = {xr.x, xr.y, xr.z, xr.w}, bw[4] = {br.x, br.y, br.z, br.w};
 #pragma unroll
@@ -270,8 +277,8 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const LutArgs a) {
               v[u][2 * h2 + 1] = xf.y * bf.y;
             }
           } else {
-            const float4 z0 = __ldcg(reinterpret_cast<const float4*>(a.zin + (int64_t)t * a.ldz + col));
-            const float4 z1 = __ldcg(reinterpret_cast<const float4*>(a.zin + (int64_t)t * a.ldz + col + 4));
+            const float4 z0 = __ldcg(reinterpret_cast<const float4*>(zg + (int64_t)t * a.ldz + col));
+            const float4 z1 = __ldcg(reinterpret_cast<const float4*>(zg + (int64_t)t * a.ldz + col + 4));
             v[u][0] = z0.x;
             v[u][1] = z0.y;
             v[u][2] = z0.z;
@@ -287,9 +294,9 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const LutArgs a) {
             float z = 0.f;
             if (i < ng && col + q < a.sm.C) {
               if (PHASE == 1)
-                z = __half2float(__ldcg(a.x + (int64_t)t * a.ldx + col + q)) * __half2float(a.colscale[col + q]);
+                z = __half2float(__ldcg(xg + (int64_t)t * a.ldx + col + q)) * __half2float(a.colscale[col + q]);
               else
-                z = __ldcg(a.zin + (int64_t)t * a.ldz + col + q);
+                z = __ldcg(zg + (int64_t)t * a.ldz + col + q);
             }
             v[u][q] = z;
           }
@@ -421,11 +428,11 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const LutArgs a) {
     for (; q < 2 * KS; ++q) v0 += pr[q * qstride];
     const float out = ((v0 + v1) + (v2 + v3)) * rs[i];
     if (PHASE == 1) {
-      a.sout[(int64_t)t * a.lds + row] = out;
+      a.sout[(int64_t)(tg0 + t) * a.lds + row] = out;
     } else if (a.ydtype == 0) {
-      reinterpret_cast<__half*>(a.y)[(int64_t)t * a.ldy + row] = __float2half_rn(out);
+      reinterpret_cast<__half*>(a.y)[(int64_t)(tg0 + t) * a.ldy + row] = __float2half_rn(out);
     } else {
-      reinterpret_cast<float*>(a.y)[(int64_t)t * a.ldy + row] = out;
+      reinterpret_cast<float*>(a.y)[(int64_t)(tg0 + t) * a.ldy + row] = out;
     }
   }
 
@@ -449,7 +456,7 @@ cudaError_t launch_np(const LutArgs& a, const LutPlan& p, cudaStream_t st) {
     if (e != cudaSuccess) return e;
   }
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((unsigned)a.sm.RB, (unsigned)p.KS, 1);
+  cfg.gridDim = dim3((unsigned)a.sm.RB, (unsigned)p.KS, (unsigned)((a.tokens + kGroupTokens - 1) / kGroupTokens));
   cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.dynamicSmemBytes = (size_t)p.smem;
   cfg.stream = st;
@@ -470,15 +477,19 @@ cudaError_t launch_np(const LutArgs& a, const LutPlan& p, cudaStream_t st) {
 
 }  // namespace
 
-// Split of one sign matrix for a pass of T <= 4 tokens: about two CTAs per SM
-// (row blocks x KS ~ 2 SMs, KS <= 16 CTAs per cluster), CTAs small enough
-// that three fit on an SM, and at most kMaxCPC chunks each.
+// Split of one sign matrix for a pass of T <= 16 tokens, run as ceil(T / 4)
+// token groups of CTAs: about two CTAs per SM (row blocks x KS x groups ~
+// 2 SMs, KS <= 16 CTAs per cluster), CTAs small enough that three fit on an
+// SM, and at most kMaxCPC chunks each.
 LutPlan plan_lut(const SignMatrix& sm, int T, int num_sms, int max_smem) {
   LutPlan p;
-  if (T < 1 || T > kMaxTokens || sm.RB < 1 || sm.NCH < 1) return p;
+  if (T < 1 || T > kMaxPassTokens || sm.RB < 1 || sm.NCH < 1) return p;
+  const int Tg = T < kGroupTokens ? T : kGroupTokens;
+  const int groups = (T + kGroupTokens - 1) / kGroupTokens;
   const int sms = num_sms > 0 ? num_sms : 148;
   const int cap = max_smem / 3 < 72 * 1024 ? max_smem / 3 : 72 * 1024;
-  int ks = (2 * sms + sm.RB - 1) / sm.RB;
+  const int64_t tiles = (int64_t)sm.RB * groups;
+  int ks = (int)((2 * sms + tiles - 1) / tiles);
   if (ks > kMaxKS) ks = kMaxKS;
   if (ks > sm.NCH) ks = sm.NCH;
   if (ks < 1) ks = 1;
@@ -486,7 +497,7 @@ LutPlan plan_lut(const SignMatrix& sm, int T, int num_sms, int max_smem) {
     const int cpc = (sm.NCH + ks - 1) / ks;
     if (cpc > kMaxCPC) continue;
     const int KS = (sm.NCH + cpc - 1) / cpc;
-    const int need = lut_smem(cpc, KS, T).total;
+    const int need = lut_smem(cpc, KS, Tg, pairs_for(Tg)).total;
     if (need <= cap || (ks == kMaxKS || ks == sm.NCH)) {
       if (need > max_smem) return p;
       p.KS = KS;
@@ -501,7 +512,7 @@ LutPlan plan_lut(const SignMatrix& sm, int T, int num_sms, int max_smem) {
 
 template <int PHASE>
 cudaError_t launch_phase(const LutArgs& a, const LutPlan& p, cudaStream_t st) {
-  switch (pairs_for(a.tokens)) {
+  switch (pairs_for(a.tokens < kGroupTokens ? a.tokens : kGroupTokens)) {
     case 0: return launch_np<PHASE, 0>(a, p, st);
     case 1: return launch_np<PHASE, 1>(a, p, st);
     default: return launch_np<PHASE, 2>(a, p, st);
