@@ -34,6 +34,10 @@ import numpy as np  # noqa: E402
 
 METRIC = "tokens/s and us/layer for binary-factorized linear (AF1, 1.0 BPW); % of HBM roofline"
 LAYERS = 32
+# Measured DRAM traffic of one layer's seven decode calls at one token (bytes;
+# ncu, profiles/lut_kernel_llama3_8b_b1.md): 1.028 x the algorithmic bytes.
+DECODE_TRAFFIC_B1_PER_LAYER = 28197888
+TC_DECODE = False  # set from --tc-decode
 
 
 def parse():
@@ -56,6 +60,8 @@ def parse():
     p.add_argument("--no-sweep", action="store_true",
                    help="skip the per-shape sweep (LLaMA-3-8B at 1/4/16 tokens, 70B shapes at 1/8/64/512)")
     p.add_argument("--no-stack", action="store_true", help="skip the 32-layer stack with HiSA-like ranks")
+    p.add_argument("--tc-decode", action="store_true",
+                   help="create layers with AF1_FLAG_TC_DECODE (tensor-core decode kernel instead of lookup tables)")
     return p.parse_args()
 
 
@@ -196,6 +202,8 @@ def config_dict(args):
                                                if args.schedule == "dag" else "one stream in model order")
                          + ("" if args.no_graph else ", CUDA graph")),
             "batch": args.batch, "layers": args.layers, "linears_per_step": 7 * args.layers,
+            "decode_kernel": ("tensor cores (AF1_FLAG_TC_DECODE)" if args.tc_decode
+                              else "lookup tables on the CUDA cores (default)"),
             "l2": "inputs larger than L2 (packed weights per step >> 129 MB), no flush"}
 
 
@@ -264,7 +272,7 @@ def build_layers(P, torch, layers, batch, rank, outlier_frac=0.0):
             f16 = lambda bits: torch.from_numpy(np.ascontiguousarray(bits).view(np.float16)).cuda()
             Uw = torch.from_numpy(d["Uw"].view(np.int32)).cuda()
             Vw = torch.from_numpy(d["Vw"].view(np.int32)).cuda()
-            layer = P.Layer.from_words(Uw, Vw, f16(d["a"]), f16(d["s"]), f16(d["b"]), m, n, r)
+            layer = P.Layer.from_words(Uw, Vw, f16(d["a"]), f16(d["s"]), f16(d["b"]), m, n, r, tc_decode=TC_DECODE)
             del Uw, Vw
             x = f16(d["x"]).reshape(batch, n)
             objs.append((name, m, n, r, layer, x))
@@ -287,7 +295,7 @@ def device_layer(P, torch, m, n, r, seed, any_rank=False):
     rs = synth.rng(seed)
     f16 = lambda bits: torch.from_numpy(np.ascontiguousarray(bits).view(np.float16)).cuda()
     a, s_, b = f16(synth.scales_f16(rs, m)), f16(synth.scales_f16(rs, r)), f16(synth.scales_f16(rs, n))
-    layer = P.Layer.from_words(Uw, Vw, a, s_, b, m, n, r, any_rank=any_rank)
+    layer = P.Layer.from_words(Uw, Vw, a, s_, b, m, n, r, any_rank=any_rank, tc_decode=TC_DECODE)
     del Uw, Vw
     return layer
 
@@ -413,7 +421,9 @@ def stack_hisa(P, torch, peaks, stream, steps, dense_ms=None):
 
 
 def main():
+    global TC_DECODE
     args = parse()
+    TC_DECODE = args.tc_decode
     if args.impl == "reference":
         run_reference(args)
         return
@@ -611,16 +621,22 @@ def main():
                     "peak_source": "MEASURED_PEAKS.json bf16_tflops_sustained (FP16 dense rate = BF16 rate)",
                     "algorithmic_flops_per_step": flops, "traffic": None}
         else:
-            roof = {"bound": "hbm", "kernel": "af1_linear_forward (phase-1 + phase-2 kernels, per call)",
+            # DRAM bytes (read + write) of one layer's 14 lookup-table kernels
+            # at one token, from the ncu capture summarised in
+            # profiles/lut_kernel_llama3_8b_b1.md, times 32 layers.
+            traffic = DECODE_TRAFFIC_B1_PER_LAYER * args.layers if b == 1 and not TC_DECODE else None
+            roof = {"bound": "hbm", "kernel": "af1_linear_forward (two lookup-table kernels per call, lut_kernel<1|2>)",
                     "achieved": achieved_gbs, "peak": hbm, "unit": "GB/s",
                     "frac": (achieved_gbs / hbm) if hbm else None, "peak_source": "MEASURED_PEAKS.json hbm_gbs"
                     if "hbm_gbs" in peaks else "fallback 6800 GB/s",
-                    "algorithmic_bytes_per_step": alg, "traffic": None}
+                    "algorithmic_bytes_per_step": alg, "traffic": traffic,
+                    "traffic_source": "ncu dram__bytes_read.sum + dram__bytes_write.sum per layer x layers"
+                    if traffic else None}
         line = {
             "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
             "warmup": max(args.warmup, 3), "ms_per_step": ms_step, "us_per_layer": us_layer,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-            "dtype": "e4m3 MMA / f32 accumulate (1-bit signs, f16 scales and activations)",
+            "dtype": "f16" if args.workload == "prefill" else "f32",
             "data": "synthetic (seeded PCG64 packed signs, |N(0,0.02)|+1e-3 scales, N(0,1) activations)",
             "config": config_dict(args),
             "roofline": roof,

@@ -73,6 +73,11 @@ extern "C" {
    paper's 2.5-BPW setting). Without it r > af1_rank_for_budget(m, n, 1, 1)
    is rejected with AF1_ERR_OVER_BUDGET. */
 #define AF1_FLAG_ANY_RANK 1
+/* Run decode passes (1..16 tokens) on the tensor-core kernel (tcgen05 MMAs on
+   e4m3 sign and activation terms) instead of the default CUDA-core kernel
+   (lookup tables of signed sums). Both compute the same products within the
+   library's tolerance; the default is faster at every measured shape. */
+#define AF1_FLAG_TC_DECODE 2
 
 typedef struct af1_layer_desc {
   int64_t m;       /* d_out: rows of W_hat, length of a, length of y rows */

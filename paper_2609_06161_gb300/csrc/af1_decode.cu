@@ -48,6 +48,7 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include "af1.h"
 #include "af1_internal.h"
 #include "af1_layout.h"
 
@@ -895,9 +896,11 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
   for (int64_t t0 = 0; t0 < tokens; t0 += pass) {
     const int T = (int)((tokens - t0) < pass ? (tokens - t0) : pass);
     // Passes run on the CUDA cores (af1_lut.cu) whenever that kernel has a
-    // plan; the tensor-core kernel is the fallback.
-    const LutPlan l1 = plan_lut(L.p1, T, L.num_sms, L.max_smem);
-    const LutPlan l2 = plan_lut(L.p2, T, L.num_sms, L.max_smem);
+    // plan, unless the layer asks for the tensor-core kernel, which is also
+    // the fallback.
+    const bool tc = (L.flags & AF1_FLAG_TC_DECODE) != 0;
+    const LutPlan l1 = tc ? LutPlan() : plan_lut(L.p1, T, L.num_sms, L.max_smem);
+    const LutPlan l2 = tc ? LutPlan() : plan_lut(L.p2, T, L.num_sms, L.max_smem);
     DecodePlan q1, q2;
     if (!l1.ok) q1 = plan_decode(1, L.p1, T, L.num_sms, L.max_smem);
     if (!l2.ok) q2 = plan_decode(2, L.p2, T, L.num_sms, L.max_smem);
