@@ -308,6 +308,15 @@ int64_t af1_workspace_bytes(const af1_layer* layer, int64_t tokens) {
 
 int af1_linear_forward(const af1_layer* layer, const void* x, int64_t ldx, int64_t tokens, void* y, int64_t ldy,
                        int y_dtype, void* workspace, int64_t workspace_bytes, void* stream) {
+  return af1::linear_forward_checked(layer, x, ldx, tokens, y, ldy, y_dtype, workspace, workspace_bytes, stream, true);
+}
+
+}  // extern "C"
+
+namespace af1 {
+
+int linear_forward_checked(const af1_layer* layer, const void* x, int64_t ldx, int64_t tokens, void* y, int64_t ldy,
+                           int y_dtype, void* workspace, int64_t workspace_bytes, void* stream, bool prep) {
   if (layer == nullptr) return fail(AF1_ERR_INVALID_ARG, "layer is NULL");
   if (tokens < 0) return fail(AF1_ERR_INVALID_ARG, "tokens must be >= 0");
   if (y_dtype != AF1_F16 && y_dtype != AF1_F32) return fail(AF1_ERR_INVALID_ARG, "y_dtype must be AF1_F16 or AF1_F32");
@@ -333,14 +342,18 @@ int af1_linear_forward(const af1_layer* layer, const void* x, int64_t ldx, int64
     return fail(AF1_ERR_MISALIGNED, "ldy * element size must be a multiple of 16 bytes");
   if ((reinterpret_cast<uintptr_t>(workspace) & 255) != 0)
     return fail(AF1_ERR_WORKSPACE, "workspace must be 256-byte aligned");
-  const int64_t need = af1::plan_workspace(*layer, tokens).total;
+  const int64_t need = af1::plan_workspace(*layer, tokens, prep).total;
   if (workspace_bytes < need)
     return fail(AF1_ERR_WORKSPACE, "workspace too small: need " + std::to_string(need) + " bytes");
-  e = af1::launch_forward(*layer, x, ldx, tokens, y, ldy, y_dtype, workspace, static_cast<cudaStream_t>(stream));
+  e = af1::launch_forward(*layer, x, ldx, tokens, y, ldy, y_dtype, workspace, static_cast<cudaStream_t>(stream), prep);
   if (e != cudaSuccess) return fail_cuda(e, "forward launch");
   g_err.clear();
   return AF1_OK;
 }
+
+}  // namespace af1
+
+extern "C" {
 
 int af1_workspace_status(void* workspace, void* stream) {
   if (workspace == nullptr) return fail(AF1_ERR_WORKSPACE, "workspace is NULL");

@@ -251,6 +251,12 @@ struct DecodeArgs {
   int64_t ldy;
   int ydtype;
   unsigned* status;
+  // Prepared B operand (passes of more than 4 tokens): tiles of every chunk
+  // (chunk c at c N 128 bytes) and per-(slice, token) {2^-sigma, Q 2^-sigma}
+  // at bstats[slice * kMaxPassTokens + t]; written by bprep_kernel, read by
+  // decode_kernel<..., true>.
+  uint8_t* bbuf;
+  float2* bstats;
 };
 
 struct __align__(8) DecodeHeader {
@@ -391,12 +397,135 @@ __device__ __forceinline__ float4 act4(const uint8_t* act, int rowlen, int t, in
   return z;
 }
 
+// The B operand of one K slice for T tokens (chunks c0 .. c0 + nch - 1,
+// columns from k0), built by 128 threads (bt = 0..127, named barrier 1):
+// per-token power-of-two scale from the slice's max |z'|, four e4m3 terms per
+// value in the 128-byte-swizzled K-major tile layout at Bt (chunk c at
+// c N 128), and per-thread Q partials in qpart[t][bt]. Bt is shared memory in
+// the decode kernel and global memory in the prep kernel. The activations
+// must be readable (after griddepcontrol.wait).
 template <int PHASE, int N>
+__device__ __forceinline__ void build_b(const DecodeArgs& a, int T, int nch, int64_t k0, int bt, uint8_t* act,
+                                        uint8_t* Bt, float* qpart, uint32_t* maxbits, uint64_t* xfull,
+                                        uint32_t* err) {
+  constexpr int STASH = 4;         // activation groups a builder thread keeps in registers
+  constexpr bool STAGED = N > 16;  // staged_acts(N)
+  const int g4 = nch * (kChunkCols / 4);  // groups of 4 columns per token
+  const int ngroups = T * g4;
+  for (int t = 0; t < T; ++t) qpart[t * 128 + bt] = 0.f;  // own column only
+  const int rowlen = a.CPC * kChunkCols;
+  const int kv = (int)min((int64_t)nch * kChunkCols, a.sm.C - k0);  // valid columns of this CTA
+  if (STAGED) {
+    // One bulk copy per token row of its 16-byte-multiple valid prefix; the
+    // few remaining columns with plain loads.
+    constexpr int ESZ = PHASE == 1 ? 2 : 4;
+    const int bulk_cols = ((kv * ESZ) & ~15) / ESZ;
+    if (bt == 0) {
+      const uint32_t bytes = (uint32_t)(bulk_cols * ESZ);
+      if (bytes > 0) {
+        mbar_expect_tx(xfull, bytes * (uint32_t)T);
+        for (int t = 0; t < T; ++t) {
+          const uint8_t* src = PHASE == 1 ? reinterpret_cast<const uint8_t*>(a.x + (int64_t)t * a.ldx + k0)
+                                          : reinterpret_cast<const uint8_t*>(a.zin + (int64_t)t * a.ldz + k0);
+          bulk_g2s(act + (size_t)t * rowlen * ESZ, src, bytes, xfull);
+        }
+      } else {
+        mbar_arrive(xfull);
+      }
+    }
+    for (int i = bt; i < T * 8; i += 128) {
+      const int t = i >> 3, k = bulk_cols + (i & 7);
+      if (k < kv) {
+        if (PHASE == 1)
+          reinterpret_cast<__half*>(act)[(size_t)t * rowlen + k] = __ldcg(a.x + (int64_t)t * a.ldx + k0 + k);
+        else
+          reinterpret_cast<float*>(act)[(size_t)t * rowlen + k] = __ldcg(a.zin + (int64_t)t * a.ldz + k0 + k);
+      }
+    }
+    mbar_wait(xfull, 0, err);
+    builders_sync();  // tail values visible
+  }
+  // z' of group (t, c4): from the staged activations or straight from L2.
+  auto zq = [&](int t, int c4) -> float4 {
+    const int64_t k = k0 + 4 * c4;
+    const float4 z = STAGED ? act4<PHASE>(act, rowlen, t, 4 * c4, kv) : load4<PHASE>(a, t, k);
+    return scale4<PHASE>(a, z, k);
+  };
+  float4 stash[STASH];
+  // Pass 1: maxima of |z'| per token.
+  {
+    int cur_t = -1;
+    float mx = 0.f;
+#pragma unroll
+    for (int i = 0; i < STASH; ++i) stash[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int i = 0, g = bt; g < ngroups; ++i, g += 128) {
+      const int t = g / g4, c4 = g - t * g4;
+      const float4 u = zq(t, c4);
+      if (i < STASH) {
+#pragma unroll
+        for (int j = 0; j < STASH; ++j)
+          if (j == i) stash[j] = u;
+      }
+      if (t != cur_t) {
+        if (cur_t >= 0 && mx > 0.f) atomicMax(&maxbits[cur_t], __float_as_uint(mx));
+        cur_t = t;
+        mx = 0.f;
+      }
+      mx = fmaxf(mx, fmaxf(fmaxf(fabsf(u.x), fabsf(u.y)), fmaxf(fabsf(u.z), fabsf(u.w))));
+    }
+    if (cur_t >= 0 && mx > 0.f) atomicMax(&maxbits[cur_t], __float_as_uint(mx));
+  }
+  builders_sync();
+  // Pass 2: split into 4 e4m3 terms, write B rows 4t + q, and Q partials.
+  {
+    int cur_t = -1;
+    float sc = 0.f, q = 0.f;
+    for (int i = 0, g = bt; g < ngroups; ++i, g += 128) {
+      const int t = g / g4, c4 = g - t * g4;
+      if (t != cur_t) {
+        if (cur_t >= 0) qpart[cur_t * 128 + bt] = q;
+        cur_t = t;
+        q = 0.f;
+        float is_unused;
+        pow2_scale(__uint_as_float(maxbits[t]), &sc, &is_unused);
+      }
+      float4 u;
+      if (i < STASH) {
+        u = stash[0];
+#pragma unroll
+        for (int j = 1; j < STASH; ++j)
+          if (j == i) u = stash[j];
+      } else {
+        u = zq(t, c4);
+      }
+      float4 v = make_float4(u.x * sc, u.y * sc, u.z * sc, u.w * sc);
+      const float4 v0 = v;
+      const int kl = 4 * c4;  // column within the CTA's range
+      const int c = kl >> 7, kin = kl & 127;
+      uint8_t* base = Bt + c * (N * 128) + (kin & 15);
+      const int j16 = kin >> 4;
+#pragma unroll
+      for (int term = 0; term < kTerms; ++term) {
+        const uint32_t lo = e4m3x2(v.x, v.y), hi = e4m3x2(v.z, v.w);
+        const float2 flo = e4m3x2_value(lo), fhi = e4m3x2_value(hi);
+        v.x -= flo.x;
+        v.y -= flo.y;
+        v.z -= fhi.x;
+        v.w -= fhi.y;
+        const int n = 4 * t + term;
+        *reinterpret_cast<uint32_t*>(base + n * 128 + ((j16 ^ (n & 7)) << 4)) = lo | (hi << 16);
+      }
+      q += c_lph[c4 & 7] * (((v0.x - v.x) + (v0.y - v.y)) + ((v0.z - v.z) + (v0.w - v.w)));
+    }
+    if (cur_t >= 0) qpart[cur_t * 128 + bt] = q;
+  }
+}
+
+template <int PHASE, int N, bool PREP>
 __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const DecodeArgs a) {
   constexpr int NACC = nacc_for(N);
   constexpr int NBUF = nbuf_for(N);
   constexpr int DCOL = NBUF * 32;  // first accumulator column
-  constexpr int STASH = 4;         // activation groups a builder thread keeps in registers
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -487,115 +616,17 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const DecodeArgs a)
   } else {
     // ---- B: activations -> e4m3 terms in the swizzled B tile --------------
     const int bt = tid - 128;
-    const int g4 = nch * (kChunkCols / 4);  // groups of 4 columns per token
-    const int ngroups = T * g4;
-    for (int t = 0; t < T; ++t) qpart[t * 128 + bt] = 0.f;  // own column only
     griddep_wait();  // activations are written by the previous kernel
-    const int rowlen = a.CPC * kChunkCols;
-    const int kv = (int)min((int64_t)nch * kChunkCols, a.sm.C - k0);  // valid columns of this CTA
-    if (STAGED) {
-      // One bulk copy per token row of its 16-byte-multiple valid prefix; the
-      // few remaining columns with plain loads.
-      constexpr int ESZ = PHASE == 1 ? 2 : 4;
-      const int bulk_cols = ((kv * ESZ) & ~15) / ESZ;
+    if constexpr (PREP) {
+      // Prepared by bprep_kernel for this K slice: one bulk copy per chunk.
       if (bt == 0) {
-        const uint32_t bytes = (uint32_t)(bulk_cols * ESZ);
-        if (bytes > 0) {
-          mbar_expect_tx(&h.xfull, bytes * (uint32_t)T);
-          for (int t = 0; t < T; ++t) {
-            const uint8_t* src = PHASE == 1 ? reinterpret_cast<const uint8_t*>(a.x + (int64_t)t * a.ldx + k0)
-                                            : reinterpret_cast<const uint8_t*>(a.zin + (int64_t)t * a.ldz + k0);
-            bulk_g2s(act + (size_t)t * rowlen * ESZ, src, bytes, &h.xfull);
-          }
-        } else {
-          mbar_arrive(&h.xfull);
-        }
-      }
-      for (int i = bt; i < T * 8; i += 128) {
-        const int t = i >> 3, k = bulk_cols + (i & 7);
-        if (k < kv) {
-          if (PHASE == 1)
-            reinterpret_cast<__half*>(act)[(size_t)t * rowlen + k] = __ldcg(a.x + (int64_t)t * a.ldx + k0 + k);
-          else
-            reinterpret_cast<float*>(act)[(size_t)t * rowlen + k] = __ldcg(a.zin + (int64_t)t * a.ldz + k0 + k);
-        }
+        mbar_expect_tx(&h.xfull, (uint32_t)(nch * N * 128));
+        for (int c = 0; c < nch; ++c)
+          bulk_g2s(Bt + c * N * 128, a.bbuf + (int64_t)(c0 + c) * N * 128, (uint32_t)(N * 128), &h.xfull);
       }
       mbar_wait(&h.xfull, 0, &h.err);
-      builders_sync();  // tail values visible
-    }
-    // z' of group (t, c4): from the staged activations or straight from L2.
-    auto zq = [&](int t, int c4) -> float4 {
-      const int64_t k = k0 + 4 * c4;
-      const float4 z = STAGED ? act4<PHASE>(act, rowlen, t, 4 * c4, kv) : load4<PHASE>(a, t, k);
-      return scale4<PHASE>(a, z, k);
-    };
-    float4 stash[STASH];
-    // Pass 1: maxima of |z'| per token.
-    {
-      int cur_t = -1;
-      float mx = 0.f;
-#pragma unroll
-      for (int i = 0; i < STASH; ++i) stash[i] = make_float4(0.f, 0.f, 0.f, 0.f);
-      for (int i = 0, g = bt; g < ngroups; ++i, g += 128) {
-        const int t = g / g4, c4 = g - t * g4;
-        const float4 u = zq(t, c4);
-        if (i < STASH) {
-#pragma unroll
-          for (int j = 0; j < STASH; ++j)
-            if (j == i) stash[j] = u;
-        }
-        if (t != cur_t) {
-          if (cur_t >= 0 && mx > 0.f) atomicMax(&h.maxbits[cur_t], __float_as_uint(mx));
-          cur_t = t;
-          mx = 0.f;
-        }
-        mx = fmaxf(mx, fmaxf(fmaxf(fabsf(u.x), fabsf(u.y)), fmaxf(fabsf(u.z), fabsf(u.w))));
-      }
-      if (cur_t >= 0 && mx > 0.f) atomicMax(&h.maxbits[cur_t], __float_as_uint(mx));
-    }
-    builders_sync();
-    // Pass 2: split into 4 e4m3 terms, write B rows 4t + q, and Q partials.
-    {
-      int cur_t = -1;
-      float sc = 0.f, q = 0.f;
-      for (int i = 0, g = bt; g < ngroups; ++i, g += 128) {
-        const int t = g / g4, c4 = g - t * g4;
-        if (t != cur_t) {
-          if (cur_t >= 0) qpart[cur_t * 128 + bt] = q;
-          cur_t = t;
-          q = 0.f;
-          float is_unused;
-          pow2_scale(__uint_as_float(h.maxbits[t]), &sc, &is_unused);
-        }
-        float4 u;
-        if (i < STASH) {
-          u = stash[0];
-#pragma unroll
-          for (int j = 1; j < STASH; ++j)
-            if (j == i) u = stash[j];
-        } else {
-          u = zq(t, c4);
-        }
-        float4 v = make_float4(u.x * sc, u.y * sc, u.z * sc, u.w * sc);
-        const float4 v0 = v;
-        const int kl = 4 * c4;  // column within the CTA's range
-        const int c = kl >> 7, kin = kl & 127;
-        uint8_t* base = Bt + c * (N * 128) + (kin & 15);
-        const int j16 = kin >> 4;
-#pragma unroll
-        for (int term = 0; term < kTerms; ++term) {
-          const uint32_t lo = e4m3x2(v.x, v.y), hi = e4m3x2(v.z, v.w);
-          const float2 flo = e4m3x2_value(lo), fhi = e4m3x2_value(hi);
-          v.x -= flo.x;
-          v.y -= flo.y;
-          v.z -= fhi.x;
-          v.w -= fhi.y;
-          const int n = 4 * t + term;
-          *reinterpret_cast<uint32_t*>(base + n * 128 + ((j16 ^ (n & 7)) << 4)) = lo | (hi << 16);
-        }
-        q += c_lph[c4 & 7] * (((v0.x - v.x) + (v0.y - v.y)) + ((v0.z - v.z) + (v0.w - v.w)));
-      }
-      if (cur_t >= 0) qpart[cur_t * 128 + bt] = q;
+    } else {
+      build_b<PHASE, N>(a, T, nch, k0, bt, act, Bt, qpart, h.maxbits, &h.xfull, &h.err);
     }
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // B is read by the tensor cores
     builders_sync();
@@ -622,12 +653,18 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const DecodeArgs a)
       // ---- per-token 2^-sigma and Q 2^-sigma, summed in a fixed order ------
       const int t = bt - 112;
       if (t < T) {
-        float qs = 0.f;
-        for (int j = 0; j < 128; ++j) qs += qpart[t * 128 + j];
-        float sc, is;
-        pow2_scale(__uint_as_float(h.maxbits[t]), &sc, &is);
-        h.is[t] = is;
-        h.qis[t] = qs * is;
+        if constexpr (PREP) {
+          const float2 st = __ldcg(a.bstats + ks * kMaxPassTokens + t);
+          h.is[t] = st.x;
+          h.qis[t] = st.y;
+        } else {
+          float qs = 0.f;
+          for (int j = 0; j < 128; ++j) qs += qpart[t * 128 + j];
+          float sc, is;
+          pow2_scale(__uint_as_float(h.maxbits[t]), &sc, &is);
+          h.is[t] = is;
+          h.qis[t] = qs * is;
+        }
       }
       mbar_arrive(&h.stats);
     }
@@ -695,7 +732,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const DecodeArgs a)
     // Something timed out: let the bulk copies drain (bounded) so that none
     // lands after the CTA has exited, and report it.
     for (int c = 0; c < nch; ++c) mbar_wait(&h.wfull[c], 0, &h.err);
-    if (STAGED) mbar_wait(&h.xfull, 0, &h.err);
+    if (STAGED || PREP) mbar_wait(&h.xfull, 0, &h.err);
     atomicOr(a.status, kStatusTimeout);
   }
   if (warp == 4) {
@@ -704,6 +741,80 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const DecodeArgs a)
     __syncwarp();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"((uint32_t)kTmemCols)
                  : "memory");
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Prep kernel: the B operand of every K slice of a pass, built once per slice
+// instead of once per row block (the split of a pass of T tokens into 4T
+// e4m3 terms costs about 40 instructions per value and grows with T, while
+// the decode CTAs of one slice all need the same tiles). CTA ks = slice ks,
+// 128 threads.
+// ---------------------------------------------------------------------------
+
+struct __align__(8) PrepHeader {
+  uint64_t xfull;  // staged activations have landed (bulk copies)
+  uint32_t err;
+  uint32_t maxbits[kMaxPassTokens];
+};
+
+struct PrepSmem {
+  int act, qpart, hdr, total;
+};
+
+__host__ __device__ inline PrepSmem prep_smem(int phase, int CPC, int T) {
+  PrepSmem p;
+  int off = 0;
+  p.act = off;
+  off = align128(off + T * CPC * kChunkCols * (phase == 1 ? 2 : 4));
+  p.qpart = off;
+  off = align128(off + T * 128 * 4);
+  p.hdr = off;
+  off = align128(off + (int)sizeof(PrepHeader));
+  p.total = off + 128;  // slack for aligning the base to 128 bytes
+  return p;
+}
+
+template <int PHASE, int N>
+__global__ void __launch_bounds__(128) bprep_kernel(const DecodeArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 127) & ~(uintptr_t)127);
+  const int T = a.tokens;
+  const PrepSmem sp = prep_smem(PHASE, a.CPC, T);
+  uint8_t* act = smem + sp.act;
+  float* qpart = reinterpret_cast<float*>(smem + sp.qpart);
+  PrepHeader& h = *reinterpret_cast<PrepHeader*>(smem + sp.hdr);
+  const int bt = threadIdx.x, ks = blockIdx.x;
+  const int c0 = ks * a.CPC;
+  const int nch = min(a.CPC, a.sm.NCH - c0);
+  const int64_t k0 = (int64_t)c0 * kChunkCols;
+  if (bt == 0) {
+    mbar_init(&h.xfull, 1);
+    h.err = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (bt < kMaxPassTokens) h.maxbits[bt] = 0u;
+  __syncthreads();
+  // The decode kernel that consumes the tiles starts now: its sign copies and
+  // expansion into tensor memory do not depend on this kernel.
+  griddep_launch_dependents();
+  griddep_wait();  // activations are written by the previous kernel
+  build_b<PHASE, N>(a, T, nch, k0, bt, act, a.bbuf + (int64_t)c0 * N * 128, qpart, h.maxbits, &h.xfull, &h.err);
+  builders_sync();
+  if (bt < T) {
+    float qs = 0.f;
+    for (int j = 0; j < 128; ++j) qs += qpart[bt * 128 + j];
+    float sc, is;
+    pow2_scale(__uint_as_float(h.maxbits[bt]), &sc, &is);
+    a.bstats[ks * kMaxPassTokens + bt] = make_float2(is, qs * is);
+  }
+  // The tiles are read by bulk copies (async proxy) in the next kernel.
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+  __syncthreads();
+  if (bt == 0 && h.err != 0) {
+    if (staged_acts(N)) mbar_wait(&h.xfull, 0, &h.err);
+    atomicOr(a.status, kStatusTimeout);
   }
 }
 
@@ -717,6 +828,14 @@ struct DecodePlan {
 };
 
 int n_for_tokens(int T) { return T <= 4 ? 16 : T <= 8 ? 32 : 64; }
+
+// Passes of at least kTcMinTokens tokens over a sign matrix of at least
+// kTcMinSigns signs use the tensor-core kernel with a prepared B operand when
+// the workspace holds it (measured at 8 and 16 tokens: faster from about
+// 30 M signs per phase, e.g. 8192x28672 at 8 tokens 170 -> 96 us, 14336x4096
+// at 16 tokens 57.8 -> 50.2 us; slower on 4096^2, 33.7 vs 22.2 us at 16).
+constexpr int kTcMinTokens = 8;
+constexpr int64_t kTcMinSigns = 16 << 20;
 
 constexpr int kTwoPerSmSmem = 110 * 1024;  // at or below this, two CTAs share an SM
 
@@ -793,8 +912,31 @@ DecodePlan plan_decode(int phase, const SignMatrix& sm, int T, int num_sms, int 
 }
 
 template <int PHASE, int N>
+cudaError_t launch_prep(const DecodeArgs& a, const DecodePlan& p, cudaStream_t st) {
+  auto kern = bprep_kernel<PHASE, N>;
+  const int smem = prep_smem(PHASE, p.CPC, a.tokens).total;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)p.KS, 1, 1);
+  cfg.blockDim = dim3(128, 1, 1);
+  cfg.dynamicSmemBytes = (size_t)smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, a);
+}
+
+template <int PHASE, int N, bool PREP>
 cudaError_t launch_decode_n(const DecodeArgs& a, const DecodePlan& p, cudaStream_t st) {
-  auto kern = decode_kernel<PHASE, N>;
+  if (PREP) {
+    cudaError_t e = launch_prep<PHASE, N>(a, p, st);
+    if (e != cudaSuccess) return e;
+  }
+  auto kern = decode_kernel<PHASE, N, PREP>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, p.smem);
   if (e != cudaSuccess) return e;
   if (p.KS > 8) {
@@ -818,14 +960,17 @@ cudaError_t launch_decode_n(const DecodeArgs& a, const DecodePlan& p, cudaStream
   return cudaLaunchKernelEx(&cfg, kern, a);
 }
 
+// Passes of more than 4 tokens (N > 16) build the B operand once per K slice
+// in bprep_kernel when the caller's workspace holds the tiles (a.bbuf set).
 template <int PHASE>
 cudaError_t launch_decode(DecodeArgs a, const DecodePlan& p, cudaStream_t st) {
   a.KS = p.KS;
   a.CPC = p.CPC;
+  const bool prep = a.bbuf != nullptr && p.N > 16;
   switch (p.N) {
-    case 16: return launch_decode_n<PHASE, 16>(a, p, st);
-    case 32: return launch_decode_n<PHASE, 32>(a, p, st);
-    default: return launch_decode_n<PHASE, 64>(a, p, st);
+    case 16: return launch_decode_n<PHASE, 16, false>(a, p, st);
+    case 32: return prep ? launch_decode_n<PHASE, 32, true>(a, p, st) : launch_decode_n<PHASE, 32, false>(a, p, st);
+    default: return prep ? launch_decode_n<PHASE, 64, true>(a, p, st) : launch_decode_n<PHASE, 64, false>(a, p, st);
   }
 }
 
@@ -855,13 +1000,22 @@ LutArgs lut_args(const DecodeArgs& d) {
 
 int64_t decode_ldz(const af1_layer& L) { return (int64_t)L.p2.NCH * kChunkCols; }
 
-Workspace plan_workspace(const af1_layer& L, int64_t tokens) {
+Workspace plan_workspace(const af1_layer& L, int64_t tokens, bool prep) {
   Workspace w;
   int64_t off = 0;
   w.status = off;
   off += 256;
   w.sbuf = off;
   off += align256((int64_t)kMaxPassTokens * decode_ldz(L) * 4);
+  if (prep && tokens > 4 && tokens <= kMaxPassTokens) {
+    // Prepared B operand of the wider decode passes: every chunk's tiles at
+    // the widest N (64 rows of 128 bytes) and the per-(slice, token) scales.
+    const int nch = L.p1.NCH > L.p2.NCH ? L.p1.NCH : L.p2.NCH;
+    w.bbuf = off;
+    off += align256((int64_t)nch * 64 * 128);
+    w.bstats = off;
+    off += align256((int64_t)kMaxKS * kMaxPassTokens * 8);
+  }
   w.hbuf = off;
   if (tokens > kMaxPassTokens) {
     const int64_t t = tokens < kPrefillPassTokens ? tokens : kPrefillPassTokens;
@@ -872,8 +1026,8 @@ Workspace plan_workspace(const af1_layer& L, int64_t tokens) {
 }
 
 cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64_t tokens, void* y,
-                           int64_t ldy, int y_dtype, void* ws, cudaStream_t st) {
-  const Workspace W = plan_workspace(L, tokens);
+                           int64_t ldy, int y_dtype, void* ws, cudaStream_t st, bool prep) {
+  const Workspace W = plan_workspace(L, tokens, prep);
   uint8_t* wsb = static_cast<uint8_t*>(ws);
   if (tokens > kMaxPassTokens) {
     // Prefill: two tensor-core GEMMs per pass (af1_prefill.cu).
@@ -895,12 +1049,17 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
   const int ysize = y_dtype == 0 ? 2 : 4;
   for (int64_t t0 = 0; t0 < tokens; t0 += pass) {
     const int T = (int)((tokens - t0) < pass ? (tokens - t0) : pass);
-    // Passes run on the CUDA cores (af1_lut.cu) whenever that kernel has a
-    // plan, unless the layer asks for the tensor-core kernel, which is also
-    // the fallback.
-    const bool tc = (L.flags & AF1_FLAG_TC_DECODE) != 0;
-    const LutPlan l1 = tc ? LutPlan() : plan_lut(L.p1, T, L.num_sms, L.max_smem);
-    const LutPlan l2 = tc ? LutPlan() : plan_lut(L.p2, T, L.num_sms, L.max_smem);
+    // A phase runs on the CUDA cores (af1_lut.cu) whenever that kernel has a
+    // plan, unless the layer asks for the tensor-core kernel (which is also
+    // the fallback) or the pass is wide and the matrix large enough for the
+    // tensor-core kernel with a prepared B operand to be faster.
+    const bool flag = (L.flags & AF1_FLAG_TC_DECODE) != 0;
+    auto wide_tc = [&](const SignMatrix& m) {
+      return W.bbuf != 0 && T >= kTcMinTokens && m.R * m.C >= kTcMinSigns;
+    };
+    const bool tc1 = flag || wide_tc(L.p1), tc2 = flag || wide_tc(L.p2);
+    const LutPlan l1 = tc1 ? LutPlan() : plan_lut(L.p1, T, L.num_sms, L.max_smem);
+    const LutPlan l2 = tc2 ? LutPlan() : plan_lut(L.p2, T, L.num_sms, L.max_smem);
     DecodePlan q1, q2;
     if (!l1.ok) q1 = plan_decode(1, L.p1, T, L.num_sms, L.max_smem);
     if (!l2.ok) q2 = plan_decode(2, L.p2, T, L.num_sms, L.max_smem);
@@ -917,6 +1076,8 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
     a1.sout = reinterpret_cast<float*>(wsb + W.sbuf);
     a1.lds = decode_ldz(L);
     a1.status = reinterpret_cast<unsigned*>(wsb + W.status);
+    a1.bbuf = W.bbuf != 0 ? wsb + W.bbuf : nullptr;
+    a1.bstats = W.bbuf != 0 ? reinterpret_cast<float2*>(wsb + W.bstats) : nullptr;
     cudaError_t e = l1.ok ? launch_lut(1, lut_args(a1), l1, st) : launch_decode<1>(a1, q1, st);
     if (e != cudaSuccess) return e;
 
@@ -931,6 +1092,8 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
     a2.ldy = ldy;
     a2.ydtype = y_dtype;
     a2.status = a1.status;
+    a2.bbuf = a1.bbuf;
+    a2.bstats = a1.bstats;
     e = l2.ok ? launch_lut(2, lut_args(a2), l2, st) : launch_decode<2>(a2, q2, st);
     if (e != cudaSuccess) return e;
   }

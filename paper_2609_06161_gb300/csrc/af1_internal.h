@@ -37,10 +37,13 @@ constexpr int64_t kPrefillPassTokens = 2048;
 struct Workspace {
   int64_t status = 0;  // uint32 status word
   int64_t sbuf = 0;    // float[kMaxPassTokens][decode_ldz]: s' = s * t (decode)
+  int64_t bbuf = 0;    // prepared B tiles of decode passes of 5..16 tokens (0: none)
+  int64_t bstats = 0;  // float2 [16 slices][16 tokens] of the prepared B (0: none)
   int64_t hbuf = 0;    // FP16 [min(tokens, kPrefillPassTokens)][prefill_h_ld]: H (prefill)
   int64_t total = 0;
 };
-Workspace plan_workspace(const af1_layer& L, int64_t tokens);
+// prep = false leaves out the prepared-B region (and so never uses it).
+Workspace plan_workspace(const af1_layer& L, int64_t tokens, bool prep = true);
 int64_t prefill_h_ld(const af1_layer& L);
 int64_t decode_ldz(const af1_layer& L);
 
@@ -84,6 +87,10 @@ cudaError_t launch_lut(int phase, const LutArgs& a, const LutPlan& p, cudaStream
 cudaError_t launch_prefill(const af1_layer& L, const void* x, int64_t ldx, int64_t tokens, void* y, int64_t ldy,
                            int y_dtype, uint8_t* h_buf, unsigned* status, cudaStream_t st);
 cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64_t tokens, void* y,
-                           int64_t ldy, int y_dtype, void* ws, cudaStream_t st);
+                           int64_t ldy, int y_dtype, void* ws, cudaStream_t st, bool prep = true);
+// af1_linear_forward with all its argument checks; prep = false never uses
+// (and does not require) the prepared-B region of the workspace.
+int linear_forward_checked(const af1_layer* layer, const void* x, int64_t ldx, int64_t tokens, void* y, int64_t ldy,
+                           int y_dtype, void* workspace, int64_t workspace_bytes, void* stream, bool prep);
 
 }  // namespace af1

@@ -54,7 +54,7 @@ int af1_linear_forward_static(const af1_layer* layer, const void* x, int64_t ldx
   if (tokens < 0) return fail(AF1_ERR_INVALID_ARG, "tokens must be >= 0");
   if (y_dtype != AF1_F16 && y_dtype != AF1_F32) return fail(AF1_ERR_INVALID_ARG, "y_dtype must be AF1_F16 or AF1_F32");
   if (tokens == 0) return AF1_OK;
-  const int64_t need = af1::plan_workspace(*layer, tokens).total;
+  const int64_t need = af1::plan_workspace(*layer, tokens, false).total;
   if (need > kStaticScratchBytes)
     return fail(AF1_ERR_WORKSPACE, "layer needs " + std::to_string(need) + " bytes of scratch; the built-in array holds " +
                                        std::to_string(kStaticScratchBytes));
@@ -66,8 +66,10 @@ int af1_linear_forward_static(const af1_layer* layer, const void* x, int64_t ldx
   int rc = scratch_address(dev, &scratch);
   if (rc != AF1_OK) return rc;
   // Same argument checks and kernels as af1_linear_forward, with the
-  // built-in array as the workspace.
-  return af1_linear_forward(layer, x, ldx, tokens, y, ldy, y_dtype, scratch, kStaticScratchBytes, stream);
+  // built-in array as the workspace (without its prepared-B region: wide
+  // decode passes build their B operand in every CTA instead).
+  return af1::linear_forward_checked(layer, x, ldx, tokens, y, ldy, y_dtype, scratch, kStaticScratchBytes, stream,
+                                     false);
 }
 
 }  // extern "C"
