@@ -282,7 +282,8 @@ __host__ __device__ inline int slice_rows(int KS) { return (kBlockRows + KS - 1)
 // with bulk copies (one per token row) before splitting them.
 __host__ __device__ inline bool staged_acts(int N) { return N > 16; }
 
-__host__ __device__ inline DecodeSmem decode_smem(int phase, int N, int CPC, int KS, int T) {
+// prep: the B operand is prepared (bprep_kernel), so no activations are staged.
+__host__ __device__ inline DecodeSmem decode_smem(int phase, int N, int CPC, int KS, int T, bool prep) {
   DecodeSmem p;
   int off = 0;
   p.bt = off;
@@ -290,7 +291,7 @@ __host__ __device__ inline DecodeSmem decode_smem(int phase, int N, int CPC, int
   p.w = off;
   off += kChunkBytes * CPC;
   p.act = off;  // T rows of CPC * 128 activations (FP16 phase 1, FP32 phase 2)
-  if (staged_acts(N)) off += T * CPC * kChunkCols * (phase == 1 ? 2 : 4);
+  if (staged_acts(N) && !prep) off += T * CPC * kChunkCols * (phase == 1 ? 2 : 4);
   p.recv = off;
   off = align128(off + KS * T * slice_rows(KS) * 4);
   p.qpart = off;
@@ -531,7 +532,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const DecodeArgs a)
   uint8_t* smem = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   const int T = a.tokens;
   const int KS = a.KS;
-  const DecodeSmem sp = decode_smem(PHASE, N, a.CPC, KS, T);
+  const DecodeSmem sp = decode_smem(PHASE, N, a.CPC, KS, T, PREP);
   constexpr bool STAGED = N > 16;  // staged_acts(N)
   uint8_t* act = smem + sp.act;
   uint8_t* Bt = smem + sp.bt;
@@ -849,7 +850,7 @@ constexpr int kTwoPerSmSmem = 110 * 1024;  // at or below this, two CTAs share a
 // CTA streams more chunks than its A ring holds, K is split twice as finely
 // (portable clusters, at most two CTAs per SM; 14336x4096 at one token
 // 20.9 -> 15.2 us).
-DecodePlan plan_decode(int phase, const SignMatrix& sm, int T, int num_sms, int max_smem) {
+DecodePlan plan_decode(int phase, const SignMatrix& sm, int T, int num_sms, int max_smem, bool prep) {
   DecodePlan p;
   p.N = n_for_tokens(T);
   const int sms = num_sms > 0 ? num_sms : 148;
@@ -871,7 +872,7 @@ DecodePlan plan_decode(int phase, const SignMatrix& sm, int T, int num_sms, int 
     const int cpc = (sm.NCH + ks - 1) / ks;
     if (cpc > kMaxCPC) continue;
     const int KS = (sm.NCH + cpc - 1) / cpc;
-    const int need = decode_smem(phase, p.N, cpc, KS, T).total;
+    const int need = decode_smem(phase, p.N, cpc, KS, T, prep).total;
     if (need <= max_smem) {
       p.KS = KS;
       p.CPC = cpc;
@@ -881,14 +882,16 @@ DecodePlan plan_decode(int phase, const SignMatrix& sm, int T, int num_sms, int 
         for (int k2 = ks + 1; k2 <= kMaxKS && k2 <= sm.NCH; ++k2) {
           const int c2 = (sm.NCH + k2 - 1) / k2;
           const int K2 = (sm.NCH + c2 - 1) / c2;
-          const int n2 = decode_smem(phase, p.N, c2, K2, T).total;
+          const int n2 = decode_smem(phase, p.N, c2, K2, T, prep).total;
           if (n2 <= kTwoPerSmSmem) {
-            if (waves(K2, n2) * c2 < waves(KS, need) * cpc) {
+            if (waves(K2, n2) * c2 < waves(p.KS, p.smem) * p.CPC) {
               p.KS = K2;
               p.CPC = c2;
               p.smem = n2 < kMinSmem ? kMinSmem : n2;
             }
-            break;
+            // Passes of one to four tokens take the first such split; wider
+            // ones (fewer chunks fit) search every finer split.
+            if (p.N <= 16) break;
           }
         }
       }
@@ -899,7 +902,7 @@ DecodePlan plan_decode(int phase, const SignMatrix& sm, int T, int num_sms, int 
         const int k2 = p.KS * 2;
         const int c2 = (sm.NCH + k2 - 1) / k2;
         const int K2 = (sm.NCH + c2 - 1) / c2;
-        const int n2 = decode_smem(phase, p.N, c2, K2, T).total;
+        const int n2 = decode_smem(phase, p.N, c2, K2, T, prep).total;
         if (n2 > max_smem) break;
         p.KS = K2;
         p.CPC = c2;
@@ -1040,8 +1043,8 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
   DecodePlan p1, p2;
   for (;;) {
     const int T = (int)(tokens < pass ? tokens : pass);
-    p1 = plan_decode(1, L.p1, T, L.num_sms, L.max_smem);
-    p2 = plan_decode(2, L.p2, T, L.num_sms, L.max_smem);
+    p1 = plan_decode(1, L.p1, T, L.num_sms, L.max_smem, false);
+    p2 = plan_decode(2, L.p2, T, L.num_sms, L.max_smem, false);
     if ((p1.ok && p2.ok) || pass <= 4) break;
     pass /= 2;
   }
@@ -1061,8 +1064,9 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
     const LutPlan l1 = tc1 ? LutPlan() : plan_lut(L.p1, T, L.num_sms, L.max_smem);
     const LutPlan l2 = tc2 ? LutPlan() : plan_lut(L.p2, T, L.num_sms, L.max_smem);
     DecodePlan q1, q2;
-    if (!l1.ok) q1 = plan_decode(1, L.p1, T, L.num_sms, L.max_smem);
-    if (!l2.ok) q2 = plan_decode(2, L.p2, T, L.num_sms, L.max_smem);
+    const bool prep = W.bbuf != 0 && n_for_tokens(T) > 16;  // launch_decode prepares B then
+    if (!l1.ok) q1 = plan_decode(1, L.p1, T, L.num_sms, L.max_smem, prep);
+    if (!l2.ok) q2 = plan_decode(2, L.p2, T, L.num_sms, L.max_smem, prep);
     if ((!l1.ok && !q1.ok) || (!l2.ok && !q2.ok)) return cudaErrorInvalidConfiguration;
 
     DecodeArgs a1 = {};
