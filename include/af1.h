@@ -173,6 +173,9 @@ AF1_API int af1_linear_forward(const af1_layer* layer, const void* x, int64_t ld
  * rejected with AF1_ERR_WORKSPACE: with up to 16 tokens every shape with
  * r <= 16256 fits; longer calls also hold min(tokens, 2048) x r FP16 rank
  * intermediates, so they fit only for short passes of small-rank layers.
+ * Passes of 8-16 tokens over large sign matrices run here without the
+ * prepared tensor-core operand that af1_linear_forward keeps in its
+ * workspace (the CUDA-core kernel takes them), so they can be slower.
  * The first call on a device looks up the array's device address (once per
  * device); make that first call before any stream capture. All calls share
  * the array and leave their intermediate results in it, so calls that may
