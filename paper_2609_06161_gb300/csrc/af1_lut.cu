@@ -104,13 +104,16 @@ __device__ __forceinline__ void cluster_arrive_relaxed() {
   asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
 }
 __device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.aligned;" ::: "memory"); }
-__device__ __forceinline__ void cluster_sync() {
-  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
-}
-__device__ __forceinline__ void st_cluster_f32(float* local, uint32_t rank, float v) {
-  uint32_t remote;
-  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(local)), "r"(rank));
-  asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(remote), "f"(v) : "memory");
+
+// v -> `local` in the shared memory of cluster CTA `rank`, completing 4
+// bytes of the transaction count of that CTA's mbarrier `bar`.
+__device__ __forceinline__ void st_async_f32(float* local, uint64_t* bar, uint32_t rank, float v) {
+  uint32_t raddr, rbar;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(raddr) : "r"(smem_u32(local)), "r"(rank));
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(rbar) : "r"(smem_u32(bar)), "r"(rank));
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.f32 [%0], %1, [%2];" ::"r"(raddr), "f"(v),
+               "r"(rbar)
+               : "memory");
 }
 __device__ __forceinline__ float lds_f32(uint32_t addr) {
   float v;
@@ -139,6 +142,7 @@ __host__ __device__ inline int slice_rows(int KS) { return (kBlockRows + KS - 1)
 __host__ __device__ inline int align128(int v) { return (v + 127) & ~127; }
 
 struct __align__(8) LutHeader {
+  uint64_t red;             // all partial sums for this CTA's rows have landed (st.async)
   uint64_t wfull[kMaxCPC];  // packed chunk c has landed
   uint32_t err;
 };
@@ -229,10 +233,14 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const LutArgs a) {
   const int my0 = ks * slice;  // first block row this CTA finalises
   const int zrow = zrow_floats(CPC);
 
-  cluster_arrive_relaxed();  // matched by cluster_wait before the first remote store
+  const int cnt = min(slice, kBlockRows - my0);  // rows this CTA finalises (may be <= 0)
 
   if (tid == 0) {
     for (int c = 0; c < nch; ++c) mbar_init(&h.wfull[c], 1);
+    // The partial sums of this CTA's rows arrive by st.async from the 2 KS
+    // word halves of the cluster, 4 bytes per row and token each.
+    mbar_init(&h.red, 1);
+    mbar_expect_tx(&h.red, cnt > 0 ? (uint32_t)(2 * KS * T * cnt * 4) : 0u);
     h.err = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -242,6 +250,9 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const LutArgs a) {
       bulk_g2s(smem + sp.w + c * kChunkBytes, src + (int64_t)c * kChunkBytes, kChunkBytes, &h.wfull[c]);
     }
   }
+  // Matched by cluster_wait before the first remote store: a peer's barrier
+  // and expected byte count are set up before any partial can reach it.
+  cluster_arrive_relaxed();
   // Row scale of row my0 + tid of the block (a layer constant): loaded now,
   // stored to shared memory once the activations are staged.
   const float rs_own = (tid < slice && my0 + tid < kBlockRows && row0 + my0 + tid < a.sm.R)
@@ -403,10 +414,12 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const LutArgs a) {
     const int src = ks * 2 + g;
 #pragma unroll
     for (int t = 0; t < NACC; ++t)
-      if (t < T) st_cluster_f32(recv + ((src * T + t) * slice + (r - owner * slice)), (uint32_t)owner, acc[t]);
+      if (t < T) st_async_f32(recv + ((src * T + t) * slice + (r - owner * slice)), &h.red, (uint32_t)owner, acc[t]);
   }
-  cluster_sync();  // all partials of the cluster have landed in their owners' buffers
-  const int cnt = min(slice, kBlockRows - my0);
+  // Exit barrier (waited for after the final sums): no CTA leaves while a
+  // peer may still store into it.
+  cluster_arrive_relaxed();
+  mbar_wait(&h.red, 0, &h.err);  // this CTA's partials have all landed
   for (int idx = tid; idx < T * cnt; idx += kThreads) {
     const int t = idx / cnt;
     const int i = idx - t * cnt;
@@ -435,6 +448,8 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const LutArgs a) {
       reinterpret_cast<float*>(a.y)[(int64_t)(tg0 + t) * a.ldy + row] = out;
     }
   }
+
+  cluster_wait();
 
   // ---- teardown ---------------------------------------------------------------
   __syncthreads();
