@@ -54,9 +54,10 @@ def parse():
                    help="decode: config 1 (1-16 tokens); prefill: config 2 (2048 tokens, tensor cores)")
     p.add_argument("--tokens", type=int, default=2048, help="prefill tokens per call")
     p.add_argument("--no-graph", action="store_true", help="eager launches instead of a CUDA graph (for profilers)")
-    p.add_argument("--schedule", choices=["dag", "serial"], default="dag",
+    p.add_argument("--schedule", choices=["dag", "serial", "group"], default="dag",
                    help="dag: a decoder layer's independent linears (q/k/v, gate/up) on parallel streams; "
-                        "serial: all 7 linears chained on one stream")
+                        "serial: all 7 linears chained on one stream; group: q|k|v and gate|up as one "
+                        "af1_linear_forward_multi call each (shared input), one stream")
     p.add_argument("--no-sweep", action="store_true",
                    help="skip the per-shape sweep (LLaMA-3-8B at 1/4/16 tokens, 70B shapes at 1/8/64/512)")
     p.add_argument("--no-stack", action="store_true", help="skip the 32-layer stack with HiSA-like ranks")
@@ -198,8 +199,10 @@ def config_dict(args):
                 "l2": "inputs larger than L2 (weights + activations per step >> 129 MB), no flush"}
     return {"workload": (f"LLaMA-3-8B-shaped AF1 decoder linears (q,k,v,o 4096x4096 r2028 / k,v 1024x4096 r800 / "
                          f"gate,up 14336x4096 r3167 / down 4096x14336 r3167) x {args.layers} layers, decode batch "
-                         f"{args.batch}, " + ("q|k|v and gate|up on parallel streams (decoder dependency DAG)"
-                                               if args.schedule == "dag" else "one stream in model order")
+                         f"{args.batch}, " + {"dag": "q|k|v and gate|up on parallel streams (decoder dependency DAG)",
+                                              "group": "q|k|v and gate|up each as one multi-layer call (shared "
+                                                       "input), one stream",
+                                              "serial": "one stream in model order"}[args.schedule]
                          + ("" if args.no_graph else ", CUDA graph")),
             "batch": args.batch, "layers": args.layers, "linears_per_step": 7 * args.layers,
             "decode_kernel": ("tensor cores (AF1_FLAG_TC_DECODE)" if args.tc_decode
@@ -385,6 +388,37 @@ def sweep(P, torch, peaks, stream):
     return out
 
 
+TC_MIN_TOKENS, TC_MIN_SIGNS = 8, 16 << 20  # the library's rule for the prepared tensor-core decode
+
+
+def phase_launches(m, n, r, b):
+    """Kernel launches of one decode call (b <= 16 tokens) per the library's
+    dispatch: a phase on the lookup-table kernel is one launch, a phase on the
+    tensor-core kernel with a prepared B operand is two (prep + decode)."""
+    if TC_DECODE:
+        return sum(2 if b > 4 else 1 for _ in (0, 1))
+    wide = b >= TC_MIN_TOKENS
+    return sum(2 if wide and R * C >= TC_MIN_SIGNS else 1 for (R, C) in ((r, n), (m, r)))
+
+
+def step_launches(objs, b, schedule):
+    """Kernel launches of one decode step of 7-linear layers."""
+    total = 0
+    for li in range(len(objs) // 7):
+        lay = objs[7 * li:7 * li + 7]
+        calls = [phase_launches(m, n, r, b) for (_nm, m, n, r, _L, _x) in lay]
+        if schedule == "group":
+            for grp in ((0, 1, 2), (4, 5)):
+                if all(calls[i] == 2 for i in grp):  # every phase on the lookup-table kernel: one launch per phase
+                    total += 2
+                else:
+                    total += sum(calls[i] for i in grp)
+            total += calls[3] + calls[6]
+        else:
+            total += sum(calls)
+    return total
+
+
 def dag_step(torch, views, stream, side, ws, ws_side):
     """One decode step over views = [(layer, x, y)] * 7 per decoder layer on
     the decoder's dependency DAG: per layer q | k | v in parallel, then o, then
@@ -520,6 +554,23 @@ def main():
     def step_dag():
         dag_step(torch, views, stream, side, ws, ws_side)
 
+    ws_multi = None
+    if len(views) % 7 == 0:
+        nbytes = max(max(P.workspace_bytes_multi([views[7 * li + j][0] for j in (0, 1, 2)], b),
+                         P.workspace_bytes_multi([views[7 * li + j][0] for j in (4, 5)], b))
+                     for li in range(len(views) // 7))
+        ws_multi = torch.zeros(nbytes, dtype=torch.uint8, device=dev)
+
+    def step_group():
+        # q, k, v read one input and gate, up another (the decoder's shared
+        # activations): one multi-layer call each.
+        for li in range(len(views) // 7):
+            q, k, v, o, gate, up, down = views[7 * li:7 * li + 7]
+            P.forward_multi([q[0], k[0], v[0]], q[1], [q[2], k[2], v[2]], ws_multi, stream=stream)
+            o[0].forward_into(o[1], o[2], ws, stream=stream)
+            P.forward_multi([gate[0], up[0]], gate[1], [gate[2], up[2]], ws_multi, stream=stream)
+            down[0].forward_into(down[1], down[2], ws, stream=stream)
+
     def make_graph(fn):
         with torch.cuda.stream(stream):
             fn()
@@ -536,7 +587,8 @@ def main():
         torch.cuda.synchronize()
         return g
 
-    step = step_dag if (args.schedule == "dag" and len(views) % 7 == 0) else step_serial
+    steps_by_name = {"dag": step_dag, "group": step_group, "serial": step_serial}
+    step = steps_by_name[args.schedule] if len(views) % 7 == 0 else step_serial
     graph = make_graph(step)
 
     def barrier():
@@ -572,22 +624,27 @@ def main():
     alg = sum(algorithmic_bytes(m, n, r, b) for (name, m, n, r, layer, x) in objs)
     achieved_gbs = alg / (ms_step * 1e-3) / 1e9
 
-    serial = None
-    if step is step_dag:
-        g2 = make_graph(step_serial)
-        for _ in range(3):
-            g2.replay()
-        torch.cuda.synchronize()
-        f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        f0.record(stream)
-        with torch.cuda.stream(stream):
-            for _ in range(args.steps):
+    # The same step on the other schedules (outside the headline's timing).
+    others = {}
+    if len(views) % 7 == 0 and args.workload == "decode":
+        for name, fn in steps_by_name.items():
+            if name == args.schedule:
+                continue
+            g2 = make_graph(fn)
+            for _ in range(3):
                 g2.replay()
-        f1.record(stream)
-        torch.cuda.synchronize()
-        sms = f0.elapsed_time(f1) / args.steps
-        serial = {"ms_per_step": sms, "us_per_layer": sms * 1e3 / len(views), "tokens_per_s": b / (sms * 1e-3)}
-        del g2
+            torch.cuda.synchronize()
+            f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            f0.record(stream)
+            with torch.cuda.stream(stream):
+                for _ in range(args.steps):
+                    g2.replay()
+            f1.record(stream)
+            torch.cuda.synchronize()
+            sms = f0.elapsed_time(f1) / args.steps
+            others[name] = {"ms_per_step": sms, "us_per_layer": sms * 1e3 / len(views), "tokens_per_s": b / (sms * 1e-3)}
+            del g2
+    serial = others.get("serial")
 
     # e2e: host buffers in pinned memory, copies inside the timed region.
     xh = torch.empty(xo, dtype=torch.float16, pin_memory=True)
@@ -658,13 +715,16 @@ def main():
             "roofline": roof,
             "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": xo * 2,
                     "d2h_bytes_per_step": yo * 2},
-            "gpu_launches": 2 * nlin * args.steps,
+            "gpu_launches": (step_launches(objs, b, args.schedule) if args.workload == "decode" and nlin % 7 == 0
+                             else 2 * nlin) * args.steps,
             "clocks": clk,
         }
         if dense is not None:
             line["dense_bf16_baseline"] = dense
         if serial is not None:
             line["serial_chain"] = serial
+        if others:
+            line["other_schedules"] = others
         if stack is not None:
             line["stack_hisa"] = stack
         if sweep_rows is not None:

@@ -161,6 +161,27 @@ AF1_API int af1_linear_forward(const af1_layer* layer, const void* x, int64_t ld
                        void* y, int64_t ldy, int y_dtype, void* workspace,
                        int64_t workspace_bytes, void* stream);
 
+/* Several layers applied to the same input, e.g. the q, k and v projections
+ * of a decoder layer (or gate and up): y_i = x . W_hat_i^T for i < count.
+ * The paper has no counterpart; it is the batching of a decoder layer's
+ * V-contractions that share x. Decode passes (up to 16 tokens) run as one
+ * launch per phase for all layers when every phase of every layer would use
+ * the CUDA-core decode kernel; otherwise, and for longer calls, the layers run
+ * one after another. Results equal af1_linear_forward per layer within the
+ * library's tolerance (count == 1: bit-identical).
+ *   layers: count (1..4) layers with the same n, on the current device.
+ *   x, ldx, tokens: as af1_linear_forward (shared by all layers).
+ *   ys[i], ldys[i]: output of layer i, as y and ldy of af1_linear_forward.
+ *   workspace: at least af1_workspace_bytes_multi(layers, count, tokens)
+ *       bytes, 256-byte aligned, zero-filled before first use, as for
+ *       af1_linear_forward; af1_workspace_status reports on it.
+ * Errors: INVALID_ARG (count out of range, NULL entries, different n or
+ * devices), BAD_POINTER, MISALIGNED, WORKSPACE, CUDA. */
+AF1_API int64_t af1_workspace_bytes_multi(const af1_layer* const* layers, int count, int64_t tokens);
+AF1_API int af1_linear_forward_multi(const af1_layer* const* layers, int count, const void* x, int64_t ldx,
+                                     int64_t tokens, void* const* ys, const int64_t* ldys, int y_dtype,
+                                     void* workspace, int64_t workspace_bytes, void* stream);
+
 /* af1_linear_forward for callers that cannot allocate device memory when
  * they run a layer: for example a runtime that reserves all GPU memory at
  * start-up and forbids later cudaMalloc calls, or a plugin whose host owns

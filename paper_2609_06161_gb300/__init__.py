@@ -73,6 +73,11 @@ _lib.af1_workspace_bytes.argtypes = [_vp, _i64]
 _lib.af1_workspace_bytes.restype = _i64
 _lib.af1_linear_forward.argtypes = [_vp, _vp, _i64, _i64, _vp, _i64, ctypes.c_int, _vp, _i64, _vp]
 _lib.af1_linear_forward.restype = ctypes.c_int
+_lib.af1_workspace_bytes_multi.argtypes = [ctypes.POINTER(_vp), ctypes.c_int, _i64]
+_lib.af1_workspace_bytes_multi.restype = _i64
+_lib.af1_linear_forward_multi.argtypes = [ctypes.POINTER(_vp), ctypes.c_int, _vp, _i64, _i64, ctypes.POINTER(_vp),
+                                          ctypes.POINTER(_i64), ctypes.c_int, _vp, _i64, _vp]
+_lib.af1_linear_forward_multi.restype = ctypes.c_int
 _lib.af1_workspace_status.argtypes = [_vp, _vp]
 _lib.af1_workspace_status.restype = ctypes.c_int
 _lib.af1_free.argtypes = [_vp]
@@ -248,3 +253,41 @@ class Layer:
             self.free()
         except Exception:
             pass
+
+
+# -- several layers sharing their input ------------------------------------------
+
+def workspace_bytes_multi(layers, tokens: int = 1) -> int:
+    """Workspace bytes of forward_multi over `layers` (1..4 Layer objects)."""
+    arr = (_vp * len(layers))(*[L._h for L in layers])
+    v = _lib.af1_workspace_bytes_multi(arr, len(layers), tokens)
+    if v < 0:
+        raise AF1Error(int(v), last_error())
+    return int(v)
+
+
+def forward_multi(layers, x: torch.Tensor, ys, workspace: torch.Tensor, stream=None) -> None:
+    """ys[i][:tokens, :m_i] = x[:tokens, :n] W_hat_i^T for layers with the same
+    n (af1_linear_forward_multi); x float16 (tokens, ldx), every ys[i] float16
+    or every one float32, all 2-D with unit column stride."""
+    if x.dim() != 2 or x.stride(1) != 1 or x.dtype != torch.float16:
+        raise ValueError("x must be 2-D float16 with contiguous rows")
+    if len(ys) != len(layers):
+        raise ValueError("one output per layer")
+    yd = AF1_F16 if ys[0].dtype == torch.float16 else AF1_F32
+    tokens = x.shape[0]
+    n = layers[0].n
+    ldx = x.stride(0) if tokens > 1 else max(x.stride(0), n + (-n) % 8)
+    ldys = []
+    for L, y in zip(layers, ys):
+        if y.dim() != 2 or y.stride(1) != 1 or y.shape[0] < tokens:
+            raise ValueError("every y must be 2-D with contiguous rows and at least `tokens` rows")
+        if (y.dtype == torch.float16) != (yd == AF1_F16) or y.dtype not in (torch.float16, torch.float32):
+            raise ValueError("outputs must all be float16 or all float32")
+        align = 8 if yd == AF1_F16 else 4
+        ldys.append(y.stride(0) if tokens > 1 else max(y.stride(0), L.m + (-L.m) % align))
+    hs = (_vp * len(layers))(*[L._h for L in layers])
+    yp = (_vp * len(ys))(*[_ptr(y) for y in ys])
+    ld = (_i64 * len(ys))(*ldys)
+    _check(_lib.af1_linear_forward_multi(hs, len(layers), _ptr(x), ldx, tokens, yp, ld, yd, _ptr(workspace),
+                                         workspace.numel() * workspace.element_size(), _stream_handle(stream)))

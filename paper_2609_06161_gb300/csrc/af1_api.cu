@@ -355,6 +355,63 @@ int linear_forward_checked(const af1_layer* layer, const void* x, int64_t ldx, i
 
 extern "C" {
 
+int64_t af1_workspace_bytes_multi(const af1_layer* const* layers, int count, int64_t tokens) {
+  if (layers == nullptr || count < 1 || count > af1::kMaxGroup)
+    return fail(AF1_ERR_INVALID_ARG, "layers must hold 1.." + std::to_string(af1::kMaxGroup) + " layers");
+  for (int i = 0; i < count; ++i)
+    if (layers[i] == nullptr) return fail(AF1_ERR_INVALID_ARG, "layers[" + std::to_string(i) + "] is NULL");
+  if (tokens < 0) return fail(AF1_ERR_INVALID_ARG, "tokens must be >= 0");
+  return af1::multi_workspace_offset(layers, count, tokens, true);
+}
+
+int af1_linear_forward_multi(const af1_layer* const* layers, int count, const void* x, int64_t ldx, int64_t tokens,
+                             void* const* ys, const int64_t* ldys, int y_dtype, void* workspace,
+                             int64_t workspace_bytes, void* stream) {
+  if (layers == nullptr || count < 1 || count > af1::kMaxGroup)
+    return fail(AF1_ERR_INVALID_ARG, "layers must hold 1.." + std::to_string(af1::kMaxGroup) + " layers");
+  if (ys == nullptr || ldys == nullptr) return fail(AF1_ERR_INVALID_ARG, "ys and ldys must not be NULL");
+  for (int i = 0; i < count; ++i) {
+    if (layers[i] == nullptr) return fail(AF1_ERR_INVALID_ARG, "layers[" + std::to_string(i) + "] is NULL");
+    if (layers[i]->n != layers[0]->n) return fail(AF1_ERR_INVALID_ARG, "the layers' n (d_in) differ");
+    if (layers[i]->device != layers[0]->device) return fail(AF1_ERR_INVALID_ARG, "the layers live on different devices");
+  }
+  if (tokens < 0) return fail(AF1_ERR_INVALID_ARG, "tokens must be >= 0");
+  if (y_dtype != AF1_F16 && y_dtype != AF1_F32) return fail(AF1_ERR_INVALID_ARG, "y_dtype must be AF1_F16 or AF1_F32");
+  if (tokens == 0) {
+    g_err.clear();
+    return AF1_OK;
+  }
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return fail_cuda(e, "cudaGetDevice");
+  if (dev != layers[0]->device) return fail(AF1_ERR_BAD_POINTER, "the current device is not the layers' device");
+  int rc;
+  if ((rc = check_device_ptr(x, "x", dev)) != AF1_OK) return rc;
+  if (ldx < layers[0]->n) return fail(AF1_ERR_INVALID_ARG, "ldx < n");
+  if ((reinterpret_cast<uintptr_t>(x) & 15) != 0) return fail(AF1_ERR_MISALIGNED, "x must be 16-byte aligned");
+  if (ldx % 8 != 0) return fail(AF1_ERR_MISALIGNED, "ldx must be a multiple of 8");
+  for (int i = 0; i < count; ++i) {
+    const std::string yi = "ys[" + std::to_string(i) + "]";
+    if ((rc = check_device_ptr(ys[i], yi.c_str(), dev)) != AF1_OK) return rc;
+    if (ldys[i] < layers[i]->m) return fail(AF1_ERR_INVALID_ARG, "ldys[" + std::to_string(i) + "] < m");
+    if ((reinterpret_cast<uintptr_t>(ys[i]) & 15) != 0) return fail(AF1_ERR_MISALIGNED, yi + " must be 16-byte aligned");
+    if (ldys[i] % (y_dtype == AF1_F16 ? 8 : 4) != 0)
+      return fail(AF1_ERR_MISALIGNED, "ldys[i] * element size must be a multiple of 16 bytes");
+  }
+  if (workspace == nullptr) return fail(AF1_ERR_WORKSPACE, "workspace is NULL");
+  if ((rc = check_device_ptr(workspace, "workspace", dev)) != AF1_OK) return AF1_ERR_WORKSPACE;
+  if ((reinterpret_cast<uintptr_t>(workspace) & 255) != 0)
+    return fail(AF1_ERR_WORKSPACE, "workspace must be 256-byte aligned");
+  const int64_t need = af1::multi_workspace_offset(layers, count, tokens, true);
+  if (workspace_bytes < need)
+    return fail(AF1_ERR_WORKSPACE, "workspace too small: need " + std::to_string(need) + " bytes");
+  e = af1::launch_forward_multi(layers, count, x, ldx, tokens, ys, ldys, y_dtype, workspace,
+                                static_cast<cudaStream_t>(stream), true);
+  if (e != cudaSuccess) return fail_cuda(e, "forward launch");
+  g_err.clear();
+  return AF1_OK;
+}
+
 int af1_workspace_status(void* workspace, void* stream) {
   if (workspace == nullptr) return fail(AF1_ERR_WORKSPACE, "workspace is NULL");
   cudaStream_t st = static_cast<cudaStream_t>(stream);

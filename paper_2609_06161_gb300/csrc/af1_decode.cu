@@ -979,23 +979,30 @@ cudaError_t launch_decode(DecodeArgs a, const DecodePlan& p, cudaStream_t st) {
 
 int64_t align256(int64_t v) { return (v + 255) / 256 * 256; }
 
+LutProblem lut_problem(const DecodeArgs& d) {
+  LutProblem q = {};
+  q.signs = d.signs;
+  q.sm = d.sm;
+  q.x = d.x;
+  q.ldx = d.ldx;
+  q.zin = d.zin;
+  q.ldz = d.ldz;
+  q.colscale = d.colscale;
+  q.rowscale = d.rowscale;
+  q.sout = d.sout;
+  q.lds = d.lds;
+  q.y = d.y;
+  q.ldy = d.ldy;
+  return q;
+}
+
 LutArgs lut_args(const DecodeArgs& d) {
   LutArgs a = {};
-  a.signs = d.signs;
-  a.sm = d.sm;
+  a.count = 1;
   a.tokens = d.tokens;
-  a.x = d.x;
-  a.ldx = d.ldx;
-  a.zin = d.zin;
-  a.ldz = d.ldz;
-  a.colscale = d.colscale;
-  a.rowscale = d.rowscale;
-  a.sout = d.sout;
-  a.lds = d.lds;
-  a.y = d.y;
-  a.ldy = d.ldy;
   a.ydtype = d.ydtype;
   a.status = d.status;
+  a.prob[0] = lut_problem(d);
   return a;
 }
 
@@ -1029,13 +1036,13 @@ Workspace plan_workspace(const af1_layer& L, int64_t tokens, bool prep) {
 }
 
 cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64_t tokens, void* y,
-                           int64_t ldy, int y_dtype, void* ws, cudaStream_t st, bool prep) {
+                           int64_t ldy, int y_dtype, void* ws, cudaStream_t st, bool prep, unsigned* status) {
   const Workspace W = plan_workspace(L, tokens, prep);
   uint8_t* wsb = static_cast<uint8_t*>(ws);
+  unsigned* stat = status != nullptr ? status : reinterpret_cast<unsigned*>(wsb + W.status);
   if (tokens > kMaxPassTokens) {
     // Prefill: two tensor-core GEMMs per pass (af1_prefill.cu).
-    return launch_prefill(L, x, ldx, tokens, y, ldy, y_dtype, wsb + W.hbuf, reinterpret_cast<unsigned*>(wsb + W.status),
-                          st);
+    return launch_prefill(L, x, ldx, tokens, y, ldy, y_dtype, wsb + W.hbuf, stat, st);
   }
   // Widest pass whose plans fit (16 tokens normally; fewer only for very
   // long contractions).
@@ -1061,8 +1068,8 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
       return W.bbuf != 0 && T >= kTcMinTokens && m.R * m.C >= kTcMinSigns;
     };
     const bool tc1 = flag || wide_tc(L.p1), tc2 = flag || wide_tc(L.p2);
-    const LutPlan l1 = tc1 ? LutPlan() : plan_lut(L.p1, T, L.num_sms, L.max_smem);
-    const LutPlan l2 = tc2 ? LutPlan() : plan_lut(L.p2, T, L.num_sms, L.max_smem);
+    const LutPlan l1 = tc1 ? LutPlan() : plan_lut(&L.p1, 1, T, L.num_sms, L.max_smem);
+    const LutPlan l2 = tc2 ? LutPlan() : plan_lut(&L.p2, 1, T, L.num_sms, L.max_smem);
     DecodePlan q1, q2;
     const bool prep = W.bbuf != 0 && n_for_tokens(T) > 16;  // launch_decode prepares B then
     if (!l1.ok) q1 = plan_decode(1, L.p1, T, L.num_sms, L.max_smem, prep);
@@ -1079,7 +1086,7 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
     a1.rowscale = reinterpret_cast<const __half*>(L.s);
     a1.sout = reinterpret_cast<float*>(wsb + W.sbuf);
     a1.lds = decode_ldz(L);
-    a1.status = reinterpret_cast<unsigned*>(wsb + W.status);
+    a1.status = stat;
     a1.bbuf = W.bbuf != 0 ? wsb + W.bbuf : nullptr;
     a1.bstats = W.bbuf != 0 ? reinterpret_cast<float2*>(wsb + W.bstats) : nullptr;
     cudaError_t e = l1.ok ? launch_lut(1, lut_args(a1), l1, st) : launch_decode<1>(a1, q1, st);
@@ -1102,6 +1109,80 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
     if (e != cudaSuccess) return e;
   }
   return cudaSuccess;
+}
+
+
+int64_t multi_workspace_offset(const af1_layer* const* Ls, int i, int64_t tokens, bool prep) {
+  int64_t off = 0;
+  for (int j = 0; j < i; ++j) off += align256(plan_workspace(*Ls[j], tokens, prep).total);
+  return off;
+}
+
+cudaError_t launch_forward_multi(const af1_layer* const* Ls, int count, const void* x, int64_t ldx, int64_t tokens,
+                                 void* const* ys, const int64_t* ldys, int y_dtype, void* ws, cudaStream_t st,
+                                 bool prep) {
+  uint8_t* wsb = static_cast<uint8_t*>(ws);
+  unsigned* status = reinterpret_cast<unsigned*>(wsb);  // layer 0's slice starts with its status word
+  const int T = (int)tokens;
+  // One launch per phase for all layers when every phase of every layer
+  // would run on the lookup-table kernel anyway and the group has a plan.
+  bool group = tokens <= kMaxPassTokens;
+  SignMatrix m1[kMaxGroup], m2[kMaxGroup];
+  for (int i = 0; i < count && group; ++i) {
+    const af1_layer& L = *Ls[i];
+    const bool wide = prep && T >= kTcMinTokens && n_for_tokens(T) > 16;
+    if ((L.flags & AF1_FLAG_TC_DECODE) != 0 || (wide && (L.p1.R * L.p1.C >= kTcMinSigns ||
+                                                         L.p2.R * L.p2.C >= kTcMinSigns)))
+      group = false;
+    m1[i] = L.p1;
+    m2[i] = L.p2;
+  }
+  LutPlan g1, g2;
+  if (group) {
+    g1 = plan_lut(m1, count, T, Ls[0]->num_sms, Ls[0]->max_smem);
+    g2 = plan_lut(m2, count, T, Ls[0]->num_sms, Ls[0]->max_smem);
+    group = g1.ok && g2.ok;
+  }
+  if (!group) {
+    // One call per layer, each with its own workspace slice, all reporting to
+    // the first slice's status word.
+    for (int i = 0; i < count; ++i) {
+      const int64_t off = multi_workspace_offset(Ls, i, tokens, prep);
+      cudaError_t e = launch_forward(*Ls[i], x, ldx, tokens, ys[i], ldys[i], y_dtype, wsb + off, st, prep, status);
+      if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
+  }
+  LutArgs a1 = {}, a2 = {};
+  a1.count = a2.count = count;
+  a1.tokens = a2.tokens = T;
+  a1.ydtype = a2.ydtype = y_dtype;
+  a1.status = a2.status = status;
+  for (int i = 0; i < count; ++i) {
+    const af1_layer& L = *Ls[i];
+    const Workspace W = plan_workspace(L, tokens, prep);
+    float* sbuf = reinterpret_cast<float*>(wsb + multi_workspace_offset(Ls, i, tokens, prep) + W.sbuf);
+    LutProblem& q1 = a1.prob[i];
+    q1.signs = L.signs1;
+    q1.sm = L.p1;
+    q1.x = static_cast<const __half*>(x);
+    q1.ldx = ldx;
+    q1.colscale = reinterpret_cast<const __half*>(L.b);
+    q1.rowscale = reinterpret_cast<const __half*>(L.s);
+    q1.sout = sbuf;
+    q1.lds = decode_ldz(L);
+    LutProblem& q2 = a2.prob[i];
+    q2.signs = L.signs2;
+    q2.sm = L.p2;
+    q2.zin = sbuf;
+    q2.ldz = decode_ldz(L);
+    q2.rowscale = reinterpret_cast<const __half*>(L.a);
+    q2.y = ys[i];
+    q2.ldy = ldys[i];
+  }
+  cudaError_t e = launch_lut(1, a1, g1, st);
+  if (e != cudaSuccess) return e;
+  return launch_lut(2, a2, g2, st);
 }
 
 }  // namespace af1

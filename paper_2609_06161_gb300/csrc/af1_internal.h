@@ -57,13 +57,14 @@ cudaError_t launch_words_to_blocks(const uint32_t* words, int64_t words_per_row,
 // Set the calling thread's af1_last_error() message; returns `code`.
 int set_error(int code, const std::string& msg);
 
-// Decode on the CUDA cores (af1_lut.cu): one sign-matrix product of a pass
-// of 1..16 tokens through lookup tables of signed sums.
-struct LutArgs {
+// Decode on the CUDA cores (af1_lut.cu): the sign-matrix products of one
+// phase of a pass of 1..16 tokens through lookup tables of signed sums, for
+// up to kMaxGroup independent problems (layers that share their input) in
+// one launch.
+constexpr int kMaxGroup = 4;
+struct LutProblem {
   const uint8_t* signs;  // af1_layout.h row-block layout
   SignMatrix sm;
-  int KS, CPC;           // set by the launcher from the plan
-  int tokens;            // T (1..16)
   const __half* x;       // phase 1 input [T][ldx] (FP16)
   int64_t ldx;
   const float* zin;      // phase 2 input [T][ldz] (FP32)
@@ -74,20 +75,39 @@ struct LutArgs {
   int64_t lds;
   void* y;                 // phase 2 output [T][ldy], FP16 (ydtype 0) or FP32
   int64_t ldy;
+  int CPC, rb0;            // set by the launcher: chunks per CTA, first grid x of the problem
+};
+struct LutArgs {
+  int count;         // problems (1..kMaxGroup)
+  int tokens;        // T (1..16)
   int ydtype;
+  int KS;            // set by the launcher: CTAs per cluster, common to all problems
   unsigned* status;
+  LutProblem prob[kMaxGroup];
 };
 struct LutPlan {
-  int KS = 0, CPC = 0, smem = 0;
+  int KS = 0, smem = 0;
+  int CPC[kMaxGroup] = {0, 0, 0, 0};
   bool ok = false;
 };
-LutPlan plan_lut(const SignMatrix& sm, int T, int num_sms, int max_smem);
+// Plan of one phase for `count` problems (sm[i]) of a pass of T tokens.
+LutPlan plan_lut(const SignMatrix* sm, int count, int T, int num_sms, int max_smem);
 cudaError_t launch_lut(int phase, const LutArgs& a, const LutPlan& p, cudaStream_t st);
 
 cudaError_t launch_prefill(const af1_layer& L, const void* x, int64_t ldx, int64_t tokens, void* y, int64_t ldy,
                            int y_dtype, uint8_t* h_buf, unsigned* status, cudaStream_t st);
+// status: the status word to report to (nullptr: the workspace's own).
 cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64_t tokens, void* y,
-                           int64_t ldy, int y_dtype, void* ws, cudaStream_t st, bool prep = true);
+                           int64_t ldy, int y_dtype, void* ws, cudaStream_t st, bool prep = true,
+                           unsigned* status = nullptr);
+// Several layers with the same input x (same n): one lookup-table launch per
+// phase for all of them when possible, else one call per layer. The
+// workspace holds one single-layer workspace per layer, each 256-aligned,
+// in order (multi_workspace_offset); status reports go to the first.
+int64_t multi_workspace_offset(const af1_layer* const* Ls, int i, int64_t tokens, bool prep);
+cudaError_t launch_forward_multi(const af1_layer* const* Ls, int count, const void* x, int64_t ldx, int64_t tokens,
+                                 void* const* ys, const int64_t* ldys, int y_dtype, void* ws, cudaStream_t st,
+                                 bool prep);
 // af1_linear_forward with all its argument checks; prep = false never uses
 // (and does not require) the prepared-B region of the workspace.
 int linear_forward_checked(const af1_layer* layer, const void* x, int64_t ldx, int64_t tokens, void* y, int64_t ldy,

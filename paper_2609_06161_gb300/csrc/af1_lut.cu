@@ -203,18 +203,26 @@ __device__ __forceinline__ void lookup_word2(uint32_t w, uint32_t pat, const uin
   }
 }
 
-template <int PHASE, int NP>
-__global__ void __launch_bounds__(kThreads, 4) lut_kernel(const LutArgs a) {
+template <int PHASE, int NP, bool MULTI>
+__global__ void __launch_bounds__(kThreads, 4) lut_kernel(const __grid_constant__ LutArgs a) {
   constexpr int NACC = NP == 0 ? 1 : 2 * NP;
   constexpr int TCB = table_chunk_bytes(NP);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  // Problem of this CTA: grid x runs over the row blocks of all problems.
+  // (One problem: fixed parameter offsets, no lookup.)
+  int pi = 0;
+  if (MULTI) {
+    for (int i = 1; i < a.count; ++i)
+      if ((int)blockIdx.x >= a.prob[i].rb0) pi = i;
+  }
+  const LutProblem& pb = a.prob[MULTI ? pi : 0];
   // Token group blockIdx.z: tokens tg0 .. tg0 + T - 1 of the pass.
   const int tg0 = (int)blockIdx.z * kGroupTokens;
   const int T = min(kGroupTokens, a.tokens - tg0);
-  const __half* xg = PHASE == 1 ? a.x + (int64_t)tg0 * a.ldx : nullptr;
-  const float* zg = PHASE == 2 ? a.zin + (int64_t)tg0 * a.ldz : nullptr;
-  const int KS = a.KS, CPC = a.CPC;
+  const __half* xg = PHASE == 1 ? pb.x + (int64_t)tg0 * pb.ldx : nullptr;
+  const float* zg = PHASE == 2 ? pb.zin + (int64_t)tg0 * pb.ldz : nullptr;
+  const int KS = a.KS, CPC = pb.CPC;
   const LutSmem sp = lut_smem(CPC, KS, T, NP);
   const uint32_t* W = reinterpret_cast<const uint32_t*>(smem + sp.w);
   float* zs = reinterpret_cast<float*>(smem + sp.z);
@@ -223,10 +231,12 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const LutArgs a) {
   LutHeader& h = *reinterpret_cast<LutHeader*>(smem + sp.hdr);
 
   const int tid = threadIdx.x;
-  const int rb = blockIdx.x, ks = blockIdx.y;
-  const int nch_total = a.sm.NCH;
+  const int rb = (int)blockIdx.x - pb.rb0, ks = blockIdx.y;
+  const int nch_total = pb.sm.NCH;
   const int c0 = ks * CPC;
-  const int nch = min(CPC, nch_total - c0);  // >= 1 by construction of KS
+  // Chunks of this CTA; 0 for the last CTAs of a problem with fewer chunks
+  // than the group's clusters have CTAs (they still finalise their rows).
+  const int nch = max(0, min(CPC, nch_total - c0));
   const int64_t row0 = (int64_t)rb * kBlockRows;
   const int64_t k0 = (int64_t)c0 * kChunkCols;
   const int slice = slice_rows(KS);
@@ -244,7 +254,7 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const LutArgs a) {
     h.err = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-    const uint8_t* src = a.signs + ((int64_t)rb * nch_total + c0) * kChunkBytes;
+    const uint8_t* src = pb.signs + ((int64_t)rb * nch_total + c0) * kChunkBytes;
     for (int c = 0; c < nch; ++c) {
       mbar_expect_tx(&h.wfull[c], kChunkBytes);
       bulk_g2s(smem + sp.w + c * kChunkBytes, src + (int64_t)c * kChunkBytes, kChunkBytes, &h.wfull[c]);
@@ -255,8 +265,8 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const LutArgs a) {
   cluster_arrive_relaxed();
   // Row scale of row my0 + tid of the block (a layer constant): loaded now,
   // stored to shared memory once the activations are staged.
-  const float rs_own = (tid < slice && my0 + tid < kBlockRows && row0 + my0 + tid < a.sm.R)
-                           ? __half2float(a.rowscale[row0 + my0 + tid])
+  const float rs_own = (tid < slice && my0 + tid < kBlockRows && row0 + my0 + tid < pb.sm.R)
+                           ? __half2float(pb.rowscale[row0 + my0 + tid])
                            : 0.f;
   __syncthreads();
 
@@ -275,10 +285,10 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const LutArgs a) {
         const int i = i0 + u * kThreads;
         const int t = i / g8, k = (i - t * g8) * 8;
         const int64_t col = k0 + k;
-        if (i < ng && col + 7 < a.sm.C) {
+        if (i < ng && col + 7 < pb.sm.C) {
           if (PHASE == 1) {
-            const uint4 xr = __ldcg(reinterpret_cast<const uint4*>(xg + (int64_t)t * a.ldx + col));
-            const uint4 br = __ldg(reinterpret_cast<const uint4*>(a.colscale + col));
+            const uint4 xr = __ldcg(reinterpret_cast<const uint4*>(xg + (int64_t)t * pb.ldx + col));
+            const uint4 br = __ldg(reinterpret_cast<const uint4*>(pb.colscale + col));
             const uint32_t xw[4] = {xr.x, xr.y, xr.z, xr.w}, bw[4] = {br.x, br.y, br.z, br.w};
 #pragma unroll
             for (int h2 = 0; h2 < 4; ++h2) {
@@ -288,8 +298,8 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const LutArgs a) {
               v[u][2 * h2 + 1] = xf.y * bf.y;
             }
           } else {
-            const float4 z0 = __ldcg(reinterpret_cast<const float4*>(zg + (int64_t)t * a.ldz + col));
-            const float4 z1 = __ldcg(reinterpret_cast<const float4*>(zg + (int64_t)t * a.ldz + col + 4));
+            const float4 z0 = __ldcg(reinterpret_cast<const float4*>(zg + (int64_t)t * pb.ldz + col));
+            const float4 z1 = __ldcg(reinterpret_cast<const float4*>(zg + (int64_t)t * pb.ldz + col + 4));
             v[u][0] = z0.x;
             v[u][1] = z0.y;
             v[u][2] = z0.z;
@@ -303,11 +313,11 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const LutArgs a) {
 #pragma unroll
           for (int q = 0; q < 8; ++q) {
             float z = 0.f;
-            if (i < ng && col + q < a.sm.C) {
+            if (i < ng && col + q < pb.sm.C) {
               if (PHASE == 1)
-                z = __half2float(__ldcg(xg + (int64_t)t * a.ldx + col + q)) * __half2float(a.colscale[col + q]);
+                z = __half2float(__ldcg(xg + (int64_t)t * pb.ldx + col + q)) * __half2float(pb.colscale[col + q]);
               else
-                z = __ldcg(zg + (int64_t)t * a.ldz + col + q);
+                z = __ldcg(zg + (int64_t)t * pb.ldz + col + q);
             }
             v[u][q] = z;
           }
@@ -424,7 +434,7 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const LutArgs a) {
     const int t = idx / cnt;
     const int i = idx - t * cnt;
     const int64_t row = row0 + my0 + i;
-    if (row >= a.sm.R) continue;
+    if (row >= pb.sm.R) continue;
     // The 2 KS partials in four interleaved chains (fixed order:
     // deterministic), so their reads overlap.
     const float* pr = recv + t * slice + i;
@@ -441,11 +451,11 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const LutArgs a) {
     for (; q < 2 * KS; ++q) v0 += pr[q * qstride];
     const float out = ((v0 + v1) + (v2 + v3)) * rs[i];
     if (PHASE == 1) {
-      a.sout[(int64_t)(tg0 + t) * a.lds + row] = out;
+      pb.sout[(int64_t)(tg0 + t) * pb.lds + row] = out;
     } else if (a.ydtype == 0) {
-      reinterpret_cast<__half*>(a.y)[(int64_t)(tg0 + t) * a.ldy + row] = __float2half_rn(out);
+      reinterpret_cast<__half*>(pb.y)[(int64_t)(tg0 + t) * pb.ldy + row] = __float2half_rn(out);
     } else {
-      reinterpret_cast<float*>(a.y)[(int64_t)(tg0 + t) * a.ldy + row] = out;
+      reinterpret_cast<float*>(pb.y)[(int64_t)(tg0 + t) * pb.ldy + row] = out;
     }
   }
 
@@ -461,17 +471,25 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const LutArgs a) {
   }
 }
 
-template <int PHASE, int NP>
+template <int PHASE, int NP, bool MULTI>
 cudaError_t launch_np(const LutArgs& a, const LutPlan& p, cudaStream_t st) {
-  auto kern = lut_kernel<PHASE, NP>;
+  auto kern = lut_kernel<PHASE, NP, MULTI>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, p.smem);
   if (e != cudaSuccess) return e;
   if (p.KS > 8) {
     e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     if (e != cudaSuccess) return e;
   }
+  LutArgs b = a;
+  b.KS = p.KS;
+  int rbs = 0;  // grid x: the row blocks of all problems, in order
+  for (int i = 0; i < a.count; ++i) {
+    b.prob[i].CPC = p.CPC[i];
+    b.prob[i].rb0 = rbs;
+    rbs += a.prob[i].sm.RB;
+  }
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((unsigned)a.sm.RB, (unsigned)p.KS, (unsigned)((a.tokens + kGroupTokens - 1) / kGroupTokens));
+  cfg.gridDim = dim3((unsigned)rbs, (unsigned)p.KS, (unsigned)((a.tokens + kGroupTokens - 1) / kGroupTokens));
   cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.dynamicSmemBytes = (size_t)p.smem;
   cfg.stream = st;
@@ -484,24 +502,21 @@ cudaError_t launch_np(const LutArgs& a, const LutPlan& p, cudaStream_t st) {
   attr[1].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  LutArgs b = a;
-  b.KS = p.KS;
-  b.CPC = p.CPC;
   return cudaLaunchKernelEx(&cfg, kern, b);
 }
 
 }  // namespace
 
+namespace {
+
 // Split of one sign matrix for a pass of T <= 16 tokens, run as ceil(T / 4)
 // token groups of CTAs: about two CTAs per SM (row blocks x KS x groups ~
 // 2 SMs, KS <= 16 CTAs per cluster), CTAs small enough that three fit on an
-// SM, and at most kMaxCPC chunks each.
-LutPlan plan_lut(const SignMatrix& sm, int T, int num_sms, int max_smem) {
-  LutPlan p;
-  if (T < 1 || T > kMaxPassTokens || sm.RB < 1 || sm.NCH < 1) return p;
+// SM, and at most kMaxCPC chunks each. Returns KS (0: no plan), *cpc and
+// *smem.
+int plan_one(const SignMatrix& sm, int T, int sms, int max_smem, int* cpc_out, int* smem_out) {
   const int Tg = T < kGroupTokens ? T : kGroupTokens;
   const int groups = (T + kGroupTokens - 1) / kGroupTokens;
-  const int sms = num_sms > 0 ? num_sms : 148;
   const int cap = max_smem / 3 < 72 * 1024 ? max_smem / 3 : 72 * 1024;
   const int64_t tiles = (int64_t)sm.RB * groups;
   int ks = (int)((2 * sms + tiles - 1) / tiles);
@@ -514,23 +529,56 @@ LutPlan plan_lut(const SignMatrix& sm, int T, int num_sms, int max_smem) {
     const int KS = (sm.NCH + cpc - 1) / cpc;
     const int need = lut_smem(cpc, KS, Tg, pairs_for(Tg)).total;
     if (need <= cap || (ks == kMaxKS || ks == sm.NCH)) {
-      if (need > max_smem) return p;
-      p.KS = KS;
-      p.CPC = cpc;
-      p.smem = need;
-      p.ok = true;
-      return p;
+      if (need > max_smem) return 0;
+      *cpc_out = cpc;
+      *smem_out = need;
+      return KS;
     }
   }
+  return 0;
+}
+
+}  // namespace
+
+// One problem: its own split. Several (layers sharing their input, one
+// launch): the largest of their splits' cluster sizes for all, each problem
+// cutting its columns into that many slices (the last CTAs of a problem with
+// fewer chunks get none).
+LutPlan plan_lut(const SignMatrix* sm, int count, int T, int num_sms, int max_smem) {
+  LutPlan p;
+  if (count < 1 || count > kMaxGroup || T < 1 || T > kMaxPassTokens) return p;
+  const int sms = num_sms > 0 ? num_sms : 148;
+  const int Tg = T < kGroupTokens ? T : kGroupTokens;
+  int KS = 0;
+  for (int i = 0; i < count; ++i) {
+    if (sm[i].RB < 1 || sm[i].NCH < 1) return p;
+    int cpc = 0, smem = 0;
+    const int k = plan_one(sm[i], T, sms, max_smem, &cpc, &smem);
+    if (k == 0) return p;
+    if (k > KS) KS = k;
+  }
+  int smem = 0;
+  for (int i = 0; i < count; ++i) {
+    const int cpc = (sm[i].NCH + KS - 1) / KS;
+    if (cpc > kMaxCPC) return p;
+    const int need = lut_smem(cpc, KS, Tg, pairs_for(Tg)).total;
+    if (need > max_smem) return p;
+    if (need > smem) smem = need;
+    p.CPC[i] = cpc;
+  }
+  p.KS = KS;
+  p.smem = smem;
+  p.ok = true;
   return p;
 }
 
 template <int PHASE>
 cudaError_t launch_phase(const LutArgs& a, const LutPlan& p, cudaStream_t st) {
+  const bool multi = a.count > 1;
   switch (pairs_for(a.tokens < kGroupTokens ? a.tokens : kGroupTokens)) {
-    case 0: return launch_np<PHASE, 0>(a, p, st);
-    case 1: return launch_np<PHASE, 1>(a, p, st);
-    default: return launch_np<PHASE, 2>(a, p, st);
+    case 0: return multi ? launch_np<PHASE, 0, true>(a, p, st) : launch_np<PHASE, 0, false>(a, p, st);
+    case 1: return multi ? launch_np<PHASE, 1, true>(a, p, st) : launch_np<PHASE, 1, false>(a, p, st);
+    default: return multi ? launch_np<PHASE, 2, true>(a, p, st) : launch_np<PHASE, 2, false>(a, p, st);
   }
 }
 

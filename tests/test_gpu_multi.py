@@ -1,0 +1,125 @@
+"""Several layers sharing one input (af1_linear_forward_multi) against the
+FP64 oracle per layer, through the C ABI."""
+import numpy as np
+import pytest
+import torch
+
+import synth
+from oracle import af1_oracle as O
+from tests.af1_cases import TOL, f16, oracle_from_signs, signs_layer
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def P():
+    import paper_2609_06161_gb300 as P
+    return P
+
+
+def _group(P, seed, n, specs, tokens, integer=False):
+    """Layers (m_i, r_i) with input width n and one shared x."""
+    ds, layers = [], []
+    for i, (m, r) in enumerate(specs):
+        if integer:
+            d = synth.integer_layer(seed + i, m, n, r, tokens)
+        else:
+            d = synth.layer_signs(seed + i, m, n, r, tokens)
+        ds.append(d)
+        layers.append(signs_layer(P, d))
+    x = ds[0]["x"]  # every layer gets the first layer's activations
+    for d in ds:
+        d["x"] = x
+    return ds, layers, x
+
+
+def _run(P, layers, x_bits, n, tokens, out_dtype=torch.float32):
+    x = f16(x_bits).reshape(tokens, n)
+    pad = (-n) % 8
+    xp = torch.zeros((tokens, n + pad), dtype=torch.float16, device="cuda")
+    xp[:, :n] = x
+    ys = []
+    for L in layers:
+        align = 8 if out_dtype == torch.float16 else 4
+        ys.append(torch.full((tokens, L.m + (-L.m) % align), float("nan"), dtype=out_dtype, device="cuda"))
+    ws = torch.zeros(P.workspace_bytes_multi(layers, tokens), dtype=torch.uint8, device="cuda")
+    P.forward_multi(layers, xp, ys, ws)
+    P.workspace_status(ws)
+    torch.cuda.synchronize()
+    return [y[:, :L.m].double().cpu().numpy() for L, y in zip(layers, ys)]
+
+
+@pytest.mark.parametrize("specs", [[(200, 77), (100, 40), (100, 40)], [(300, 120), (64, 30)],
+                                   [(256, 200), (129, 60), (64, 33), (1000, 321)], [(520, 600)]])
+@pytest.mark.parametrize("tokens", [1, 3, 5, 8, 16, 17])
+def test_multi_matches_oracle(P, specs, tokens):
+    n = 700
+    ds, layers, x = _group(P, 40 + tokens + len(specs), n, specs, tokens)
+    ys = _run(P, layers, x, n, tokens)
+    for d, y in zip(ds, ys):
+        err = O.rowwise_rel_err(y, oracle_from_signs(d, n))
+        assert err <= TOL, err
+    for L in layers:
+        L.free()
+
+
+@pytest.mark.parametrize("tokens", [1, 4, 7, 16])
+def test_multi_integer_bit_exact(P, tokens):
+    n = 256
+    ds, layers, x = _group(P, 70 + tokens, n, [(130, 100), (64, 40), (200, 120)], tokens, integer=True)
+    ys = _run(P, layers, x, n, tokens)
+    for d, y in zip(ds, ys):
+        np.testing.assert_array_equal(y, oracle_from_signs(d, n))
+    for L in layers:
+        L.free()
+
+
+@pytest.mark.parametrize("tokens", [1, 4, 16])
+def test_multi_single_layer_identical(P, tokens):
+    """count == 1 runs exactly the kernels of af1_linear_forward."""
+    n = 4096
+    d = synth.layer_signs(90 + tokens, 1024, n, 800, tokens)
+    layer = signs_layer(P, d)
+    (y_multi,) = _run(P, [layer], d["x"], n, tokens)
+    x = f16(d["x"]).reshape(tokens, n)
+    y_one = layer.forward(x, out_dtype=torch.float32).double().cpu().numpy()
+    np.testing.assert_array_equal(y_multi, y_one)
+    layer.free()
+
+
+def test_multi_llama_qkv_full_size(P):
+    """q, k, v of a LLaMA-3-8B-shaped layer at their 1.0-BPW ranks, one token,
+    sampled rows against the oracle."""
+    n, tokens = 4096, 1
+    specs = [(4096, O.rank_for_budget(4096, n, 1)), (1024, O.rank_for_budget(1024, n, 1)),
+             (1024, O.rank_for_budget(1024, n, 1))]
+    ds = [synth.layer_words(300 + i, m, n, r, tokens) for i, (m, r) in enumerate(specs)]
+    from tests.af1_cases import words_layer
+    layers = [words_layer(P, d, m, n, r) for d, (m, r) in zip(ds, specs)]
+    ys = _run(P, layers, ds[0]["x"], n, tokens)
+    for d, (m, r), y in zip(ds, specs, ys):
+        rows = np.sort(synth.rng(m).choice(m, size=128, replace=False))
+        ref = O.forward_from_packed(d["Uw"], d["Vw"], d["a"], d["s"], d["b"], ds[0]["x"], m, n, r, rows=rows)
+        assert O.rowwise_rel_err(y[:, rows], ref) <= TOL
+    for L in layers:
+        L.free()
+
+
+def test_multi_errors(P):
+    d1 = synth.layer_signs(95, 64, 96, 20, 1)
+    d2 = synth.layer_signs(96, 64, 128, 20, 1)
+    L1, L2 = signs_layer(P, d1), signs_layer(P, d2)
+    x = torch.zeros((1, 96), dtype=torch.float16, device="cuda")
+    y = torch.zeros((1, 64), dtype=torch.float32, device="cuda")
+    ws = torch.zeros(1 << 20, dtype=torch.uint8, device="cuda")
+    with pytest.raises(P.AF1Error) as e:
+        P.forward_multi([L1, L2], x, [y, y], ws)  # different n
+    assert e.value.code == -1
+    with pytest.raises(P.AF1Error) as e:
+        P.forward_multi([L1] * 5, x, [y] * 5, ws)  # more than 4 layers
+    assert e.value.code == -1
+    with pytest.raises(P.AF1Error) as e:
+        P.forward_multi([L1, L1], x, [y, y], ws[:256])  # workspace too small
+    assert e.value.code == -8
+    L1.free()
+    L2.free()
