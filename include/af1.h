@@ -63,6 +63,7 @@ extern "C" {
 #define AF1_ERR_CUDA (-6)          /* a CUDA runtime error (message has details)    */
 #define AF1_ERR_TIMEOUT (-7)       /* a bounded device wait gave up                 */
 #define AF1_ERR_WORKSPACE (-8)     /* workspace missing, too small or misaligned    */
+#define AF1_ERR_IO (-9)            /* a layer file could not be read or written     */
 
 /* ---- output dtypes for af1_linear_forward -------------------------------- */
 #define AF1_F16 0
@@ -78,6 +79,13 @@ extern "C" {
    (lookup tables of signed sums). Both compute the same products within the
    library's tolerance; the default is faster at every measured shape. */
 #define AF1_FLAG_TC_DECODE 2
+/* The scale vectors a, s, b passed to af1_pack_layer / af1_load_packed_layer
+   are BF16 bit patterns (the paper's storage type) instead of FP16. The layer
+   converts them to FP16 on the device, exactly; a value FP16 cannot hold
+   exactly (beyond +-65504, nonzero below 2^-24, more significant bits than
+   FP16 has at that magnitude, NaN) fails the call with AF1_ERR_INVALID_ARG.
+   Both types cost 16 bits, so the bit budget is unchanged. */
+#define AF1_FLAG_BF16_SCALES 4
 
 typedef struct af1_layer_desc {
   int64_t m;       /* d_out: rows of W_hat, length of a, length of y rows */
@@ -127,6 +135,36 @@ AF1_API int af1_pack_layer(const af1_layer_desc* desc, const int8_t* U, const in
 AF1_API int af1_load_packed_layer(const af1_layer_desc* desc, const uint32_t* U_words,
                           const uint32_t* V_words, const uint16_t* a, const uint16_t* s,
                           const uint16_t* b, void* stream, af1_layer** out);
+
+/* The layer's factors and scales in the exchange format: canonical packed
+ * words U [m x W(r)] and V [r x W(n)] (uint32) and FP16 bit patterns of a, s,
+ * b (for a layer made from BF16 scales: their exact FP16 values). Every output
+ * is an optional device pointer (NULL skips it). Stream-ordered, asynchronous.
+ * Errors: INVALID_ARG, BAD_POINTER, CUDA. */
+AF1_API int af1_export_layer(const af1_layer* layer, uint32_t* U_words, uint32_t* V_words, uint16_t* a,
+                             uint16_t* s, uint16_t* b, void* stream);
+
+/* Layer files. Layout (little-endian): the 40-byte header below, then U words
+ * (m x W(r) uint32), V words (r x W(n) uint32), a (m FP16), s (r FP16), b
+ * (n FP16), with no padding between the arrays. flags holds the layer's
+ * AF1_FLAG_ANY_RANK / AF1_FLAG_TC_DECODE bits. */
+#define AF1_FILE_MAGIC "AF1LAYER"
+#define AF1_FILE_VERSION 1u
+typedef struct af1_file_header {
+  char magic[8];     /* AF1_FILE_MAGIC, no terminating NUL */
+  uint32_t version;  /* AF1_FILE_VERSION */
+  uint32_t flags;
+  int64_t m, n, r;
+} af1_file_header;
+
+/* Write a layer to `path` (host file). Synchronizes the device work it
+ * queues (on the legacy default stream). Errors: INVALID_ARG, CUDA, IO. */
+AF1_API int af1_save_layer(const af1_layer* layer, const char* path);
+
+/* Read a layer file and build the layer (as af1_load_packed_layer, on
+ * `stream`, which is synchronized). Errors: INVALID_ARG, OVER_BUDGET, CUDA,
+ * IO (missing, truncated or foreign file). */
+AF1_API int af1_load_layer(const char* path, void* stream, af1_layer** out);
 
 /* Copy the description of a layer into *desc. */
 AF1_API int af1_layer_get_desc(const af1_layer* layer, af1_layer_desc* desc);

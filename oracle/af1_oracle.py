@@ -163,6 +163,14 @@ def f16_bits_to_f64(h) -> np.ndarray:
     return h.view(np.float16).astype(np.float64)
 
 
+def bf16_bits_to_f64(h) -> np.ndarray:
+    """BF16 bit patterns (uint16) -> float64, exact: a BF16 value is the
+    FP32 value whose upper 16 bits are the pattern and lower 16 bits zero
+    (1 sign, 8 exponent, 7 mantissa bits; the paper's scale type)."""
+    h = np.ascontiguousarray(np.asarray(h, dtype=np.uint16))
+    return (h.astype(np.uint32) << np.uint32(16)).view(np.float32).astype(np.float64)
+
+
 # ---------------------------------------------------------------------------
 # Reconstruction and forward (Eq. double_factor_equiv, Eq. binary_paths)
 # ---------------------------------------------------------------------------
@@ -214,20 +222,22 @@ def forward_factored(U, V, a, s, b, X, rows=None) -> np.ndarray:
     return (st @ Uf.T) * a[rows][None, :]
 
 
-def forward_from_packed(Uw, Vw, a_h, s_h, b_h, X_h, d_out, d_in, r, rows=None):
+def forward_from_packed(Uw, Vw, a_h, s_h, b_h, X_h, d_out, d_in, r, rows=None, scale_dtype="f16"):
     """Full oracle forward from the deployable format: canonical packed words
-    plus FP16 bit patterns of a (d_out), s (r), b (d_in) and X (T x d_in).
-    Unpacks the signs, widens everything to FP64 exactly and evaluates
-    forward_factored. Returns float64 (T x d_out), or (T x len(rows))."""
+    plus FP16 bit patterns of a (d_out), s (r), b (d_in) and X (T x d_in)
+    (scale_dtype="bf16": a, s, b are BF16 bit patterns instead). Unpacks the
+    signs, widens everything to FP64 exactly and evaluates forward_factored.
+    Returns float64 (T x d_out), or (T x len(rows))."""
     U = unpack_U(Uw, r)
     if U.shape[0] != d_out:
         raise ValueError("U rows != d_out")
     V = unpack_V(Vw, d_in)
     if V.shape[1] != r:
         raise ValueError("V rank mismatch")
-    a = f16_bits_to_f64(a_h)
-    s = f16_bits_to_f64(s_h)
-    b = f16_bits_to_f64(b_h)
+    dec = {"f16": f16_bits_to_f64, "bf16": bf16_bits_to_f64}[scale_dtype]
+    a = dec(a_h)
+    s = dec(s_h)
+    b = dec(b_h)
     X = f16_bits_to_f64(X_h).reshape(-1, d_in)
     return forward_factored(U, V, a, s, b, X, rows=rows)
 

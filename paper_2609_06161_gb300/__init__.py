@@ -37,10 +37,17 @@ AF1_F16 = 0
 AF1_F32 = 1
 AF1_FLAG_ANY_RANK = 1
 AF1_FLAG_TC_DECODE = 2
+AF1_FLAG_BF16_SCALES = 4
 
 
-def _flags(any_rank: bool, tc_decode: bool) -> int:
-    return (AF1_FLAG_ANY_RANK if any_rank else 0) | (AF1_FLAG_TC_DECODE if tc_decode else 0)
+def _flags(any_rank: bool, tc_decode: bool, scales=()) -> int:
+    """Layer flags; BF16 scale tensors select AF1_FLAG_BF16_SCALES."""
+    dts = {t.dtype for t in scales}
+    if len(dts) > 1 or not dts <= {torch.float16, torch.bfloat16}:
+        raise ValueError("a, s and b must all be float16 or all bfloat16")
+    bf16 = dts == {torch.bfloat16}
+    return ((AF1_FLAG_ANY_RANK if any_rank else 0) | (AF1_FLAG_TC_DECODE if tc_decode else 0)
+            | (AF1_FLAG_BF16_SCALES if bf16 else 0))
 _ERR_NAMES = {
     -1: "AF1_ERR_INVALID_ARG", -2: "AF1_ERR_BAD_POINTER", -3: "AF1_ERR_MISALIGNED",
     -4: "AF1_ERR_OVER_BUDGET", -5: "AF1_ERR_INVALID_SIGN", -6: "AF1_ERR_CUDA",
@@ -78,6 +85,12 @@ _lib.af1_workspace_bytes_multi.restype = _i64
 _lib.af1_linear_forward_multi.argtypes = [ctypes.POINTER(_vp), ctypes.c_int, _vp, _i64, _i64, ctypes.POINTER(_vp),
                                           ctypes.POINTER(_i64), ctypes.c_int, _vp, _i64, _vp]
 _lib.af1_linear_forward_multi.restype = ctypes.c_int
+_lib.af1_export_layer.argtypes = [_vp, _vp, _vp, _vp, _vp, _vp, _vp]
+_lib.af1_export_layer.restype = ctypes.c_int
+_lib.af1_save_layer.argtypes = [_vp, ctypes.c_char_p]
+_lib.af1_save_layer.restype = ctypes.c_int
+_lib.af1_load_layer.argtypes = [ctypes.c_char_p, _vp, ctypes.POINTER(_vp)]
+_lib.af1_load_layer.restype = ctypes.c_int
 _lib.af1_workspace_status.argtypes = [_vp, _vp]
 _lib.af1_workspace_status.restype = ctypes.c_int
 _lib.af1_free.argtypes = [_vp]
@@ -167,7 +180,7 @@ class Layer:
         if return_words:
             Uw = torch.empty((m, words_per_row(r)), dtype=torch.int32, device=U.device)
             Vw = torch.empty((r, words_per_row(n)), dtype=torch.int32, device=U.device)
-        d = _Desc(m, n, r, _flags(any_rank, tc_decode), 0)
+        d = _Desc(m, n, r, _flags(any_rank, tc_decode, (a, s, b)), 0)
         h = _vp()
         _check(_lib.af1_pack_layer(ctypes.byref(d), _ptr(U), _ptr(V), _ptr(a), _ptr(s), _ptr(b),
                                    _ptr(Uw), _ptr(Vw), _stream_handle(stream), ctypes.byref(h)))
@@ -181,11 +194,36 @@ class Layer:
         """Uw: (m, W(r)), Vw: (r, W(n)) canonical packed words (int32/uint32)."""
         Uw, Vw = Uw.contiguous(), Vw.contiguous()
         a, s, b = a.contiguous(), s.contiguous(), b.contiguous()
-        d = _Desc(m, n, r, _flags(any_rank, tc_decode), 0)
+        d = _Desc(m, n, r, _flags(any_rank, tc_decode, (a, s, b)), 0)
         h = _vp()
         _check(_lib.af1_load_packed_layer(ctypes.byref(d), _ptr(Uw), _ptr(Vw), _ptr(a), _ptr(s), _ptr(b),
                                           _stream_handle(stream), ctypes.byref(h)))
         return cls(h.value, m, n, r)
+
+    @classmethod
+    def load(cls, path: str, stream=None):
+        """A layer from a file written by save() (af1_load_layer)."""
+        h = _vp()
+        _check(_lib.af1_load_layer(str(path).encode(), _stream_handle(stream), ctypes.byref(h)))
+        d = _Desc()
+        _check(_lib.af1_layer_get_desc(h, ctypes.byref(d)))
+        return cls(h.value, d.m, d.n, d.r)
+
+    def save(self, path: str) -> None:
+        """Write the layer to a file (af1_save_layer; format in include/af1.h)."""
+        _check(_lib.af1_save_layer(self._h, str(path).encode()))
+
+    def export(self, stream=None):
+        """(Uw, Vw, a, s, b): canonical packed words (int32, (m, W(r)) and
+        (r, W(n))) and FP16 scales, on the layer's device (af1_export_layer)."""
+        dev = torch.device("cuda", torch.cuda.current_device())
+        Uw = torch.empty((self.m, words_per_row(self.r)), dtype=torch.int32, device=dev)
+        Vw = torch.empty((self.r, words_per_row(self.n)), dtype=torch.int32, device=dev)
+        a = torch.empty(self.m, dtype=torch.float16, device=dev)
+        s = torch.empty(self.r, dtype=torch.float16, device=dev)
+        b = torch.empty(self.n, dtype=torch.float16, device=dev)
+        _check(_lib.af1_export_layer(self._h, _ptr(Uw), _ptr(Vw), _ptr(a), _ptr(s), _ptr(b), _stream_handle(stream)))
+        return Uw, Vw, a, s, b
 
     # -- queries ---------------------------------------------------------------
     def workspace_bytes(self, tokens: int = 1) -> int:

@@ -6,6 +6,7 @@
 #include <stdint.h>
 
 #include <cstdio>
+#include <cstring>
 #include <new>
 #include <string>
 
@@ -68,7 +69,7 @@ int check_desc(const af1_layer_desc* d) {
   if (d->m <= 0 || d->n <= 0 || d->r <= 0) return fail(AF1_ERR_INVALID_ARG, "m, n and r must be positive");
   if (d->m > ((int64_t)1 << 30) || d->n > af1::kMaxCols || d->r > af1::kMaxCols)
     return fail(AF1_ERR_INVALID_ARG, "m must be <= 2^30 and n, r <= " + std::to_string(af1::kMaxCols));
-  if (d->reserved != 0 || (d->flags & ~(AF1_FLAG_ANY_RANK | AF1_FLAG_TC_DECODE)) != 0)
+  if (d->reserved != 0 || (d->flags & ~(AF1_FLAG_ANY_RANK | AF1_FLAG_TC_DECODE | AF1_FLAG_BF16_SCALES)) != 0)
     return fail(AF1_ERR_INVALID_ARG, "unknown flags or non-zero reserved field");
   if (!(d->flags & AF1_FLAG_ANY_RANK)) {
     int64_t rmax = 0;
@@ -140,13 +141,25 @@ void destroy_layer(af1_layer* L) {
   delete L;
 }
 
-int copy_scales(af1_layer* L, const uint16_t* a, const uint16_t* s, const uint16_t* b, cudaStream_t st) {
-  cudaError_t e = cudaMemcpyAsync(L->a, a, 2 * L->m, cudaMemcpyDeviceToDevice, st);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(L->s, s, 2 * L->r, cudaMemcpyDeviceToDevice, st);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(L->b, b, 2 * L->n, cudaMemcpyDeviceToDevice, st);
-  if (e != cudaSuccess) return fail_cuda(e, "cudaMemcpyAsync(scales)");
+// The layer keeps FP16 scales. BF16 inputs (AF1_FLAG_BF16_SCALES) are
+// converted exactly; a value FP16 cannot hold sets *bad.
+int copy_scales(af1_layer* L, const uint16_t* a, const uint16_t* s, const uint16_t* b, cudaStream_t st,
+                uint32_t* bad) {
+  cudaError_t e;
+  if (L->flags & AF1_FLAG_BF16_SCALES) {
+    e = af1::launch_bf16_to_f16(a, L->a, L->m, bad, st);
+    if (e == cudaSuccess) e = af1::launch_bf16_to_f16(s, L->s, L->r, bad, st);
+    if (e == cudaSuccess) e = af1::launch_bf16_to_f16(b, L->b, L->n, bad, st);
+  } else {
+    e = cudaMemcpyAsync(L->a, a, 2 * L->m, cudaMemcpyDeviceToDevice, st);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(L->s, s, 2 * L->r, cudaMemcpyDeviceToDevice, st);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(L->b, b, 2 * L->n, cudaMemcpyDeviceToDevice, st);
+  }
+  if (e != cudaSuccess) return fail_cuda(e, "copying the scales");
   return AF1_OK;
 }
+
+const char* kBf16Msg = "a BF16 scale has no exact FP16 value (out of range or below its resolution)";
 
 int check_scales(const uint16_t* a, const uint16_t* s, const uint16_t* b, int dev) {
   int rc = check_device_ptr(a, "a", dev);
@@ -217,7 +230,7 @@ int af1_pack_layer(const af1_layer_desc* desc, const int8_t* U, const int8_t* V,
     cudaFree(scratch);
     return rc;
   }
-  e = cudaMemsetAsync(flag, 0, 4, st);
+  e = cudaMemsetAsync(flag, 0, 8, st);
   // U: m rows of r signs, row-major. V^T: r rows of n signs read from the
   // n x r row-major V (row stride 1, column stride r).
   if (e == cudaSuccess) e = af1::launch_pack_signs(U, m, r, r, 1, Uw, wu, flag, st);
@@ -229,15 +242,16 @@ int af1_pack_layer(const af1_layer_desc* desc, const int8_t* U, const int8_t* V,
     cudaFree(scratch);
     return fail_cuda(e, "pack kernels");
   }
-  rc = copy_scales(L, a, s, b, st);
-  uint32_t hflag = 0;
+  rc = copy_scales(L, a, s, b, st, flag + 1);
+  uint32_t hflag[2] = {0, 0};
   if (rc == AF1_OK) {
-    e = cudaMemcpyAsync(&hflag, flag, 4, cudaMemcpyDeviceToHost, st);
+    e = cudaMemcpyAsync(hflag, flag, 8, cudaMemcpyDeviceToHost, st);
     if (e == cudaSuccess) e = cudaStreamSynchronize(st);
     if (e != cudaSuccess) rc = fail_cuda(e, "pack synchronize");
   }
   cudaFree(scratch);
-  if (rc == AF1_OK && hflag != 0) rc = fail(AF1_ERR_INVALID_SIGN, "a sign entry is not exactly +1 or -1");
+  if (rc == AF1_OK && hflag[0] != 0) rc = fail(AF1_ERR_INVALID_SIGN, "a sign entry is not exactly +1 or -1");
+  if (rc == AF1_OK && hflag[1] != 0) rc = fail(AF1_ERR_INVALID_ARG, kBf16Msg);
   if (rc != AF1_OK) {
     destroy_layer(L);
     return rc;
@@ -269,11 +283,25 @@ int af1_load_packed_layer(const af1_layer_desc* desc, const uint32_t* U_words, c
     destroy_layer(L);
     return fail_cuda(e, "pack kernels");
   }
-  rc = copy_scales(L, a, s, b, st);
+  uint32_t* bad = nullptr;
+  if (desc->flags & AF1_FLAG_BF16_SCALES) {
+    e = cudaMalloc(&bad, 256);
+    if (e == cudaSuccess) e = cudaMemsetAsync(bad, 0, 4, st);
+    if (e != cudaSuccess) {
+      if (bad) cudaFree(bad);
+      destroy_layer(L);
+      return fail_cuda(e, "cudaMalloc(flag)");
+    }
+  }
+  rc = copy_scales(L, a, s, b, st, bad);
+  uint32_t hbad = 0;
   if (rc == AF1_OK) {
-    e = cudaStreamSynchronize(st);
+    e = bad ? cudaMemcpyAsync(&hbad, bad, 4, cudaMemcpyDeviceToHost, st) : cudaSuccess;
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
     if (e != cudaSuccess) rc = fail_cuda(e, "load synchronize");
   }
+  if (bad) cudaFree(bad);
+  if (rc == AF1_OK && hbad != 0) rc = fail(AF1_ERR_INVALID_ARG, kBf16Msg);
   if (rc != AF1_OK) {
     destroy_layer(L);
     return rc;
@@ -298,6 +326,114 @@ int af1_layer_device_bytes(const af1_layer* layer, int64_t* sign_bytes, int64_t*
   if (sign_bytes) *sign_bytes = layer->sign_bytes;
   if (scale_bytes) *scale_bytes = layer->scale_bytes;
   return AF1_OK;
+}
+
+int af1_export_layer(const af1_layer* layer, uint32_t* U_words, uint32_t* V_words, uint16_t* a, uint16_t* s,
+                     uint16_t* b, void* stream) {
+  if (layer == nullptr) return fail(AF1_ERR_INVALID_ARG, "layer is NULL");
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return fail_cuda(e, "cudaGetDevice");
+  if (dev != layer->device) return fail(AF1_ERR_BAD_POINTER, "the current device is not the layer's device");
+  int rc;
+  if (U_words && (rc = check_device_ptr(U_words, "U_words", dev)) != AF1_OK) return rc;
+  if (V_words && (rc = check_device_ptr(V_words, "V_words", dev)) != AF1_OK) return rc;
+  if (a && (rc = check_device_ptr(a, "a", dev)) != AF1_OK) return rc;
+  if (s && (rc = check_device_ptr(s, "s", dev)) != AF1_OK) return rc;
+  if (b && (rc = check_device_ptr(b, "b", dev)) != AF1_OK) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  e = cudaSuccess;
+  if (U_words) e = af1::launch_blocks_to_words(layer->signs2, layer->p2, words_per_row(layer->r), U_words, st);
+  if (e == cudaSuccess && V_words)
+    e = af1::launch_blocks_to_words(layer->signs1, layer->p1, words_per_row(layer->n), V_words, st);
+  if (e == cudaSuccess && a) e = cudaMemcpyAsync(a, layer->a, 2 * layer->m, cudaMemcpyDeviceToDevice, st);
+  if (e == cudaSuccess && s) e = cudaMemcpyAsync(s, layer->s, 2 * layer->r, cudaMemcpyDeviceToDevice, st);
+  if (e == cudaSuccess && b) e = cudaMemcpyAsync(b, layer->b, 2 * layer->n, cudaMemcpyDeviceToDevice, st);
+  if (e != cudaSuccess) return fail_cuda(e, "export");
+  g_err.clear();
+  return AF1_OK;
+}
+
+int af1_save_layer(const af1_layer* layer, const char* path) {
+  if (layer == nullptr || path == nullptr) return fail(AF1_ERR_INVALID_ARG, "layer or path is NULL");
+  const int64_t m = layer->m, n = layer->n, r = layer->r;
+  const int64_t nu = m * words_per_row(r), nv = r * words_per_row(n);
+  const int64_t bytes = 4 * (nu + nv) + 2 * (m + r + n);
+  uint8_t* d = nullptr;
+  cudaError_t e = cudaMalloc(&d, (size_t)(bytes + 1024));
+  if (e != cudaSuccess) return fail_cuda(e, "cudaMalloc(save)");
+  uint32_t* dU = reinterpret_cast<uint32_t*>(d);
+  uint32_t* dV = dU + nu;
+  uint16_t* da = reinterpret_cast<uint16_t*>(dV + nv);
+  uint16_t* ds = da + m;
+  uint16_t* db = ds + r;
+  int rc = af1_export_layer(layer, dU, dV, da, ds, db, nullptr);
+  std::string host((size_t)bytes, '\0');
+  if (rc == AF1_OK) {
+    e = cudaMemcpy(&host[0], d, (size_t)bytes, cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) rc = fail_cuda(e, "cudaMemcpy(save)");
+  }
+  cudaFree(d);
+  if (rc != AF1_OK) return rc;
+  af1_file_header hdr = {};
+  std::memcpy(hdr.magic, AF1_FILE_MAGIC, 8);
+  hdr.version = AF1_FILE_VERSION;
+  hdr.flags = (uint32_t)(layer->flags & ~AF1_FLAG_BF16_SCALES);  // the file stores FP16 scales
+  hdr.m = m;
+  hdr.n = n;
+  hdr.r = r;
+  FILE* f = std::fopen(path, "wb");
+  if (f == nullptr) return fail(AF1_ERR_IO, std::string("cannot open ") + path + " for writing");
+  const bool ok = std::fwrite(&hdr, sizeof(hdr), 1, f) == 1 && std::fwrite(host.data(), 1, host.size(), f) == host.size();
+  const bool closed = std::fclose(f) == 0;
+  if (!ok || !closed) return fail(AF1_ERR_IO, std::string("writing ") + path + " failed");
+  g_err.clear();
+  return AF1_OK;
+}
+
+int af1_load_layer(const char* path, void* stream, af1_layer** out) {
+  if (out == nullptr || path == nullptr) return fail(AF1_ERR_INVALID_ARG, "path or out is NULL");
+  *out = nullptr;
+  FILE* f = std::fopen(path, "rb");
+  if (f == nullptr) return fail(AF1_ERR_IO, std::string("cannot open ") + path);
+  af1_file_header hdr = {};
+  if (std::fread(&hdr, sizeof(hdr), 1, f) != 1 || std::memcmp(hdr.magic, AF1_FILE_MAGIC, 8) != 0 ||
+      hdr.version != AF1_FILE_VERSION) {
+    std::fclose(f);
+    return fail(AF1_ERR_IO, std::string(path) + " is not an AF1 layer file of version " +
+                                std::to_string(AF1_FILE_VERSION));
+  }
+  af1_layer_desc desc = {hdr.m, hdr.n, hdr.r, (int32_t)hdr.flags, 0};
+  int rc = check_desc(&desc);
+  if (rc != AF1_OK || (desc.flags & AF1_FLAG_BF16_SCALES)) {
+    std::fclose(f);
+    return rc != AF1_OK ? rc : fail(AF1_ERR_IO, std::string(path) + ": invalid flags");
+  }
+  const int64_t m = hdr.m, n = hdr.n, r = hdr.r;
+  const int64_t nu = m * words_per_row(r), nv = r * words_per_row(n);
+  const int64_t bytes = 4 * (nu + nv) + 2 * (m + r + n);
+  std::string host((size_t)bytes, '\0');
+  const bool ok = std::fread(&host[0], 1, host.size(), f) == host.size();
+  std::fclose(f);
+  if (!ok) return fail(AF1_ERR_IO, std::string(path) + " is truncated");
+  uint8_t* d = nullptr;
+  cudaError_t e = cudaMalloc(&d, (size_t)(bytes + 1024));
+  if (e != cudaSuccess) return fail_cuda(e, "cudaMalloc(load)");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  e = cudaMemcpyAsync(d, host.data(), (size_t)bytes, cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);  // `host` is pageable and freed on return
+  if (e != cudaSuccess) {
+    cudaFree(d);
+    return fail_cuda(e, "cudaMemcpyAsync(load)");
+  }
+  const uint32_t* dU = reinterpret_cast<const uint32_t*>(d);
+  const uint32_t* dV = dU + nu;
+  const uint16_t* da = reinterpret_cast<const uint16_t*>(dV + nv);
+  const uint16_t* ds = da + m;
+  const uint16_t* db = ds + r;
+  rc = af1_load_packed_layer(&desc, dU, dV, da, ds, db, stream, out);  // synchronizes `stream`
+  cudaFree(d);
+  return rc;
 }
 
 int64_t af1_workspace_bytes(const af1_layer* layer, int64_t tokens) {

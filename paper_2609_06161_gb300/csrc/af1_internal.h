@@ -54,6 +54,9 @@ cudaError_t launch_pack_signs(const int8_t* src, int64_t rows, int64_t cols, int
                               uint32_t* bad_flag, cudaStream_t st);
 cudaError_t launch_words_to_blocks(const uint32_t* words, int64_t words_per_row, const SignMatrix& sm,
                                    uint8_t* out, cudaStream_t st);
+cudaError_t launch_blocks_to_words(const uint8_t* blocks, const SignMatrix& sm, int64_t wpr, uint32_t* words,
+                                   cudaStream_t st);
+cudaError_t launch_bf16_to_f16(const uint16_t* src, uint16_t* dst, int64_t count, uint32_t* bad, cudaStream_t st);
 // Set the calling thread's af1_last_error() message; returns `code`.
 int set_error(int code, const std::string& msg);
 

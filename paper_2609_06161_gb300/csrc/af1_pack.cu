@@ -6,6 +6,10 @@
 // (2) words_to_blocks: canonical words -> the internal row-block layout
 //     described in af1_layout.h. The bit count is unchanged (1 bit per sign);
 //     only the order differs, plus the zero rows of a partial row block.
+// (3) blocks_to_words: the inverse, for exporting a layer.
+// (4) bf16_to_f16: BF16 scale bit patterns -> FP16 bit patterns, flagging
+//     any value FP16 does not represent exactly.
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -66,7 +70,53 @@ __global__ void words_to_blocks_kernel(const uint32_t* __restrict__ words, int64
   out[t] = v;
 }
 
+// One thread per canonical word: the inverse gather of words_to_blocks
+// (padding columns and rows beyond R are absent from, or zero in, the
+// canonical words).
+__global__ void blocks_to_words_kernel(const uint32_t* __restrict__ blocks, SignMatrix sm, int64_t wpr,
+                                       uint32_t* __restrict__ words) {
+  const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= sm.R * wpr) return;
+  const int64_t row = t / wpr, kw = t - row * wpr;
+  uint32_t v = 0;
+  if (kw < (int64_t)sm.NCH * kChunkWords) {
+    const uint32_t src = blocks[word_index(sm, row, kw)];
+#pragma unroll
+    for (int b = 0; b < 32; ++b) v |= ((src >> b) & 1u) << bit_col(b);
+  }
+  words[t] = v;
+}
+
+// BF16 value -> FP16 bits when FP16 holds the same value exactly (finite,
+// inside the FP16 range, no mantissa bit below its resolution); else *bad.
+__global__ void bf16_to_f16_kernel(const uint16_t* __restrict__ src, uint16_t* __restrict__ dst, int64_t count,
+                                   uint32_t* bad) {
+  const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= count) return;
+  const float f = __uint_as_float((uint32_t)src[t] << 16);
+  const __half h = __float2half_rn(f);
+  if (!(__half2float(h) == f)) atomicOr(bad, 1u);  // also catches NaN
+  dst[t] = __half_as_ushort(h);
+}
+
 }  // namespace
+
+cudaError_t launch_blocks_to_words(const uint8_t* blocks, const SignMatrix& sm, int64_t wpr, uint32_t* words,
+                                   cudaStream_t st) {
+  const int64_t total = sm.R * wpr;
+  if (total == 0) return cudaSuccess;
+  const int threads = 256;
+  blocks_to_words_kernel<<<(unsigned)((total + threads - 1) / threads), threads, 0, st>>>(
+      reinterpret_cast<const uint32_t*>(blocks), sm, wpr, words);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_bf16_to_f16(const uint16_t* src, uint16_t* dst, int64_t count, uint32_t* bad, cudaStream_t st) {
+  if (count == 0) return cudaSuccess;
+  const int threads = 256;
+  bf16_to_f16_kernel<<<(unsigned)((count + threads - 1) / threads), threads, 0, st>>>(src, dst, count, bad);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_pack_signs(const int8_t* src, int64_t rows, int64_t cols, int64_t row_stride,
                               int64_t col_stride, uint32_t* words, int64_t wpr, uint32_t* bad_flag,

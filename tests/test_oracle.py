@@ -6,6 +6,7 @@ from fractions import Fraction
 import numpy as np
 import pytest
 
+import synth
 from oracle import af1_oracle as O
 from tests.golden_io import load
 
@@ -251,6 +252,39 @@ def test_f16_widening_exact():
     assert v[0] == 1.0 and v[1] == -2.0 and v[2] == 2.0 ** -24 and v[3] == 65504.0
     assert v[4] == 1365 / 4096  # 0x3555: exponent 13 -> 2^-2 * (1 + 341/1024)
     assert v[5] == 0.0 and np.signbit(v[5])
+
+
+def test_bf16_widening_exact():
+    # BF16 = the upper half of an FP32: 1 sign, 8 exponent (bias 127), 7 mantissa bits.
+    bits = np.array([0x3F80, 0xC000, 0x3C23, 0x7F7F, 0x0001, 0x8000], dtype=np.uint16)
+    v = O.bf16_bits_to_f64(bits)
+    assert v[0] == 1.0 and v[1] == -2.0
+    assert v[2] == 163 / 16384  # exponent 120 -> 2^-7 * (1 + 35/128)
+    assert v[3] == 255 * 2.0 ** 120  # largest finite: 2^127 * (1 + 127/128)
+    assert v[4] == 2.0 ** -133  # smallest subnormal: 2^-126 * 2^-7
+    assert v[5] == 0.0 and np.signbit(v[5])
+
+
+def test_forward_bf16_scales_equal_f16_scales_of_equal_value():
+    """Scales whose BF16 and FP16 patterns hold the same values (dyadic
+    numbers with few significant bits) give the same forward; each of a, s, b
+    is decoded as BF16 (a pattern read as FP16 instead would change it)."""
+    g = synth.rng(5)
+    m, n, r, T = 9, 14, 6, 2
+    U, V = synth.signs(g, m, r), synth.signs(g, n, r)
+    vals = [0.5, 0.25, 1.5, 0.125, 2.0, 0.75]
+    def pick(k):
+        v = np.array([vals[i % len(vals)] for i in range(k)], dtype=np.float32)
+        f16 = v.astype(np.float16).view(np.uint16)
+        b16 = (v.view(np.uint32) >> np.uint32(16)).astype(np.uint16)
+        return f16, b16
+    (a16, ab), (s16, sb), (b16_, bb) = pick(m), pick(r), pick(n)
+    X = synth.activations_f16(g, T, n)
+    Uw, Vw = O.pack_U(U), O.pack_V(V)
+    y16 = O.forward_from_packed(Uw, Vw, a16, s16, b16_, X, m, n, r)
+    ybf = O.forward_from_packed(Uw, Vw, ab, sb, bb, X, m, n, r, scale_dtype="bf16")
+    np.testing.assert_array_equal(y16, ybf)
+    assert not np.array_equal(O.bf16_bits_to_f64(ab), O.f16_bits_to_f64(ab))
 
 
 # --------------------------------------------------------------------------
