@@ -252,6 +252,37 @@ AF1_API int af1_workspace_status(void* workspace, void* stream);
  * device before freeing, so queued work that reads the layer completes. */
 AF1_API void af1_free(af1_layer* layer);
 
+/* HiSA budget arithmetic (AF1 Sec. 3.2, "Hierarchical Shapley Allocation"),
+ * host-only, from Shapley scores the caller estimated (which needs a model
+ * and calibration data, outside this library). The paper has these as
+ * formulas; these functions state them once, in double precision.
+ *
+ * Layer budgets, Eq. hisa_layer_budget:
+ *   B_out[l] = B_total exp(phi[l] / tau) / sum_j exp(phi[j] / tau).
+ * With equal-size layers and a per-layer budget in bits per weight, B_total
+ * is L times the target average (e.g. L for 1.0 BPW). Errors: INVALID_ARG
+ * (L <= 0, tau <= 0, non-finite inputs, NULL). */
+AF1_API int af1_hisa_layer_budgets(const double* phi, int64_t L, double B_total, double tau, double* B_out);
+
+/* Module budgets within one layer (Eq. hisa_mad_norm, the logistic map and
+ * Soft-OR fusion, Eq. hisa_module_budget): for the N submodules with
+ * directional and magnitude Shapley scores phi_dir[i], phi_mag[i] and
+ * parameter counts params[i],
+ *   z_c = (phi_c - median) / (1.4826 MAD + eps),  P_c = 1 / (1 + exp(-z_c)),
+ *   v = 1 - (1 - P_dir)(1 - P_mag),  w = (v / params + eps)^alpha,
+ *   b_out[i] = B_l (sum_k params[k]) w_i / sum_j params[j] w_j,
+ * so that the parameter-weighted mean of b_out is B_l (bits per weight).
+ * The paper's defaults: alpha = 0.2; eps is not given (1e-8 is a reading).
+ * Errors: INVALID_ARG. */
+AF1_API int af1_hisa_module_budgets(const double* phi_dir, const double* phi_mag, const int64_t* params,
+                                    int64_t N, double B_l, double alpha, double eps, double* b_out);
+
+/* Budget-to-rank conversion (App. "Budget-to-rank conversion"):
+ * r = Round(b m n / (m + n)) (round half up; dominant sign bits only),
+ * clipped to [1, 32768]. For the exact storage rule use
+ * af1_rank_for_budget. Errors: INVALID_ARG. */
+AF1_API int af1_budget_to_rank(double b, int64_t m, int64_t n, int64_t* r_out);
+
 /* Message for the last error on the calling thread ("" if none). */
 AF1_API const char* af1_last_error(void);
 

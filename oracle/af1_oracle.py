@@ -261,3 +261,57 @@ def rowwise_rel_err(y, y_ref) -> float:
     den = np.abs(y_ref).max(axis=1)
     den = np.where(den > 0, den, 1.0)
     return float((num / den).max())
+
+
+# ---------------------------------------------------------------------------
+# HiSA budget math (Sec. 3.2 "Hierarchical Shapley Allocation"), as functions
+# of given Shapley scores. Plain loops over Python floats.
+# ---------------------------------------------------------------------------
+
+def hisa_layer_budgets(phi, B_total: float, tau: float):
+    """Eq. hisa_layer_budget: B_l = B_total exp(phi_l / tau) / sum_j exp(phi_j / tau).
+    The largest exponent is subtracted first (the ratio is unchanged)."""
+    top = max(p / tau for p in phi)
+    e = [math.exp(p / tau - top) for p in phi]
+    tot = sum(e)
+    return [B_total * v / tot for v in e]
+
+
+def _median(values):
+    v = sorted(values)
+    k = len(v)
+    return v[k // 2] if k % 2 else (v[k // 2 - 1] + v[k // 2]) / 2.0
+
+
+def mad_z(phi, eps: float):
+    """Eq. hisa_mad_norm: (phi_i - median) / (1.4826 MAD + eps), MAD the
+    median absolute deviation from the median."""
+    med = _median(phi)
+    mad = _median([abs(p - med) for p in phi])
+    return [(p - med) / (1.4826 * mad + eps) for p in phi]
+
+
+def hisa_module_budgets(phi_dir, phi_mag, params, B_l: float, alpha: float, eps: float):
+    """Module budgets of one layer: MAD z-scores of both distortion scores,
+    logistic map P = 1 / (1 + exp(-z)), Soft-OR fusion
+    v = 1 - (1 - P_dir)(1 - P_mag), size-aware density
+    w = (v / |W| + eps)^alpha and Eq. hisa_module_budget
+    b_i = B_l (sum_k |W_k|) w_i / sum_j |W_j| w_j (bits per weight; the
+    parameter-weighted mean of the b_i is B_l)."""
+    zd, zm = mad_z(phi_dir, eps), mad_z(phi_mag, eps)
+    w = []
+    for i in range(len(params)):
+        pd = 1.0 / (1.0 + math.exp(-zd[i]))
+        pm = 1.0 / (1.0 + math.exp(-zm[i]))
+        v = 1.0 - (1.0 - pd) * (1.0 - pm)
+        w.append((v / params[i] + eps) ** alpha)
+    total = float(sum(params))
+    den = sum(params[j] * w[j] for j in range(len(params)))
+    return [B_l * total * w[i] / den for i in range(len(params))]
+
+
+def budget_to_rank(b: float, d_out: int, d_in: int, r_max: int = 32768) -> int:
+    """App. "Budget-to-rank conversion": r = Round(b d_out d_in / (d_out + d_in))
+    (round half up), clipped to [1, r_max]."""
+    r = math.floor(b * d_out * d_in / (d_out + d_in) + 0.5)
+    return min(max(r, 1), r_max)

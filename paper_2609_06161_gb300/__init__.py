@@ -91,6 +91,14 @@ _lib.af1_save_layer.argtypes = [_vp, ctypes.c_char_p]
 _lib.af1_save_layer.restype = ctypes.c_int
 _lib.af1_load_layer.argtypes = [ctypes.c_char_p, _vp, ctypes.POINTER(_vp)]
 _lib.af1_load_layer.restype = ctypes.c_int
+_dp = ctypes.POINTER(ctypes.c_double)
+_lib.af1_hisa_layer_budgets.argtypes = [_dp, _i64, ctypes.c_double, ctypes.c_double, _dp]
+_lib.af1_hisa_layer_budgets.restype = ctypes.c_int
+_lib.af1_hisa_module_budgets.argtypes = [_dp, _dp, ctypes.POINTER(_i64), _i64, ctypes.c_double, ctypes.c_double,
+                                         ctypes.c_double, _dp]
+_lib.af1_hisa_module_budgets.restype = ctypes.c_int
+_lib.af1_budget_to_rank.argtypes = [ctypes.c_double, _i64, _i64, ctypes.POINTER(_i64)]
+_lib.af1_budget_to_rank.restype = ctypes.c_int
 _lib.af1_workspace_status.argtypes = [_vp, _vp]
 _lib.af1_workspace_status.restype = ctypes.c_int
 _lib.af1_free.argtypes = [_vp]
@@ -329,3 +337,35 @@ def forward_multi(layers, x: torch.Tensor, ys, workspace: torch.Tensor, stream=N
     ld = (_i64 * len(ys))(*ldys)
     _check(_lib.af1_linear_forward_multi(hs, len(layers), _ptr(x), ldx, tokens, yp, ld, yd, _ptr(workspace),
                                          workspace.numel() * workspace.element_size(), _stream_handle(stream)))
+
+
+# -- HiSA budget arithmetic (host) --------------------------------------------------
+
+def _dbl(v):
+    a = (ctypes.c_double * len(v))(*[float(x) for x in v])
+    return a
+
+
+def hisa_layer_budgets(phi, B_total: float, tau: float = 1.0):
+    """Layer budgets from layer Shapley scores (af1_hisa_layer_budgets)."""
+    out = (ctypes.c_double * len(phi))()
+    _check(_lib.af1_hisa_layer_budgets(_dbl(phi), len(phi), B_total, tau, out))
+    return list(out)
+
+
+def hisa_module_budgets(phi_dir, phi_mag, params, B_l: float, alpha: float = 0.2, eps: float = 1e-8):
+    """Module budgets (bits per weight) within one layer (af1_hisa_module_budgets)."""
+    n = len(params)
+    if len(phi_dir) != n or len(phi_mag) != n:
+        raise ValueError("one score pair per module")
+    out = (ctypes.c_double * n)()
+    p = (_i64 * n)(*[int(x) for x in params])
+    _check(_lib.af1_hisa_module_budgets(_dbl(phi_dir), _dbl(phi_mag), p, n, B_l, alpha, eps, out))
+    return list(out)
+
+
+def budget_to_rank(b: float, m: int, n: int) -> int:
+    """r = Round(b m n / (m + n)), clipped to [1, 32768] (af1_budget_to_rank)."""
+    r = _i64()
+    _check(_lib.af1_budget_to_rank(b, m, n, ctypes.byref(r)))
+    return r.value
