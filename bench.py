@@ -35,8 +35,8 @@ import numpy as np  # noqa: E402
 METRIC = "tokens/s and us/layer for binary-factorized linear (AF1, 1.0 BPW); % of HBM roofline"
 LAYERS = 32
 # Measured DRAM traffic of one layer's seven decode calls at one token (bytes;
-# ncu, profiles/lut_kernel_llama3_8b_b1.md): 1.028 x the algorithmic bytes.
-DECODE_TRAFFIC_B1_PER_LAYER = 28197888
+# ncu, profiles/lut_kernel_llama3_8b_b1.md): 1.026 x the algorithmic bytes.
+DECODE_TRAFFIC_B1_PER_LAYER = 28147456
 TC_DECODE = False  # set from --tc-decode
 
 
