@@ -86,6 +86,12 @@ extern "C" {
    FP16 has at that magnitude, NaN) fails the call with AF1_ERR_INVALID_ARG.
    Both types cost 16 bits, so the bit budget is unchanged. */
 #define AF1_FLAG_BF16_SCALES 4
+/* Run decode passes of 1 or 2 tokens on the streaming CUDA-core kernel (one
+   wave of CTAs, each streaming an equal share of the sign chunks) whenever it
+   has a plan. Without the flag it runs only where its plan beats the default
+   clustered kernel (matrices whose clustered split needs more than one wave
+   of CTAs). Results agree within the library's tolerance. */
+#define AF1_FLAG_STREAM_DECODE 8
 
 typedef struct af1_layer_desc {
   int64_t m;       /* d_out: rows of W_hat, length of a, length of y rows */
@@ -147,7 +153,7 @@ AF1_API int af1_export_layer(const af1_layer* layer, uint32_t* U_words, uint32_t
 /* Layer files. Layout (little-endian): the 40-byte header below, then U words
  * (m x W(r) uint32), V words (r x W(n) uint32), a (m FP16), s (r FP16), b
  * (n FP16), with no padding between the arrays. flags holds the layer's
- * AF1_FLAG_ANY_RANK / AF1_FLAG_TC_DECODE bits. */
+ * AF1_FLAG_ANY_RANK / AF1_FLAG_TC_DECODE / AF1_FLAG_STREAM_DECODE bits. */
 #define AF1_FILE_MAGIC "AF1LAYER"
 #define AF1_FILE_VERSION 1u
 typedef struct af1_file_header {

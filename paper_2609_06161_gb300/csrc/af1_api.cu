@@ -69,7 +69,8 @@ int check_desc(const af1_layer_desc* d) {
   if (d->m <= 0 || d->n <= 0 || d->r <= 0) return fail(AF1_ERR_INVALID_ARG, "m, n and r must be positive");
   if (d->m > ((int64_t)1 << 30) || d->n > af1::kMaxCols || d->r > af1::kMaxCols)
     return fail(AF1_ERR_INVALID_ARG, "m must be <= 2^30 and n, r <= " + std::to_string(af1::kMaxCols));
-  if (d->reserved != 0 || (d->flags & ~(AF1_FLAG_ANY_RANK | AF1_FLAG_TC_DECODE | AF1_FLAG_BF16_SCALES)) != 0)
+  if (d->reserved != 0 || (d->flags & ~(AF1_FLAG_ANY_RANK | AF1_FLAG_TC_DECODE | AF1_FLAG_BF16_SCALES |
+                                                AF1_FLAG_STREAM_DECODE)) != 0)
     return fail(AF1_ERR_INVALID_ARG, "unknown flags or non-zero reserved field");
   if (!(d->flags & AF1_FLAG_ANY_RANK)) {
     int64_t rmax = 0;

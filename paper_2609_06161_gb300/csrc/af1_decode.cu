@@ -1035,6 +1035,49 @@ Workspace plan_workspace(const af1_layer& L, int64_t tokens, bool prep) {
   return w;
 }
 
+namespace {
+
+// Kernel of one phase of a decode pass of T tokens: the tensor-core kernel
+// (tc), the streaming CUDA-core kernel (stream.ok) or the clustered one
+// (lut.ok); tc also when neither CUDA-core kernel has a plan.
+struct PhaseChoice {
+  bool tc = false;
+  LutPlan lut;
+  StreamPlan stream;
+};
+
+PhaseChoice choose_phase(const af1_layer& L, int phase, const SignMatrix& m, int T, const Workspace& W) {
+  PhaseChoice c;
+  // The tensor-core kernel when the layer asks for it, or for wide passes
+  // over matrices large enough for it (with a prepared B operand) to be the
+  // faster one.
+  if ((L.flags & AF1_FLAG_TC_DECODE) != 0 || (W.bbuf != 0 && T >= kTcMinTokens && m.R * m.C >= kTcMinSigns)) {
+    c.tc = true;
+    return c;
+  }
+  c.lut = plan_lut(&m, 1, T, L.num_sms, L.max_smem);
+  if (T <= 2) {
+    // The streaming kernel where the clustered split needs more than one
+    // wave of CTAs (each wave pays the CTAs' start-up and reduction), or
+    // wherever it has a plan when the layer asks for it. (On one-wave
+    // matrices it is faster alone but slower when several layers run at once
+    // on parallel streams, as a decoder's q|k|v and gate|up do: measured.)
+    const bool flag = (L.flags & AF1_FLAG_STREAM_DECODE) != 0;
+    bool want = flag || !c.lut.ok;
+    if (!want) {
+      const int sms = L.num_sms > 0 ? L.num_sms : 148;
+      int per_sm = 233472 / (c.lut.smem + 1024);
+      per_sm = per_sm > 4 ? 4 : per_sm;
+      want = (int64_t)m.RB * c.lut.KS > (int64_t)sms * per_sm;
+    }
+    if (want) c.stream = plan_stream(phase, m, T, L.num_sms, L.max_smem);
+  }
+  if (!c.stream.ok && !c.lut.ok) c.tc = true;
+  return c;
+}
+
+}  // namespace
+
 cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64_t tokens, void* y,
                            int64_t ldy, int y_dtype, void* ws, cudaStream_t st, bool prep, unsigned* status) {
   const Workspace W = plan_workspace(L, tokens, prep);
@@ -1059,22 +1102,12 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
   const int ysize = y_dtype == 0 ? 2 : 4;
   for (int64_t t0 = 0; t0 < tokens; t0 += pass) {
     const int T = (int)((tokens - t0) < pass ? (tokens - t0) : pass);
-    // A phase runs on the CUDA cores (af1_lut.cu) whenever that kernel has a
-    // plan, unless the layer asks for the tensor-core kernel (which is also
-    // the fallback) or the pass is wide and the matrix large enough for the
-    // tensor-core kernel with a prepared B operand to be faster.
-    const bool flag = (L.flags & AF1_FLAG_TC_DECODE) != 0;
-    auto wide_tc = [&](const SignMatrix& m) {
-      return W.bbuf != 0 && T >= kTcMinTokens && m.R * m.C >= kTcMinSigns;
-    };
-    const bool tc1 = flag || wide_tc(L.p1), tc2 = flag || wide_tc(L.p2);
-    const LutPlan l1 = tc1 ? LutPlan() : plan_lut(&L.p1, 1, T, L.num_sms, L.max_smem);
-    const LutPlan l2 = tc2 ? LutPlan() : plan_lut(&L.p2, 1, T, L.num_sms, L.max_smem);
+    const PhaseChoice c1 = choose_phase(L, 1, L.p1, T, W), c2 = choose_phase(L, 2, L.p2, T, W);
     DecodePlan q1, q2;
     const bool prep = W.bbuf != 0 && n_for_tokens(T) > 16;  // launch_decode prepares B then
-    if (!l1.ok) q1 = plan_decode(1, L.p1, T, L.num_sms, L.max_smem, prep);
-    if (!l2.ok) q2 = plan_decode(2, L.p2, T, L.num_sms, L.max_smem, prep);
-    if ((!l1.ok && !q1.ok) || (!l2.ok && !q2.ok)) return cudaErrorInvalidConfiguration;
+    if (c1.tc) q1 = plan_decode(1, L.p1, T, L.num_sms, L.max_smem, prep);
+    if (c2.tc) q2 = plan_decode(2, L.p2, T, L.num_sms, L.max_smem, prep);
+    if ((c1.tc && !q1.ok) || (c2.tc && !q2.ok)) return cudaErrorInvalidConfiguration;
 
     DecodeArgs a1 = {};
     a1.signs = L.signs1;
@@ -1089,7 +1122,9 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
     a1.status = stat;
     a1.bbuf = W.bbuf != 0 ? wsb + W.bbuf : nullptr;
     a1.bstats = W.bbuf != 0 ? reinterpret_cast<float2*>(wsb + W.bstats) : nullptr;
-    cudaError_t e = l1.ok ? launch_lut(1, lut_args(a1), l1, st) : launch_decode<1>(a1, q1, st);
+    cudaError_t e = c1.tc         ? launch_decode<1>(a1, q1, st)
+                    : c1.stream.ok ? launch_stream(1, lut_problem(a1), T, 0, c1.stream, stat, st)
+                                   : launch_lut(1, lut_args(a1), c1.lut, st);
     if (e != cudaSuccess) return e;
 
     DecodeArgs a2 = {};
@@ -1105,7 +1140,9 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
     a2.status = a1.status;
     a2.bbuf = a1.bbuf;
     a2.bstats = a1.bstats;
-    e = l2.ok ? launch_lut(2, lut_args(a2), l2, st) : launch_decode<2>(a2, q2, st);
+    e = c2.tc         ? launch_decode<2>(a2, q2, st)
+        : c2.stream.ok ? launch_stream(2, lut_problem(a2), T, y_dtype, c2.stream, stat, st)
+                       : launch_lut(2, lut_args(a2), c2.lut, st);
     if (e != cudaSuccess) return e;
   }
   return cudaSuccess;
@@ -1125,15 +1162,15 @@ cudaError_t launch_forward_multi(const af1_layer* const* Ls, int count, const vo
   unsigned* status = reinterpret_cast<unsigned*>(wsb);  // layer 0's slice starts with its status word
   const int T = (int)tokens;
   // One launch per phase for all layers when every phase of every layer
-  // would run on the lookup-table kernel anyway and the group has a plan.
+  // would run on the clustered lookup-table kernel anyway and the group has
+  // a plan.
   bool group = tokens <= kMaxPassTokens;
   SignMatrix m1[kMaxGroup], m2[kMaxGroup];
   for (int i = 0; i < count && group; ++i) {
     const af1_layer& L = *Ls[i];
-    const bool wide = prep && T >= kTcMinTokens && n_for_tokens(T) > 16;
-    if ((L.flags & AF1_FLAG_TC_DECODE) != 0 || (wide && (L.p1.R * L.p1.C >= kTcMinSigns ||
-                                                         L.p2.R * L.p2.C >= kTcMinSigns)))
-      group = false;
+    const Workspace W = plan_workspace(L, tokens, prep);
+    const PhaseChoice c1 = choose_phase(L, 1, L.p1, T, W), c2 = choose_phase(L, 2, L.p2, T, W);
+    if (c1.tc || c2.tc || c1.stream.ok || c2.stream.ok) group = false;
     m1[i] = L.p1;
     m2[i] = L.p2;
   }

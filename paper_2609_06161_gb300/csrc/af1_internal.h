@@ -97,6 +97,20 @@ struct LutPlan {
 LutPlan plan_lut(const SignMatrix* sm, int count, int T, int num_sms, int max_smem);
 cudaError_t launch_lut(int phase, const LutArgs& a, const LutPlan& p, cudaStream_t st);
 
+// Decode passes of 1..2 tokens over matrices too large for one wave of the
+// clustered kernel (af1_stream.cu): clusters of KS CTAs per super row of G
+// row blocks, CPC chunks per CTA, streamed through a ring of NSC slots, in
+// one wave.
+struct StreamPlan {
+  int G = 0, KS = 0, CPC = 0, NSC = 0, smem = 0;
+  bool ok = false;
+};
+// Plan of `phase` for a pass of T tokens over sm on the current device (not
+// ok when no split runs in one wave).
+StreamPlan plan_stream(int phase, const SignMatrix& sm, int T, int num_sms, int max_smem);
+cudaError_t launch_stream(int phase, const LutProblem& prob, int tokens, int ydtype, const StreamPlan& p,
+                          unsigned* status, cudaStream_t st);
+
 cudaError_t launch_prefill(const af1_layer& L, const void* x, int64_t ldx, int64_t tokens, void* y, int64_t ldy,
                            int y_dtype, uint8_t* h_buf, unsigned* status, cudaStream_t st);
 // status: the status word to report to (nullptr: the workspace's own).

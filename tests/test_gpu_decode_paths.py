@@ -92,7 +92,7 @@ def test_unknown_flag_rejected(P):
     U = torch.from_numpy(d["U"]).cuda()
     V = torch.from_numpy(d["V"]).cuda()
     a, s, b = (torch.from_numpy(d[k].view(np.float16)).cuda() for k in ("a", "s", "b"))
-    desc = P._Desc(64, 96, 20, 4 | P.AF1_FLAG_ANY_RANK, 0)
+    desc = P._Desc(64, 96, 20, 64 | P.AF1_FLAG_ANY_RANK, 0)
     h = ctypes.c_void_p()
     rc = P._lib.af1_pack_layer(ctypes.byref(desc), U.data_ptr(), V.data_ptr(), a.data_ptr(), s.data_ptr(),
                                b.data_ptr(), None, None, None, ctypes.byref(h))
