@@ -368,65 +368,70 @@ cudaError_t launch_np(const StreamArgs& a, const StreamPlan& p, cudaStream_t st)
 
 }  // namespace
 
-// Every (G, KS) split that runs in one wave of CTAs at 3 (else 2) CTAs per
-// SM (the device runs all SRB clusters at once), with a ring deep enough to
-// cover a copy (about 2 us under load) when it fits, and no deeper than the
-// slice; the one with the smallest modelled time on its busiest SM: lookups
-// of G x CPC tiles at the measured per-SM rate for that many CTAs, table
-// builds (about a twentieth of a tile's lookups per chunk), and the wait for
-// refills the slots ahead do not cover. Not ok when no split fits in one
-// wave.
+// Every (G, KS) split whose SRB clusters the device runs at once (one wave)
+// with at most 3 CTAs per SM (the register budget of 288 threads), each CTA
+// padded with shared memory so that no SM holds more than its share
+// ceil(CTAs / SMs) (the block scheduler would otherwise fill some SMs and
+// leave others idle); the padding deepens the ring, up to the whole slice.
+// The chosen split has the smallest modelled time on an SM: lookups of G x
+// CPC tiles at the measured per-SM rate for that many CTAs, table builds
+// (about a twentieth of a tile's lookups per chunk), and the wait for
+// refills the slots ahead do not cover (a copy takes about 2 us under load).
+// Not ok when no split fits in one wave.
 StreamPlan search_stream(int phase, const SignMatrix& sm, int T, int num_sms, int max_smem) {
   StreamPlan p;
   if (T < 1 || T > kMaxStreamTokens || sm.RB < 1 || sm.NCH < 1) return p;
   const int sms = num_sms > 0 ? num_sms : 148;
   int64_t best = -1;
-  for (int per_sm = 3; per_sm >= 2; --per_sm) {
-    for (int G = 1; G <= kMaxStreamG; G *= 2) {
-      const int64_t SRB = (sm.RB + G - 1) / G;
-      const int64_t kmax = (int64_t)sms * per_sm / SRB;
-      for (int k = 1; k <= kMaxStreamKS && k <= kmax && k <= sm.NCH; ++k) {
-        const int CPC = (sm.NCH + k - 1) / k;
-        const int KS = (sm.NCH + CPC - 1) / CPC;
-        if (KS != k) continue;  // the same split as a smaller k
-        const int budget = (kSmemPerSM / per_sm - kSmemPerCTA) < max_smem ? kSmemPerSM / per_sm - kSmemPerCTA
-                                                                           : max_smem;
-        const int64_t ctas = SRB * KS;
-        const int64_t on_sm = (ctas + sms - 1) / sms;  // CTAs on the busiest SM
-        // Lookup rate per SM (signs per ns, one token) with 1, 2, >= 3 CTAs
-        // of 8 lookup warps: a probe of the inner loop on GB300.
-        const double rate = on_sm >= 3 ? 155.0 : on_sm == 2 ? 149.0 : 130.0;
-        const double tile_ns = 16384.0 * (double)on_sm / rate * (T == 2 ? 1.35 : 1.0);
-        const int base = stream_smem(CPC, KS, T, G, 0).total;
-        const int fit = (budget - base) / (G * kChunkBytes);
-        int NSC = (int)(kCopyNs / (G * tile_ns)) + 2;  // the slots ahead cover a copy
-        NSC = NSC > 4 ? NSC : 4;
-        NSC = NSC < fit ? NSC : fit;
-        NSC = NSC < CPC ? NSC : CPC;
-        NSC = NSC < kMaxRing ? NSC : kMaxRing;
-        if (NSC < 2 && NSC < CPC) continue;
-        if (per_sm < 3 && 3 * (stream_smem(CPC, KS, T, G, 2).total + kSmemPerCTA) <= kSmemPerSM)
-          continue;  // counted with 3 per SM
-        const int smem = stream_smem(CPC, KS, T, G, NSC).total;
-        if (SRB > max_active_clusters(phase, T, G, KS, smem)) continue;  // more than one wave
-        double ns = (G * CPC + 0.05 * CPC) * tile_ns;
-        if (NSC < CPC) {
-          const double cover = (NSC - 1) * G * tile_ns;
-          if (cover < kCopyNs) ns += (kCopyNs - cover) * ((CPC - 1) / NSC);
-        }
-        const int64_t score = (int64_t)ns;
-        if (best < 0 || score < best) {
-          best = score;
-          p.G = G;
-          p.KS = KS;
-          p.CPC = CPC;
-          p.NSC = NSC;
-          p.smem = smem;
-          p.ok = true;
-        }
+  for (int G = 1; G <= kMaxStreamG; G *= 2) {
+    const int64_t SRB = (sm.RB + G - 1) / G;
+    for (int k = 1; k <= kMaxStreamKS && k <= sm.NCH; ++k) {
+      const int CPC = (sm.NCH + k - 1) / k;
+      const int KS = (sm.NCH + CPC - 1) / CPC;
+      if (KS != k) continue;  // the same split as a smaller k
+      const int64_t ctas = SRB * KS;
+      const int on_sm = (int)((ctas + sms - 1) / sms);  // CTAs per SM, spread evenly
+      if (on_sm > 3) break;                             // larger k only adds CTAs
+      // Shared memory per CTA: at most this SM's share, at least enough that
+      // one more CTA does not fit.
+      int budget = kSmemPerSM / on_sm - kSmemPerCTA;
+      budget = budget < max_smem ? budget : max_smem;
+      const int floor_smem = on_sm < 3 ? kSmemPerSM / (on_sm + 1) - kSmemPerCTA + 256 : 0;
+      // Lookup rate per SM (signs per ns, one token) with 1, 2, >= 3 CTAs
+      // of 8 lookup warps: a probe of the inner loop on GB300.
+      const double rate = on_sm >= 3 ? 155.0 : on_sm == 2 ? 149.0 : 130.0;
+      const double tile_ns = 16384.0 * (double)on_sm / rate * (T == 2 ? 1.35 : 1.0);
+      const int base = stream_smem(CPC, KS, T, G, 0).total;
+      if (base > budget) continue;
+      int NSC = (budget > floor_smem ? floor_smem - base : 0) / (G * kChunkBytes);  // slots the padding pays for
+      const int need = (int)(kCopyNs / (G * tile_ns)) + 2;  // slots ahead that cover a copy
+      const int fit = (budget - base) / (G * kChunkBytes);
+      NSC = NSC > need ? NSC : need;
+      NSC = NSC > 4 ? NSC : 4;
+      NSC = NSC < fit ? NSC : fit;
+      NSC = NSC < CPC ? NSC : CPC;
+      NSC = NSC < kMaxRing ? NSC : kMaxRing;
+      if (NSC < 2 && NSC < CPC) continue;
+      int smem = stream_smem(CPC, KS, T, G, NSC).total;
+      smem = smem > floor_smem ? smem : floor_smem;
+      if (smem > budget) continue;
+      if (SRB > max_active_clusters(phase, T, G, KS, smem)) continue;  // more than one wave
+      double ns = (G * CPC + 0.05 * CPC) * tile_ns;
+      if (NSC < CPC) {
+        const double cover = (NSC - 1) * G * tile_ns;
+        if (cover < kCopyNs) ns += (kCopyNs - cover) * ((CPC - 1) / NSC);
+      }
+      const int64_t score = (int64_t)ns;
+      if (best < 0 || score < best) {
+        best = score;
+        p.G = G;
+        p.KS = KS;
+        p.CPC = CPC;
+        p.NSC = NSC;
+        p.smem = smem;
+        p.ok = true;
       }
     }
-    if (p.ok) return p;
   }
   return p;
 }
