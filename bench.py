@@ -61,6 +61,10 @@ def parse():
     p.add_argument("--no-sweep", action="store_true",
                    help="skip the per-shape sweep (LLaMA-3-8B at 1/4/16 tokens, 70B shapes at 1/8/64/512)")
     p.add_argument("--no-stack", action="store_true", help="skip the 32-layer stack with HiSA-like ranks")
+    p.add_argument("--shape", default=None, metavar="MxN",
+                   help="time one linear of this shape (1.0-BPW rank) at --batch tokens instead of the stack: "
+                        "--steps calls rotating over copies larger than L2; prints one JSON line (per-shape "
+                        "measurement and profiling, e.g. with --no-graph under ncu)")
     p.add_argument("--tc-decode", action="store_true",
                    help="create layers with AF1_FLAG_TC_DECODE (tensor-core decode kernel instead of lookup tables)")
     return p.parse_args()
@@ -523,6 +527,9 @@ def main():
         b = args.batch
         if not 1 <= b <= 16:
             raise SystemExit("--batch must be in 1..16 for the decode path")
+    if args.shape:
+        run_shape(P, torch, args)
+        return
     dev = torch.device("cuda", torch.cuda.current_device())
     objs = build_layers(P, torch, args.layers, b, rank, outlier_frac=0.01 if args.workload == "prefill" else 0.0)
     ws = torch.zeros(max(o[4].workspace_bytes(b) for o in objs), dtype=torch.uint8, device=dev)
@@ -737,6 +744,54 @@ def main():
         print(json.dumps(line))
     if world > 1:
         dist.destroy_process_group()
+
+
+def run_shape(P, torch, args):
+    """One linear of shape --shape at its 1.0-BPW rank and --batch tokens:
+    --warmup then --steps calls, each on the next of enough copies of the
+    layer to exceed twice the L2 (every call streams its signs from HBM), in
+    a CUDA graph or (--no-graph) as eager launches for profilers."""
+    import math
+    m, n = (int(v) for v in args.shape.lower().split("x"))
+    b = args.batch
+    r = P.rank_for_budget(m, n)
+    packed = r * (m + n) // 8 + 2 * (m + n + r)
+    copies = max(2, min(128, math.ceil(2 * L2_BYTES / packed)))
+    layers = [device_layer(P, torch, m, n, r, 7000 + c) for c in range(copies)]
+    g = torch.Generator(device="cuda")
+    g.manual_seed(9000 + b)
+    x = torch.randn((b, n), generator=g, device="cuda", dtype=torch.float16)
+    y = torch.empty((b, m), device="cuda", dtype=torch.float16)
+    ws = torch.zeros(layers[0].workspace_bytes(b), dtype=torch.uint8, device="cuda")
+    stream = torch.cuda.Stream()
+    calls = max(args.steps, 1)
+
+    def run(k):
+        for i in range(k):
+            layers[i % copies].forward_into(x, y, ws, stream=stream)
+
+    if args.no_graph:
+        with torch.cuda.stream(stream):
+            run(max(args.warmup, 1))
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        with torch.cuda.stream(stream):
+            run(calls)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        us = e0.elapsed_time(e1) * 1e3 / calls
+    else:
+        us = time_graph(torch, lambda: run(copies), stream, max(1, calls // copies)) * 1e3 / copies
+    P.workspace_status(ws)
+    peaks = load_peaks()
+    alg = algorithmic_bytes(m, n, r, b)
+    line = {"shape": f"{m}x{n}", "rank": r, "tokens": b, "us_per_call": us, "copies": copies,
+            "graph": not args.no_graph, "algorithmic_bytes": alg, "achieved_gbs": alg / (us * 1e-6) / 1e9,
+            "hbm_frac": alg / (us * 1e-6) / 1e9 / peaks.get("hbm_gbs", 6800.0)}
+    print(json.dumps(line))
+    for L in layers:
+        L.free()
 
 
 def load_peaks():
