@@ -453,6 +453,58 @@ def dag_step(torch, views, stream, side, ws, ws_side):
         down[0].forward_into(down[1], down[2], ws, stream=stream)
 
 
+def mlp_swiglu(P, torch, stream, steps):
+    """LLaMA-3-8B MLP blocks at one token: gate | up (parallel streams), then
+    the down projection of h = FP16(SiLU(gate) * up). Fused: the down call
+    forms h itself (af1_linear_forward_swiglu); unfused: h by torch
+    elementwise ops, then af1_linear_forward. 32 blocks rotate (weights far
+    larger than L2); CUDA graph."""
+    blocks = 32
+    rank = P.rank_for_budget
+    mk = lambda m, n, seed: device_layer(P, torch, m, n, rank(m, n), seed)
+    gates = [mk(14336, 4096, 5000 + 3 * i) for i in range(blocks)]
+    ups = [mk(14336, 4096, 5001 + 3 * i) for i in range(blocks)]
+    downs = [mk(4096, 14336, 5002 + 3 * i) for i in range(blocks)]
+    g = torch.Generator(device="cuda")
+    g.manual_seed(77)
+    x = torch.randn((1, 4096), generator=g, device="cuda", dtype=torch.float16)
+    gy = torch.empty((1, 14336), device="cuda", dtype=torch.float16)
+    uy = torch.empty_like(gy)
+    h = torch.empty_like(gy)
+    y = torch.empty((1, 4096), device="cuda", dtype=torch.float16)
+    nbytes = max(downs[0].workspace_bytes_swiglu(1), gates[0].workspace_bytes(1))
+    ws = torch.zeros(nbytes, dtype=torch.uint8, device="cuda")
+    ws_side = torch.zeros_like(ws)
+    side = torch.cuda.Stream()
+
+    def run(fused):
+        for i in range(blocks):
+            ev = torch.cuda.Event()
+            ev.record(stream)
+            side.wait_event(ev)
+            gates[i].forward_into(x, gy, ws, stream=stream)
+            ups[i].forward_into(x, uy, ws_side, stream=side)
+            e = torch.cuda.Event()
+            e.record(side)
+            stream.wait_event(e)
+            if fused:
+                downs[i].forward_swiglu_into(gy, uy, y, ws, stream=stream)
+            else:
+                with torch.cuda.stream(stream):
+                    h.copy_(torch.nn.functional.silu(gy.float()).mul_(uy.float()))
+                downs[i].forward_into(h, y, ws, stream=stream)
+
+    reps = max(2, steps // 10)
+    fused_us = time_graph(torch, lambda: run(True), stream, reps) * 1e3 / blocks
+    unfused_us = time_graph(torch, lambda: run(False), stream, reps) * 1e3 / blocks
+    for L in gates + ups + downs:
+        L.free()
+    return {"workload": "32 LLaMA-3-8B MLP blocks, 1 token: gate | up on two streams, then down on "
+                        "h = FP16(SiLU(gate) * up); CUDA graph",
+            "fused_us_per_block": fused_us, "unfused_us_per_block": unfused_us,
+            "unfused": "h by torch elementwise ops (FP32 SiLU and product, FP16 store), then af1_linear_forward"}
+
+
 def stack_hisa(P, torch, peaks, stream, steps, dense_ms=None):
     """32-layer LLaMA-3-8B stack with HiSA-like per-matrix ranks (+-30 %
     around the 1.0-BPW rank, renormalised to 1.0 BPW over the stack), one
@@ -681,12 +733,13 @@ def main():
     if not args.no_dense and rank == 0:
         dense = dense_bf16(torch, objs, b, args, stream)
     peaks = load_peaks()
-    sweep_rows = stack = None
+    sweep_rows = stack = mlp = None
     if args.workload == "decode" and rank == 0:
         # Extra measurements, outside the timed region of the headline number.
         if not args.no_stack:
             stack = stack_hisa(P, torch, peaks, stream, args.steps,
                                dense_ms=dense["ms_per_step"] if dense and b == 1 else None)
+            mlp = mlp_swiglu(P, torch, stream, args.steps)
         if not args.no_sweep:
             sweep_rows = sweep(P, torch, peaks, stream)
 
@@ -734,6 +787,8 @@ def main():
             line["other_schedules"] = others
         if stack is not None:
             line["stack_hisa"] = stack
+        if mlp is not None:
+            line["mlp_swiglu"] = mlp
         if sweep_rows is not None:
             line["sweep"] = sweep_rows
         if not args.no_cpu and world == 1 and args.workload == "decode":

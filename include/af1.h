@@ -205,6 +205,23 @@ AF1_API int af1_linear_forward(const af1_layer* layer, const void* x, int64_t ld
                        void* y, int64_t ldy, int y_dtype, void* workspace,
                        int64_t workspace_bytes, void* stream);
 
+/* SwiGLU input of a down projection (the MLP of the LLaMA models the paper
+ * compresses): y = h . W_hat^T with h = FP16(SiLU(g) * u) elementwise,
+ * SiLU(z) = z / (1 + e^-z) in FP32, from the outputs g and u of the gate and
+ * up projections, without h in memory where the kernel allows it.
+ *   g, u: FP16 [tokens x n], both with row stride ldx, each under the rules
+ *       of x in af1_linear_forward (16-byte aligned, ldx % 8 == 0).
+ *   workspace: at least af1_workspace_bytes_swiglu(layer, tokens) bytes.
+ * Other arguments, stream semantics and errors as af1_linear_forward
+ * (u NULL: INVALID_ARG). Decode passes on the CUDA-core kernels form h while
+ * they stage their activations; the tensor-core kernels (AF1_FLAG_TC_DECODE,
+ * wide passes, prefill) first write h into the workspace. Both give the same
+ * h. */
+AF1_API int64_t af1_workspace_bytes_swiglu(const af1_layer* layer, int64_t tokens);
+AF1_API int af1_linear_forward_swiglu(const af1_layer* layer, const void* g, const void* u, int64_t ldx,
+                                      int64_t tokens, void* y, int64_t ldy, int y_dtype, void* workspace,
+                                      int64_t workspace_bytes, void* stream);
+
 /* Several layers applied to the same input, e.g. the q, k and v projections
  * of a decoder layer (or gate and up): y_i = x . W_hat_i^T for i < count.
  * The paper has no counterpart; it is the batching of a decoder layer's

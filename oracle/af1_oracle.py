@@ -171,6 +171,36 @@ def bf16_bits_to_f64(h) -> np.ndarray:
     return (h.astype(np.uint32) << np.uint32(16)).view(np.float32).astype(np.float64)
 
 
+def f64_to_f16_bits(v) -> np.ndarray:
+    """float64 -> FP16 bit patterns, rounded once to nearest (ties to even);
+    beyond the FP16 range the result is +-inf."""
+    with np.errstate(over="ignore"):
+        return np.asarray(v, dtype=np.float64).astype(np.float16).view(np.uint16)
+
+
+# ---------------------------------------------------------------------------
+# SwiGLU input of a down projection (the MLP of the LLaMA models the paper
+# compresses: h = SiLU(x W_gate^T) * (x W_up^T), SiLU(z) = z * sigmoid(z)).
+# Not part of AF1 itself; the fused entry point takes h from the gate and up
+# outputs.
+# ---------------------------------------------------------------------------
+
+def silu_f64(z) -> np.ndarray:
+    """SiLU(z) = z / (1 + e^-z) in float64."""
+    z = np.asarray(z, dtype=np.float64)
+    with np.errstate(over="ignore"):
+        return z / (1.0 + np.exp(-z))
+
+
+def swiglu_f16(g_h, u_h) -> np.ndarray:
+    """h = SiLU(g) * u from FP16 bit patterns g and u (same shape), in
+    float64, rounded once to FP16: the activations the down projection sees.
+    Returns FP16 bit patterns."""
+    g = f16_bits_to_f64(g_h)
+    u = f16_bits_to_f64(u_h)
+    return f64_to_f16_bits(silu_f64(g) * u).reshape(np.shape(g_h))
+
+
 # ---------------------------------------------------------------------------
 # Reconstruction and forward (Eq. double_factor_equiv, Eq. binary_paths)
 # ---------------------------------------------------------------------------

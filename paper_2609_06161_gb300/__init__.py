@@ -81,6 +81,10 @@ _lib.af1_workspace_bytes.argtypes = [_vp, _i64]
 _lib.af1_workspace_bytes.restype = _i64
 _lib.af1_linear_forward.argtypes = [_vp, _vp, _i64, _i64, _vp, _i64, ctypes.c_int, _vp, _i64, _vp]
 _lib.af1_linear_forward.restype = ctypes.c_int
+_lib.af1_workspace_bytes_swiglu.argtypes = [_vp, _i64]
+_lib.af1_workspace_bytes_swiglu.restype = _i64
+_lib.af1_linear_forward_swiglu.argtypes = [_vp, _vp, _vp, _i64, _i64, _vp, _i64, ctypes.c_int, _vp, _i64, _vp]
+_lib.af1_linear_forward_swiglu.restype = ctypes.c_int
 _lib.af1_workspace_bytes_multi.argtypes = [ctypes.POINTER(_vp), ctypes.c_int, _i64]
 _lib.af1_workspace_bytes_multi.restype = _i64
 _lib.af1_linear_forward_multi.argtypes = [ctypes.POINTER(_vp), ctypes.c_int, _vp, _i64, _i64, ctypes.POINTER(_vp),
@@ -290,6 +294,56 @@ class Layer:
         y = torch.empty((tokens, ldy), dtype=out_dtype, device=x.device)
         ws = workspace if workspace is not None else self.make_workspace(tokens, x.device)
         self.forward_into(x, y, ws, stream)
+        return y[:, :self.m]
+
+    def workspace_bytes_swiglu(self, tokens: int = 1) -> int:
+        v = _lib.af1_workspace_bytes_swiglu(self._h, tokens)
+        if v < 0:
+            raise AF1Error(int(v), last_error())
+        return int(v)
+
+    def forward_swiglu_into(self, g: torch.Tensor, u: torch.Tensor, y: torch.Tensor, workspace: torch.Tensor,
+                            stream=None) -> None:
+        """y[:tokens, :m] = h W_hat^T with h = FP16(SiLU(g) * u)
+        (af1_linear_forward_swiglu); g and u float16 (tokens, ldx) with the
+        same strides, y float16 or float32 (tokens, ldy)."""
+        for t in (g, u, y):
+            if t.dim() != 2 or t.stride(1) != 1:
+                raise ValueError("g, u and y must be 2-D with contiguous rows")
+        if g.dtype != torch.float16 or u.dtype != torch.float16:
+            raise ValueError("g and u must be float16")
+        if g.shape != u.shape or g.stride() != u.stride():
+            raise ValueError("g and u must have the same shape and strides")
+        if y.dtype == torch.float16:
+            yd = AF1_F16
+        elif y.dtype == torch.float32:
+            yd = AF1_F32
+        else:
+            raise ValueError("y must be float16 or float32")
+        tokens = g.shape[0]
+        if y.shape[0] < tokens:
+            raise ValueError("y has fewer rows than g")
+        ldx = g.stride(0) if tokens > 1 else max(g.stride(0), self.n + (-self.n) % 8)
+        ldy = y.stride(0) if tokens > 1 else max(y.stride(0), self.m + (-self.m) % (8 if yd == AF1_F16 else 4))
+        _check(_lib.af1_linear_forward_swiglu(self._h, _ptr(g), _ptr(u), ldx, tokens, _ptr(y), ldy, yd,
+                                              _ptr(workspace), workspace.numel() * workspace.element_size(),
+                                              _stream_handle(stream)))
+
+    def forward_swiglu(self, g: torch.Tensor, u: torch.Tensor, out_dtype=torch.float16,
+                       workspace: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+        if g.dim() == 1:
+            g, u = g.unsqueeze(0), u.unsqueeze(0)
+        tokens = g.shape[0]
+        pad = (-self.n) % 8
+        gp = torch.zeros((tokens, self.n + pad), dtype=torch.float16, device=g.device)
+        up = torch.zeros_like(gp)
+        gp[:, :self.n] = g
+        up[:, :self.n] = u
+        align = 8 if out_dtype == torch.float16 else 4
+        y = torch.empty((tokens, self.m + (-self.m) % align), dtype=out_dtype, device=g.device)
+        ws = workspace if workspace is not None else torch.zeros(self.workspace_bytes_swiglu(tokens),
+                                                                 dtype=torch.uint8, device=g.device)
+        self.forward_swiglu_into(gp, up, y, ws, stream)
         return y[:, :self.m]
 
     def free(self) -> None:

@@ -453,7 +453,8 @@ int af1_linear_forward(const af1_layer* layer, const void* x, int64_t ldx, int64
 namespace af1 {
 
 int linear_forward_checked(const af1_layer* layer, const void* x, int64_t ldx, int64_t tokens, void* y, int64_t ldy,
-                           int y_dtype, void* workspace, int64_t workspace_bytes, void* stream, bool prep) {
+                           int y_dtype, void* workspace, int64_t workspace_bytes, void* stream, bool prep,
+                           const void* x2) {
   if (layer == nullptr) return fail(AF1_ERR_INVALID_ARG, "layer is NULL");
   if (tokens < 0) return fail(AF1_ERR_INVALID_ARG, "tokens must be >= 0");
   if (y_dtype != AF1_F16 && y_dtype != AF1_F32) return fail(AF1_ERR_INVALID_ARG, "y_dtype must be AF1_F16 or AF1_F32");
@@ -466,7 +467,10 @@ int linear_forward_checked(const af1_layer* layer, const void* x, int64_t ldx, i
   if (e != cudaSuccess) return fail_cuda(e, "cudaGetDevice");
   if (dev != layer->device) return fail(AF1_ERR_BAD_POINTER, "the current device is not the layer's device");
   int rc;
-  if ((rc = check_device_ptr(x, "x", dev)) != AF1_OK) return rc;
+  if ((rc = check_device_ptr(x, x2 != nullptr ? "g" : "x", dev)) != AF1_OK) return rc;
+  if (x2 != nullptr && (rc = check_device_ptr(x2, "u", dev)) != AF1_OK) return rc;
+  if (x2 != nullptr && (reinterpret_cast<uintptr_t>(x2) & 15) != 0)
+    return fail(AF1_ERR_MISALIGNED, "u must be 16-byte aligned");
   if ((rc = check_device_ptr(y, "y", dev)) != AF1_OK) return rc;
   if (workspace == nullptr) return fail(AF1_ERR_WORKSPACE, "workspace is NULL");
   if ((rc = check_device_ptr(workspace, "workspace", dev)) != AF1_OK) return AF1_ERR_WORKSPACE;
@@ -479,10 +483,11 @@ int linear_forward_checked(const af1_layer* layer, const void* x, int64_t ldx, i
     return fail(AF1_ERR_MISALIGNED, "ldy * element size must be a multiple of 16 bytes");
   if ((reinterpret_cast<uintptr_t>(workspace) & 255) != 0)
     return fail(AF1_ERR_WORKSPACE, "workspace must be 256-byte aligned");
-  const int64_t need = af1::plan_workspace(*layer, tokens, prep).total;
+  const int64_t need = af1::plan_workspace(*layer, tokens, prep, x2 != nullptr).total;
   if (workspace_bytes < need)
     return fail(AF1_ERR_WORKSPACE, "workspace too small: need " + std::to_string(need) + " bytes");
-  e = af1::launch_forward(*layer, x, ldx, tokens, y, ldy, y_dtype, workspace, static_cast<cudaStream_t>(stream), prep);
+  e = af1::launch_forward(*layer, x, ldx, tokens, y, ldy, y_dtype, workspace, static_cast<cudaStream_t>(stream), prep,
+                          nullptr, x2);
   if (e != cudaSuccess) return fail_cuda(e, "forward launch");
   g_err.clear();
   return AF1_OK;
@@ -491,6 +496,20 @@ int linear_forward_checked(const af1_layer* layer, const void* x, int64_t ldx, i
 }  // namespace af1
 
 extern "C" {
+
+int64_t af1_workspace_bytes_swiglu(const af1_layer* layer, int64_t tokens) {
+  if (layer == nullptr) return fail(AF1_ERR_INVALID_ARG, "layer is NULL");
+  if (tokens < 0) return fail(AF1_ERR_INVALID_ARG, "tokens must be >= 0");
+  return af1::plan_workspace(*layer, tokens, true, true).total;
+}
+
+int af1_linear_forward_swiglu(const af1_layer* layer, const void* g, const void* u, int64_t ldx, int64_t tokens,
+                              void* y, int64_t ldy, int y_dtype, void* workspace, int64_t workspace_bytes,
+                              void* stream) {
+  if (u == nullptr) return fail(AF1_ERR_INVALID_ARG, "u is NULL");
+  return af1::linear_forward_checked(layer, g, ldx, tokens, y, ldy, y_dtype, workspace, workspace_bytes, stream, true,
+                                     u);
+}
 
 int64_t af1_workspace_bytes_multi(const af1_layer* const* layers, int count, int64_t tokens) {
   if (layers == nullptr || count < 1 || count > af1::kMaxGroup)

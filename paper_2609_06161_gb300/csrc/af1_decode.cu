@@ -1010,7 +1010,9 @@ LutArgs lut_args(const DecodeArgs& d) {
 
 int64_t decode_ldz(const af1_layer& L) { return (int64_t)L.p2.NCH * kChunkCols; }
 
-Workspace plan_workspace(const af1_layer& L, int64_t tokens, bool prep) {
+int64_t swiglu_ld(const af1_layer& L) { return (L.n + 7) / 8 * 8; }
+
+Workspace plan_workspace(const af1_layer& L, int64_t tokens, bool prep, bool swiglu) {
   Workspace w;
   int64_t off = 0;
   w.status = off;
@@ -1030,6 +1032,11 @@ Workspace plan_workspace(const af1_layer& L, int64_t tokens, bool prep) {
   if (tokens > kMaxPassTokens) {
     const int64_t t = tokens < kPrefillPassTokens ? tokens : kPrefillPassTokens;
     off += align256(t * prefill_h_ld(L) * 2);
+  }
+  if (swiglu) {
+    const int64_t t = tokens < kPrefillPassTokens ? tokens : kPrefillPassTokens;
+    w.hx = off;
+    off += align256(t * swiglu_ld(L) * 2);
   }
   w.total = off;
   return w;
@@ -1079,13 +1086,29 @@ PhaseChoice choose_phase(const af1_layer& L, int phase, const SignMatrix& m, int
 }  // namespace
 
 cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64_t tokens, void* y,
-                           int64_t ldy, int y_dtype, void* ws, cudaStream_t st, bool prep, unsigned* status) {
-  const Workspace W = plan_workspace(L, tokens, prep);
+                           int64_t ldy, int y_dtype, void* ws, cudaStream_t st, bool prep, unsigned* status,
+                           const void* x2) {
+  const Workspace W = plan_workspace(L, tokens, prep, x2 != nullptr);
   uint8_t* wsb = static_cast<uint8_t*>(ws);
   unsigned* stat = status != nullptr ? status : reinterpret_cast<unsigned*>(wsb + W.status);
+  const int ysize = y_dtype == 0 ? 2 : 4;
+  const __half* gx = static_cast<const __half*>(x);
+  const __half* ux = static_cast<const __half*>(x2);
+  __half* hx = x2 != nullptr ? reinterpret_cast<__half*>(wsb + W.hx) : nullptr;
+  const int64_t ldh = swiglu_ld(L);
   if (tokens > kMaxPassTokens) {
-    // Prefill: two tensor-core GEMMs per pass (af1_prefill.cu).
-    return launch_prefill(L, x, ldx, tokens, y, ldy, y_dtype, wsb + W.hbuf, stat, st);
+    // Prefill: two tensor-core GEMMs per pass (af1_prefill.cu); the SwiGLU
+    // input is formed first, one pass of tokens at a time.
+    if (x2 == nullptr) return launch_prefill(L, x, ldx, tokens, y, ldy, y_dtype, wsb + W.hbuf, stat, st);
+    for (int64_t t0 = 0; t0 < tokens; t0 += kPrefillPassTokens) {
+      const int64_t T = (tokens - t0) < kPrefillPassTokens ? (tokens - t0) : kPrefillPassTokens;
+      cudaError_t e = launch_swiglu(gx + t0 * ldx, ux + t0 * ldx, ldx, T, L.n, hx, ldh, st);
+      if (e == cudaSuccess)
+        e = launch_prefill(L, hx, ldh, T, static_cast<uint8_t*>(y) + t0 * ldy * ysize, ldy, y_dtype, wsb + W.hbuf,
+                           stat, st);
+      if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
   }
   // Widest pass whose plans fit (16 tokens normally; fewer only for very
   // long contractions).
@@ -1099,7 +1122,6 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
     pass /= 2;
   }
   if (!p1.ok || !p2.ok) return cudaErrorInvalidConfiguration;
-  const int ysize = y_dtype == 0 ? 2 : 4;
   for (int64_t t0 = 0; t0 < tokens; t0 += pass) {
     const int T = (int)((tokens - t0) < pass ? (tokens - t0) : pass);
     PhaseChoice c1 = choose_phase(L, 1, L.p1, T, W), c2 = choose_phase(L, 2, L.p2, T, W);
@@ -1127,9 +1149,27 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
     a1.status = stat;
     a1.bbuf = W.bbuf != 0 ? wsb + W.bbuf : nullptr;
     a1.bstats = W.bbuf != 0 ? reinterpret_cast<float2*>(wsb + W.bstats) : nullptr;
-    cudaError_t e = c1.tc         ? launch_decode<1>(a1, q1, st)
-                    : c1.stream.ok ? launch_stream(1, lut_problem(a1), T, 0, c1.stream, stat, st)
-                                   : launch_lut(1, lut_args(a1), c1.lut, st);
+    cudaError_t e = cudaSuccess;
+    // SwiGLU input: the CUDA-core kernels form h while staging; the
+    // tensor-core kernel reads it from the workspace.
+    const __half* u1 = x2 != nullptr ? ux + t0 * ldx : nullptr;
+    if (u1 != nullptr && c1.tc) {
+      e = launch_swiglu(a1.x, u1, ldx, T, L.n, hx, ldh, st);
+      if (e != cudaSuccess) return e;
+      a1.x = hx;
+      a1.ldx = ldh;
+    }
+    if (c1.tc) {
+      e = launch_decode<1>(a1, q1, st);
+    } else if (c1.stream.ok) {
+      LutProblem q = lut_problem(a1);
+      q.x2 = u1;
+      e = launch_stream(1, q, T, 0, c1.stream, stat, st);
+    } else {
+      LutArgs la = lut_args(a1);
+      la.prob[0].x2 = u1;
+      e = launch_lut(1, la, c1.lut, st);
+    }
     if (e != cudaSuccess) return e;
 
     DecodeArgs a2 = {};

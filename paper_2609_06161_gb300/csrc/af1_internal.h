@@ -40,10 +40,15 @@ struct Workspace {
   int64_t bbuf = 0;    // prepared B tiles of decode passes of 5..16 tokens (0: none)
   int64_t bstats = 0;  // float2 [16 slices][16 tokens] of the prepared B (0: none)
   int64_t hbuf = 0;    // FP16 [min(tokens, kPrefillPassTokens)][prefill_h_ld]: H (prefill)
+  int64_t hx = 0;      // FP16 [min(tokens, kPrefillPassTokens)][swiglu_ld]: SwiGLU input h (0: none)
   int64_t total = 0;
 };
-// prep = false leaves out the prepared-B region (and so never uses it).
-Workspace plan_workspace(const af1_layer& L, int64_t tokens, bool prep = true);
+// prep = false leaves out the prepared-B region (and so never uses it);
+// swiglu adds the region the SwiGLU entry point forms h in for the kernels
+// that cannot form it while staging (tensor-core decode and prefill).
+Workspace plan_workspace(const af1_layer& L, int64_t tokens, bool prep = true, bool swiglu = false);
+// Row stride (elements) of the SwiGLU input h in the workspace.
+int64_t swiglu_ld(const af1_layer& L);
 int64_t prefill_h_ld(const af1_layer& L);
 int64_t decode_ldz(const af1_layer& L);
 
@@ -57,6 +62,10 @@ cudaError_t launch_words_to_blocks(const uint32_t* words, int64_t words_per_row,
 cudaError_t launch_blocks_to_words(const uint8_t* blocks, const SignMatrix& sm, int64_t wpr, uint32_t* words,
                                    cudaStream_t st);
 cudaError_t launch_bf16_to_f16(const uint16_t* src, uint16_t* dst, int64_t count, uint32_t* bad, cudaStream_t st);
+// h[t][j] = FP16(SiLU(g[t][j]) u[t][j]) for t < tokens, j < n (rows of g and
+// u at stride ldx, of h at ldh).
+cudaError_t launch_swiglu(const __half* g, const __half* u, int64_t ldx, int64_t tokens, int64_t n, __half* h,
+                          int64_t ldh, cudaStream_t st);
 // Set the calling thread's af1_last_error() message; returns `code`.
 int set_error(int code, const std::string& msg);
 
@@ -69,6 +78,7 @@ struct LutProblem {
   const uint8_t* signs;  // af1_layout.h row-block layout
   SignMatrix sm;
   const __half* x;       // phase 1 input [T][ldx] (FP16)
+  const __half* x2;      // phase 1, SwiGLU input: x is g, x2 is u, the input h = FP16(SiLU(g) u) (nullptr: x)
   int64_t ldx;
   const float* zin;      // phase 2 input [T][ldz] (FP32)
   int64_t ldz;
@@ -114,9 +124,11 @@ cudaError_t launch_stream(int phase, const LutProblem& prob, int tokens, int ydt
 cudaError_t launch_prefill(const af1_layer& L, const void* x, int64_t ldx, int64_t tokens, void* y, int64_t ldy,
                            int y_dtype, uint8_t* h_buf, unsigned* status, cudaStream_t st);
 // status: the status word to report to (nullptr: the workspace's own).
+// x2 != nullptr: the SwiGLU entry point (x is g, x2 is u; the workspace was
+// planned with swiglu = true).
 cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64_t tokens, void* y,
                            int64_t ldy, int y_dtype, void* ws, cudaStream_t st, bool prep = true,
-                           unsigned* status = nullptr);
+                           unsigned* status = nullptr, const void* x2 = nullptr);
 // Several layers with the same input x (same n): one lookup-table launch per
 // phase for all of them when possible, else one call per layer. The
 // workspace holds one single-layer workspace per layer, each 256-aligned,
@@ -128,6 +140,7 @@ cudaError_t launch_forward_multi(const af1_layer* const* Ls, int count, const vo
 // af1_linear_forward with all its argument checks; prep = false never uses
 // (and does not require) the prepared-B region of the workspace.
 int linear_forward_checked(const af1_layer* layer, const void* x, int64_t ldx, int64_t tokens, void* y, int64_t ldy,
-                           int y_dtype, void* workspace, int64_t workspace_bytes, void* stream, bool prep);
+                           int y_dtype, void* workspace, int64_t workspace_bytes, void* stream, bool prep,
+                           const void* x2 = nullptr);
 
 }  // namespace af1

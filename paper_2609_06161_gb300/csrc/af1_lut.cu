@@ -78,7 +78,8 @@ __host__ __device__ inline LutSmem lut_smem(int CPC, int KS, int T, int np) {
 // Kernel
 // ---------------------------------------------------------------------------
 
-template <int PHASE, int NP, bool MULTI>
+// SWIGLU (phase 1, one problem): the input is h = FP16(SiLU(x) x2).
+template <int PHASE, int NP, bool MULTI, bool SWIGLU>
 __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const __grid_constant__ LutArgs a) {
   constexpr int NACC = NP == 0 ? 1 : 2 * NP;
   constexpr int TCB = table_chunk_bytes(NP);
@@ -96,6 +97,7 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const __grid_constant_
   const int tg0 = (int)blockIdx.z * kGroupTokens;
   const int T = min(kGroupTokens, a.tokens - tg0);
   const __half* xg = PHASE == 1 ? pb.x + (int64_t)tg0 * pb.ldx : nullptr;
+  const __half* x2g = SWIGLU ? pb.x2 + (int64_t)tg0 * pb.ldx : nullptr;
   const float* zg = PHASE == 2 ? pb.zin + (int64_t)tg0 * pb.ldz : nullptr;
   const int KS = a.KS, CPC = pb.CPC;
   const LutSmem sp = lut_smem(CPC, KS, T, NP);
@@ -147,7 +149,7 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const __grid_constant_
 
   // ---- activations of the CTA's columns -> zs[t][k + k / 32] (FP32) -------
   griddep_wait();
-  stage_activations<PHASE, kThreads>(pb, xg, zg, T, nch, k0, zs, zrow, tid);
+  stage_activations<PHASE, kThreads, SWIGLU>(pb, xg, x2g, zg, T, nch, k0, zs, zrow, tid);
   if (tid < slice) rs[tid] = rs_own;
   __syncthreads();
 
@@ -229,9 +231,9 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const __grid_constant_
   }
 }
 
-template <int PHASE, int NP, bool MULTI>
+template <int PHASE, int NP, bool MULTI, bool SWIGLU = false>
 cudaError_t launch_np(const LutArgs& a, const LutPlan& p, cudaStream_t st) {
-  auto kern = lut_kernel<PHASE, NP, MULTI>;
+  auto kern = lut_kernel<PHASE, NP, MULTI, SWIGLU>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, p.smem);
   if (e != cudaSuccess) return e;
   if (p.KS > 8) {
@@ -333,6 +335,13 @@ LutPlan plan_lut(const SignMatrix* sm, int count, int T, int num_sms, int max_sm
 template <int PHASE>
 cudaError_t launch_phase(const LutArgs& a, const LutPlan& p, cudaStream_t st) {
   const bool multi = a.count > 1;
+  if (PHASE == 1 && !multi && a.prob[0].x2 != nullptr) {
+    switch (pairs_for(a.tokens < kGroupTokens ? a.tokens : kGroupTokens)) {
+      case 0: return launch_np<PHASE, 0, false, true>(a, p, st);
+      case 1: return launch_np<PHASE, 1, false, true>(a, p, st);
+      default: return launch_np<PHASE, 2, false, true>(a, p, st);
+    }
+  }
   switch (pairs_for(a.tokens < kGroupTokens ? a.tokens : kGroupTokens)) {
     case 0: return multi ? launch_np<PHASE, 0, true>(a, p, st) : launch_np<PHASE, 0, false>(a, p, st);
     case 1: return multi ? launch_np<PHASE, 1, true>(a, p, st) : launch_np<PHASE, 1, false>(a, p, st);

@@ -120,15 +120,21 @@ __host__ __device__ constexpr int zrow_floats(int CPC) { return CPC * kChunkCols
 // Activations, tables, lookups
 // ---------------------------------------------------------------------------
 
+// SwiGLU input h = FP16(SiLU(g) u), SiLU(g) = g / (1 + e^-g) in FP32.
+__device__ __forceinline__ float swiglu_h(float g, float u) {
+  return __half2float(__float2half_rn(g / (1.f + expf(-g)) * u));
+}
+
 // Activations of `nch` chunks from column k0 on -> zs[t][k + k / 32]
 // (FP32), k the column within the staged chunks. Phase 1 stages z = b * x
-// (an FP16 x FP16 product, exact in FP32), phase 2 its FP32 input; columns
-// >= C stage 0. Written by the previous kernel, the inputs are read through
-// L2 (ld.global.cg), 8 columns per load, a batch of loads per thread in
-// flight at once.
-template <int PHASE, int THREADS>
-__device__ __forceinline__ void stage_activations(const LutProblem& pb, const __half* xg, const float* zg, int T,
-                                                  int nch, int64_t k0, float* zs, int zrow, int tid) {
+// (an FP16 x FP16 product, exact in FP32; SWIGLU: x = swiglu_h(xg, x2g)),
+// phase 2 its FP32 input; columns >= C stage 0. Written by the previous
+// kernel, the inputs are read through L2 (ld.global.cg), 8 columns per load,
+// a batch of loads per thread in flight at once.
+template <int PHASE, int THREADS, bool SWIGLU = false>
+__device__ __forceinline__ void stage_activations(const LutProblem& pb, const __half* xg, const __half* x2g,
+                                                  const float* zg, int T, int nch, int64_t k0, float* zs, int zrow,
+                                                  int tid) {
   const int g8 = nch * (kChunkCols / 8);  // 8-column groups per token
   const int ng = T * g8;
   constexpr int kBatch = 2;
@@ -144,10 +150,23 @@ __device__ __forceinline__ void stage_activations(const LutProblem& pb, const __
           const uint4 xr = __ldcg(reinterpret_cast<const uint4*>(xg + (int64_t)t * pb.ldx + col));
           const uint4 br = __ldg(reinterpret_cast<const uint4*>(pb.colscale + col));
           const uint32_t xw[4] = {xr.x, xr.y, xr.z, xr.w}, bw[4] = {br.x, br.y, br.z, br.w};
+          uint32_t uw[4] = {0u, 0u, 0u, 0u};
+          if constexpr (SWIGLU) {
+            const uint4 ur = __ldcg(reinterpret_cast<const uint4*>(x2g + (int64_t)t * pb.ldx + col));
+            uw[0] = ur.x;
+            uw[1] = ur.y;
+            uw[2] = ur.z;
+            uw[3] = ur.w;
+          }
 #pragma unroll
           for (int h2 = 0; h2 < 4; ++h2) {
-            const float2 xf = __half22float2(*reinterpret_cast<const __half2*>(&xw[h2]));
+            float2 xf = __half22float2(*reinterpret_cast<const __half2*>(&xw[h2]));
             const float2 bf = __half22float2(*reinterpret_cast<const __half2*>(&bw[h2]));
+            if constexpr (SWIGLU) {
+              const float2 uf = __half22float2(*reinterpret_cast<const __half2*>(&uw[h2]));
+              xf.x = swiglu_h(xf.x, uf.x);
+              xf.y = swiglu_h(xf.y, uf.y);
+            }
             v[u][2 * h2] = xf.x * bf.x;
             v[u][2 * h2 + 1] = xf.y * bf.y;
           }
@@ -168,9 +187,11 @@ __device__ __forceinline__ void stage_activations(const LutProblem& pb, const __
         for (int q = 0; q < 8; ++q) {
           float z = 0.f;
           if (i < ng && col + q < pb.sm.C) {
-            if (PHASE == 1)
-              z = __half2float(__ldcg(xg + (int64_t)t * pb.ldx + col + q)) * __half2float(pb.colscale[col + q]);
-            else
+            if (PHASE == 1) {
+              float xv = __half2float(__ldcg(xg + (int64_t)t * pb.ldx + col + q));
+              if constexpr (SWIGLU) xv = swiglu_h(xv, __half2float(__ldcg(x2g + (int64_t)t * pb.ldx + col + q)));
+              z = xv * __half2float(pb.colscale[col + q]);
+            } else
               z = __ldcg(zg + (int64_t)t * pb.ldz + col + q);
           }
           v[u][q] = z;

@@ -99,6 +99,39 @@ __global__ void bf16_to_f16_kernel(const uint16_t* __restrict__ src, uint16_t* _
   dst[t] = __half_as_ushort(h);
 }
 
+// h = FP16(SiLU(g) u) elementwise (SiLU(g) = g / (1 + e^-g) in FP32): the
+// SwiGLU input of a down projection, for the kernels that read their
+// activations from memory. Thread i handles 8 columns of one row.
+__global__ void swiglu_kernel(const __half* __restrict__ g, const __half* __restrict__ u, int64_t ldx,
+                              int64_t tokens, int64_t n, __half* __restrict__ h, int64_t ldh) {
+  const int64_t g8 = (n + 7) / 8;
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= tokens * g8) return;
+  const int64_t t = i / g8, j = (i - t * g8) * 8;
+  const __half* gr = g + t * ldx + j;
+  const __half* ur = u + t * ldx + j;
+  __half* hr = h + t * ldh + j;
+  if (j + 8 <= n) {
+    const uint4 gv = *reinterpret_cast<const uint4*>(gr);
+    const uint4 uv = *reinterpret_cast<const uint4*>(ur);
+    const uint32_t gw[4] = {gv.x, gv.y, gv.z, gv.w}, uw[4] = {uv.x, uv.y, uv.z, uv.w};
+    uint32_t hw[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const float2 gf = __half22float2(*reinterpret_cast<const __half2*>(&gw[k]));
+      const float2 uf = __half22float2(*reinterpret_cast<const __half2*>(&uw[k]));
+      const __half2 hv = __floats2half2_rn(gf.x / (1.f + expf(-gf.x)) * uf.x, gf.y / (1.f + expf(-gf.y)) * uf.y);
+      hw[k] = *reinterpret_cast<const uint32_t*>(&hv);
+    }
+    *reinterpret_cast<uint4*>(hr) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+  } else {
+    for (int64_t k = 0; j + k < n; ++k) {
+      const float gf = __half2float(gr[k]), uf = __half2float(ur[k]);
+      hr[k] = __float2half_rn(gf / (1.f + expf(-gf)) * uf);
+    }
+  }
+}
+
 }  // namespace
 
 cudaError_t launch_blocks_to_words(const uint8_t* blocks, const SignMatrix& sm, int64_t wpr, uint32_t* words,
@@ -108,6 +141,15 @@ cudaError_t launch_blocks_to_words(const uint8_t* blocks, const SignMatrix& sm, 
   const int threads = 256;
   blocks_to_words_kernel<<<(unsigned)((total + threads - 1) / threads), threads, 0, st>>>(
       reinterpret_cast<const uint32_t*>(blocks), sm, wpr, words);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_swiglu(const __half* g, const __half* u, int64_t ldx, int64_t tokens, int64_t n, __half* h,
+                          int64_t ldh, cudaStream_t st) {
+  const int64_t total = tokens * ((n + 7) / 8);
+  if (total == 0) return cudaSuccess;
+  const int threads = 256;
+  swiglu_kernel<<<(unsigned)((total + threads - 1) / threads), threads, 0, st>>>(g, u, ldx, tokens, n, h, ldh);
   return cudaGetLastError();
 }
 

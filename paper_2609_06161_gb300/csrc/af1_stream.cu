@@ -95,7 +95,8 @@ struct StreamArgs {
   unsigned* status;
 };
 
-template <int PHASE, int NP, int G>
+// SWIGLU (phase 1): the input is h = FP16(SiLU(x) x2).
+template <int PHASE, int NP, int G, bool SWIGLU>
 __global__ void __launch_bounds__(kStreamThreads, 3) stream_kernel(const __grid_constant__ StreamArgs a) {
   constexpr int NACC = NP == 0 ? 1 : 2 * NP;
   constexpr int TCB = table_chunk_bytes(NP);
@@ -174,7 +175,8 @@ __global__ void __launch_bounds__(kStreamThreads, 3) stream_kernel(const __grid_
   // ---- consumers: activations of the CTA's chunks, tables --------------------
   griddep_wait();
   const int zrow = zrow_floats(CPC);
-  stage_activations<PHASE, kConsumers>(pb, pb.x, pb.zin, T, nch, (int64_t)c0 * kChunkCols, zs, zrow, tid);
+  stage_activations<PHASE, kConsumers, SWIGLU>(pb, pb.x, pb.x2, pb.zin, T, nch, (int64_t)c0 * kChunkCols, zs, zrow,
+                                               tid);
   named_sync(kBarConsumers, kConsumers);
   build_tables<NP, kConsumers>(smem + sp.tbl, zs, zrow, T, nch, tid);
   named_sync(kBarConsumers, kConsumers);
@@ -274,9 +276,9 @@ __global__ void __launch_bounds__(kStreamThreads, 3) stream_kernel(const __grid_
 }
 
 // Kernel attributes for a launch with `smem` bytes and clusters of KS.
-template <int PHASE, int NP, int G>
+template <int PHASE, int NP, int G, bool SWIGLU = false>
 cudaError_t prepare_kernel(int smem, int KS) {
-  auto kern = stream_kernel<PHASE, NP, G>;
+  auto kern = stream_kernel<PHASE, NP, G, SWIGLU>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e == cudaSuccess && KS > 8) e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   return e;
@@ -298,7 +300,7 @@ int active_clusters(int smem, int KS) {
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   int n = 0;
-  if (cudaOccupancyMaxActiveClusters(&n, stream_kernel<PHASE, NP, G>, &cfg) != cudaSuccess) {
+  if (cudaOccupancyMaxActiveClusters(&n, stream_kernel<PHASE, NP, G, false>, &cfg) != cudaSuccess) {
     cudaGetLastError();  // clear: the query failing only rules the split out
     return 0;
   }
@@ -334,10 +336,10 @@ int max_active_clusters(int phase, int T, int G, int KS, int smem) {
   return n;
 }
 
-template <int PHASE, int NP, int G>
+template <int PHASE, int NP, int G, bool SWIGLU>
 cudaError_t launch_g(const StreamArgs& a, const StreamPlan& p, cudaStream_t st) {
-  auto kern = stream_kernel<PHASE, NP, G>;
-  cudaError_t e = prepare_kernel<PHASE, NP, G>(p.smem, p.KS);
+  auto kern = stream_kernel<PHASE, NP, G, SWIGLU>;
+  cudaError_t e = prepare_kernel<PHASE, NP, G, SWIGLU>(p.smem, p.KS);
   if (e != cudaSuccess) return e;
   const int SRB = (a.p.sm.RB + G - 1) / G;
   cudaLaunchConfig_t cfg = {};
@@ -357,12 +359,12 @@ cudaError_t launch_g(const StreamArgs& a, const StreamPlan& p, cudaStream_t st) 
   return cudaLaunchKernelEx(&cfg, kern, a);
 }
 
-template <int PHASE, int NP>
+template <int PHASE, int NP, bool SWIGLU = false>
 cudaError_t launch_np(const StreamArgs& a, const StreamPlan& p, cudaStream_t st) {
   switch (p.G) {
-    case 1: return launch_g<PHASE, NP, 1>(a, p, st);
-    case 2: return launch_g<PHASE, NP, 2>(a, p, st);
-    default: return launch_g<PHASE, NP, 4>(a, p, st);
+    case 1: return launch_g<PHASE, NP, 1, SWIGLU>(a, p, st);
+    case 2: return launch_g<PHASE, NP, 2, SWIGLU>(a, p, st);
+    default: return launch_g<PHASE, NP, 4, SWIGLU>(a, p, st);
   }
 }
 
@@ -466,6 +468,8 @@ cudaError_t launch_stream(int phase, const LutProblem& prob, int tokens, int ydt
   a.CPC = p.CPC;
   a.NSC = p.NSC;
   a.status = status;
+  if (phase == 1 && prob.x2 != nullptr)
+    return tokens == 1 ? launch_np<1, 0, true>(a, p, st) : launch_np<1, 1, true>(a, p, st);
   if (phase == 1) return tokens == 1 ? launch_np<1, 0>(a, p, st) : launch_np<1, 1>(a, p, st);
   return tokens == 1 ? launch_np<2, 0>(a, p, st) : launch_np<2, 1>(a, p, st);
 }

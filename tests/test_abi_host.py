@@ -102,5 +102,8 @@ def test_host_validation_errors():
     assert lib.af1_load_packed_layer(ctypes.byref(d), None, None, None, None, None, None, ctypes.byref(h)) == -1
     assert lib.af1_linear_forward(None, None, 0, 1, None, 0, 0, None, 0, None) == -1
     assert lib.af1_workspace_bytes(None, 1) == -1
+    assert lib.af1_workspace_bytes_swiglu(None, 1) == -1
+    assert lib.af1_linear_forward_swiglu(None, None, None, 0, 1, None, 0, 0, None, 0, None) == -1
+    assert "u is NULL" in P.last_error()
     lib.af1_free(None)  # NULL-safe
     assert P.version().startswith("af1-gb300")

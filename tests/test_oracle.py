@@ -338,3 +338,35 @@ def test_rowwise_rel_err():
     assert O.rowwise_rel_err(y, ref) == pytest.approx(1e-3)
     assert O.rowwise_rel_err(ref, ref) == 0.0
     assert O.rowwise_rel_err(np.zeros((0, 3)), np.zeros((0, 3))) == 0.0
+
+
+# ---- SwiGLU input of a down projection (oracle side) -----------------------
+
+def test_silu_against_the_tanh_form_and_the_odd_part():
+    # SiLU(z) = z sigmoid(z) = (z / 2) (1 + tanh(z / 2)), and SiLU(z) - SiLU(-z) = z
+    # because sigmoid(z) + sigmoid(-z) = 1.
+    z = np.linspace(-30.0, 30.0, 2001)
+    # (the tanh form cancels for z << 0: compare absolutely there)
+    np.testing.assert_allclose(O.silu_f64(z), 0.5 * z * (1.0 + np.tanh(0.5 * z)), rtol=1e-13, atol=1e-14)
+    np.testing.assert_allclose(O.silu_f64(z) - O.silu_f64(-z), z, rtol=1e-13, atol=1e-13)
+    assert O.silu_f64(0.0) == 0.0
+    assert O.silu_f64(1.0) == pytest.approx(0.7310585786300049, rel=1e-15)   # 1 / (1 + 1/e)
+    assert O.silu_f64(-1e4) == 0.0 or abs(O.silu_f64(-1e4)) < 1e-300          # no overflow to NaN
+
+
+def test_swiglu_f16_rounds_once():
+    g = np.array([0.0, 1.0, -1.0, 2.0, 20.0, -20.0, 3.0, 65504.0], dtype=np.float16)
+    u = np.array([5.0, 1.0, 1.0, -0.5, 2.0, 1.0, 0.0, 1.0], dtype=np.float16)
+    h = O.swiglu_f16(g.view(np.uint16), u.view(np.uint16)).view(np.float16).astype(np.float64)
+    ref = [0.0,
+           float(np.float16(0.7310585786300049)),        # SiLU(1)
+           float(np.float16(-0.2689414213699951)),       # SiLU(-1) = SiLU(1) - 1
+           float(np.float16(-0.5 * 1.7615941559557649)),  # SiLU(2) * -0.5
+           40.0,                                           # SiLU(20) = 20 - 4e-8 -> 20, times 2
+           float(np.float16(-20.0 / (1.0 + np.exp(20.0)))),  # about -4.1e-8: a subnormal
+           0.0,
+           65504.0]                                        # SiLU(65504) = 65504 exactly in FP16
+    np.testing.assert_array_equal(h, ref)
+    # Sign symmetry of round to nearest: negating u negates h.
+    hn = O.swiglu_f16(g.view(np.uint16), (-u).view(np.uint16)).view(np.float16).astype(np.float64)
+    np.testing.assert_array_equal(hn, -h)
