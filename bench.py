@@ -453,6 +453,46 @@ def dag_step(torch, views, stream, side, ws, ws_side):
         down[0].forward_into(down[1], down[2], ws, stream=stream)
 
 
+def nabf_bench(P, torch):
+    """NABF (the factorization that produces the layer) on synthetic
+    weights: a rank-512 structure plus noise, LLaMA-3-8B 4096 x 4096 at the
+    1.0-BPW rank and a 1024 x 1024 sample, with per-column / per-row
+    calibration scales; wall time per iteration on the GPU (the call
+    synchronizes), and the FP64 oracle on the host for the small sample."""
+    import time
+    import synth
+    out = {"workload": "NABF on synthetic W (rank-512 structure + N(0, 0.01) noise, i, o ~ U(0.5, 2)), "
+                       "rho 1e-2, eta 0.01, 20 power iterations; wall time per iteration (iterations 1..5 "
+                       "minus the initialization)"}
+    for (m, n) in ((1024, 1024), (4096, 4096)):
+        r = P.rank_for_budget(m, n)
+        g = synth.rng(m)
+        k = min(512, r // 2)
+        W = (g.normal(size=(m, k)) @ g.normal(size=(k, n)) * 0.01 + g.normal(0.0, 0.01, size=(m, n))).astype(np.float32)
+        i_s, o_s = g.uniform(0.5, 2.0, n).astype(np.float32), g.uniform(0.5, 2.0, m).astype(np.float32)
+        Wt, it, ot = (torch.from_numpy(v).cuda() for v in (W, i_s, o_s))
+        times = {}
+        for iters in (0, 5):
+            P.nabf_factorize(Wt, r, iters=iters, rho=1e-2, in_scale=it, out_scale=ot)  # warm-up (library loads)
+            t0 = time.perf_counter()
+            res = P.nabf_factorize(Wt, r, iters=iters, rho=1e-2, in_scale=it, out_scale=ot)
+            times[iters] = time.perf_counter() - t0
+        row = {"m": m, "n": n, "r": r, "gpu_ms_per_iteration": (times[5] - times[0]) / 5 * 1e3,
+               "gpu_init_ms": times[0] * 1e3, "objective": res["objective"], "q_left": res["q_left"],
+               "q_right": res["q_right"]}
+        if m == 1024:
+            from oracle import af1_nabf_oracle as N
+            t0 = time.perf_counter()
+            N.nabf(W, r, 0, rho=1e-2, in_scale=i_s, out_scale=o_s)
+            t1 = time.perf_counter()
+            ref = N.nabf(W, r, 2, rho=1e-2, in_scale=i_s, out_scale=o_s)
+            t2 = time.perf_counter()
+            row["cpu_oracle_s_per_iteration"] = ((t2 - t1) - (t1 - t0)) / 2
+            row["cpu_oracle_objective_2_iters"] = list(ref["objective"])
+        out[f"{m}x{n}"] = row
+    return out
+
+
 def mlp_swiglu(P, torch, stream, steps):
     """LLaMA-3-8B MLP blocks at one token: gate | up (parallel streams), then
     the down projection of h = FP16(SiLU(gate) * up). Fused: the down call
@@ -733,13 +773,14 @@ def main():
     if not args.no_dense and rank == 0:
         dense = dense_bf16(torch, objs, b, args, stream)
     peaks = load_peaks()
-    sweep_rows = stack = mlp = None
+    sweep_rows = stack = mlp = nabf = None
     if args.workload == "decode" and rank == 0:
         # Extra measurements, outside the timed region of the headline number.
         if not args.no_stack:
             stack = stack_hisa(P, torch, peaks, stream, args.steps,
                                dense_ms=dense["ms_per_step"] if dense and b == 1 else None)
             mlp = mlp_swiglu(P, torch, stream, args.steps)
+            nabf = nabf_bench(P, torch)
         if not args.no_sweep:
             sweep_rows = sweep(P, torch, peaks, stream)
 
@@ -789,6 +830,8 @@ def main():
             line["stack_hisa"] = stack
         if mlp is not None:
             line["mlp_swiglu"] = mlp
+        if nabf is not None:
+            line["nabf"] = nabf
         if sweep_rows is not None:
             line["sweep"] = sweep_rows
         if not args.no_cpu and world == 1 and args.workload == "decode":

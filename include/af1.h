@@ -205,6 +205,48 @@ AF1_API int af1_linear_forward(const af1_layer* layer, const void* x, int64_t ld
                        void* y, int64_t ldy, int y_dtype, void* workspace,
                        int64_t workspace_bytes, void* stream);
 
+/* ---- NABF: the factorization that produces an AF1 layer ---------------------
+ * Algorithm NABF (Null-space-Aware Binary Factorization; App. "ADMM-SVID
+ * Framework in DBF", "Adaptive Residual-Energy Cutoff") on the GPU: the
+ * surrogate W' = o * W * i^T is factorized as A B with A = a * A_pm1 * m1^T,
+ * B = m2 * B_pm1 * b^T by alternating ADMM proxies, SVID projections (signs
+ * and a rank-1 magnitude fit by power iteration), null-space compensation and
+ * closed-form scale fits. Readings: initialization by a randomized range
+ * finder (W' Omega, Omega +-1 from SplitMix64(seed, j r + k), top bit -> -1,
+ * then the right proxy with a zero prior and SVID of both), Sign(0) = +1,
+ * power iteration from the all-ones vector with the singular value split
+ * evenly, duals updated with the compensated factors. Dense products,
+ * Cholesky / triangular solves and symmetric eigendecompositions use cuBLAS
+ * and cuSOLVER, loaded at run time (AF1_ERR_CUDA if they cannot be loaded). */
+typedef struct af1_nabf_params {
+  int32_t iters;        /* T: alternating iterations, >= 0 */
+  int32_t power_iters;  /* power iterations per SVID projection, >= 1 */
+  double rho;           /* ADMM penalty, > 0 */
+  double eta;           /* residual-energy cutoff of the null-space projector, in [0, 1) (paper: 0.01) */
+  double eps;           /* stabilizer of the cutoff fraction and of the scale fits, >= 0 */
+  uint64_t seed;        /* seed of the initial +-1 draw */
+  int32_t compensate;   /* 1: NABF; 0: plain ADMM-SVID (no compensation) */
+  int32_t reserved;     /* must be 0 */
+} af1_nabf_params;
+
+/* Factorize W (device, FP32, row-major m x n) at rank r (0 < r <= min(m, n)).
+ *   in_scale (n) / out_scale (m): the surrogate's i and o (device FP32), or
+ *       NULL for ones.
+ *   Outputs, device: U (int8 +-1, row-major m x r) = A_pm1, V (int8 +-1,
+ *       row-major n x r) = B_pm1^T, a (m), s (r) = m1 * m2, b (n) as FP32,
+ *       with the surrogate scaling undone (a / o, b / i): the AF1 layer
+ *       W_hat = Diag(a) U Diag(s) V^T Diag(b) (pack with af1_pack_layer after
+ *       converting the scales to FP16).
+ *   history (host, may be NULL): 3 (iters + 1) doubles: the relative
+ *       objective |W' - A B|_F^2 / |W'|_F^2 after the initialization and after
+ *       each iteration, then the numbers of trailing eigenvectors the left and
+ *       right null-space projectors kept per iteration (0 at index 0).
+ * Synchronizes the stream; allocates and frees its own scratch. Errors:
+ * INVALID_ARG, CUDA (including a proxy that is not positive definite). */
+AF1_API int af1_nabf_factorize(const float* W, int64_t m, int64_t n, int64_t r, const float* in_scale,
+                               const float* out_scale, const af1_nabf_params* params, int8_t* U, int8_t* V,
+                               float* a, float* s, float* b, double* history, void* stream);
+
 /* SwiGLU input of a down projection (the MLP of the LLaMA models the paper
  * compresses): y = h . W_hat^T with h = FP16(SiLU(g) * u) elementwise,
  * SiLU(z) = z / (1 + e^-z) in FP32, from the outputs g and u of the gate and

@@ -104,6 +104,17 @@ _lib.af1_hisa_module_budgets.argtypes = [_dp, _dp, ctypes.POINTER(_i64), _i64, c
 _lib.af1_hisa_module_budgets.restype = ctypes.c_int
 _lib.af1_budget_to_rank.argtypes = [ctypes.c_double, _i64, _i64, ctypes.POINTER(_i64)]
 _lib.af1_budget_to_rank.restype = ctypes.c_int
+
+
+class _NabfParams(ctypes.Structure):
+    _fields_ = [("iters", ctypes.c_int32), ("power_iters", ctypes.c_int32), ("rho", ctypes.c_double),
+                ("eta", ctypes.c_double), ("eps", ctypes.c_double), ("seed", ctypes.c_uint64),
+                ("compensate", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+
+
+_lib.af1_nabf_factorize.argtypes = [_vp, _i64, _i64, _i64, _vp, _vp, ctypes.POINTER(_NabfParams), _vp, _vp, _vp,
+                                    _vp, _vp, _dp, _vp]
+_lib.af1_nabf_factorize.restype = ctypes.c_int
 _lib.af1_workspace_status.argtypes = [_vp, _vp]
 _lib.af1_workspace_status.restype = ctypes.c_int
 _lib.af1_free.argtypes = [_vp]
@@ -426,3 +437,32 @@ def budget_to_rank(b: float, m: int, n: int) -> int:
     r = _i64()
     _check(_lib.af1_budget_to_rank(b, m, n, ctypes.byref(r)))
     return r.value
+
+
+# -- NABF: factorize a weight matrix into an AF1 layer -----------------------------
+
+def nabf_factorize(W: torch.Tensor, r: int, iters: int = 10, rho: float = 1.0, eta: float = 0.01,
+                   eps: float = 1e-8, power_iters: int = 20, seed: int = 0, in_scale=None, out_scale=None,
+                   compensate: bool = True, stream=None) -> dict:
+    """Algorithm NABF on W (float32 CUDA tensor, m x n) at rank r
+    (af1_nabf_factorize). Returns U (int8 m x r), V (int8 n x r), a, s, b
+    (float32, the surrogate scaling undone), the relative objective per
+    iteration and the null-space sizes kept per iteration (left, right)."""
+    W = W.contiguous().float()
+    m, n = W.shape
+    dev = W.device
+    U = torch.empty((m, r), dtype=torch.int8, device=dev)
+    V = torch.empty((n, r), dtype=torch.int8, device=dev)
+    a = torch.empty(m, dtype=torch.float32, device=dev)
+    s_ = torch.empty(r, dtype=torch.float32, device=dev)
+    b = torch.empty(n, dtype=torch.float32, device=dev)
+    i_s = None if in_scale is None else in_scale.contiguous().float()
+    o_s = None if out_scale is None else out_scale.contiguous().float()
+    hist = (ctypes.c_double * (3 * (iters + 1)))()
+    p = _NabfParams(iters, power_iters, rho, eta, eps, seed & ((1 << 64) - 1), 1 if compensate else 0, 0)
+    _check(_lib.af1_nabf_factorize(_ptr(W), m, n, r, _ptr(i_s), _ptr(o_s), ctypes.byref(p), _ptr(U), _ptr(V),
+                                   _ptr(a), _ptr(s_), _ptr(b), hist, _stream_handle(stream)))
+    h = list(hist)
+    k = iters + 1
+    return {"U": U, "V": V, "a": a, "s": s_, "b": b, "objective": h[:k], "q_left": [int(v) for v in h[k:2 * k]],
+            "q_right": [int(v) for v in h[2 * k:]]}

@@ -17,7 +17,7 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 OUT = os.path.join(HERE, "libaf1.so")
 BUILD_DIR = os.path.join(HERE, "_build")
-SOURCES = ["af1_api.cu", "af1_pack.cu", "af1_decode.cu", "af1_lut.cu", "af1_stream.cu", "af1_prefill.cu", "af1_noalloc.cu", "af1_hisa.cu"]
+SOURCES = ["af1_api.cu", "af1_pack.cu", "af1_decode.cu", "af1_lut.cu", "af1_stream.cu", "af1_prefill.cu", "af1_noalloc.cu", "af1_hisa.cu", "af1_nabf.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden",
          "--expt-relaxed-constexpr", "-I", INCLUDE]
@@ -51,7 +51,7 @@ def build(verbose: bool = False) -> str:
             sys.stderr.write(log)
     objs = [o for o, _ in results]
     tmp = OUT + ".tmp"
-    cmd = [cc, *ARCH, "-shared", "-cudart", "shared", "-o", tmp, *objs,
+    cmd = [cc, *ARCH, "-shared", "-cudart", "shared", "-o", tmp, *objs, "-ldl",
            "-Xlinker", "-rpath,/usr/local/cuda/lib64"]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:

@@ -105,5 +105,12 @@ def test_host_validation_errors():
     assert lib.af1_workspace_bytes_swiglu(None, 1) == -1
     assert lib.af1_linear_forward_swiglu(None, None, None, 0, 1, None, 0, 0, None, 0, None) == -1
     assert "u is NULL" in P.last_error()
+    prm = P._NabfParams(3, 10, 1.0, 0.01, 1e-8, 0, 1, 0)
+    assert lib.af1_nabf_factorize(None, 8, 8, 4, None, None, None, None, None, None, None, None, None, None) == -1
+    assert lib.af1_nabf_factorize(None, 8, 8, 9, None, None, ctypes.byref(prm), None, None, None, None, None, None,
+                                  None) == -1  # r > min(m, n)
+    bad = P._NabfParams(3, 10, 0.0, 0.01, 1e-8, 0, 1, 0)  # rho = 0
+    assert lib.af1_nabf_factorize(None, 8, 8, 4, None, None, ctypes.byref(bad), None, None, None, None, None, None,
+                                  None) == -1
     lib.af1_free(None)  # NULL-safe
     assert P.version().startswith("af1-gb300")
