@@ -620,7 +620,7 @@ def main():
         if not 1 <= b <= 16:
             raise SystemExit("--batch must be in 1..16 for the decode path")
     if args.shape:
-        run_shape(P, torch, args)
+        run_shape(P, torch, args, b)
         return
     dev = torch.device("cuda", torch.cuda.current_device())
     objs = build_layers(P, torch, args.layers, b, rank, outlier_frac=0.01 if args.workload == "prefill" else 0.0)
@@ -844,14 +844,14 @@ def main():
         dist.destroy_process_group()
 
 
-def run_shape(P, torch, args):
-    """One linear of shape --shape at its 1.0-BPW rank and --batch tokens:
+def run_shape(P, torch, args, b):
+    """One linear of shape --shape at its 1.0-BPW rank and b tokens (--batch,
+    or --tokens with --workload prefill):
     --warmup then --steps calls, each on the next of enough copies of the
     layer to exceed twice the L2 (every call streams its signs from HBM), in
     a CUDA graph or (--no-graph) as eager launches for profilers."""
     import math
     m, n = (int(v) for v in args.shape.lower().split("x"))
-    b = args.batch
     r = P.rank_for_budget(m, n)
     packed = r * (m + n) // 8 + 2 * (m + n + r)
     copies = max(2, min(128, math.ceil(2 * L2_BYTES / packed)))
@@ -884,9 +884,12 @@ def run_shape(P, torch, args):
     P.workspace_status(ws)
     peaks = load_peaks()
     alg = algorithmic_bytes(m, n, r, b)
+    fl = 2 * b * r * (m + n)
     line = {"shape": f"{m}x{n}", "rank": r, "tokens": b, "us_per_call": us, "copies": copies,
             "graph": not args.no_graph, "algorithmic_bytes": alg, "achieved_gbs": alg / (us * 1e-6) / 1e9,
-            "hbm_frac": alg / (us * 1e-6) / 1e9 / peaks.get("hbm_gbs", 6800.0)}
+            "hbm_frac": alg / (us * 1e-6) / 1e9 / peaks.get("hbm_gbs", 6800.0),
+            "flops": fl, "achieved_tflops": fl / (us * 1e-6) / 1e12,
+            "tensor_frac": fl / (us * 1e-6) / 1e12 / peaks.get("bf16_tflops_sustained", 1700.0)}
     print(json.dumps(line))
     for L in layers:
         L.free()

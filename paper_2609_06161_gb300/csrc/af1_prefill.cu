@@ -254,8 +254,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
   const uint32_t tmem = bar.tmem_addr;
 
-  griddep_launch_dependents();
-
   if (warp == 0) {
     // ---- activation producer: one TMA copy per stage ---------------------
     griddep_wait();  // the activations are written by the previous kernel
@@ -365,6 +363,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(&bar.full_a[(nk - 1) % STAGES]);
     }
+    // The next kernel may launch once this CTA has expanded its weights: its
+    // own expansion needs no input and would otherwise compete with this
+    // one's for the SMs. Measured against a trigger right after the
+    // tensor-memory allocation: the 2048-token prefill step 4.18 -> 4.04 ms,
+    // 64 tokens 4096^2 37.9 -> 31.3 us, 8192^2 56.7 -> 47.9, 1024 x 8192
+    // 33.4 -> 26.2, 28672 x 8192 at 128 tokens 179 -> 127; only 28672 x 8192
+    // at 64 tokens lost (95 -> 120), where GEMM 1 leaves SMs idle.
+    griddep_launch_dependents();
     // ---- epilogue: TMEM -> registers -> global ---------------------------
     if (lane == 0) mbar_wait(&bar.done, 0, &bar.err);
     __syncwarp();
@@ -514,7 +520,10 @@ cudaError_t launch_gemm_bn(const PrefillArgs& a, const __half* act, int64_t ld_a
 // Tiling of one GEMM: the smallest token tile of 64 / 128 / 256 that covers
 // the pass, made smaller while the grid would leave half the SMs idle; with
 // tiles of 64, short passes (few row blocks x token tiles) split K over a
-// cluster of 2, 4 or 8 CTAs (every CTA keeps at least two K-stages).
+// cluster of 2, 4 or 8 CTAs (every CTA keeps at least two K-stages) while
+// the grid fits one CTA per SM, or two per SM for contractions of 256
+// K-stages or more (measured: 8192 x 28672 at 64 tokens 164 -> 108 us; the
+// same on shorter contractions lost, e.g. 4096^2 31 -> 40 us).
 template <bool GEMM1>
 cudaError_t launch_gemm(const PrefillArgs& a, const __half* act, int64_t ld_act, int num_sms, cudaStream_t st) {
   const int64_t rb = a.sm.RB;
@@ -525,7 +534,8 @@ cudaError_t launch_gemm(const PrefillArgs& a, const __half* act, int64_t ld_act,
   const int64_t base = rb * ((a.tokens + 63) / 64);
   const int nk = (int)((a.sm.C + BK - 1) / BK);
   int ks = 1;
-  while (ks < 8 && base * ks * 2 <= num_sms && nk >= 4 * ks) ks *= 2;
+  const int64_t room = nk >= 256 ? 2 * (int64_t)num_sms : (int64_t)num_sms;
+  while (ks < 8 && base * ks * 2 <= room && nk >= 4 * ks) ks *= 2;
   // every CTA of the split needs at least one stage
   while (ks > 1 && (ks - 1) * ((nk + ks - 1) / ks) >= nk) ks /= 2;
   switch (ks) {
