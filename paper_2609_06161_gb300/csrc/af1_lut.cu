@@ -149,6 +149,13 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const __grid_constant_
 
   // ---- activations of the CTA's columns -> zs[t][k + k / 32] (FP32) -------
   griddep_wait();
+  // Phase 1's dependent is the same call's phase 2: let it launch now, so its
+  // CTAs copy their U words from HBM while this kernel computes (they hold
+  // no input of another call). Measured against launching it after the
+  // lookups (below): config-1 stack 6.33 -> 6.22 us per linear on the DAG
+  // schedule, 6.42 -> 6.13 grouped, 8.62 -> 8.42 serial; letting phase 2's
+  // own dependents launch this early too lost on the DAG (6.43).
+  if (PHASE == 1) griddep_launch_dependents();
   stage_activations<PHASE, kThreads, SWIGLU>(pb, xg, x2g, zg, T, nch, k0, zs, zrow, tid);
   if (tid < slice) rs[tid] = rs_own;
   __syncthreads();
@@ -171,12 +178,12 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const __grid_constant_
     }
   }
 
-  // Let the next kernel launch only now: its CTAs would otherwise hold SM
-  // slots (waiting for this kernel) that sibling kernels on other streams
-  // need, and its sign copies still get the reduction's time as a head start
-  // (measured: config-1 stack 7.40 -> 6.53 us per linear on the DAG schedule,
-  // trigger at the start vs here).
-  griddep_launch_dependents();
+  // Phase 2 lets the next kernel launch only now: its CTAs would otherwise
+  // hold SM slots (waiting for this kernel) that sibling kernels on other
+  // streams need, and its sign copies still get the reduction's time as a
+  // head start (measured: config-1 stack 7.40 -> 6.53 us per linear on the
+  // DAG schedule, trigger at the start vs here).
+  if (PHASE == 2) griddep_launch_dependents();
   // ---- partial sums -> owner CTA of each row -> final sums -------------------
   cluster_wait();  // every CTA of the cluster has started
   {
