@@ -36,7 +36,7 @@ METRIC = "tokens/s and us/layer for binary-factorized linear (AF1, 1.0 BPW); % o
 LAYERS = 32
 # Measured DRAM traffic of one layer's seven decode calls at one token (bytes;
 # ncu, profiles/lut_kernel_llama3_8b_b1.md): 1.026 x the algorithmic bytes.
-DECODE_TRAFFIC_B1_PER_LAYER = 28147456
+DECODE_TRAFFIC_B1_PER_LAYER = 28145408
 TC_DECODE = False  # set from --tc-decode
 
 
