@@ -853,7 +853,7 @@ constexpr int kTwoPerSmSmem = 110 * 1024;  // at or below this, two CTAs share a
 DecodePlan plan_decode(int phase, const SignMatrix& sm, int T, int num_sms, int max_smem, bool prep) {
   DecodePlan p;
   p.N = n_for_tokens(T);
-  const int sms = num_sms > 0 ? num_sms : 148;
+  const int sms = num_sms > 0 ? num_sms : kDefaultSms;
   int ks = sms / (sm.RB > 0 ? sm.RB : 1);
   if (ks < 1) ks = 1;
   if (ks > kMaxKS) ks = kMaxKS;
@@ -1072,7 +1072,7 @@ PhaseChoice choose_phase(const af1_layer& L, int phase, const SignMatrix& m, int
     const bool flag = (L.flags & AF1_FLAG_STREAM_DECODE) != 0;
     bool want = flag || !c.lut.ok;
     if (!want) {
-      const int sms = L.num_sms > 0 ? L.num_sms : 148;
+      const int sms = L.num_sms > 0 ? L.num_sms : kDefaultSms;
       int per_sm = 233472 / (c.lut.smem + 1024);
       per_sm = per_sm > 4 ? 4 : per_sm;
       want = (int64_t)m.RB * c.lut.KS > (int64_t)sms * per_sm;

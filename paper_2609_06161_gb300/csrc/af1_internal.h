@@ -32,6 +32,8 @@ namespace af1 {
 
 // Tokens per prefill pass (calls with more than kMaxPassTokens tokens).
 constexpr int64_t kPrefillPassTokens = 2048;
+// SM count the planners assume when the caller passes none (a GB300 has 152).
+constexpr int kDefaultSms = 152;
 
 // Workspace carve-up for one layer and one forward call of `tokens` tokens.
 struct Workspace {

@@ -314,7 +314,7 @@ int plan_one(const SignMatrix& sm, int T, int sms, int max_smem, int* cpc_out, i
 LutPlan plan_lut(const SignMatrix* sm, int count, int T, int num_sms, int max_smem) {
   LutPlan p;
   if (count < 1 || count > kMaxGroup || T < 1 || T > kMaxPassTokens) return p;
-  const int sms = num_sms > 0 ? num_sms : 148;
+  const int sms = num_sms > 0 ? num_sms : kDefaultSms;
   const int Tg = T < kGroupTokens ? T : kGroupTokens;
   int KS = 0;
   for (int i = 0; i < count; ++i) {

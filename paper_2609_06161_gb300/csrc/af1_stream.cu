@@ -383,7 +383,7 @@ cudaError_t launch_np(const StreamArgs& a, const StreamPlan& p, cudaStream_t st)
 StreamPlan search_stream(int phase, const SignMatrix& sm, int T, int num_sms, int max_smem) {
   StreamPlan p;
   if (T < 1 || T > kMaxStreamTokens || sm.RB < 1 || sm.NCH < 1) return p;
-  const int sms = num_sms > 0 ? num_sms : 148;
+  const int sms = num_sms > 0 ? num_sms : kDefaultSms;
   int64_t best = -1;
   for (int G = 1; G <= kMaxStreamG; G *= 2) {
     const int64_t SRB = (sm.RB + G - 1) / G;
