@@ -194,20 +194,21 @@ def run_reference(args):
     print(json.dumps(line))
 
 
+SCHEDULES = {"dag": "q|k|v and gate|up on parallel streams (decoder dependency DAG)",
+             "group": "q|k|v and gate|up each as one multi-layer call (shared input), one stream",
+             "serial": "one stream in model order"}
+
+
 def config_dict(args):
     if args.workload == "prefill":
         return {"workload": (f"LLaMA-3-8B-shaped AF1 linears (q,k,v,o,gate,up,down at 1.0-BPW ranks) x {args.layers} "
                              f"layers, prefill {args.tokens} tokens per call, FP16 N(0,1) activations with 1% outlier "
-                             f"channels x20, one stream in model order" + ("" if args.no_graph else ", CUDA graph")),
+                             f"channels x20, " + SCHEDULES[args.schedule] + ("" if args.no_graph else ", CUDA graph")),
                 "tokens": args.tokens, "layers": args.layers, "linears_per_step": 7 * args.layers,
                 "l2": "inputs larger than L2 (weights + activations per step >> 129 MB), no flush"}
     return {"workload": (f"LLaMA-3-8B-shaped AF1 decoder linears (q,k,v,o 4096x4096 r2028 / k,v 1024x4096 r800 / "
                          f"gate,up 14336x4096 r3167 / down 4096x14336 r3167) x {args.layers} layers, decode batch "
-                         f"{args.batch}, " + {"dag": "q|k|v and gate|up on parallel streams (decoder dependency DAG)",
-                                              "group": "q|k|v and gate|up each as one multi-layer call (shared "
-                                                       "input), one stream",
-                                              "serial": "one stream in model order"}[args.schedule]
-                         + ("" if args.no_graph else ", CUDA graph")),
+                         f"{args.batch}, " + SCHEDULES[args.schedule] + ("" if args.no_graph else ", CUDA graph")),
             "batch": args.batch, "layers": args.layers, "linears_per_step": 7 * args.layers,
             "decode_kernel": ("tensor cores (AF1_FLAG_TC_DECODE)" if args.tc_decode
                               else "lookup tables on the CUDA cores (default)"),
