@@ -154,7 +154,21 @@ def time_oracle_layer(data):
     return time.perf_counter() - t0
 
 
-def cpu_baseline(batch, min_seconds=10.0):
+def resolve_workload(args):
+    """Tokens per call of the workload; the prefill workload defaults to 4
+    layers (a step of 28 calls at 2048 tokens)."""
+    if args.workload == "prefill":
+        if args.tokens <= 16:
+            raise SystemExit("--tokens must be > 16 for the prefill path")
+        if args.layers == LAYERS:
+            args.layers = 4
+        return args.tokens
+    if not 1 <= args.batch <= 16:
+        raise SystemExit("--batch must be in 1..16 for the decode path")
+    return args.batch
+
+
+def cpu_baseline(batch, layers, min_seconds=10.0):
     data = oracle_layer_sample(batch)
     times = []
     t_start = time.perf_counter()
@@ -163,32 +177,33 @@ def cpu_baseline(batch, min_seconds=10.0):
         if time.perf_counter() - t_start >= min_seconds:
             break
     per_layer = float(np.median(times))
-    value = batch / (per_layer * LAYERS)
+    value = batch / (per_layer * layers)
     return {"value": value, "unit": "tokens/s", "cores": NCORES, "kind": "oracle",
             "sample": (f"FP64 numpy oracle (unpack + factored forward) on the 7 linears of one decoder layer, "
-                       f"batch {batch}, {len(times)} repetitions ({sum(times):.1f} s), median scaled x{LAYERS} layers; "
+                       f"{batch} tokens per call, {len(times)} repetitions ({sum(times):.1f} s), median scaled x{layers} layers; "
                        f"BLAS threads {NCORES}, unpacking single-threaded")}
 
 
-def run_reference(args):
+def run_reference(args, b):
     world, rank, _ = dist_env()
     if rank != 0:
         return
-    data = oracle_layer_sample(args.batch)
+    data = oracle_layer_sample(b)
     for _ in range(max(args.warmup, 0)):
         time_oracle_layer(data)
     times = [time_oracle_layer(data) for _ in range(args.steps)]
     step = float(np.mean(times))
-    value = args.batch / (step * LAYERS)
+    value = b / (step * args.layers)
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": step * LAYERS * 1e3,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": step * args.layers * 1e3,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic (seeded PCG64 signs/scales/activations)",
         "config": config_dict(args),
         "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": NCORES, "kind": "oracle",
                          "sample": (f"each step: FP64 oracle forward of the 7 linears of one decoder layer "
-                                    f"(1/{LAYERS} of the workload), batch {args.batch}; value scaled x{LAYERS}")},
+                                    f"(1/{args.layers} of the workload), {b} tokens per call; value scaled "
+                                    f"x{args.layers}")},
         "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line))
@@ -596,8 +611,9 @@ def main():
     global TC_DECODE
     args = parse()
     TC_DECODE = args.tc_decode
+    b = resolve_workload(args)
     if args.impl == "reference":
-        run_reference(args)
+        run_reference(args, b)
         return
     import torch
     import torch.distributed as dist
@@ -610,16 +626,6 @@ def main():
         torch.cuda.set_device(0)
     import paper_2609_06161_gb300 as P
 
-    if args.workload == "prefill":
-        b = args.tokens
-        if b <= 16:
-            raise SystemExit("--tokens must be > 16 for the prefill path")
-        if args.layers == LAYERS:
-            args.layers = 4
-    else:
-        b = args.batch
-        if not 1 <= b <= 16:
-            raise SystemExit("--batch must be in 1..16 for the decode path")
     if args.shape:
         run_shape(P, torch, args, b)
         return
@@ -836,7 +842,7 @@ def main():
         if sweep_rows is not None:
             line["sweep"] = sweep_rows
         if not args.no_cpu and world == 1 and args.workload == "decode":
-            line["cpu_baseline"] = cpu_baseline(b)
+            line["cpu_baseline"] = cpu_baseline(b, args.layers)
         if args.workload == "prefill":
             line["dtype"] = "f16 tcgen05 MMA / f32 accumulate (1-bit signs expanded to +-b, f16 activations)"
             line["us_per_layer"] = ms_step * 1e3 / nlin
