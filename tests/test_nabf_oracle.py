@@ -99,3 +99,34 @@ def test_nabf_improves_on_its_initialisation_and_dbf_has_no_projector():
         out = N.nabf(W, r, iters=8, rho=1.0, compensate=comp)
         assert out["objective"][-1] < out["objective"][0]
         assert (np.all(out["q_left"] == 0) and np.all(out["q_right"] == 0)) == (not comp)
+
+
+def test_proxies_satisfy_first_order_optimality(monkeypatch):
+    """The ADMM proxies (Sec. 3.1) are regularised least-squares minimisers:
+    the gradient of |W' - A0 B|^2 + rho |B|^2 vanishes at the initial right
+    proxy B0, and that of |W' - A B|^2 + rho |A - A_prev|^2 at the first left
+    proxy (duals still zero), A_prev and B being the SVID projections of the
+    initialisation. The initial sketch is W' times the SplitMix64 signs."""
+    g = np.random.default_rng(6)
+    m, n, r, rho = 30, 24, 6, 0.7
+    W = g.normal(size=(m, n))
+    calls = []
+    real = N.svid
+
+    def spy(Z, power_iters):
+        out = real(Z, power_iters)
+        calls.append((np.array(Z, dtype=np.float64), out))
+        return out
+
+    monkeypatch.setattr(N, "svid", spy)
+    N.nabf(W, r, iters=1, rho=rho, seed=3)
+    assert len(calls) == 4  # init A, init B, then the left and right projections of iteration 1
+    (A0, (A_init, *_)), (B0, (B_init, *_)), (Ah, _) = calls[0], calls[1], calls[2]
+    np.testing.assert_allclose(A0, W @ N.splitmix64_signs(3, n * r).reshape(n, r), rtol=1e-12, atol=1e-12)
+    grad_B = -A0.T @ (W - A0 @ B0) + rho * B0
+    assert np.abs(grad_B).max() <= 1e-9 * np.abs(A0.T @ W).max()
+    grad_A = -(W - Ah @ B_init) @ B_init.T + rho * (Ah - A_init)
+    assert np.abs(grad_A).max() <= 1e-9 * np.abs(W @ B_init.T).max()
+    # A transposed operand or a dropped regulariser fails the same check.
+    wrong = np.linalg.solve(B_init @ B_init.T, (W @ B_init.T).T).T
+    assert np.abs(-(W - wrong @ B_init) @ B_init.T + rho * (wrong - A_init)).max() > 1e-3
