@@ -132,6 +132,19 @@ def dist_env():
     return world, rank, local
 
 
+def max_over_ranks(dist, torch, world, value, device):
+    """The job's time: the largest of the ranks' times (every rank gets it)."""
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_tokens_per_s(tokens_per_rank_step, world, steps, seconds):
+    """Whole-job throughput: every rank's tokens over the slowest rank's time."""
+    return tokens_per_rank_step * world * steps / seconds
+
+
 # ---------------------------------------------------------------------------
 # CPU oracle timing (cpu_baseline and the reference arm)
 # ---------------------------------------------------------------------------
@@ -718,13 +731,9 @@ def main():
     barrier()
     ms = e0.elapsed_time(e1)
     clk = clocks.stop()
-    t = torch.tensor([ms], dtype=torch.float64, device=dev)
-    if world > 1:
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    ms_max = float(t.item())
+    ms_max = max_over_ranks(dist, torch, world, ms, dev)
     ms_step = ms_max / args.steps
-    tokens_per_step = b * world
-    value = tokens_per_step / (ms_step * 1e-3)
+    value = job_tokens_per_s(b, world, args.steps, ms_max * 1e-3)
     nlin = len(views)
     us_layer = ms_step * 1e3 / nlin
     alg = sum(algorithmic_bytes(m, n, r, b) for (name, m, n, r, layer, x) in objs)
@@ -771,10 +780,7 @@ def main():
             yh.copy_(ybuf, non_blocking=True)
         stream.synchronize()
     e2e_s = time.perf_counter() - t0
-    te = torch.tensor([e2e_s], dtype=torch.float64, device=dev)
-    if world > 1:
-        dist.all_reduce(te, op=dist.ReduceOp.MAX)
-    e2e_value = tokens_per_step * args.steps / float(te.item())
+    e2e_value = job_tokens_per_s(b, world, args.steps, max_over_ranks(dist, torch, world, e2e_s, dev))
 
     dense = None
     if not args.no_dense and rank == 0:

@@ -56,3 +56,40 @@ def test_workload_bounds(monkeypatch):
         monkeypatch.setattr(sys, "argv", ["bench.py"] + argv)
         with pytest.raises(SystemExit):
             bench.resolve_workload(bench.parse())
+
+
+def _rank_worker(rank, world, port, q):
+    import torch
+    import torch.distributed as dist
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    sys.path.insert(0, ROOT)
+    import bench
+    # Rank g took 10 + 5 g seconds for 3 steps of 4 tokens.
+    t = bench.max_over_ranks(dist, torch, world, 10.0 + 5.0 * rank, "cpu")
+    q.put((rank, t, bench.job_tokens_per_s(4, world, 3, t)))
+    dist.destroy_process_group()
+
+
+def test_job_time_is_the_slowest_rank():
+    """Under several ranks the bench times the job by its slowest rank and
+    counts every rank's tokens (two gloo processes on the CPU)."""
+    import socket
+    import torch.multiprocessing as mp
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        port = s.getsockname()[1]
+    world = 2
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    procs = [ctx.Process(target=_rank_worker, args=(g, world, port, q)) for g in range(world)]
+    for p in procs:
+        p.start()
+    for p in procs:
+        p.join(120)
+        assert p.exitcode == 0
+    got = sorted(q.get(timeout=10) for _ in range(world))
+    for rank, t, v in got:
+        assert t == 15.0
+        assert v == pytest.approx(4 * 2 * 3 / 15.0)
