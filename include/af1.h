@@ -308,10 +308,118 @@ AF1_API int af1_linear_forward_multi(const af1_layer* const* layers, int count, 
 AF1_API int af1_linear_forward_static(const af1_layer* layer, const void* x, int64_t ldx, int64_t tokens,
                                       void* y, int64_t ldy, int y_dtype, void* stream);
 
+/* Status of the built-in scratch array of af1_linear_forward_static on the
+ * current device: synchronizes `stream`, then returns AF1_OK, or
+ * AF1_ERR_TIMEOUT if a bounded device-side wait of a static call gave up
+ * since the last check. On AF1_ERR_TIMEOUT the whole array is zeroed again
+ * (status word and bookkeeping), so the next static call starts clean.
+ * Allocates nothing. Errors: CUDA. */
+AF1_API int af1_static_status(void* stream);
+
 /* Synchronize `stream` and report the status word the kernels keep in a
  * workspace: AF1_OK, or AF1_ERR_TIMEOUT if a bounded device-side wait gave
  * up since the workspace was last cleared (the word is then reset to 0). */
 AF1_API int af1_workspace_status(void* workspace, void* stream);
+
+/* Budget of every bounded device-side wait (mbarrier phases, dependency
+ * counters), in clock64() cycles, for the kernels launched after this call
+ * on any thread (default 2e9, about 1 s at 2 GHz). A launch captured in a
+ * CUDA graph keeps the budget it was captured with. A wait that exceeds it
+ * gives up and the call reports AF1_ERR_TIMEOUT through its status word.
+ * Errors: INVALID_ARG (cycles < 1). */
+AF1_API int af1_set_wait_cycles(int64_t cycles);
+AF1_API int64_t af1_get_wait_cycles(void);
+
+/* ---- A decode step as one launch ---------------------------------------------
+ * Many linears (e.g. the 7 of each decoder layer of a model) in dependent
+ * levels, run by ONE persistent kernel. Each linear computes
+ * y = x . W_hat^T (AF1 Sec. 3.1, Eq. final_reconstruction, right to left);
+ * the paper has no counterpart for the batching, which removes the kernel
+ * boundary per phase that separate calls pay.
+ * Dependencies: an input that is exactly the output of a linear of an
+ * earlier level (same pointer and row stride, matching width, FP16 outputs)
+ * is chained: the consumer reads the producer's results as soon as they
+ * exist, rounded exactly as the stored output (so a decoder's o projection
+ * can read q's output and down can read gate's and up's through x2). Any
+ * other input of a linear at level L > 0 is read only after every linear of
+ * the levels below L has stored its output, as kernels in stream order
+ * would. An input may not be the output of the same or a later level.
+ * Results agree with af1_linear_forward per linear within the library's
+ * tolerance; with integer-exact inputs they are identical. */
+typedef struct af1_step_linear {
+  const af1_layer* layer;
+  const void* x;    /* FP16 [tokens x n], row stride ldx (ldx >= n, ldx % 8 == 0), 16-byte aligned */
+  const void* x2;   /* NULL, or FP16 u of the same shape: the input is then h = FP16(SiLU(x) u),
+                       SiLU(z) = z / (1 + e^-z) in FP32 (x is the gate output g) */
+  int64_t ldx;
+  void* y;          /* [tokens x m] of the step's y_dtype, row stride ldy, 16-byte aligned */
+  int64_t ldy;
+  int32_t level;    /* >= 0; linears of one level are independent of each other */
+  int32_t reserved; /* must be 0 */
+} af1_step_linear;
+
+/* Level 0 waits until af1_step_open_gate has set the workspace's gate word
+ * (a hand-off from another stream without an event); each run closes the
+ * gate again when it ends. */
+#define AF1_STEP_WAIT_GATE 1
+
+typedef struct af1_step af1_step; /* opaque plan, owns a small device table */
+
+/* Plan a step over `count` linears for `tokens` rows (1..4) with outputs of
+ * y_dtype (AF1_F16 or AF1_F32). The pointers in lin are baked into the plan:
+ * each run reads the x buffers and writes the y buffers given here. Layers
+ * must outlive the plan. Allocates the plan's device table (synchronous).
+ * Errors: INVALID_ARG, BAD_POINTER, MISALIGNED, CUDA. */
+AF1_API int af1_step_create(const af1_step_linear* lin, int count, int64_t tokens, int y_dtype, int32_t flags,
+                            af1_step** out);
+
+/* The schedule af1_step_create would build, computed on the host alone (no
+ * GPU needed): for linears of shapes (m[i], n[i], r[i]) at level[i], `tokens`
+ * rows and `ctas` CTAs. producer[i] >= 0 names the linear (of an earlier
+ * level) whose output is linear i's input, producer2[i] >= 0 the one whose
+ * output is its SwiGLU up operand; -1 (or a NULL array) means none: an
+ * external input. Problem 2j is phase 1 (t = V^T (b x), an r x n sign
+ * matrix) and 2j + 1 phase 2 (u = U s', m x r) of linear order_out[j] (the
+ * linears sorted by level, stably). Tile k is tasks_out[7k .. 7k + 6] =
+ * {problem, first row block, row blocks G, first 128-column chunk, chunks,
+ * K slice, kind}: kind 0 computes partial sums over the chunks, kind 1 (on
+ * phase-2 problems, chunks 0) stores the G row blocks of y; a level's kind-1
+ * tiles run after the next level's phase-1 tiles when every linear of that
+ * level has a producer, else before them. CTA c runs tiles
+ * cta_first_out[c] .. cta_first_out[c + 1] - 1 in that order; ks_out[q] is
+ * the number of K slices of problem q. Every output
+ * pointer may be NULL (tasks_out needs max_tasks >= *ntasks). Errors:
+ * INVALID_ARG. */
+AF1_API int af1_step_plan_dry(const int64_t* m, const int64_t* n, const int64_t* r, const int32_t* level,
+                              const int32_t* producer, const int32_t* producer2, int count, int64_t tokens,
+                              int32_t ctas, int32_t* order_out, int32_t* tasks_out, int64_t max_tasks,
+                              int32_t* cta_first_out, int32_t* ks_out, int64_t* ntasks, double* model_us);
+
+/* Workspace bytes af1_step_run needs (>= 256: a header of run bookkeeping
+ * and the split-K partial sums of every phase, 8 bytes each). */
+AF1_API int64_t af1_step_workspace_bytes(const af1_step* step);
+
+/* Plan summary: CTAs of the launch, tiles, levels and the planner's modelled
+ * critical path in microseconds (any pointer may be NULL). */
+AF1_API int af1_step_info(const af1_step* step, int64_t* ctas, int64_t* tasks, int64_t* levels, double* model_us);
+
+/* Run the step on `stream`: one cooperative kernel launch (every CTA of the
+ * launch is resident). workspace: device memory of af1_step_workspace_bytes,
+ * 256-byte aligned, zero-filled before its first use; every completed run
+ * leaves the header ready for the next one, so one workspace serves any
+ * sequence of runs on one stream. Runs that may overlap on the GPU need
+ * different workspaces. A bounded wait that gave up is reported by
+ * af1_workspace_status(workspace, stream) (the run's bookkeeping is closed
+ * even then, so the workspace stays usable). Asynchronous; errors:
+ * INVALID_ARG, WORKSPACE, BAD_POINTER, CUDA. */
+AF1_API int af1_step_run(const af1_step* step, void* workspace, int64_t workspace_bytes, void* stream);
+
+/* Open the gate of a step created with AF1_STEP_WAIT_GATE (stream-ordered
+ * write of the workspace's gate word). Errors: WORKSPACE, CUDA. */
+AF1_API int af1_step_open_gate(void* workspace, void* stream);
+
+/* Release a plan (synchronizes the device first). NULL is a no-op. */
+AF1_API void af1_step_destroy(af1_step* step);
 
 /* Release a layer and its device buffers. NULL is a no-op. Synchronizes the
  * device before freeing, so queued work that reads the layer completes. */

@@ -18,8 +18,8 @@ import os
 import torch
 
 __all__ = [
-    "AF1Error", "Layer", "rank_for_budget", "workspace_status", "last_error", "version", "lib_path",
-    "words_per_row", "AF1_F16", "AF1_F32",
+    "AF1Error", "Layer", "Step", "rank_for_budget", "workspace_status", "static_status", "last_error", "version",
+    "lib_path", "words_per_row", "set_wait_cycles", "get_wait_cycles", "AF1_F16", "AF1_F32",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -117,6 +117,33 @@ _lib.af1_nabf_factorize.argtypes = [_vp, _i64, _i64, _i64, _vp, _vp, ctypes.POIN
 _lib.af1_nabf_factorize.restype = ctypes.c_int
 _lib.af1_workspace_status.argtypes = [_vp, _vp]
 _lib.af1_workspace_status.restype = ctypes.c_int
+_lib.af1_static_status.argtypes = [_vp]
+_lib.af1_static_status.restype = ctypes.c_int
+_lib.af1_set_wait_cycles.argtypes = [_i64]
+_lib.af1_set_wait_cycles.restype = ctypes.c_int
+_lib.af1_get_wait_cycles.argtypes = []
+_lib.af1_get_wait_cycles.restype = _i64
+
+
+class _StepLinear(ctypes.Structure):
+    _fields_ = [("layer", _vp), ("x", _vp), ("x2", _vp), ("ldx", _i64), ("y", _vp), ("ldy", _i64),
+                ("level", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+
+
+_lib.af1_step_create.argtypes = [ctypes.POINTER(_StepLinear), ctypes.c_int, _i64, ctypes.c_int, ctypes.c_int32,
+                                 ctypes.POINTER(_vp)]
+_lib.af1_step_create.restype = ctypes.c_int
+_lib.af1_step_workspace_bytes.argtypes = [_vp]
+_lib.af1_step_workspace_bytes.restype = _i64
+_lib.af1_step_info.argtypes = [_vp, ctypes.POINTER(_i64), ctypes.POINTER(_i64), ctypes.POINTER(_i64),
+                               ctypes.POINTER(ctypes.c_double)]
+_lib.af1_step_info.restype = ctypes.c_int
+_lib.af1_step_run.argtypes = [_vp, _vp, _i64, _vp]
+_lib.af1_step_run.restype = ctypes.c_int
+_lib.af1_step_open_gate.argtypes = [_vp, _vp]
+_lib.af1_step_open_gate.restype = ctypes.c_int
+_lib.af1_step_destroy.argtypes = [_vp]
+_lib.af1_step_destroy.restype = None
 _lib.af1_free.argtypes = [_vp]
 _lib.af1_free.restype = None
 _lib.af1_last_error.argtypes = []
@@ -176,6 +203,21 @@ def _ptr(t) -> int:
 def workspace_status(workspace: torch.Tensor, stream=None) -> None:
     """Synchronize and raise AF1Error(AF1_ERR_TIMEOUT) if a bounded device wait gave up."""
     _check(_lib.af1_workspace_status(_ptr(workspace), _stream_handle(stream)))
+
+
+def static_status(stream=None) -> None:
+    """af1_static_status: raise AF1Error(AF1_ERR_TIMEOUT) if a wait of a
+    call of af1_linear_forward_static gave up (the array is then reset)."""
+    _check(_lib.af1_static_status(_stream_handle(stream)))
+
+
+def set_wait_cycles(cycles: int) -> None:
+    """Budget (clock64 cycles) of every bounded device wait of later launches."""
+    _check(_lib.af1_set_wait_cycles(int(cycles)))
+
+
+def get_wait_cycles() -> int:
+    return int(_lib.af1_get_wait_cycles())
 
 
 class Layer:
@@ -466,3 +508,93 @@ def nabf_factorize(W: torch.Tensor, r: int, iters: int = 10, rho: float = 1.0, e
     k = iters + 1
     return {"U": U, "V": V, "a": a, "s": s_, "b": b, "objective": h[:k], "q_left": [int(v) for v in h[k:2 * k]],
             "q_right": [int(v) for v in h[2 * k:]]}
+
+
+# -- a decode step as one launch -------------------------------------------------------
+
+AF1_STEP_WAIT_GATE = 1
+
+
+def _row_stride(t: torch.Tensor, cols: int, align: int) -> int:
+    if t.dim() != 2 or t.stride(1) != 1:
+        raise ValueError("step tensors must be 2-D with contiguous rows")
+    return t.stride(0) if t.shape[0] > 1 else max(t.stride(0), cols + (-cols) % align)
+
+
+class Step:
+    """af1_step_*: many linears in dependent levels as one persistent launch.
+
+    linears: sequence of (layer, x, y, level) or (layer, x, y, level, x2)
+    tuples; x (and x2, the `up` output of a SwiGLU input) float16
+    (tokens, ldx), y float16 or float32 (tokens, ldy), all on the current
+    device. The tensors are kept alive by this object; every run reads the
+    x buffers and writes the y buffers given here."""
+
+    def __init__(self, linears, gate: bool = False):
+        items = []
+        keep = []
+        tokens = None
+        ydt = None
+        for item in linears:
+            layer, x, y, level = item[:4]
+            x2 = item[4] if len(item) > 4 else None
+            if x.dtype != torch.float16 or (x2 is not None and x2.dtype != torch.float16):
+                raise ValueError("x and x2 must be float16")
+            if y.dtype not in (torch.float16, torch.float32):
+                raise ValueError("y must be float16 or float32")
+            ydt = ydt or y.dtype
+            if y.dtype != ydt:
+                raise ValueError("all outputs must have one dtype")
+            tokens = tokens or x.shape[0]
+            if x.shape[0] != tokens or y.shape[0] < tokens:
+                raise ValueError("all inputs must have the same number of rows")
+            yd = AF1_F16 if ydt == torch.float16 else AF1_F32
+            ldx = _row_stride(x, layer.n, 8)
+            if x2 is not None and (x2.shape != x.shape or x2.stride() != x.stride()):
+                raise ValueError("x2 must have the shape and strides of x")
+            ldy = _row_stride(y, layer.m, 8 if yd == AF1_F16 else 4)
+            items.append(_StepLinear(layer._h, _ptr(x), _ptr(x2), ldx, _ptr(y), ldy, int(level), 0))
+            keep += [layer, x, y, x2]
+        arr = (_StepLinear * len(items))(*items)
+        h = _vp()
+        yd = AF1_F16 if ydt == torch.float16 else AF1_F32
+        _check(_lib.af1_step_create(arr, len(items), tokens, yd, AF1_STEP_WAIT_GATE if gate else 0,
+                                    ctypes.byref(h)))
+        self._h = h.value
+        self._keep = keep
+        self.tokens = tokens
+
+    def workspace_bytes(self) -> int:
+        v = _lib.af1_step_workspace_bytes(self._h)
+        if v < 0:
+            raise AF1Error(int(v), last_error())
+        return int(v)
+
+    def make_workspace(self, device=None) -> torch.Tensor:
+        return torch.zeros(self.workspace_bytes(), dtype=torch.uint8,
+                           device=device or torch.device("cuda", torch.cuda.current_device()))
+
+    def info(self) -> dict:
+        c, t, lv, us = _i64(), _i64(), _i64(), ctypes.c_double()
+        _check(_lib.af1_step_info(self._h, ctypes.byref(c), ctypes.byref(t), ctypes.byref(lv), ctypes.byref(us)))
+        return {"ctas": c.value, "tasks": t.value, "levels": lv.value, "model_us": us.value}
+
+    def run(self, workspace: torch.Tensor, stream=None) -> None:
+        _check(_lib.af1_step_run(self._h, _ptr(workspace), workspace.numel() * workspace.element_size(),
+                                 _stream_handle(stream)))
+
+    @staticmethod
+    def open_gate(workspace: torch.Tensor, stream=None) -> None:
+        _check(_lib.af1_step_open_gate(_ptr(workspace), _stream_handle(stream)))
+
+    def destroy(self) -> None:
+        if getattr(self, "_h", None):
+            _lib.af1_step_destroy(self._h)
+            self._h = None
+            self._keep = []
+
+    def __del__(self):
+        try:
+            self.destroy()
+        except Exception:
+            pass

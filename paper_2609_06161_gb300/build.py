@@ -17,7 +17,7 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 OUT = os.path.join(HERE, "libaf1.so")
 BUILD_DIR = os.path.join(HERE, "_build")
-SOURCES = ["af1_api.cu", "af1_pack.cu", "af1_decode.cu", "af1_lut.cu", "af1_stream.cu", "af1_prefill.cu", "af1_noalloc.cu", "af1_hisa.cu", "af1_nabf.cu"]
+SOURCES = ["af1_api.cu", "af1_pack.cu", "af1_decode.cu", "af1_lut.cu", "af1_stream.cu", "af1_prefill.cu", "af1_noalloc.cu", "af1_hisa.cu", "af1_nabf.cu", "af1_step.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden",
          "--expt-relaxed-constexpr", "-I", INCLUDE]

@@ -5,6 +5,7 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
 #include <cstdio>
 #include <cstring>
 #include <new>
@@ -171,9 +172,14 @@ int check_scales(const uint16_t* a, const uint16_t* s, const uint16_t* b, int de
 
 }  // namespace
 
+namespace {
+std::atomic<long long> g_wait_cycles{af1::kDefaultWaitCycles};
+}  // namespace
+
 namespace af1 {
 // Record a failure in the calling thread's af1_last_error() message.
 int set_error(int code, const std::string& msg) { return fail(code, msg); }
+long long wait_budget() { return g_wait_cycles.load(std::memory_order_relaxed); }
 }  // namespace af1
 
 extern "C" {
@@ -473,7 +479,8 @@ int linear_forward_checked(const af1_layer* layer, const void* x, int64_t ldx, i
     return fail(AF1_ERR_MISALIGNED, "u must be 16-byte aligned");
   if ((rc = check_device_ptr(y, "y", dev)) != AF1_OK) return rc;
   if (workspace == nullptr) return fail(AF1_ERR_WORKSPACE, "workspace is NULL");
-  if ((rc = check_device_ptr(workspace, "workspace", dev)) != AF1_OK) return AF1_ERR_WORKSPACE;
+  if (check_device_ptr(workspace, "workspace", dev) != AF1_OK)
+    return fail(AF1_ERR_WORKSPACE, "workspace is not device memory of the current device");
   if (ldx < layer->n) return fail(AF1_ERR_INVALID_ARG, "ldx < n");
   if (ldy < layer->m) return fail(AF1_ERR_INVALID_ARG, "ldy < m");
   if ((reinterpret_cast<uintptr_t>(x) & 15) != 0 || (reinterpret_cast<uintptr_t>(y) & 15) != 0)
@@ -555,7 +562,8 @@ int af1_linear_forward_multi(const af1_layer* const* layers, int count, const vo
       return fail(AF1_ERR_MISALIGNED, "ldys[i] * element size must be a multiple of 16 bytes");
   }
   if (workspace == nullptr) return fail(AF1_ERR_WORKSPACE, "workspace is NULL");
-  if ((rc = check_device_ptr(workspace, "workspace", dev)) != AF1_OK) return AF1_ERR_WORKSPACE;
+  if (check_device_ptr(workspace, "workspace", dev) != AF1_OK)
+    return fail(AF1_ERR_WORKSPACE, "workspace is not device memory of the current device");
   if ((reinterpret_cast<uintptr_t>(workspace) & 255) != 0)
     return fail(AF1_ERR_WORKSPACE, "workspace must be 256-byte aligned");
   const int64_t need = af1::multi_workspace_offset(layers, count, tokens, true);
@@ -583,6 +591,15 @@ int af1_workspace_status(void* workspace, void* stream) {
   g_err.clear();
   return AF1_OK;
 }
+
+int af1_set_wait_cycles(int64_t cycles) {
+  if (cycles < 1) return fail(AF1_ERR_INVALID_ARG, "cycles must be >= 1");
+  g_wait_cycles.store(cycles, std::memory_order_relaxed);
+  g_err.clear();
+  return AF1_OK;
+}
+
+int64_t af1_get_wait_cycles(void) { return g_wait_cycles.load(std::memory_order_relaxed); }
 
 void af1_free(af1_layer* layer) { destroy_layer(layer); }
 

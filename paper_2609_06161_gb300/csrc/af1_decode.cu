@@ -51,6 +51,7 @@
 #include "af1.h"
 #include "af1_internal.h"
 #include "af1_layout.h"
+#include "af1_ptx.cuh"
 
 namespace af1 {
 namespace {
@@ -60,70 +61,11 @@ constexpr int kTmemCols = 256;        // per CTA: two CTAs fit on one SM
 constexpr int kMaxCPC = 64;           // column chunks per CTA (one mbarrier each)
 constexpr int kMaxKS = 16;            // CTAs per cluster
 constexpr int kMinSmem = 80 * 1024;   // at most two CTAs per SM: their tensor memory always fits
-constexpr long long kWaitCycles = 2000000000ll;  // ~1 s at 2 GHz
-constexpr unsigned kStatusTimeout = 1u;
 
 // ---------------------------------------------------------------------------
 // PTX helpers (hand-written: mbarrier, bulk copy, PDL, cluster, tcgen05, FP8)
 // ---------------------------------------------------------------------------
 
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
-}
-__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
-}
-__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
-               : "memory");
-}
-__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
-  uint32_t done;
-  asm volatile(
-      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
-      : "=r"(done)
-      : "r"(smem_u32(bar)), "r"(parity)
-      : "memory");
-  return done != 0;
-}
-// Bounded wait: false (and the CTA error flag set) if the phase did not
-// complete within kWaitCycles.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint32_t* err) {
-  if (mbar_try_wait(bar, parity)) return true;
-  const long long t0 = clock64();
-  while (!mbar_try_wait(bar, parity)) {
-    if (clock64() - t0 > kWaitCycles) {
-      atomicOr(err, 1u);
-      return false;
-    }
-  }
-  return true;
-}
-__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
-  asm volatile(
-      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-          smem_u32(dst)),
-      "l"(src), "r"(bytes), "r"(smem_u32(bar))
-      : "memory");
-}
-__device__ __forceinline__ void griddep_launch_dependents() {
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-}
-__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
-
-// Split cluster barrier: arrive (relaxed) at start, wait before the first
-// write into a peer's shared memory (the peer must have started).
-__device__ __forceinline__ void cluster_arrive_relaxed() {
-  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
-}
-__device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.aligned;" ::: "memory"); }
-// Cluster-wide barrier with release/acquire semantics for shared memory.
-__device__ __forceinline__ void cluster_sync() {
-  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
-}
 __device__ __forceinline__ void st_cluster_f32(float* local, uint32_t rank, float v) {
   uint32_t remote;
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(local)), "r"(rank));
@@ -251,6 +193,7 @@ struct DecodeArgs {
   int64_t ldy;
   int ydtype;
   unsigned* status;
+  long long wait_cycles;  // budget of every bounded wait (clock64 cycles)
   // Prepared B operand (passes of more than 4 tokens): tiles of every chunk
   // (chunk c at c N 128 bytes) and per-(slice, token) {2^-sigma, Q 2^-sigma}
   // at bstats[slice * kMaxPassTokens + t]; written by bprep_kernel, read by
@@ -443,7 +386,7 @@ __device__ __forceinline__ void build_b(const DecodeArgs& a, int T, int nch, int
           reinterpret_cast<float*>(act)[(size_t)t * rowlen + k] = __ldcg(a.zin + (int64_t)t * a.ldz + k0 + k);
       }
     }
-    mbar_wait(xfull, 0, err);
+    mbar_wait(xfull, 0, err, a.wait_cycles);
     builders_sync();  // tail values visible
   }
   // z' of group (t, c4): from the staged activations or straight from L2.
@@ -598,10 +541,10 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const DecodeArgs a)
     for (int c = 0; c < nch && ok; ++c) {
       const int b = c % NBUF, use = c / NBUF;
       if (use >= 1) {
-        ok = mbar_wait(&h.aempty[b], (use - 1) & 1, &h.err);
+        ok = mbar_wait(&h.aempty[b], (use - 1) & 1, &h.err, a.wait_cycles);
         tc_fence_after();
       }
-      if (ok) ok = mbar_wait(&h.wfull[c], 0, &h.err);
+      if (ok) ok = mbar_wait(&h.wfull[c], 0, &h.err, a.wait_cycles);
       if (!ok) break;
       uint32_t r[32];
       const uint32_t* wc = W + c * (kChunkBytes / 4);
@@ -625,7 +568,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const DecodeArgs a)
         for (int c = 0; c < nch; ++c)
           bulk_g2s(Bt + c * N * 128, a.bbuf + (int64_t)(c0 + c) * N * 128, (uint32_t)(N * 128), &h.xfull);
       }
-      mbar_wait(&h.xfull, 0, &h.err);
+      mbar_wait(&h.xfull, 0, &h.err, a.wait_cycles);
     } else {
       build_b<PHASE, N>(a, T, nch, k0, bt, act, Bt, qpart, h.maxbits, &h.xfull, &h.err);
     }
@@ -638,7 +581,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const DecodeArgs a)
       bool ok = true;
       for (int c = 0; c < nch && ok; ++c) {
         const int b = c % NBUF, use = c / NBUF;
-        ok = mbar_wait(&h.afull[b], use & 1, &h.err);
+        ok = mbar_wait(&h.afull[b], use & 1, &h.err, a.wait_cycles);
         if (!ok) break;
         tc_fence_after();
 #pragma unroll
@@ -677,7 +620,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const DecodeArgs a)
   griddep_wait();  // outputs may still be read by the previous kernel until it completes
   cluster_wait();  // every CTA of the cluster has started
   if (warp < 4) {
-    const bool ok = mbar_wait(&h.ddone, 0, &h.err) && mbar_wait(&h.stats, 0, &h.err);
+    const bool ok = mbar_wait(&h.ddone, 0, &h.err, a.wait_cycles) && mbar_wait(&h.stats, 0, &h.err, a.wait_cycles);
     tc_fence_after();
     const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
     const int i = tid;  // block row
@@ -732,13 +675,13 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const DecodeArgs a)
   if (tid == 128 && h.err != 0) {
     // Something timed out: let the bulk copies drain (bounded) so that none
     // lands after the CTA has exited, and report it.
-    for (int c = 0; c < nch; ++c) mbar_wait(&h.wfull[c], 0, &h.err);
-    if (STAGED || PREP) mbar_wait(&h.xfull, 0, &h.err);
+    for (int c = 0; c < nch; ++c) mbar_wait(&h.wfull[c], 0, &h.err, a.wait_cycles);
+    if (STAGED || PREP) mbar_wait(&h.xfull, 0, &h.err, a.wait_cycles);
     atomicOr(a.status, kStatusTimeout);
   }
   if (warp == 4) {
     tc_fence_after();
-    if (lane == 0) mbar_wait(&h.ddone, 0, &h.err);  // no MMA may still read tensor memory
+    if (lane == 0) mbar_wait(&h.ddone, 0, &h.err, a.wait_cycles);  // no MMA may still read tensor memory
     __syncwarp();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"((uint32_t)kTmemCols)
                  : "memory");
@@ -814,7 +757,7 @@ __global__ void __launch_bounds__(128) bprep_kernel(const DecodeArgs a) {
   asm volatile("fence.proxy.async.global;" ::: "memory");
   __syncthreads();
   if (bt == 0 && h.err != 0) {
-    if (staged_acts(N)) mbar_wait(&h.xfull, 0, &h.err);
+    if (staged_acts(N)) mbar_wait(&h.xfull, 0, &h.err, a.wait_cycles);
     atomicOr(a.status, kStatusTimeout);
   }
 }
@@ -1002,6 +945,7 @@ LutArgs lut_args(const DecodeArgs& d) {
   a.tokens = d.tokens;
   a.ydtype = d.ydtype;
   a.status = d.status;
+  a.wait_cycles = d.wait_cycles;
   a.prob[0] = lut_problem(d);
   return a;
 }
@@ -1147,6 +1091,7 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
     a1.sout = reinterpret_cast<float*>(wsb + W.sbuf);
     a1.lds = decode_ldz(L);
     a1.status = stat;
+    a1.wait_cycles = wait_budget();
     a1.bbuf = W.bbuf != 0 ? wsb + W.bbuf : nullptr;
     a1.bstats = W.bbuf != 0 ? reinterpret_cast<float2*>(wsb + W.bstats) : nullptr;
     cudaError_t e = cudaSuccess;
@@ -1183,6 +1128,7 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
     a2.ldy = ldy;
     a2.ydtype = y_dtype;
     a2.status = a1.status;
+    a2.wait_cycles = a1.wait_cycles;
     a2.bbuf = a1.bbuf;
     a2.bstats = a1.bstats;
     e = c2.tc         ? launch_decode<2>(a2, q2, st)
@@ -1240,6 +1186,7 @@ cudaError_t launch_forward_multi(const af1_layer* const* Ls, int count, const vo
   a1.tokens = a2.tokens = T;
   a1.ydtype = a2.ydtype = y_dtype;
   a1.status = a2.status = status;
+  a1.wait_cycles = a2.wait_cycles = wait_budget();
   for (int i = 0; i < count; ++i) {
     const af1_layer& L = *Ls[i];
     const Workspace W = plan_workspace(L, tokens, prep);

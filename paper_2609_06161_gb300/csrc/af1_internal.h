@@ -68,6 +68,11 @@ cudaError_t launch_bf16_to_f16(const uint16_t* src, uint16_t* dst, int64_t count
 // u at stride ldx, of h at ldh).
 cudaError_t launch_swiglu(const __half* g, const __half* u, int64_t ldx, int64_t tokens, int64_t n, __half* h,
                           int64_t ldh, cudaStream_t st);
+// Budget, in clock64() cycles, of every bounded device-side wait of the
+// kernels launched from now on (af1_set_wait_cycles; process-wide). The
+// default is about 1 s at the GB300's 2 GHz clock.
+constexpr long long kDefaultWaitCycles = 2000000000ll;
+long long wait_budget();
 // Set the calling thread's af1_last_error() message; returns `code`.
 int set_error(int code, const std::string& msg);
 
@@ -98,6 +103,7 @@ struct LutArgs {
   int ydtype;
   int KS;            // set by the launcher: CTAs per cluster, common to all problems
   unsigned* status;
+  long long wait_cycles;  // budget of every bounded wait (clock64 cycles)
   LutProblem prob[kMaxGroup];
 };
 struct LutPlan {

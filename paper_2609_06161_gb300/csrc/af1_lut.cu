@@ -173,7 +173,7 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const __grid_constant_
     const uint32_t tbl0 = smem_u32(smem + sp.tbl);
     bool ok = true;
     for (int c = 0; c < nch; ++c) {
-      if (ok) ok = mbar_wait(&h.wfull[c], 0, &h.err);
+      if (ok) ok = mbar_wait(&h.wfull[c], 0, &h.err, a.wait_cycles);
       lookup_chunk<NP>(tbl0 + (uint32_t)(c * TCB), W + c * (kChunkBytes / 4) + r, g, acc);
     }
   }
@@ -196,7 +196,7 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const __grid_constant_
   // Exit barrier (waited for after the final sums): no CTA leaves while a
   // peer may still store into it.
   cluster_arrive_relaxed();
-  mbar_wait(&h.red, 0, &h.err);  // this CTA's partials have all landed
+  mbar_wait(&h.red, 0, &h.err, a.wait_cycles);  // this CTA's partials have all landed
   for (int idx = tid; idx < T * cnt; idx += kThreads) {
     const int t = idx / cnt;
     const int i = idx - t * cnt;
@@ -233,7 +233,7 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const __grid_constant_
   if (tid == 0 && h.err != 0) {
     // A wait gave up: let the bulk copies drain (bounded) so that none lands
     // after the CTA has exited, and report it.
-    for (int c = 0; c < nch; ++c) mbar_wait(&h.wfull[c], 0, &h.err);
+    for (int c = 0; c < nch; ++c) mbar_wait(&h.wfull[c], 0, &h.err, a.wait_cycles);
     atomicOr(a.status, kStatusTimeout);
   }
 }

@@ -1,6 +1,6 @@
 // af1_lut_common.cuh — pieces shared by the two CUDA-core decode kernels
 // (af1_lut.cu: clustered split-K tiles; af1_stream.cu: balanced streaming
-// ranges): PTX helpers, the layout of the lookup tables of signed sums, the
+// ranges): the layout of the lookup tables of signed sums, the
 // staging of activations, the table build and the lookups of one chunk.
 //
 // Tables. For every group of 4 columns {k_0..k_3} and every token, the 16 sums
@@ -24,64 +24,10 @@
 
 #include "af1_internal.h"
 #include "af1_layout.h"
+#include "af1_ptx.cuh"
 
 namespace af1 {
 namespace {
-
-constexpr long long kWaitCycles = 2000000000ll;  // ~1 s at 2 GHz
-constexpr unsigned kStatusTimeout = 1u;
-
-// ---------------------------------------------------------------------------
-// PTX helpers (mbarrier, bulk copy, PDL, cluster)
-// ---------------------------------------------------------------------------
-
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
-}
-__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
-               : "memory");
-}
-__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
-  uint32_t done;
-  asm volatile(
-      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
-      : "=r"(done)
-      : "r"(smem_u32(bar)), "r"(parity)
-      : "memory");
-  return done != 0;
-}
-// Bounded wait: false (and the CTA error flag set) if the phase did not
-// complete within kWaitCycles.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint32_t* err) {
-  if (mbar_try_wait(bar, parity)) return true;
-  const long long t0 = clock64();
-  while (!mbar_try_wait(bar, parity)) {
-    if (clock64() - t0 > kWaitCycles) {
-      atomicOr(err, 1u);
-      return false;
-    }
-  }
-  return true;
-}
-__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
-  asm volatile(
-      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-          smem_u32(dst)),
-      "l"(src), "r"(bytes), "r"(smem_u32(bar))
-      : "memory");
-}
-__device__ __forceinline__ void griddep_launch_dependents() {
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-}
-__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
-__device__ __forceinline__ void cluster_arrive_relaxed() {
-  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
-}
-__device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.aligned;" ::: "memory"); }
 
 // v -> `local` in the shared memory of cluster CTA `rank`, completing 4
 // bytes of the transaction count of that CTA's mbarrier `bar`.

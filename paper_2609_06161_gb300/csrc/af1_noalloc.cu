@@ -72,4 +72,30 @@ int af1_linear_forward_static(const af1_layer* layer, const void* x, int64_t ldx
                                      false);
 }
 
+// Status word of the built-in array (offset 0 of the array, where every
+// forward call keeps its workspace status). A timeout leaves the array's
+// bookkeeping undefined, so the whole array is zeroed after reporting one.
+int af1_static_status(void* stream) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return fail(AF1_ERR_CUDA, std::string("cudaGetDevice: ") + cudaGetErrorString(e));
+  if (dev < 0 || dev >= kMaxDevices) return fail(AF1_ERR_CUDA, "device index out of range");
+  void* scratch = nullptr;
+  int rc = scratch_address(dev, &scratch);
+  if (rc != AF1_OK) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  uint32_t word = 0;
+  e = cudaMemcpyAsync(&word, scratch, 4, cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  if (e != cudaSuccess) return fail(AF1_ERR_CUDA, std::string("af1_static_status: ") + cudaGetErrorString(e));
+  if (word != 0) {
+    e = cudaMemsetAsync(scratch, 0, (size_t)kStaticScratchBytes, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return fail(AF1_ERR_CUDA, std::string("af1_static_status: ") + cudaGetErrorString(e));
+    return fail(AF1_ERR_TIMEOUT, "a bounded device-side wait of a static call gave up; the built-in array was reset");
+  }
+  af1::set_error(AF1_OK, "");
+  return AF1_OK;
+}
+
 }  // extern "C"

@@ -31,6 +31,7 @@
 
 #include "af1_internal.h"
 #include "af1_layout.h"
+#include "af1_ptx.cuh"
 
 namespace af1 {
 namespace {
@@ -39,8 +40,6 @@ constexpr int BM = 128;  // features per CTA (MMA M, TMEM lanes)
 constexpr int BK = 64;   // K per stage: one 128-byte swizzle row of FP16
 constexpr int kMaxStages = 6;
 constexpr int kThreads = 256;
-constexpr long long kWaitCycles = 2000000000ll;
-constexpr unsigned kStatusTimeout = 1u;
 
 template <int BN>
 __host__ __device__ constexpr int tile_b_bytes() {
@@ -68,6 +67,7 @@ struct PrefillArgs {
   int64_t ld_out;
   int out_f32;
   unsigned* status;
+  long long wait_cycles;  // budget of every bounded wait (clock64 cycles)
 };
 
 struct __align__(8) PrefillBarriers {
@@ -79,46 +79,6 @@ struct __align__(8) PrefillBarriers {
   uint32_t err;
 };
 
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-
-__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
-}
-__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
-}
-__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
-               : "memory");
-}
-__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
-  uint32_t done;
-  asm volatile(
-      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
-      : "=r"(done)
-      : "r"(smem_u32(bar)), "r"(parity)
-      : "memory");
-  return done != 0;
-}
-// Bounded wait; on timeout records the error in the CTA flag and returns.
-__device__ __forceinline__ void mbar_wait(uint64_t* bar, uint32_t parity, uint32_t* err) {
-  if (mbar_try_wait(bar, parity)) return;
-  const long long t0 = clock64();
-  while (!mbar_try_wait(bar, parity)) {
-    if (clock64() - t0 > kWaitCycles) {
-      atomicOr(err, 1u);
-      return;
-    }
-  }
-}
-
-__device__ __forceinline__ void griddep_launch_dependents() {
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-}
-__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
-
 __device__ __forceinline__ void tmem_ld16(uint32_t addr, uint32_t (&r)[16]) {
   asm volatile(
       "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
@@ -128,10 +88,7 @@ __device__ __forceinline__ void tmem_ld16(uint32_t addr, uint32_t (&r)[16]) {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
-// Cluster helpers for the split-K reduction.
-__device__ __forceinline__ void cluster_sync() {
-  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
-}
+// Cluster helper for the split-K reduction.
 __device__ __forceinline__ void st_cluster_f32(float* local, uint32_t rank, float v) {
   uint32_t remote;
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(local)), "r"(rank));
@@ -260,7 +217,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       for (int it = 0; it < nk; ++it) {
         const int s = it % STAGES;
-        if (it >= STAGES) mbar_wait(&bar.empty[s], ((it / STAGES) & 1) ^ 1, &bar.err);
+        if (it >= STAGES) mbar_wait(&bar.empty[s], ((it / STAGES) & 1) ^ 1, &bar.err, a.wait_cycles);
         mbar_expect_tx(&bar.full_b[s], (uint32_t)kTileB);
         tma_load_2d(tileB + s * kTileB, &act_map, (it0 + it) * BK, t0, &bar.full_b[s]);
       }
@@ -273,8 +230,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int it = 0; it < nk; ++it) {
         const int s = it % STAGES;
         const uint32_t ph = (it / STAGES) & 1;
-        mbar_wait(&bar.full_a[s], ph, &bar.err);
-        mbar_wait(&bar.full_b[s], ph, &bar.err);
+        mbar_wait(&bar.full_a[s], ph, &bar.err, a.wait_cycles);
+        mbar_wait(&bar.full_b[s], ph, &bar.err, a.wait_cycles);
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 #pragma unroll
         for (int kk = 0; kk < BK / 16; ++kk) {
@@ -335,7 +292,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) mbar_arrive(&bar.full_a[(it - 1) % STAGES]);
       }
       if (it >= STAGES) {
-        if (lane == 0) mbar_wait(&bar.empty[s], ((it / STAGES) & 1) ^ 1, &bar.err);
+        if (lane == 0) mbar_wait(&bar.empty[s], ((it / STAGES) & 1) ^ 1, &bar.err, a.wait_cycles);
         __syncwarp();
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
       }
@@ -372,7 +329,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // at 64 tokens lost (95 -> 120), where GEMM 1 leaves SMs idle.
     griddep_launch_dependents();
     // ---- epilogue: TMEM -> registers -> global ---------------------------
-    if (lane == 0) mbar_wait(&bar.done, 0, &bar.err);
+    if (lane == 0) mbar_wait(&bar.done, 0, &bar.err, a.wait_cycles);
     __syncwarp();
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     if (KS == 1) {
@@ -445,7 +402,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (bar.err != 0 && threadIdx.x == 0) {
     // A wait gave up: let TMA copies that may still be in flight land
     // (bounded) before the CTA exits, and report it.
-    for (int s = 0; s < STAGES; ++s) mbar_wait(&bar.full_b[s], 0, &bar.err);
+    for (int s = 0; s < STAGES; ++s) mbar_wait(&bar.full_b[s], 0, &bar.err, a.wait_cycles);
     atomicOr(a.status, kStatusTimeout);
   }
   if (warp == 1) {
@@ -565,6 +522,7 @@ cudaError_t launch_prefill(const af1_layer& L, const void* x, int64_t ldx, int64
     g1.ld_out = ldh;
     g1.out_f32 = 0;
     g1.status = status;
+    g1.wait_cycles = wait_budget();
     cudaError_t e = launch_gemm<true>(g1, static_cast<const __half*>(x) + t0 * ldx, ldx, L.num_sms, st);
     if (e != cudaSuccess) return e;
     PrefillArgs g2 = {};
@@ -577,6 +535,7 @@ cudaError_t launch_prefill(const af1_layer& L, const void* x, int64_t ldx, int64
     g2.ld_out = ldy;
     g2.out_f32 = y_dtype == 0 ? 0 : 1;
     g2.status = status;
+    g2.wait_cycles = g1.wait_cycles;
     e = launch_gemm<false>(g2, reinterpret_cast<const __half*>(h_buf), ldh, L.num_sms, st);
     if (e != cudaSuccess) return e;
   }

@@ -81,18 +81,12 @@ __host__ __device__ inline StreamSmem stream_smem(int CPC, int KS, int T, int G,
   return p;
 }
 
-__device__ __forceinline__ void named_sync(int id, int threads) {
-  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
-}
-__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
-}
-
 struct StreamArgs {
   LutProblem p;        // CPC and rb0 unused
   int tokens, ydtype;  // T (1..2)
   int KS, CPC, NSC;    // CTAs per cluster (grid y), chunks per CTA, ring slots
   unsigned* status;
+  long long wait_cycles;  // budget of every bounded wait (clock64 cycles)
 };
 
 // SWIGLU (phase 1): the input is h = FP16(SiLU(x) x2).
@@ -151,7 +145,7 @@ __global__ void __launch_bounds__(kStreamThreads, 3) stream_kernel(const __grid_
       uint32_t par = 0;  // parity of the slot's release to wait for
       const uint8_t* src = pb.signs + ((int64_t)srb * G * NCH + c0) * kChunkBytes;
       for (int k = 0; k < nch; ++k) {
-        if (k >= NSC && ok) ok = mbar_wait(&h.empty[s], par, &h.err);
+        if (k >= NSC && ok) ok = mbar_wait(&h.empty[s], par, &h.err, a.wait_cycles);
         mbar_expect_tx(&h.full[s], (uint32_t)(nrb * kChunkBytes));
         for (int gi = 0; gi < nrb; ++gi)
           bulk_g2s(ring + (s * G + gi) * kChunkBytes, src + ((int64_t)gi * NCH + k) * kChunkBytes, kChunkBytes,
@@ -199,7 +193,7 @@ __global__ void __launch_bounds__(kStreamThreads, 3) stream_kernel(const __grid_
     int s = 0;
     uint32_t par = 0;
     for (int k = 0; k < nch; ++k) {
-      if (ok) ok = mbar_wait(&h.full[s], par, &h.err);
+      if (ok) ok = mbar_wait(&h.full[s], par, &h.err, a.wait_cycles);
       const uint32_t tb = tbl0 + (uint32_t)(k * TCB);
 #pragma unroll
       for (int gi = 0; gi < G; ++gi)
@@ -231,7 +225,7 @@ __global__ void __launch_bounds__(kStreamThreads, 3) stream_kernel(const __grid_
   // Exit barrier (waited for after the final sums): no CTA leaves while a
   // peer may still store into it.
   cluster_arrive_relaxed();
-  mbar_wait(&h.red, 0, &h.err);
+  mbar_wait(&h.red, 0, &h.err, a.wait_cycles);
   for (int idx = tid; idx < T * cnt; idx += kConsumers) {
     const int t = idx / cnt;
     const int i = idx - t * cnt;
@@ -269,7 +263,7 @@ __global__ void __launch_bounds__(kStreamThreads, 3) stream_kernel(const __grid_
     // k < nch with k mod NSC = s.
     for (int s2 = 0; s2 < NSC && s2 < nch; ++s2) {
       const int kl = s2 + ((nch - 1 - s2) / NSC) * NSC;
-      mbar_wait(&h.full[s2], (uint32_t)((kl / NSC) & 1), &h.err);
+      mbar_wait(&h.full[s2], (uint32_t)((kl / NSC) & 1), &h.err, a.wait_cycles);
     }
     atomicOr(a.status, kStatusTimeout);
   }
@@ -468,6 +462,7 @@ cudaError_t launch_stream(int phase, const LutProblem& prob, int tokens, int ydt
   a.CPC = p.CPC;
   a.NSC = p.NSC;
   a.status = status;
+  a.wait_cycles = wait_budget();
   if (phase == 1 && prob.x2 != nullptr)
     return tokens == 1 ? launch_np<1, 0, true>(a, p, st) : launch_np<1, 1, true>(a, p, st);
   if (phase == 1) return tokens == 1 ? launch_np<1, 0>(a, p, st) : launch_np<1, 1>(a, p, st);

@@ -59,6 +59,13 @@ def scales_f16(g: np.random.Generator, size: int) -> np.ndarray:
     return v.astype(np.float16).view(np.uint16)
 
 
+def unit_gain_scales_f16(g: np.random.Generator, size: int, level: float) -> np.ndarray:
+    """FP16 bit patterns of level * U(0.5, 1.5): scales for chains of layers
+    whose activations should stay of order one (level ~ 1 / sqrt(n r) for the
+    rank scale, 1 for the row and column scales)."""
+    return (level * g.uniform(0.5, 1.5, size=size)).astype(np.float16).view(np.uint16)
+
+
 def activations_f16(g: np.random.Generator, tokens: int, d_in: int, outlier_frac: float = 0.0,
                     outlier_gain: float = 20.0) -> np.ndarray:
     """FP16 bit patterns of N(0, 1) activations (tokens x d_in); a seeded

@@ -28,13 +28,14 @@ def test_reference_arm_line():
     assert "1/2 of the workload" in cb["sample"]
     e2e = line["e2e"]
     assert e2e["value"] == line["value"] and e2e["h2d_bytes_per_step"] == 0 and e2e["d2h_bytes_per_step"] == 0
-    # tokens per step / step time: one token per step over the 2 layers timed.
-    assert line["value"] == pytest.approx(1e3 * line["config"]["batch"] / line["ms_per_step"], rel=1e-9)
+    # ms_per_step is the measured step (one decoder layer's 7 linears); the
+    # value scales it to the workload's layers.
+    assert line["value"] == pytest.approx(1e3 * line["config"]["batch"] / (line["ms_per_step"] * 2), rel=1e-9)
     assert "x 2 layers" in line["config"]["workload"]
 
 
 @pytest.mark.parametrize("workload", ["decode", "prefill"])
-@pytest.mark.parametrize("schedule", ["dag", "serial", "group"])
+@pytest.mark.parametrize("schedule", ["dag", "serial", "group", "step"])
 def test_config_names_the_schedule(monkeypatch, workload, schedule):
     sys.path.insert(0, ROOT)
     import bench

@@ -1,6 +1,7 @@
 """af1_linear_forward_static, the forward entry point that allocates nothing
 (its scratch is an array built into the library), against af1_linear_forward
-on the same layer and input, twice in a row, through the C ABI.
+on the same layer and input, twice in a row, through the C ABI, and both
+against the FP64 oracle; af1_static_status then reports no timed-out wait.
 
 Kept in a file of its own that sorts last, so that a run stopping at the
 first failure has already run every other test."""
@@ -37,6 +38,7 @@ def test_static_scratch_entry_matches_workspace_entry():
             x = xp
         ldy = m + (-m) % 4
         ws = layer.make_workspace(tokens)
+        oracle = O.forward_from_packed(O.pack_U(d["U"]), O.pack_V(d["V"]), d["a"], d["s"], d["b"], d["x"], m, n, r)
         y_ref = torch.empty((tokens, ldy), dtype=torch.float32, device="cuda")
         rc = fwd(layer._h, x.data_ptr(), ldx, tokens, y_ref.data_ptr(), ldy, 1, ws.data_ptr(),
                  ws.numel(), stream)
@@ -50,6 +52,8 @@ def test_static_scratch_entry_matches_workspace_entry():
             b = y_ref[:, :m].double().cpu().numpy()
             assert np.isfinite(a).all()
             assert O.rowwise_rel_err(a, b) <= TOL
+            assert O.rowwise_rel_err(a, oracle) <= TOL
+        P.static_status()  # raises AF1Error(AF1_ERR_TIMEOUT) if a wait of a static call gave up
         layer.free()
 
 
