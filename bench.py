@@ -1,11 +1,14 @@
 """Benchmark: AF1 binary-factorized linears (decode path by default).
 
-Workload: the seven linears of a LLaMA-3-8B decoder layer (q, k, v, o, gate,
-up, down) at their exact 1.0-BPW ranks, replicated over 32 layers with
-distinct seeded synthetic weights (0.87 GB of packed signs per step, far
-above the 129 MB L2, so no flush is needed). One step is one decode token
-batch (default 1 token) through all 224 linears, issued in model order on one
-stream through af1_linear_forward and replayed as a CUDA graph.
+Workload (default): a 32-layer LLaMA-3-8B-shaped linear stack, the seven
+linears of each decoder layer (q, k, v, o, gate, up, down) with HiSA-like
+ranks: each matrix's exact 1.0-BPW rank times a seeded factor in [0.7, 1.3],
+renormalised so the whole stack stays within 1.0 bit per weight. Distinct
+seeded synthetic weights (about 0.87 GB of packed signs per step, far above
+the 129 MB L2, so no flush is needed). One step is one decode token (batch
+1 by default) through all 224 linears through af1_linear_forward on the
+decoder's dependency DAG, replayed as a CUDA graph. `--ranks uniform` uses
+every matrix's 1.0-BPW rank instead.
 
 `--workload prefill` times the tensor-core prefill path instead: the same
 seven linears over 4 layers at 2048 tokens per call (1 % outlier channels),
@@ -54,10 +57,14 @@ def parse():
                    help="decode: config 1 (1-16 tokens); prefill: config 2 (2048 tokens, tensor cores)")
     p.add_argument("--tokens", type=int, default=2048, help="prefill tokens per call")
     p.add_argument("--no-graph", action="store_true", help="eager launches instead of a CUDA graph (for profilers)")
-    p.add_argument("--schedule", choices=["dag", "serial", "group"], default="dag",
+    p.add_argument("--schedule", choices=["dag", "serial", "group", "step"], default="dag",
                    help="dag: a decoder layer's independent linears (q/k/v, gate/up) on parallel streams; "
                         "serial: all 7 linears chained on one stream; group: q|k|v and gate|up as one "
-                        "af1_linear_forward_multi call each (shared input), one stream")
+                        "af1_linear_forward_multi call each (shared input), one stream; step: the whole step "
+                        "as one persistent launch (af1_step_run) with the DAG's level order")
+    p.add_argument("--ranks", choices=["hisa", "uniform"], default="hisa",
+                   help="decode stack ranks: hisa = 1.0-BPW rank x U(0.7, 1.3), renormalised to 1.0 BPW over the "
+                        "stack (the default workload); uniform = every matrix at its 1.0-BPW rank")
     p.add_argument("--no-sweep", action="store_true",
                    help="skip the per-shape sweep (LLaMA-3-8B at 1/4/16 tokens, 70B shapes at 1/8/64/512)")
     p.add_argument("--no-stack", action="store_true", help="skip the 32-layer stack with HiSA-like ranks")
@@ -68,6 +75,18 @@ def parse():
     p.add_argument("--tc-decode", action="store_true",
                    help="create layers with AF1_FLAG_TC_DECODE (tensor-core decode kernel instead of lookup tables)")
     return p.parse_args()
+
+
+def workload_ranks(args, rank_fn=None, bits_fn=None):
+    """Rank of every linear of the stack, in model order (7 per layer)."""
+    import synth
+    if rank_fn is None:
+        import paper_2609_06161_gb300 as P
+        rank_fn = P.rank_for_budget
+    mn = [(m, n) for _ in range(args.layers) for (_nm, m, n) in synth.LLAMA3_8B_LINEARS]
+    if args.workload == "decode" and args.ranks == "hisa":
+        return hisa_ranks(mn, rank_fn=rank_fn, bits_fn=bits_fn)
+    return [int(rank_fn(m, n)) for (m, n) in mn]
 
 
 def shapes(rank_fn=None):
@@ -86,7 +105,7 @@ def oracle_shapes():
     return shapes(lambda m, n: O.rank_for_budget(m, n, 1))
 
 
-def hisa_ranks(mn, seed=3):
+def hisa_ranks(mn, seed=3, rank_fn=None, bits_fn=None):
     """HiSA-like rank allocation over the matrices `mn` = [(m, n), ...]: each
     1.0-BPW rank scaled by a seeded factor in [0.7, 1.3], then renormalised
     so that the total storage stays within 1.0 bit per weight: one common
@@ -94,16 +113,19 @@ def hisa_ranks(mn, seed=3):
     (slack below one rank step)."""
     import math
     import synth
-    import paper_2609_06161_gb300 as P
-    base = [P.rank_for_budget(m, n) for (m, n) in mn]
+    if rank_fn is None or bits_fn is None:
+        import paper_2609_06161_gb300 as P
+        rank_fn = rank_fn or P.rank_for_budget
+        bits_fn = bits_fn or P.storage_bits
+    base = [rank_fn(m, n) for (m, n) in mn]
     f, order = synth.hisa_rank_factors(seed, len(mn))
     drawn = [max(1, int(round(b * fi))) for b, fi in zip(base, f)]
     budget = sum(m * n for (m, n) in mn)
-    fixed = sum(P.storage_bits(m, n, 1) - (m + n + 16) for (m, n) in mn)  # 16 (m + n) per matrix
+    fixed = sum(bits_fn(m, n, 1) - (m + n + 16) for (m, n) in mn)  # 16 (m + n) per matrix
     per = sum(r * (m + n + 16) for r, (m, n) in zip(drawn, mn))
     c = (budget - fixed) / per
     ranks = [max(1, math.floor(c * r)) for r in drawn]
-    total = sum(P.storage_bits(m, n, r) for r, (m, n) in zip(ranks, mn))
+    total = sum(bits_fn(m, n, r) for r, (m, n) in zip(ranks, mn))
     while total > budget:  # floor of a positive factor cannot overshoot; kept as a guard
         i = max(range(len(ranks)), key=lambda j: ranks[j])
         total -= mn[i][0] + mn[i][1] + 16
@@ -149,11 +171,19 @@ def job_tokens_per_s(tokens_per_rank_step, world, steps, seconds):
 # CPU oracle timing (cpu_baseline and the reference arm)
 # ---------------------------------------------------------------------------
 
-def oracle_layer_sample(batch, seed_base=0):
-    """The 7 linears of one decoder layer, as canonical packed words."""
+def oracle_ranks(args):
+    """The stack's ranks by the oracle's rank rule (the host legs need no GPU
+    library)."""
+    from oracle import af1_oracle as O
+    return workload_ranks(args, rank_fn=lambda m, n: O.rank_for_budget(m, n, 1), bits_fn=O.storage_bits)
+
+
+def oracle_layer_sample(batch, ranks7, seed_base=0):
+    """The 7 linears of one decoder layer (ranks ranks7), as canonical packed words."""
     import synth
     data = []
-    for i, (name, m, n, r) in enumerate(oracle_shapes()):
+    for i, (name, m, n) in enumerate(synth.LLAMA3_8B_LINEARS):
+        r = ranks7[i]
         d = synth.layer_words(seed_base + i, m, n, r, batch)
         data.append((name, m, n, r, d))
     return data
@@ -181,8 +211,8 @@ def resolve_workload(args):
     return args.batch
 
 
-def cpu_baseline(batch, layers, min_seconds=10.0):
-    data = oracle_layer_sample(batch)
+def cpu_baseline(batch, layers, ranks7, min_seconds=10.0):
+    data = oracle_layer_sample(batch, ranks7)
     times = []
     t_start = time.perf_counter()
     while True:
@@ -201,7 +231,11 @@ def run_reference(args, b):
     world, rank, _ = dist_env()
     if rank != 0:
         return
-    data = oracle_layer_sample(b)
+    if args.workload == "prefill":
+        ranks7 = [r for (_nm, _m, _n, r) in oracle_shapes()]
+    else:
+        ranks7 = oracle_ranks(args)[:7]
+    data = oracle_layer_sample(b, ranks7)
     for _ in range(max(args.warmup, 0)):
         time_oracle_layer(data)
     times = [time_oracle_layer(data) for _ in range(args.steps)]
@@ -209,14 +243,14 @@ def run_reference(args, b):
     value = b / (step * args.layers)
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": step * args.layers * 1e3,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": step * 1e3,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic (seeded PCG64 signs/scales/activations)",
         "config": config_dict(args),
         "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": NCORES, "kind": "oracle",
                          "sample": (f"each step: FP64 oracle forward of the 7 linears of one decoder layer "
-                                    f"(1/{args.layers} of the workload), {b} tokens per call; value scaled "
-                                    f"x{args.layers}")},
+                                    f"(1/{args.layers} of the workload), {b} tokens per call; ms_per_step is "
+                                    f"that measured step, value = tokens / (step time x {args.layers} layers)")},
         "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line))
@@ -224,7 +258,8 @@ def run_reference(args, b):
 
 SCHEDULES = {"dag": "q|k|v and gate|up on parallel streams (decoder dependency DAG)",
              "group": "q|k|v and gate|up each as one multi-layer call (shared input), one stream",
-             "serial": "one stream in model order"}
+             "serial": "one stream in model order",
+             "step": "the whole step as one persistent launch (af1_step_run) in the decoder's level order"}
 
 
 def config_dict(args):
@@ -234,10 +269,15 @@ def config_dict(args):
                              f"channels x20, " + SCHEDULES[args.schedule] + ("" if args.no_graph else ", CUDA graph")),
                 "tokens": args.tokens, "layers": args.layers, "linears_per_step": 7 * args.layers,
                 "l2": "inputs larger than L2 (weights + activations per step >> 129 MB), no flush"}
-    return {"workload": (f"LLaMA-3-8B-shaped AF1 decoder linears (q,k,v,o 4096x4096 r2028 / k,v 1024x4096 r800 / "
-                         f"gate,up 14336x4096 r3167 / down 4096x14336 r3167) x {args.layers} layers, decode batch "
-                         f"{args.batch}, " + SCHEDULES[args.schedule] + ("" if args.no_graph else ", CUDA graph")),
-            "batch": args.batch, "layers": args.layers, "linears_per_step": 7 * args.layers,
+    if args.ranks == "hisa":
+        ranks = ("HiSA-like ranks: each matrix's 1.0-BPW rank x U(0.7, 1.3) (seeded), renormalised to 1.0 BPW over "
+                 "the stack")
+    else:
+        ranks = "1.0-BPW ranks (q,o r2028 / k,v r800 / gate,up,down r3167)"
+    return {"workload": (f"LLaMA-3-8B-shaped AF1 decoder linears (q,o 4096x4096 / k,v 1024x4096 / gate,up 14336x4096 "
+                         f"/ down 4096x14336), {ranks}, x {args.layers} layers, decode batch {args.batch}, "
+                         + SCHEDULES[args.schedule] + ("" if args.no_graph else ", CUDA graph")),
+            "batch": args.batch, "layers": args.layers, "linears_per_step": 7 * args.layers, "ranks": args.ranks,
             "decode_kernel": ("tensor cores (AF1_FLAG_TC_DECODE)" if args.tc_decode
                               else "lookup tables on the CUDA cores (default)"),
             "l2": "inputs larger than L2 (packed weights per step >> 129 MB), no flush"}
@@ -299,16 +339,21 @@ class Clocks:
 # The AF1 arm
 # ---------------------------------------------------------------------------
 
-def build_layers(P, torch, layers, batch, rank, outlier_frac=0.0):
+def build_layers(P, torch, layers, batch, rank, outlier_frac=0.0, ranks=None):
+    """7 linears per layer with seeded synthetic words; ranks: one per linear
+    (default: every matrix's 1.0-BPW rank)."""
     import synth
     objs = []
     for li in range(layers):
         for si, (name, m, n, r) in enumerate(shapes()):
+            if ranks is not None:
+                r = ranks[7 * li + si]
             d = synth.layer_words(100000 * (rank + 1) + 7 * li + si, m, n, r, batch, outlier_frac=outlier_frac)
             f16 = lambda bits: torch.from_numpy(np.ascontiguousarray(bits).view(np.float16)).cuda()
             Uw = torch.from_numpy(d["Uw"].view(np.int32)).cuda()
             Vw = torch.from_numpy(d["Vw"].view(np.int32)).cuda()
-            layer = P.Layer.from_words(Uw, Vw, f16(d["a"]), f16(d["s"]), f16(d["b"]), m, n, r, tc_decode=TC_DECODE)
+            layer = P.Layer.from_words(Uw, Vw, f16(d["a"]), f16(d["s"]), f16(d["b"]), m, n, r, tc_decode=TC_DECODE,
+                                       any_rank=ranks is not None)
             del Uw, Vw
             x = f16(d["x"]).reshape(batch, n)
             objs.append((name, m, n, r, layer, x))
@@ -574,25 +619,21 @@ def mlp_swiglu(P, torch, stream, steps):
             "unfused": "h by torch elementwise ops (FP32 SiLU and product, FP16 store), then af1_linear_forward"}
 
 
-def stack_hisa(P, torch, peaks, stream, steps, dense_ms=None):
-    """32-layer LLaMA-3-8B stack with HiSA-like per-matrix ranks (+-30 %
-    around the 1.0-BPW rank, renormalised to 1.0 BPW over the stack), one
-    decode token per step, all 224 linears chained on one stream as a CUDA
-    graph, and again on the decoder's dependency DAG."""
+def stack_other_ranks(P, torch, peaks, stream, steps, args):
+    """The 32-layer stack with the other rank allocation than the headline's
+    (uniform 1.0-BPW ranks when the headline uses HiSA-like ranks, and vice
+    versa), one token, on the decoder DAG, CUDA graph; weights drawn on the
+    device."""
     import synth
+    other = "uniform" if args.ranks == "hisa" else "hisa"
     mn = [(m, n) for _ in range(LAYERS) for (_nm, m, n) in synth.LLAMA3_8B_LINEARS]
-    ranks = hisa_ranks(mn)
+    ranks = hisa_ranks(mn) if other == "hisa" else [P.rank_for_budget(m, n) for (m, n) in mn]
     layers = [device_layer(P, torch, m, n, r, 20000 + i, any_rank=True) for i, ((m, n), r) in enumerate(zip(mn, ranks))]
     gx = torch.Generator(device="cuda")
     gx.manual_seed(31)
     xs = [torch.randn((1, n), generator=gx, device="cuda", dtype=torch.float16) for (m, n) in mn]
     ys = [torch.empty((1, m), device="cuda", dtype=torch.float16) for (m, n) in mn]
     ws = torch.zeros(max(L.workspace_bytes(1) for L in layers), dtype=torch.uint8, device="cuda")
-
-    def run():
-        for L, x, y in zip(layers, xs, ys):
-            L.forward_into(x, y, ws, stream=stream)
-    ms = time_graph(torch, run, stream, max(5, min(steps, 20)))
     side = [torch.cuda.Stream(), torch.cuda.Stream()]
     ws_side = [torch.zeros_like(ws), torch.zeros_like(ws)]
     views = list(zip(layers, xs, ys))
@@ -600,22 +641,63 @@ def stack_hisa(P, torch, peaks, stream, steps, dense_ms=None):
                         max(5, min(steps, 20)))
     alg = sum(algorithmic_bytes(m, n, r, 1) for (m, n), r in zip(mn, ranks))
     bits = sum(P.storage_bits(m, n, r) for (m, n), r in zip(mn, ranks))
-    out = {"workload": "32 x 7 LLaMA-3-8B linears, HiSA-like ranks (+-30 %, renormalised), 1 token, one stream "
-                       "(top level) and on the decoder DAG (dag); dense BF16 on one stream",
-           "ms_per_token": ms, "tokens_per_s": 1e3 / ms, "us_per_linear": ms * 1e3 / len(mn),
-           "bpw": bits / sum(m * n for (m, n) in mn), "rank_min": min(ranks), "rank_max": max(ranks),
-           "achieved_gbs": alg / (ms * 1e-3) / 1e9, "frac": alg / (ms * 1e-3) / 1e9 / peaks.get("hbm_gbs", 6800.0)}
-    out["dag"] = {"schedule": "q|k|v and gate|up on parallel streams (decoder dependency DAG)",
-                  "ms_per_token": ms_dag, "tokens_per_s": 1e3 / ms_dag, "us_per_linear": ms_dag * 1e3 / len(mn),
-                  "achieved_gbs": alg / (ms_dag * 1e-3) / 1e9,
-                  "frac": alg / (ms_dag * 1e-3) / 1e9 / peaks.get("hbm_gbs", 6800.0)}
-    if dense_ms is not None:
-        out["dense_bf16_ms_per_token"] = dense_ms
-        out["speedup_vs_dense_bf16"] = dense_ms / ms
-        out["dag"]["speedup_vs_dense_bf16"] = dense_ms / ms_dag
+    out = {"workload": f"32 x 7 LLaMA-3-8B linears, {other} ranks, 1 token, decoder DAG, CUDA graph",
+           "ranks": other, "ms_per_token": ms_dag, "tokens_per_s": 1e3 / ms_dag,
+           "us_per_linear": ms_dag * 1e3 / len(mn), "bpw": bits / sum(m * n for (m, n) in mn),
+           "rank_min": min(ranks), "rank_max": max(ranks), "achieved_gbs": alg / (ms_dag * 1e-3) / 1e9,
+           "frac": alg / (ms_dag * 1e-3) / 1e9 / peaks.get("hbm_gbs", 6800.0)}
     for L in layers:
         L.free()
     del layers, xs, ys, ws, ws_side, views
+    torch.cuda.empty_cache()
+    return out
+
+
+def chained_views(objs, b, dev, torch):
+    """The stack's linears reading each other's outputs as a decoder does:
+    q, k, v read the layer input, o reads q, gate and up read o, down reads
+    h = FP16(SiLU(gate) up), the next layer reads down (the first layer's input
+    is an external buffer). Returns (linear, x, y, level[, x2]) items."""
+    items = []
+    x = objs[0][5]
+    for li in range(len(objs) // 7):
+        lay = objs[7 * li:7 * li + 7]
+        yv = [torch.empty((b, m), dtype=torch.float16, device=dev) for (_n, m, n, r, L, xx) in lay]
+        base = 4 * li
+        items += [(lay[0][4], x, yv[0], base), (lay[1][4], x, yv[1], base), (lay[2][4], x, yv[2], base),
+                  (lay[3][4], yv[0], yv[3], base + 1), (lay[4][4], yv[3], yv[4], base + 2),
+                  (lay[5][4], yv[3], yv[5], base + 2), (lay[6][4], yv[4], yv[6], base + 3, yv[5])]
+        x = yv[6]
+    return items
+
+
+def prefill_extra(P, torch, peaks, stream, steps):
+    """Config 2 inside the default run: the seven LLaMA-3-8B linears at their
+    1.0-BPW ranks over 4 layers, 2048 tokens per call (FP16 N(0, 1) with a
+    seeded 1 % of channels x20), the tensor-core prefill kernels on the
+    decoder DAG, CUDA graph."""
+    T, nl = 2048, 4
+    objs = build_layers(P, torch, nl, T, 7, outlier_frac=0.01)
+    ys = [torch.empty((T, m), dtype=torch.float16, device="cuda") for (_n, m, n, r, L, x) in objs]
+    ws = torch.zeros(max(o[4].workspace_bytes(T) for o in objs), dtype=torch.uint8, device="cuda")
+    side = [torch.cuda.Stream(), torch.cuda.Stream()]
+    ws_side = [torch.zeros_like(ws), torch.zeros_like(ws)]
+    views = [(o[4], o[5], y) for o, y in zip(objs, ys)]
+    ms = time_graph(torch, lambda: dag_step(torch, views, stream, side, ws, ws_side), stream, max(5, min(steps, 20)))
+    P.workspace_status(ws)
+    flops = sum(2 * T * r * (m + n) for (_n, m, n, r, L, x) in objs)
+    tflops = flops / (ms * 1e-3) / 1e12
+    tpeak = peaks.get("bf16_tflops_sustained", 1700.0)
+    out = {"workload": "config 2: LLaMA-3-8B linears (1.0-BPW ranks) x 4 layers, 2048 tokens per call, FP16 N(0,1) "
+                       "activations with 1% outlier channels x20, decoder DAG, CUDA graph",
+           "ms_per_step": ms, "tokens_per_s": T / (ms * 1e-3),
+           "roofline": {"bound": "tensor", "kernel": "prefill_kernel (tcgen05 kind::f16, two GEMMs per call)",
+                        "achieved": tflops, "peak": tpeak, "unit": "TFLOP/s", "frac": tflops / tpeak,
+                        "peak_source": "MEASURED_PEAKS.json bf16_tflops_sustained (FP16 dense rate = BF16 rate)",
+                        "algorithmic_flops_per_step": flops}}
+    for (_n, m, n, r, L, x) in objs:
+        L.free()
+    del objs, ys, ws, ws_side, views
     torch.cuda.empty_cache()
     return out
 
@@ -643,7 +725,9 @@ def main():
         run_shape(P, torch, args, b)
         return
     dev = torch.device("cuda", torch.cuda.current_device())
-    objs = build_layers(P, torch, args.layers, b, rank, outlier_frac=0.01 if args.workload == "prefill" else 0.0)
+    ranks = workload_ranks(args)
+    objs = build_layers(P, torch, args.layers, b, rank, outlier_frac=0.01 if args.workload == "prefill" else 0.0,
+                        ranks=ranks if args.workload == "decode" else None)
     ws = torch.zeros(max(o[4].workspace_bytes(b) for o in objs), dtype=torch.uint8, device=dev)
     # Inputs and outputs live in one device buffer each so the e2e leg can move
     # them with a single copy per direction.
@@ -706,7 +790,21 @@ def main():
         torch.cuda.synchronize()
         return g
 
+    # The whole step as one persistent launch, in the DAG's level order.
+    step_plan = None
+    if len(views) % 7 == 0 and b <= 4 and args.workload == "decode":
+        lv7 = [0, 0, 0, 1, 2, 2, 3]
+        step_plan = P.Step([(L, xv, yv, 4 * (i // 7) + lv7[i % 7]) for i, (L, xv, yv) in enumerate(views)])
+        ws_step = step_plan.make_workspace(dev)
+
+    def step_one_launch():
+        step_plan.run(ws_step, stream=stream)
+
     steps_by_name = {"dag": step_dag, "group": step_group, "serial": step_serial}
+    if step_plan is not None:
+        steps_by_name["step"] = step_one_launch
+    if args.schedule == "step" and step_plan is None:
+        raise SystemExit("--schedule step needs the 7-linear decode workload with at most 4 tokens")
     step = steps_by_name[args.schedule] if len(views) % 7 == 0 else step_serial
     graph = make_graph(step)
 
@@ -759,6 +857,29 @@ def main():
             sms = f0.elapsed_time(f1) / args.steps
             others[name] = {"ms_per_step": sms, "us_per_layer": sms * 1e3 / len(views), "tokens_per_s": b / (sms * 1e-3)}
             del g2
+        if step_plan is not None:
+            # The one-launch step with the decoder's data flow: each linear
+            # reads its producer's output (the same weights and level order).
+            chained = P.Step(chained_views(objs, b, dev, torch))
+            ws_ch = chained.make_workspace(dev)
+            with torch.cuda.stream(stream):
+                for _ in range(3):
+                    chained.run(ws_ch, stream=stream)
+            torch.cuda.synchronize()
+            f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            f0.record(stream)
+            for _ in range(args.steps):
+                chained.run(ws_ch, stream=stream)
+            f1.record(stream)
+            torch.cuda.synchronize()
+            P.workspace_status(ws_ch, stream)
+            sms = f0.elapsed_time(f1) / args.steps
+            others["step_chained"] = {"ms_per_step": sms, "us_per_layer": sms * 1e3 / len(views),
+                                      "tokens_per_s": b / (sms * 1e-3),
+                                      "inputs": "q,k,v <- layer input, o <- q, gate,up <- o, down <- SwiGLU(gate, up), "
+                                                "next layer <- down"}
+            chained.destroy()
+            del ws_ch
     serial = others.get("serial")
 
     # e2e: host buffers in pinned memory, copies inside the timed region.
@@ -786,14 +907,17 @@ def main():
     if not args.no_dense and rank == 0:
         dense = dense_bf16(torch, objs, b, args, stream)
     peaks = load_peaks()
-    sweep_rows = stack = mlp = nabf = None
+    sweep_rows = stack = mlp = nabf = prefill = None
     if args.workload == "decode" and rank == 0:
         # Extra measurements, outside the timed region of the headline number.
+        if step_plan is not None:
+            step_plan.destroy()
+            step_plan = None
         if not args.no_stack:
-            stack = stack_hisa(P, torch, peaks, stream, args.steps,
-                               dense_ms=dense["ms_per_step"] if dense and b == 1 else None)
+            stack = stack_other_ranks(P, torch, peaks, stream, args.steps, args)
             mlp = mlp_swiglu(P, torch, stream, args.steps)
             nabf = nabf_bench(P, torch)
+            prefill = prefill_extra(P, torch, peaks, stream, args.steps)
         if not args.no_sweep:
             sweep_rows = sweep(P, torch, peaks, stream)
 
@@ -811,8 +935,12 @@ def main():
             # DRAM bytes (read + write) of one layer's 14 lookup-table kernels
             # at one token, from the ncu capture summarised in
             # profiles/lut_kernel_llama3_8b_b1.md, times 32 layers.
-            traffic = DECODE_TRAFFIC_B1_PER_LAYER * args.layers if b == 1 and not TC_DECODE else None
-            roof = {"bound": "hbm", "kernel": "af1_linear_forward (two lookup-table kernels per call, lut_kernel<1|2>)",
+            traffic = (DECODE_TRAFFIC_B1_PER_LAYER * args.layers
+                       if b == 1 and not TC_DECODE and args.ranks == "uniform" and args.schedule == "dag" else None)
+            kname = ("af1_step_run (one persistent step_kernel launch per step)" if args.schedule == "step" else
+                     "af1_linear_forward (two lookup-table kernels per call, lut_kernel<1|2>, stream_kernel<1|2> "
+                     "for the largest matrices)")
+            roof = {"bound": "hbm", "kernel": kname,
                     "achieved": achieved_gbs, "peak": hbm, "unit": "GB/s",
                     "frac": (achieved_gbs / hbm) if hbm else None, "peak_source": "MEASURED_PEAKS.json hbm_gbs"
                     if "hbm_gbs" in peaks else "fallback 6800 GB/s",
@@ -829,8 +957,8 @@ def main():
             "roofline": roof,
             "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": xo * 2,
                     "d2h_bytes_per_step": yo * 2},
-            "gpu_launches": (step_launches(objs, b, args.schedule) if args.workload == "decode" and nlin % 7 == 0
-                             else 2 * nlin) * args.steps,
+            "gpu_launches": ((1 if args.schedule == "step" else step_launches(objs, b, args.schedule))
+                             if args.workload == "decode" and nlin % 7 == 0 else 2 * nlin) * args.steps,
             "clocks": clk,
         }
         if dense is not None:
@@ -840,7 +968,9 @@ def main():
         if others:
             line["other_schedules"] = others
         if stack is not None:
-            line["stack_hisa"] = stack
+            line["stack_other_ranks"] = stack
+        if prefill is not None:
+            line["prefill"] = prefill
         if mlp is not None:
             line["mlp_swiglu"] = mlp
         if nabf is not None:
@@ -848,7 +978,7 @@ def main():
         if sweep_rows is not None:
             line["sweep"] = sweep_rows
         if not args.no_cpu and world == 1 and args.workload == "decode":
-            line["cpu_baseline"] = cpu_baseline(b, args.layers)
+            line["cpu_baseline"] = cpu_baseline(b, args.layers, oracle_ranks(args)[:7])
         if args.workload == "prefill":
             line["dtype"] = "f16 tcgen05 MMA / f32 accumulate (1-bit signs expanded to +-b, f16 activations)"
             line["us_per_layer"] = ms_step * 1e3 / nlin
