@@ -7,10 +7,11 @@
 // Per iteration: the ADMM proxies A_hat = (W' B^T + rho (A - U_A))
 // (B B^T + rho I)^-1 and B_hat = (A^T A + rho I)^-1 (A^T W' + rho (B - U_B)),
 // their SVID projections (signs and a rank-1 magnitude fit by power
-// iteration), the null-space compensation (A_target = A_hat - E_A P_B with P_B
-// the projector onto the trailing eigenvectors of B B^T carrying at most eta
-// of its spectral energy) and the closed-form scale fits gamma* / eta*
-// (Eq. gamma_solution) folded into m1 / m2, then the dual updates.
+// iteration), the null-space compensation (Sec. 3.1: the projection
+// residual A_hat - A_q is removed along P_B, the projector onto the trailing
+// eigenvectors of B B^T carrying at most eta of its spectral energy) and the
+// closed-form scale fits gamma* / eta* (Eq. gamma_solution) folded into
+// m1 / m2, then the dual updates.
 //
 // The dense linear algebra goes to the vendor libraries, loaded at run time
 // (the rest of the library does not depend on them): SGEMM (cuBLAS), the
@@ -416,7 +417,7 @@ class Run {
     if (Zq != nullptr) svid_assemble_kernel<<<blocks_for(rows * cols), kT, 0, st_>>>(Z, rows, cols, rs, cs, Zq);
   }
 
-  // NullProj (App. "Adaptive Residual-Energy Cutoff"): P = U_hat U_hat^T over
+  // Null-space projector (App. "Adaptive Residual-Energy Cutoff"): P = U_hat U_hat^T over
   // the q trailing eigenvectors of the symmetric C whose residual-energy
   // fraction is <= eta. Returns q, or -1 on a library failure.
   int64_t null_projector(const float* C, int64_t r, double eta, double eps, float* EV, float* w, float* work,
@@ -546,7 +547,7 @@ int nabf_run(const float* W, int64_t m, int64_t n, int64_t r, const float* in_sc
     run.svid(ZA, m, r, pit, rsA, csA, Aq, sigma);
     int64_t ql = 0;
     if (P.compensate) {
-      combine_kernel<<<blocks_for(mr), kT, 0, st>>>(Ah, Aq, 1.f, -1.f, mr, Et);  // E_A
+      combine_kernel<<<blocks_for(mr), kT, 0, st>>>(Ah, Aq, 1.f, -1.f, mr, Et);  // residual A_hat - A_q
       ql = run.null_projector(CB, r, P.eta, P.eps, EV, w, work, lwork, info, Pm);
       if (ql < 0) return run.fail(AF1_ERR_CUDA, "eigendecomposition of B B^T");
       if (cudaMemcpyAsync(At, Ah, (size_t)mr * 4, cudaMemcpyDeviceToDevice, st) != cudaSuccess)
@@ -572,7 +573,7 @@ int nabf_run(const float* W, int64_t m, int64_t n, int64_t r, const float* in_sc
     run.svid(ZB, r, n, pit, rsB, csB, Bq, sigma);
     int64_t qr = 0;
     if (P.compensate) {
-      combine_kernel<<<blocks_for(rn), kT, 0, st>>>(Bh, Bq, 1.f, -1.f, rn, Eb);  // E_B
+      combine_kernel<<<blocks_for(rn), kT, 0, st>>>(Bh, Bq, 1.f, -1.f, rn, Eb);  // residual B_hat - B_q
       qr = run.null_projector(CA, r, P.eta, P.eps, EV, w, work, lwork, info, Pm);
       if (qr < 0) return run.fail(AF1_ERR_CUDA, "eigendecomposition of A^T A");
       if (cudaMemcpyAsync(Bt, Bh, (size_t)rn * 4, cudaMemcpyDeviceToDevice, st) != cudaSuccess)

@@ -54,13 +54,22 @@ def slice_packed(Uw: torch.Tensor, Vw: torch.Tensor, s: torch.Tensor, r0: int, r
 
 
 def forward_rank_split(layer_g, x: torch.Tensor, y32: torch.Tensor, workspace: torch.Tensor, group=None,
-                       stream=None) -> torch.Tensor:
+                       stream=None, host_reduce: bool = False) -> torch.Tensor:
     """This GPU's partial (FP32) followed by the all-reduce (sum) over the
-    process group; y32 (tokens, m) float32 holds the layer output on return."""
+    process group; y32 (tokens, m) float32 holds the layer output on return.
+    host_reduce: all-reduce a host copy (for process groups whose backend
+    reduces host tensors, e.g. gloo) and copy the sum back."""
     import torch.distributed as dist
     if layer_g is None:
         y32.zero_()  # a GPU without ranks contributes zeros
     else:
         layer_g.forward_into(x, y32, workspace, stream=stream)
-    dist.all_reduce(y32, op=dist.ReduceOp.SUM, group=group)
+    if host_reduce:
+        if stream is not None:
+            stream.synchronize()
+        yh = y32.cpu()
+        dist.all_reduce(yh, op=dist.ReduceOp.SUM, group=group)
+        y32.copy_(yh)
+    else:
+        dist.all_reduce(y32, op=dist.ReduceOp.SUM, group=group)
     return y32

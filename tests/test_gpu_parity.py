@@ -174,6 +174,26 @@ def test_full_size_sampled_rows(P, m, n, tokens):
     layer.free()
 
 
+FULL_70B = [(8192, 8192), (1024, 8192), (28672, 8192), (8192, 28672)]
+
+
+@pytest.mark.parametrize("m,n", FULL_70B)
+@pytest.mark.parametrize("tokens", [8, 64, 512])
+def test_full_size_70b_sampled_rows(P, m, n, tokens):
+    """The 70B-class shapes of the decode/prefill crossover sweep at their
+    full size: 8 tokens (decode; the prepared tensor-core operand on the large
+    matrices) and 64 / 512 tokens (prefill; split K over a cluster at 64,
+    including the long-K split of the 8192 x 28672 first GEMM)."""
+    r = O.rank_for_budget(m, n, 1)
+    d = synth.layer_words(3000 + m // 1024 + n // 1024 + tokens, m, n, r, tokens)
+    layer = words_layer(P, d, m, n, r)
+    y = run_gpu(layer, d["x"], n)
+    rows = np.sort(synth.rng(tokens + 7).choice(m, size=128, replace=False))
+    ref = O.forward_from_packed(d["Uw"], d["Vw"], d["a"], d["s"], d["b"], d["x"], m, n, r, rows=rows)
+    assert O.rowwise_rel_err(y[:, rows], ref) <= TOL
+    layer.free()
+
+
 # ---------------------------------------------------------------------------
 # Workspace, streams, graphs and errors
 # ---------------------------------------------------------------------------

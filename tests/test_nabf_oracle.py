@@ -130,3 +130,48 @@ def test_proxies_satisfy_first_order_optimality(monkeypatch):
     # A transposed operand or a dropped regulariser fails the same check.
     wrong = np.linalg.solve(B_init @ B_init.T, (W @ B_init.T).T).T
     assert np.abs(-(W - wrong @ B_init) @ B_init.T + rho * (wrong - A_init)).max() > 1e-3
+
+
+def _admm_left(Wp, B, rho, project, dual, iters):
+    """The oracle's left-factor ADMM step (proxy, projection of proxy + dual,
+    dual step) iterated with B held fixed."""
+    m, r = Wp.shape[0], B.shape[0]
+    A = np.zeros((m, r))
+    U = np.zeros_like(A)
+    with np.errstate(all="ignore"):
+        for _ in range(iters):
+            Ah = N.left_proxy(Wp, B, A, U, rho)
+            A = project(Ah + U)
+            U = dual(U, Ah, A)
+    return A
+
+
+def test_dual_update_pinned_by_a_convex_constraint():
+    """Scaled ADMM converges to the constrained least-squares minimiser when
+    the projection is onto a convex set (App. "ADMM subproblem"). Take the
+    set of m x r matrices whose columns S are zero: its Euclidean projection
+    zeroes those columns and min |W' - A B|^2 over it has the closed form
+    A_free = W' B_free^T (B_free B_free^T)^-1, A_S = 0. B is not orthonormal,
+    so without the dual (or with its sign flipped) the iteration ends
+    elsewhere: both mutants are rejected."""
+    g = np.random.default_rng(5)
+    m, n, r = 12, 30, 6
+    Wp = g.normal(size=(m, n))
+    B = g.normal(size=(r, r)) @ g.normal(size=(r, n)) / 3  # correlated rows
+    S = [1, 4]
+    free = [j for j in range(r) if j not in S]
+
+    def project(Z):
+        Z = Z.copy()
+        Z[:, S] = 0.0
+        return Z
+
+    Bf = B[free]
+    A_star = np.zeros((m, r))
+    A_star[:, free] = Wp @ Bf.T @ np.linalg.inv(Bf @ Bf.T)
+    A = _admm_left(Wp, B, 3.0, project, N.dual_step, 400)
+    np.testing.assert_allclose(A, A_star, atol=1e-9)
+    flipped = _admm_left(Wp, B, 3.0, project, lambda U, P, F: U - P + F, 400)
+    dropped = _admm_left(Wp, B, 3.0, project, lambda U, P, F: U, 400)
+    for bad in (flipped, dropped):
+        assert not np.all(np.isfinite(bad)) or np.abs(bad - A_star).max() > 1e-2
