@@ -40,6 +40,11 @@ LAYERS = 32
 # Measured DRAM traffic of one layer's seven decode calls at one token (bytes;
 # ncu, profiles/lut_kernel_llama3_8b_b1.md): 1.026 x the algorithmic bytes.
 DECODE_TRAFFIC_B1_PER_LAYER = 28145408
+# The same for the HiSA-rank stack on the DAG schedule: DRAM bytes (read +
+# write) of one step's 84 lookup-table launches over 6 layers, divided by that
+# step's algorithmic bytes (ncu, profiles/lut_kernel_llama3_8b_hisa_b1.md);
+# a full step's traffic is this ratio times its algorithmic bytes.
+DECODE_TRAFFIC_RATIO_HISA_B1 = 170377216 / 164560648
 TC_DECODE = False  # set from --tc-decode
 
 
@@ -935,8 +940,10 @@ def main():
             # DRAM bytes (read + write) of one layer's 14 lookup-table kernels
             # at one token, from the ncu capture summarised in
             # profiles/lut_kernel_llama3_8b_b1.md, times 32 layers.
-            traffic = (DECODE_TRAFFIC_B1_PER_LAYER * args.layers
-                       if b == 1 and not TC_DECODE and args.ranks == "uniform" and args.schedule == "dag" else None)
+            traffic = None
+            if b == 1 and not TC_DECODE and args.schedule == "dag":
+                traffic = (DECODE_TRAFFIC_B1_PER_LAYER * args.layers if args.ranks == "uniform"
+                           else int(round(DECODE_TRAFFIC_RATIO_HISA_B1 * alg)))
             kname = ("af1_step_run (one persistent step_kernel launch per step)" if args.schedule == "step" else
                      "af1_linear_forward (two lookup-table kernels per call, lut_kernel<1|2>, stream_kernel<1|2> "
                      "for the largest matrices)")
@@ -945,8 +952,9 @@ def main():
                     "frac": (achieved_gbs / hbm) if hbm else None, "peak_source": "MEASURED_PEAKS.json hbm_gbs"
                     if "hbm_gbs" in peaks else "fallback 6800 GB/s",
                     "algorithmic_bytes_per_step": alg, "traffic": traffic,
-                    "traffic_source": "ncu dram__bytes_read.sum + dram__bytes_write.sum per layer x layers"
-                    if traffic else None}
+                    "traffic_source": ("ncu dram__bytes_read.sum + dram__bytes_write.sum of the step's lookup-table "
+                                       "launches, captured on a smaller stack of the same workload and scaled "
+                                       "(uniform: per layer x layers; HiSA: by algorithmic bytes)") if traffic else None}
         line = {
             "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
             "warmup": max(args.warmup, 3), "ms_per_step": ms_step, "us_per_layer": us_layer,
