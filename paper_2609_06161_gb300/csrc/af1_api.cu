@@ -111,6 +111,8 @@ int create_layer(const af1_layer_desc* d, cudaStream_t st, af1_layer** out) {
   L->p2 = af1::make_sign_matrix(d->m, d->r);
   const int64_t t1 = af1::sign_matrix_bytes(L->p1);
   const int64_t t2 = af1::sign_matrix_bytes(L->p2);
+  // Each scale array is zero-padded to a multiple of 256 bytes: the prefill
+  // kernel copies column scales in whole 64-column stages.
   const int64_t sa = align256(2 * d->m), ss = align256(2 * d->r), sb = align256(2 * d->n);
   const int64_t total = align256(t1) + align256(t2) + sa + ss + sb;
   e = cudaMalloc(&L->alloc, (size_t)total);

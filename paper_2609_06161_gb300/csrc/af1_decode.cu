@@ -976,6 +976,12 @@ Workspace plan_workspace(const af1_layer& L, int64_t tokens, bool prep, bool swi
   if (tokens > kMaxPassTokens) {
     const int64_t t = tokens < kPrefillPassTokens ? tokens : kPrefillPassTokens;
     off += align256(t * prefill_h_ld(L) * 2);
+    if (prep) {
+      w.pbuf = off;
+      off += align256(prefill_part_bytes(L, tokens));
+      w.pcnt = off;
+      off += align256(prefill_count_bytes(L, tokens));
+    }
   }
   if (swiglu) {
     const int64_t t = tokens < kPrefillPassTokens ? tokens : kPrefillPassTokens;
@@ -1043,13 +1049,15 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
   if (tokens > kMaxPassTokens) {
     // Prefill: two tensor-core GEMMs per pass (af1_prefill.cu); the SwiGLU
     // input is formed first, one pass of tokens at a time.
-    if (x2 == nullptr) return launch_prefill(L, x, ldx, tokens, y, ldy, y_dtype, wsb + W.hbuf, stat, st);
+    float* part = W.pbuf != 0 ? reinterpret_cast<float*>(wsb + W.pbuf) : nullptr;
+    unsigned* count = W.pcnt != 0 ? reinterpret_cast<unsigned*>(wsb + W.pcnt) : nullptr;
+    if (x2 == nullptr) return launch_prefill(L, x, ldx, tokens, y, ldy, y_dtype, wsb + W.hbuf, part, count, stat, st);
     for (int64_t t0 = 0; t0 < tokens; t0 += kPrefillPassTokens) {
       const int64_t T = (tokens - t0) < kPrefillPassTokens ? (tokens - t0) : kPrefillPassTokens;
       cudaError_t e = launch_swiglu(gx + t0 * ldx, ux + t0 * ldx, ldx, T, L.n, hx, ldh, st);
       if (e == cudaSuccess)
         e = launch_prefill(L, hx, ldh, T, static_cast<uint8_t*>(y) + t0 * ldy * ysize, ldy, y_dtype, wsb + W.hbuf,
-                           stat, st);
+                           part, count, stat, st);
       if (e != cudaSuccess) return e;
     }
     return cudaSuccess;

@@ -43,15 +43,22 @@ struct Workspace {
   int64_t bstats = 0;  // float2 [16 slices][16 tokens] of the prepared B (0: none)
   int64_t hbuf = 0;    // FP16 [min(tokens, kPrefillPassTokens)][prefill_h_ld]: H (prefill)
   int64_t hx = 0;      // FP16 [min(tokens, kPrefillPassTokens)][swiglu_ld]: SwiGLU input h (0: none)
+  int64_t pbuf = 0;    // FP32 partial tiles of the prefill GEMMs (0: none; one tile per CTA then)
+  int64_t pcnt = 0;    // uint32 per prefill tile: contributors arrived (zero between calls)
   int64_t total = 0;
 };
-// prep = false leaves out the prepared-B region (and so never uses it);
+// prep = false leaves out the prepared-B region and the prefill's partial
+// tiles (and so never uses them: the prefill then runs one CTA per tile);
 // swiglu adds the region the SwiGLU entry point forms h in for the kernels
 // that cannot form it while staging (tensor-core decode and prefill).
 Workspace plan_workspace(const af1_layer& L, int64_t tokens, bool prep = true, bool swiglu = false);
 // Row stride (elements) of the SwiGLU input h in the workspace.
 int64_t swiglu_ld(const af1_layer& L);
 int64_t prefill_h_ld(const af1_layer& L);
+// Bytes of the prefill's partial tiles and tile counters for a call of
+// `tokens` (> kMaxPassTokens) tokens.
+int64_t prefill_part_bytes(const af1_layer& L, int64_t tokens);
+int64_t prefill_count_bytes(const af1_layer& L, int64_t tokens);
 int64_t decode_ldz(const af1_layer& L);
 
 // Kernel launchers (stream-ordered, asynchronous). Return cudaSuccess or the
@@ -129,8 +136,10 @@ StreamPlan plan_stream(int phase, const SignMatrix& sm, int T, int num_sms, int 
 cudaError_t launch_stream(int phase, const LutProblem& prob, int tokens, int ydtype, const StreamPlan& p,
                           unsigned* status, cudaStream_t st);
 
+// part == nullptr: one CTA per output tile (no partial tiles).
 cudaError_t launch_prefill(const af1_layer& L, const void* x, int64_t ldx, int64_t tokens, void* y, int64_t ldy,
-                           int y_dtype, uint8_t* h_buf, unsigned* status, cudaStream_t st);
+                           int y_dtype, uint8_t* h_buf, float* part, unsigned* count, unsigned* status,
+                           cudaStream_t st);
 // status: the status word to report to (nullptr: the workspace's own).
 // x2 != nullptr: the SwiGLU entry point (x is g, x2 is u; the workspace was
 // planned with swiglu = true).

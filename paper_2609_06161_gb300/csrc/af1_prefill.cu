@@ -5,29 +5,56 @@
 //   GEMM1: H[t][k] = s_k * sum_j B[k][j] * (b_j x[t][j])    (B = V^T, r x n)
 //   GEMM2: y[t][i] = a_i * sum_k U[i][k] * H[t][k]          (U, m x r)
 //
-// A CTA computes D = A . B^T for 128 features x BN tokens (BN = 64, 128 or
-// 256), D in tensor memory (128 lanes x BN FP32 columns). Per K-stage of 64:
-//   * one thread of warp 0 loads the BN x 64 FP16 activation tile (B) with
-//     one TMA copy (cp.async.bulk.tensor, 128-byte swizzle, zero fill past
-//     the tokens / columns): the K-major layout the MMA descriptor describes;
-//   * warps 4-7 (one feature row per thread = tensor-memory lane) expand the
-//     packed signs of the 128 x 64 weight tile into FP16 (+-b_j for GEMM1,
-//     +-1 for GEMM2: exact) and store them into a ring of A buffers in
-//     tensor memory (tcgen05.st, 32 columns per stage); each thread loads
-//     the next stage's sign words (and column scales) while it expands the
-//     current one. A in tensor memory leaves shared-memory bandwidth to B
-//     (measured: 848 vs 735 TFLOP/s with A in shared memory);
-//   * one thread of warp 1 issues four tcgen05.mma.kind::f16 (K = 16 each,
-//     N = BN, A from tensor memory, B from shared memory) and commits them to
-//     the stage's "empty" mbarrier.
-// Warps 4-7 then read D back with tcgen05.ld (warp w owns TMEM lanes
-// 32 (w % 4) .. +31), apply the per-feature scale and store FP16 / FP32.
+// Output tiles are 128 features x BN tokens (BN = 16, 32, 64, 128 or 256),
+// with K cut into stages of 64. The kernel is persistent and stream-K: the grid
+// (at most one CTA per SM) splits the (tile, K-stage) iterations into equal
+// contiguous ranges, so a CTA runs a few whole tiles plus, at either end of
+// its range, part of a tile shared with its neighbour. A shared tile's
+// contributors store FP32 partial tiles in the workspace and count
+// themselves on the tile's counter; the last to arrive sums the partials in
+// a fixed order (so results do not depend on timing), applies the feature
+// scale, stores the output and clears the counter. No CTA waits for
+// another. Without room for the partials (the built-in-scratch entry) the
+// grid is one CTA per tile.
+//
+// Roles of the 12 warps of a CTA, over the CTA's stages in order:
+//   * warp 0, one thread: copies each stage's packed signs (128 rows x 2
+//     words: 1 KB contiguous in the row-block layout) and, for GEMM1, its 64
+//     column scales into a ring of 14 small slots (cp.async.bulk), up to 14
+//     stages ahead and independent of the MMA (with the signs loaded by the
+//     expanders one stage ahead, each stage waited about 1,500 cycles on the
+//     load against 600 of MMA work); then the BN x 64 FP16 activation tile
+//     (B) of the stage by TMA (cp.async.bulk.tensor, 128-byte swizzle, zero
+//     fill past the tokens / columns) into a ring of 8 stages (6 for BN =
+//     256);
+//   * warps 4-7 expand the signs into FP16 (+-b_j for GEMM1, +-1 for GEMM2:
+//     exact) and store them into a ring of A buffers (one per stage) in
+//     tensor memory
+//     (tcgen05.st; warp w writes rows 32 (w % 4) .. +31, one row per thread
+//     = tensor-memory lane; eight warps with half a stage each were slower);
+//     A in tensor memory leaves shared-memory bandwidth to B;
+//   * warp 1, one thread: four tcgen05.mma.kind::f16 per stage (K = 16,
+//     N = BN, A from tensor memory, B from shared memory) into an
+//     accumulator (D, FP32, BN columns). Tiles of up to 128 tokens alternate
+//     between two accumulators, so the epilogue of one tile overlaps the
+//     MMAs of the next; tiles of 256 have one (two would leave no tensor
+//     memory for A), and the MMAs of the next tile wait for its read-back.
+//     Measured: this one thread needs about 175 cycles per MMA whatever N,
+//     so N = 128 tiles ran at half the rate of N = 256;
+//   * warps 8-11 read an accumulator back (tcgen05.ld), apply the feature
+//     scale and stage 16 tokens at a time in shared memory, which one thread
+//     writes out with a TMA store (or a bulk copy for a partial tile) while
+//     the warps go on to the next 16 (stores from the warps themselves were
+//     latency-bound in the store queue, and the MMA waits for this read-back
+//     when a tile has one accumulator).
 // All mbarrier waits are bounded; a wait that gives up sets the status word.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
+
+#include <cstring>
 
 #include "af1_internal.h"
 #include "af1_layout.h"
@@ -36,47 +63,102 @@
 namespace af1 {
 namespace {
 
-constexpr int BM = 128;  // features per CTA (MMA M, TMEM lanes)
-constexpr int BK = 64;   // K per stage: one 128-byte swizzle row of FP16
-constexpr int kMaxStages = 6;
-constexpr int kThreads = 256;
+constexpr int BM = 128;      // features per tile (MMA M, tensor-memory lanes)
+constexpr int BOX = 64;      // K per activation box: one 128-byte swizzle row of FP16
+constexpr int kThreads = 512;
+constexpr int kTmemCols = 512;  // accumulators (2 x BN, or 1 x 256) + one A buffer per stage
+constexpr int kExpandWarps = 8;  // warps 4..11
+constexpr int kEpiWarp0 = 12;    // warps 12..15
+constexpr int kMaxStages = 8;
+constexpr int kMaxWSlots = 14;
 
+// K per stage: 128 for tiles of 256 tokens, 64 otherwise. One thread issues
+// the MMAs and every operation of its loop besides them leaves the tensor
+// pipe idle (measured: 134 cycles per MMA back to back, N = 128 or 256; a
+// commit adds 77 and a completed mbarrier check 67), so long stages and one
+// barrier per stage keep it busy.
+template <int BN>
+__host__ __device__ constexpr int bk() {
+  return BN == 256 ? 128 : 64;
+}
+__host__ __device__ constexpr int bk_of(int bn) { return bn == 256 ? 128 : 64; }
 template <int BN>
 __host__ __device__ constexpr int tile_b_bytes() {
-  return BN * BK * 2;
+  return BN * bk<BN>() * 2;
 }
-// Pipeline depth: 6 stages for tiles of 256 tokens (192 KB of activation
-// tiles; tensor memory holds D in 256 columns plus an A ring of 6 x 32), 4
-// for the smaller tiles.
+// Stages of the activation ring (shared memory) and of the A ring (tensor
+// memory, bk / 2 columns each), and accumulators.
 template <int BN>
 __host__ __device__ constexpr int stages() {
-  return BN == 256 ? 6 : 4;
+  return BN == 256 ? 3 : 8;
+}
+template <int BN>
+__host__ __device__ constexpr int accumulators() {
+  return BN == 256 ? 1 : 2;
+}
+static_assert(accumulators<256>() * 256 + stages<256>() * bk<256>() / 2 <= kTmemCols, "tensor memory");
+static_assert(accumulators<128>() * 128 + stages<128>() * bk<128>() / 2 <= kTmemCols, "tensor memory");
+// Sign ring: slots of one stage's packed words (bk / 32 words x 128 rows)
+// followed by its bk FP16 column scales (GEMM1).
+template <int BN>
+__host__ __device__ constexpr int wsign_bytes() {
+  return bk<BN>() / 32 * kBlockRows * 4;
+}
+template <int BN>
+__host__ __device__ constexpr int wslot_bytes() {
+  return wsign_bytes<BN>() + bk<BN>() * 2;
+}
+template <int BN>
+__host__ __device__ constexpr int wslots() {
+  return BN == 256 ? 6 : 14;
+}
+// Stages of K per CTA below which the stream-K grid is made smaller (more
+// CTAs per tile means more partial tiles for its last contributor to sum).
+constexpr int min_stages_per_cta(int bn) { return bn == 256 ? 8 : bn <= 32 ? 8 : 16; }
+// At least 116 KB so that two CTAs never share an SM (each allocates all of
+// its tensor memory).
+// Epilogue staging: two buffers of one 16-token x 128-row chunk (FP32 at
+// most), [token][row].
+constexpr int kEpiStageBytes = 16 * 128 * 4;
+template <int BN>
+__host__ __device__ constexpr int smem_used() {
+  return stages<BN>() * tile_b_bytes<BN>() + wslots<BN>() * wslot_bytes<BN>() + 2 * kEpiStageBytes +
+         1024 /* barriers */ + 1024 /* base alignment */;
 }
 template <int BN>
 __host__ __device__ constexpr int smem_bytes() {
-  return stages<BN>() * tile_b_bytes<BN>() + 1024 /* barriers */ + 1024 /* base alignment */;
+  return smem_used<BN>() < 116 * 1024 ? 116 * 1024 : smem_used<BN>();
 }
+static_assert(smem_used<256>() <= 227 * 1024, "shared memory");
 
 struct PrefillArgs {
   const uint32_t* signs;  // packed signs, af1_layout.h row-block layout
   SignMatrix sm;          // R = features, C = K
   int tokens;
-  const __half* colscale;  // GEMM1: b (length C); GEMM2: nullptr (+-1)
+  const __half* colscale;  // GEMM1: b (length C, zero-padded to 128-column stages); GEMM2: nullptr (+-1)
   const __half* rowscale;  // GEMM1: s (length R); GEMM2: a
   void* out;               // GEMM1: H [tokens][ld_out] FP16; GEMM2: y
   int64_t ld_out;
   int out_f32;
+  int out_vec;             // out and ld_out allow 16-byte stores
+  float* part;             // partial tiles: 2 slots per CTA of 128 rows x BN FP32 (nullptr: one tile per CTA)
+  unsigned* count;         // two counters per tile: tickets taken, partials stored (zero between calls)
   unsigned* status;
   long long wait_cycles;  // budget of every bounded wait (clock64 cycles)
 };
 
 struct __align__(8) PrefillBarriers {
-  uint64_t full_a[kMaxStages];  // the 4 expander warps have stored the stage's A
-  uint64_t full_b[kMaxStages];  // the TMA tile has landed
-  uint64_t empty[kMaxStages];   // the stage's MMAs are done
-  uint64_t done;
+  uint64_t full[kMaxStages];     // the stage's activation tile has landed and its A is stored
+  uint64_t empty[kMaxStages];    // the stage's MMAs are done
+  uint64_t full_w[kMaxWSlots];   // a stage's signs (and column scales) have landed
+  uint64_t empty_w[kMaxWSlots];  // the expander warps have read them
+  uint64_t dfull[2];           // accumulator d holds a finished tile (or segment)
+  uint64_t dempty[2];          // the epilogue has read accumulator d
+  uint32_t issued_b, issued_w; // copies issued (drained when a wait gave up)
+  uint64_t red;                // partial tiles copied in for a reduction
   uint32_t tmem_addr;
   uint32_t err;
+  uint32_t last;               // epilogue: this CTA completes the shared tile
 };
 
 __device__ __forceinline__ void tmem_ld16(uint32_t addr, uint32_t (&r)[16]) {
@@ -86,13 +168,6 @@ __device__ __forceinline__ void tmem_ld16(uint32_t addr, uint32_t (&r)[16]) {
         "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
       : "r"(addr));
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-}
-
-// Cluster helper for the split-K reduction.
-__device__ __forceinline__ void st_cluster_f32(float* local, uint32_t rank, float v) {
-  uint32_t remote;
-  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(local)), "r"(rank));
-  asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(remote), "f"(v) : "memory");
 }
 
 // 2-D TMA load of the box at (x = column, y = token) into shared memory,
@@ -127,12 +202,6 @@ __device__ __forceinline__ void mma_f16_ts(uint32_t d_tmem, uint32_t a_tmem, uin
       "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate ? 1u : 0u)
       : "memory");
 }
-// Tensor-memory columns: D (BN) then the A ring (stages x 32), rounded up
-// to a power of two.
-template <int BN>
-__host__ __device__ constexpr uint32_t tmem_cols() {
-  return (BN + stages<BN>() * 32) <= 256 ? 256u : 512u;
-}
 __device__ __forceinline__ void mma_commit(uint64_t* bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
                : "memory");
@@ -145,159 +214,308 @@ __device__ __forceinline__ uint32_t signed_pair(uint32_t pair_bytes, int p, uint
   return v ^ (~sh & 0x80008000u);
 }
 
-// Column scales of stage columns kc .. kc + 63 as 8 groups of 8 FP16
-// values, 0 beyond C.
-__device__ __forceinline__ void load_colscale(const __half* cs, int64_t kc, int64_t C, uint4 (&out)[8]) {
+// TMA store of the [16 tokens][128 rows] box at (x = row, y = token) from
+// shared memory, and a plain bulk store; both in the thread's bulk group.
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, const void* src, int x, int y) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(x), "r"(y), "r"(smem_u32(src))
+               : "memory");
+}
+__device__ __forceinline__ void bulk_s2g(void* dst, const void* src, uint32_t bytes) {
+  asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(dst), "r"(smem_u32(src)),
+               "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// At most one group still reading its shared-memory source.
+__device__ __forceinline__ void bulk_wait_read1() { asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory"); }
+// Every group complete (its writes performed).
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+__device__ __forceinline__ void tmem_ld16_nowait(uint32_t addr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+        "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(addr));
+}
+__device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+
+// A warp's 32-row x 16-token chunk, held one row per lane (v[q] = token
+// q), to dst[token][row] (leading dimension ld): through a 16 x 32 staging
+// tile in shared memory, so that each lane stores 16 contiguous bytes (one
+// 2-byte store per lane and token was latency-bound in the store queue:
+// about 70 cycles per store instruction). Rows row0 .. +31 (those below
+// nrow), tokens tok0 .. +15 (those below ntok).
+template <typename T>
+__device__ __forceinline__ void store_chunk(const float (&v)[16], T* stage, T* dst, int64_t ld, int64_t row0,
+                                            int64_t nrow, int64_t tok0, int64_t ntok, bool vec, int lane) {
 #pragma unroll
-  for (int j = 0; j < 8; ++j) {
-    const int64_t k = kc + 8 * j;
-    if (k + 7 < C) {
-      out[j] = __ldg(reinterpret_cast<const uint4*>(cs + k));
-    } else {
-      const uint16_t* c16 = reinterpret_cast<const uint16_t*>(cs);
-      uint32_t e[8];
+  for (int q = 0; q < 16; ++q) {
+    if constexpr (sizeof(T) == 2)
+      stage[q * 32 + lane] = __float2half_rn(v[q]);
+    else
+      stage[q * 32 + lane] = v[q];
+  }
+  __syncwarp();
+  constexpr int VE = 16 / (int)sizeof(T);  // elements per 16-byte vector
+  constexpr int VPR = 32 / VE;              // vectors per token
 #pragma unroll
-      for (int q = 0; q < 8; ++q) e[q] = k + q < C ? c16[k + q] : 0u;
-      out[j] = make_uint4(e[0] | (e[1] << 16), e[2] | (e[3] << 16), e[4] | (e[5] << 16), e[6] | (e[7] << 16));
+  for (int vi = lane; vi < 16 * VPR; vi += 32) {
+    const int tk = vi / VPR, cg = vi % VPR;
+    const int64_t tok = tok0 + tk, row = row0 + cg * VE;
+    if (tok < ntok) {
+      const T* src = stage + tk * 32 + cg * VE;
+      T* p = dst + tok * ld + row;
+      if (vec && row + VE <= nrow) {
+        *reinterpret_cast<uint4*>(p) = *reinterpret_cast<const uint4*>(src);
+      } else {
+        for (int e = 0; e < VE; ++e)
+          if (row + e < nrow) p[e] = src[e];
+      }
     }
   }
+  __syncwarp();
 }
 
-// KS > 1: split-K over a cluster of KS CTAs along z. CTA ks runs the stages
-// [ks spk, (ks + 1) spk) and the partial tiles are summed through
-// distributed shared memory (each CTA finalises 128 / KS rows, summing the
-// KS partials in a fixed order), reusing the activation stages as the
-// receive buffer once every MMA of the cluster is done.
-template <bool GEMM1, int BN, int KS>
+// The CTA that runs iteration i of I split over G CTAs: CTA c runs
+// [floor(c I / G), floor((c + 1) I / G)).
+__device__ __forceinline__ int cta_of(int64_t i, int64_t I, int G) { return (int)(((i + 1) * G - 1) / I); }
+__device__ __forceinline__ int64_t range_start(int c, int64_t I, int G) { return (int64_t)c * I / G; }
+
+template <bool GEMM1, int BN>
 __global__ void __launch_bounds__(kThreads, 1)
-    prefill_kernel(const __grid_constant__ CUtensorMap act_map, const PrefillArgs a) {
+    prefill_kernel(const __grid_constant__ CUtensorMap act_map, const __grid_constant__ CUtensorMap out_map,
+                   const PrefillArgs a) {
+  constexpr int BK = bk<BN>();
   constexpr int kTileB = tile_b_bytes<BN>();
-  constexpr int STAGES = stages<BN>();
+  constexpr int kBoxBytes = BN * BOX * 2;
+  constexpr int kStages = stages<BN>();
+  constexpr int ND = accumulators<BN>();
+  constexpr int kWSlots = wslots<BN>();
+  constexpr int kWSignBytes = wsign_bytes<BN>();
+  constexpr int kWSlotBytes = wslot_bytes<BN>();
+  constexpr int kACols = BK / 2;       // tensor-memory columns of one stage's A
+  constexpr int kWPS = BK / 32;        // sign words per row and stage
+  constexpr int kWPW = kWPS / 2;       // ... per expander warp (two warps per row)
   extern __shared__ uint8_t smem_raw[];
   // 1024-byte alignment for the swizzled operand tiles.
   uint8_t* smem = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   uint8_t* tileB = smem;
-  PrefillBarriers& bar = *reinterpret_cast<PrefillBarriers*>(smem + STAGES * kTileB);
+  uint8_t* wring = smem + kStages * kTileB;
+  uint8_t* estage = wring + kWSlots * kWSlotBytes;
+  PrefillBarriers& bar = *reinterpret_cast<PrefillBarriers*>(estage + 2 * kEpiStageBytes);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const SignMatrix& tm = a.sm;
-  const int f0 = blockIdx.x * BM;  // first feature (row of the sign matrix)
-  const int t0 = blockIdx.y * BN;  // first token
-  const int nk_all = (int)((tm.C + BK - 1) / BK);
-  const int ks = KS > 1 ? (int)blockIdx.z : 0;
-  const int spk = (nk_all + KS - 1) / KS;  // stages per CTA (>= 1 for every ks, by the host plan)
-  const int it0 = ks * spk;
-  const int nk = min(nk_all, it0 + spk) - it0;  // this CTA's stages: it0 .. it0 + nk - 1
+  const int RB = tm.RB;
+  const int nk = (int)((tm.C + BK - 1) / BK);        // K stages per tile
+  const int NT = (a.tokens + BN - 1) / BN;           // token tiles
+  const int64_t I = (int64_t)RB * NT * nk;           // iterations: tile t = tt * RB + rb, stage k
+  const int G = (int)gridDim.x;
+  const int c = (int)blockIdx.x;
+  const int64_t i0 = range_start(c, I, G);
+  const int n = (int)(range_start(c + 1, I, G) - i0);  // this CTA's stages
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < STAGES; ++s) {
-      mbar_init(&bar.full_a[s], 4);
-      mbar_init(&bar.full_b[s], 1);
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&bar.full[s], 1 + kExpandWarps);  // the producer's expect_tx arrival + one per expander warp
       mbar_init(&bar.empty[s], 1);
     }
-    mbar_init(&bar.done, 1);
+    for (int s = 0; s < kWSlots; ++s) {
+      mbar_init(&bar.full_w[s], 1);
+      mbar_init(&bar.empty_w[s], kExpandWarps);
+    }
+    for (int d = 0; d < ND; ++d) {
+      mbar_init(&bar.dfull[d], 1);
+      mbar_init(&bar.dempty[d], 4);
+    }
+    mbar_init(&bar.red, 1);
     bar.err = 0;
+    bar.issued_b = 0;
+    bar.issued_w = 0;
+    bar.last = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&act_map)) : "memory");
   }
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&bar.tmem_addr)),
-                 "r"(tmem_cols<BN>())
+                 "r"(kTmemCols)
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
   __syncthreads();
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-  const uint32_t tmem = bar.tmem_addr;
+  const uint32_t tmem = bar.tmem_addr;  // accumulators at columns 0 (and BN), A buffers from ND BN
 
   if (warp == 0) {
-    // ---- activation producer: one TMA copy per stage ---------------------
+    // ---- producer -----------------------------------------------------------
+    // Stage j of this CTA is iteration i0 + j: tile t = (i0 + j) / nk, K stage
+    // k = (i0 + j) % nk. Its signs are words 2k and 2k + 1 of the 128 rows of
+    // row block t % RB (256 consecutive words); its column scales lie inside
+    // the layer's 256-byte-padded, zero-filled scale array.
+    // Two cursors over the stages (signs run ahead of the activation tiles),
+    // each kept as (row block, token tile, K stage): no division per stage
+    // in this single thread's loop (three 64-bit divisions per stage made
+    // it the bottleneck).
+    struct Cursor {
+      int rb, tt, k;
+    };
+    const int t_first = (int)(i0 / nk);
+    const Cursor c0 = {t_first % RB, t_first / RB, (int)(i0 - (int64_t)t_first * nk)};
+    auto advance = [&](Cursor& cu) {
+      if (++cu.k == nk) {
+        cu.k = 0;
+        if (++cu.rb == RB) {
+          cu.rb = 0;
+          ++cu.tt;
+        }
+      }
+    };
+    Cursor cw = c0, cb = c0;
+    int wi = 0;  // next stage whose signs are copied (at cursor cw)
+    auto issue_w = [&](int j) {
+      const int ws = j % kWSlots;
+      if (j >= kWSlots) mbar_wait(&bar.empty_w[ws], ((j / kWSlots) & 1) ^ 1, &bar.err, a.wait_cycles);
+      uint8_t* dst = wring + ws * kWSlotBytes;
+      mbar_expect_tx(&bar.full_w[ws], (uint32_t)(GEMM1 ? kWSlotBytes : kWSignBytes));
+      bulk_g2s(dst, a.signs + ((int64_t)cw.rb * tm.NCH * kChunkWords + (int64_t)kWPS * cw.k) * kBlockRows,
+               (uint32_t)kWSignBytes, &bar.full_w[ws]);
+      if (GEMM1) bulk_g2s(dst + kWSignBytes, a.colscale + (int64_t)cw.k * BK, (uint32_t)(BK * 2), &bar.full_w[ws]);
+      advance(cw);
+    };
+    if (lane == 0) {
+      // The signs are constants: copy the first ones before the dependency wait.
+      for (; wi < n && wi < kWSlots; ++wi) issue_w(wi);
+    }
     griddep_wait();  // the activations are written by the previous kernel
     if (lane == 0) {
-      for (int it = 0; it < nk; ++it) {
-        const int s = it % STAGES;
-        if (it >= STAGES) mbar_wait(&bar.empty[s], ((it / STAGES) & 1) ^ 1, &bar.err, a.wait_cycles);
-        mbar_expect_tx(&bar.full_b[s], (uint32_t)kTileB);
-        tma_load_2d(tileB + s * kTileB, &act_map, (it0 + it) * BK, t0, &bar.full_b[s]);
+      for (int j = 0; j < n; ++j) {
+        for (; wi < n && wi < j + kWSlots; ++wi) issue_w(wi);
+        const int s = j % kStages;
+        if (j >= kStages) mbar_wait(&bar.empty[s], ((j / kStages) & 1) ^ 1, &bar.err, a.wait_cycles);
+        mbar_expect_tx(&bar.full[s], (uint32_t)kTileB);
+#pragma unroll
+        for (int bx = 0; bx < BK / BOX; ++bx)
+          tma_load_2d(tileB + s * kTileB + bx * kBoxBytes, &act_map, cb.k * BK + bx * BOX, cb.tt * BN, &bar.full[s]);
+        advance(cb);
       }
+      bar.issued_b = (uint32_t)n;
+      bar.issued_w = (uint32_t)wi;
     }
     __syncwarp();
   } else if (warp == 1) {
-    // ---- MMA issuer ---------------------------------------------------------
+    // ---- MMA issuer -----------------------------------------------------------
     if (lane == 0) {
+      // The barriers of stage j + 1 are checked before the last MMA of
+      // stage j is issued, while three MMAs are queued (checked after it,
+      // the pipe drained during the two checks: about 200 cycles per stage).
       const uint32_t b0 = smem_u32(tileB);
-      for (int it = 0; it < nk; ++it) {
-        const int s = it % STAGES;
-        const uint32_t ph = (it / STAGES) & 1;
-        mbar_wait(&bar.full_a[s], ph, &bar.err, a.wait_cycles);
-        mbar_wait(&bar.full_b[s], ph, &bar.err, a.wait_cycles);
-        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+      int u = 0;  // segment (tile or part of one) of this CTA
+      uint32_t d_tmem = tmem;
+      bool first = true;
+      int k = (int)(i0 % nk);  // K stage of stage j, kept incrementally
+      auto wait_stage = [&](int j) { mbar_wait(&bar.full[j % kStages], (j / kStages) & 1, &bar.err, a.wait_cycles); };
+      if (n > 0) wait_stage(0);
+      asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+      for (int j = 0; j < n; ++j) {
+        const int s = j % kStages;
+        const bool seg_end = j == n - 1 || k == nk - 1;
+        // MMA kk: K 16 kk .. + 15 of the stage = tensor-memory columns 8 kk ..
+        // of its A buffer and, of its activation tile, box kk / 4, 32-byte
+        // step kk % 4 of the swizzled rows.
 #pragma unroll
-        for (int kk = 0; kk < BK / 16; ++kk) {
-          mma_f16_ts<BN>(tmem, tmem + (uint32_t)(BN + s * 32 + kk * 8), smem_desc(b0 + s * kTileB + kk * 32),
-                         it > 0 || kk > 0);
+        for (int kk = 0; kk < BK / 16 - 1; ++kk) {
+          mma_f16_ts<BN>(d_tmem, tmem + (uint32_t)(ND * BN + s * kACols + kk * 8),
+                         smem_desc(b0 + s * kTileB + (kk / 4) * kBoxBytes + (kk % 4) * 32), !(first && kk == 0));
         }
+        // Stage j + 1: its accumulator must be free (with one accumulator
+        // that needs this segment's epilogue, so it waits after the commit).
+        const bool ahead = j + 1 < n && !(seg_end && ND == 1);
+        if (ahead) {
+          if (seg_end && u + 1 >= ND)
+            mbar_wait(&bar.dempty[(u + 1) % ND], (((u + 1) / ND) & 1) ^ 1, &bar.err, a.wait_cycles);
+          wait_stage(j + 1);
+        }
+        constexpr int kl = BK / 16 - 1;
+        mma_f16_ts<BN>(d_tmem, tmem + (uint32_t)(ND * BN + s * kACols + kl * 8),
+                       smem_desc(b0 + s * kTileB + (kl / 4) * kBoxBytes + (kl % 4) * 32), true);
         mma_commit(&bar.empty[s]);
+        if (seg_end) mma_commit(&bar.dfull[u % ND]);
+        if (j + 1 < n) {
+          if (seg_end) {
+            ++u;
+            d_tmem = tmem + (uint32_t)((u % ND) * BN);
+            first = true;
+            if (!ahead) {
+              if (u >= ND) mbar_wait(&bar.dempty[u % ND], ((u / ND) & 1) ^ 1, &bar.err, a.wait_cycles);
+              wait_stage(j + 1);
+            }
+          } else {
+            first = false;
+          }
+          asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        }
+        if (++k == nk) k = 0;
       }
-      mma_commit(&bar.done);
     }
     __syncwarp();
-  } else if (warp >= 4) {
-    // ---- weight expansion: one feature row per thread --------------------
-    const int R = threadIdx.x - 128;  // 0..127 = TMEM lane of this thread
-    const int64_t frow = f0 + R;
-    const bool row_ok = frow < tm.R;
-    // Words of this row: index (rb * 4 NCH + kw) * 128 + R (rows past R are
-    // zero words of the padded block). Stage `it` uses words 2 it and
-    // 2 it + 1; the next stage's words are loaded while the current stage is
-    // expanded.
-    const uint32_t* rowp =
-        a.signs + (int64_t)blockIdx.x * tm.NCH * kChunkWords * kBlockRows + R + (int64_t)(2 * it0) * kBlockRows;
-    uint32_t w0 = __ldg(rowp), w1 = __ldg(rowp + kBlockRows);
-    uint4 cs[8];
-    if (GEMM1) load_colscale(a.colscale, (int64_t)it0 * BK, tm.C, cs);
-    for (int it = 0; it < nk; ++it) {
-      const int s = it % STAGES;
-      uint32_t n0 = 0u, n1 = 0u;
-      uint4 ncs[8];
-      if (it + 1 < nk) {
-        n0 = __ldg(rowp + (int64_t)(2 * it + 2) * kBlockRows);
-        n1 = __ldg(rowp + (int64_t)(2 * it + 3) * kBlockRows);
-        if (GEMM1) load_colscale(a.colscale, (int64_t)(it0 + it + 1) * BK, tm.C, ncs);
-      }
-      uint32_t av[32];
+  } else if (warp >= 4 && warp < kEpiWarp0) {
+    // ---- weight expansion: warp w, rows 32 (w % 4) + lane, half h = (w - 4)
+    //      / 4 of the stage: its words h kWPW .. + kWPW - 1 (32 K each) ------
+    const int q = warp & 3, h = (warp - 4) >> 2;
+    const int R = q * 32 + lane;  // TMEM lane = row of the block
+    const uint32_t lane_base = (uint32_t)(q * 32) << 16;
+    for (int j = 0; j < n; ++j) {
+      const int s = j % kStages;
+      const int ws = j % kWSlots;
+      mbar_wait(&bar.full_w[ws], (j / kWSlots) & 1, &bar.err, a.wait_cycles);
+      const uint32_t* wslot = reinterpret_cast<const uint32_t*>(wring + ws * kWSlotBytes);
+      uint32_t av[16 * kWPW];
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        // Stage columns 8j .. 8j+7 (tensor-memory columns 4j .. 4j+3, two
-        // FP16 values each) = columns 4p + e of word j / 4 with p = 2 (j % 4)
-        // (first 4) and p + 1 (last 4).
-        const uint32_t wd = (j < 4) ? w0 : w1;
-        const int p = 2 * (j & 3);
-        const uint32_t b01 = __byte_perm(wd, 0u, 0x1404);  // bytes 0,1 -> bytes 1,3 (e = 0, 1)
-        const uint32_t b23 = __byte_perm(wd, 0u, 0x3424);  // bytes 2,3 -> bytes 1,3 (e = 2, 3)
-        uint4 sv = make_uint4(0x3C003C00u, 0x3C003C00u, 0x3C003C00u, 0x3C003C00u);  // +-1 for GEMM2
-        if (GEMM1) sv = cs[j];
-        av[4 * j + 0] = signed_pair(b01, p, sv.x);
-        av[4 * j + 1] = signed_pair(b23, p, sv.y);
-        av[4 * j + 2] = signed_pair(b01, p + 1, sv.z);
-        av[4 * j + 3] = signed_pair(b23, p + 1, sv.w);
+      for (int ww = 0; ww < kWPW; ++ww) {
+        const int word = h * kWPW + ww;  // word of the stage: K 32 word .. + 31
+        const uint32_t wd = wslot[word * kBlockRows + R];
+        uint4 cs[4];
+        if (GEMM1) {
+#pragma unroll
+          for (int jj = 0; jj < 4; ++jj) cs[jj] = reinterpret_cast<const uint4*>(wslot + kWPS * kBlockRows)[4 * word + jj];
+        }
+#pragma unroll
+        for (int jj = 0; jj < 4; ++jj) {
+          // K 32 word + 8 jj .. + 7 (tensor-memory columns 16 word + 4 jj ..
+          // + 3, two FP16 values each) = columns 4p + e of the word with
+          // p = 2 jj (first 4) and p + 1 (last 4).
+          const int p = 2 * jj;
+          const uint32_t b01 = __byte_perm(wd, 0u, 0x1404);  // bytes 0,1 -> bytes 1,3 (e = 0, 1)
+          const uint32_t b23 = __byte_perm(wd, 0u, 0x3424);  // bytes 2,3 -> bytes 1,3 (e = 2, 3)
+          uint4 sv = make_uint4(0x3C003C00u, 0x3C003C00u, 0x3C003C00u, 0x3C003C00u);  // +-1 for GEMM2
+          if (GEMM1) sv = cs[jj];
+          av[16 * ww + 4 * jj + 0] = signed_pair(b01, p, sv.x);
+          av[16 * ww + 4 * jj + 1] = signed_pair(b23, p, sv.y);
+          av[16 * ww + 4 * jj + 2] = signed_pair(b01, p + 1, sv.z);
+          av[16 * ww + 4 * jj + 3] = signed_pair(b23, p + 1, sv.w);
+        }
       }
+      // The words and scales are in registers: hand the slot back.
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bar.empty_w[ws]);
       // The previous stage's store was left in flight while this stage was
-      // expanded: complete it and hand that stage to the MMA issuer.
-      if (it > 0) {
+      // expanded: complete it and count this warp on that stage.
+      if (j > 0) {
         asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
         asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
         __syncwarp();
-        if (lane == 0) mbar_arrive(&bar.full_a[(it - 1) % STAGES]);
+        if (lane == 0) mbar_arrive(&bar.full[(j - 1) % kStages]);
       }
-      if (it >= STAGES) {
-        if (lane == 0) mbar_wait(&bar.empty[s], ((it / STAGES) & 1) ^ 1, &bar.err, a.wait_cycles);
+      if (j >= kStages) {
+        if (lane == 0) mbar_wait(&bar.empty[s], ((j / kStages) & 1) ^ 1, &bar.err, a.wait_cycles);
         __syncwarp();
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
       }
-      {
-        const uint32_t addr = tmem + ((uint32_t)((warp & 3) * 32) << 16) + (uint32_t)(BN + s * 32);
+      const uint32_t addr = tmem + lane_base + (uint32_t)(ND * BN + s * kACols + 16 * kWPW * h);
+      if constexpr (kWPW == 2) {
         asm volatile(
             "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
             "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(addr),
@@ -306,108 +524,252 @@ __global__ void __launch_bounds__(kThreads, 1)
             "r"(av[16]), "r"(av[17]), "r"(av[18]), "r"(av[19]), "r"(av[20]), "r"(av[21]), "r"(av[22]), "r"(av[23]),
             "r"(av[24]), "r"(av[25]), "r"(av[26]), "r"(av[27]), "r"(av[28]), "r"(av[29]), "r"(av[30]), "r"(av[31])
             : "memory");
-      }
-      w0 = n0;
-      w1 = n1;
-      if (GEMM1) {
-#pragma unroll
-        for (int j = 0; j < 8; ++j) cs[j] = ncs[j];
+      } else {
+        asm volatile(
+            "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(
+                addr),
+            "r"(av[0]), "r"(av[1]), "r"(av[2]), "r"(av[3]), "r"(av[4]), "r"(av[5]), "r"(av[6]), "r"(av[7]),
+            "r"(av[8]), "r"(av[9]), "r"(av[10]), "r"(av[11]), "r"(av[12]), "r"(av[13]), "r"(av[14]), "r"(av[15])
+            : "memory");
       }
     }
-    if (nk > 0) {
+    if (n > 0) {
       asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
       asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
       __syncwarp();
-      if (lane == 0) mbar_arrive(&bar.full_a[(nk - 1) % STAGES]);
+      if (lane == 0) mbar_arrive(&bar.full[(n - 1) % kStages]);
     }
     // The next kernel may launch once this CTA has expanded its weights: its
     // own expansion needs no input and would otherwise compete with this
-    // one's for the SMs. Measured against a trigger right after the
-    // tensor-memory allocation: the 2048-token prefill step 4.18 -> 4.04 ms,
-    // 64 tokens 4096^2 37.9 -> 31.3 us, 8192^2 56.7 -> 47.9, 1024 x 8192
-    // 33.4 -> 26.2, 28672 x 8192 at 128 tokens 179 -> 127; only 28672 x 8192
-    // at 64 tokens lost (95 -> 120), where GEMM 1 leaves SMs idle.
+    // one's for the SMs.
     griddep_launch_dependents();
-    // ---- epilogue: TMEM -> registers -> global ---------------------------
-    if (lane == 0) mbar_wait(&bar.done, 0, &bar.err, a.wait_cycles);
-    __syncwarp();
-    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-    if (KS == 1) {
-      griddep_wait();  // the output may still be read by the previous kernel until it completes
-      const float rsc = row_ok ? __half2float(a.rowscale[frow]) : 0.f;
-      const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
-#pragma unroll 1
-      for (int c0 = 0; c0 < BN; c0 += 16) {
-        uint32_t r[16];
-        tmem_ld16(tmem + lane_base + (uint32_t)c0, r);
-        if (row_ok) {
+  } else if (warp >= kEpiWarp0) {
+    // ---- epilogue: accumulator -> registers -> output or partial tile --------
+    const int q = warp & 3;
+    const int R = q * 32 + lane;
+    const uint32_t lane_base = (uint32_t)(q * 32) << 16;
+    const bool tma_out = a.out_vec != 0;  // else each warp stores its own rows
+    griddep_wait();  // the outputs (and partial tiles) may still be read by the previous kernel
+    uint32_t red_phase = 0;  // completions of bar.red seen
+    int ebuf = 0;            // staging buffer of the next chunk
+    // One 16-token chunk of the tile (this thread's row R, v[q] = token
+    // c0 + q), staged [token][row] and written by one thread: into the
+    // output (TMA store; rows and tokens past the matrix are not written)
+    // or, with part != nullptr, into a partial slot (bulk copy).
+    auto emit = [&](const float (&v)[16], float* part, int c0, int64_t row_base, int64_t tok) {
+      uint8_t* buf = estage + ebuf * kEpiStageBytes;
+      if (R == 0) bulk_wait_read1();  // the store issued from this buffer two chunks ago has read it
+      named_sync(1, 128);
+      if (part != nullptr || a.out_f32) {
+        float* b = reinterpret_cast<float*>(buf);
 #pragma unroll
-          for (int q = 0; q < 16; ++q) {
-            const int64_t tok = t0 + c0 + q;
-            if (tok < a.tokens) {
-              const float v = __uint_as_float(r[q]) * rsc;
-              if (a.out_f32)
-                reinterpret_cast<float*>(a.out)[tok * a.ld_out + frow] = v;
-              else
-                reinterpret_cast<__half*>(a.out)[tok * a.ld_out + frow] = __float2half_rn(v);
+        for (int qq = 0; qq < 16; ++qq) b[qq * BM + R] = v[qq];
+      } else {
+        __half* b = reinterpret_cast<__half*>(buf);
+#pragma unroll
+        for (int qq = 0; qq < 16; ++qq) b[qq * BM + R] = __float2half_rn(v[qq]);
+      }
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      named_sync(1, 128);
+      if (R == 0) {
+        if (part != nullptr)
+          bulk_s2g(part + (size_t)c0 * BM, buf, 16 * BM * 4);
+        else
+          tma_store_2d(&out_map, buf, (int)row_base, (int)tok);
+        bulk_commit();
+      }
+      ebuf ^= 1;
+    };
+    auto emit_out = [&](const float (&v)[16], int64_t row0, int64_t row_base, int64_t tok) {
+      if (tma_out) {
+        emit(v, nullptr, 0, row_base, tok);
+      } else if (a.out_f32) {
+        store_chunk<float>(v, reinterpret_cast<float*>(estage) + q * 512, reinterpret_cast<float*>(a.out), a.ld_out,
+                           row0, tm.R, tok, a.tokens, false, lane);
+      } else {
+        store_chunk<__half>(v, reinterpret_cast<__half*>(estage) + q * 1024, reinterpret_cast<__half*>(a.out),
+                            a.ld_out, row0, tm.R, tok, a.tokens, false, lane);
+      }
+    };
+    int64_t i = i0;
+    const int64_t iend = i0 + n;
+    for (int u = 0; i < iend; ++u) {
+      const int t = (int)(i / nk);
+      const int ka = (int)(i - (int64_t)t * nk);
+      const int kb = (int)min((int64_t)nk, (int64_t)ka + (iend - i));
+      i += kb - ka;
+      const int d = u % ND;
+      if (lane == 0) mbar_wait(&bar.dfull[d], (u / ND) & 1, &bar.err, a.wait_cycles);
+      __syncwarp();
+      asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+      const uint32_t dcol = tmem + lane_base + (uint32_t)(d * BN);
+      const int rb = t % RB, tok0 = (t / RB) * BN;
+      const int64_t frow = (int64_t)rb * BM + R;
+      const float rsc = frow < tm.R ? __half2float(a.rowscale[frow]) : 0.f;
+      const int64_t row_base = (int64_t)rb * BM;
+      const int64_t row0 = row_base + q * 32;  // first row of this warp's quadrant
+      if (ka == 0 && kb == nk) {
+        // A whole tile: scale and store; the next chunk's read-back is in
+        // flight while this one is staged.
+        uint32_t r[16];
+        tmem_ld16(dcol, r);
+#pragma unroll 1
+        for (int c0 = 0; c0 < BN; c0 += 16) {
+          float v[16];
+#pragma unroll
+          for (int qq = 0; qq < 16; ++qq) v[qq] = __uint_as_float(r[qq]) * rsc;
+          if (c0 + 16 < BN) tmem_ld16_nowait(dcol + (uint32_t)(c0 + 16), r);
+          emit_out(v, row0, row_base, tok0 + c0);
+          tmem_wait_ld();
+        }
+        asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bar.dempty[d]);
+      } else {
+        // Part of a shared tile (CTAs cf .. cl contribute). Each takes a
+        // ticket when its accumulator is final; the last ticket sums the
+        // tile, the others store their partial into their slot (0 for the
+        // segment the CTA's range starts with, 1 for the one it ends with;
+        // [token][row] over the tile's 128 rows) and count it as stored. The
+        // summing CTA keeps its own part in tensor memory and waits (bounded)
+        // only for CTAs that hold a ticket, i.e. that are resident and only
+        // storing. Sums run in contributor order, so the result does not
+        // depend on which CTA sums.
+        const int64_t it0 = (int64_t)t * nk;
+        const int cf = cta_of(it0, I, G), cl = cta_of(it0 + nk - 1, I, G);
+        unsigned* tickets = a.count + 2 * (size_t)t;
+        unsigned* stored = tickets + 1;
+        if (R == 0) bar.last = atom_add_acq_rel_gpu(tickets, 1u) == (unsigned)(cl - cf) ? 1u : 0u;
+        named_sync(1, 128);
+        const bool last = bar.last != 0;
+        named_sync(1, 128);  // bar.last is reused by the next shared tile
+        if (!last) {
+          const int slot = 2 * c + (i0 >= it0 ? 0 : 1);
+          float* P = a.part + (size_t)slot * BN * BM;
+          uint32_t r[16];
+          tmem_ld16(dcol, r);
+#pragma unroll 1
+          for (int c0 = 0; c0 < BN; c0 += 16) {
+            float v[16];
+#pragma unroll
+            for (int qq = 0; qq < 16; ++qq) v[qq] = __uint_as_float(r[qq]);
+            if (c0 + 16 < BN) tmem_ld16_nowait(dcol + (uint32_t)(c0 + 16), r);
+            emit(v, P, c0, 0, 0);
+            tmem_wait_ld();
+          }
+          asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&bar.dempty[d]);
+          // The partial's copies complete (their writes performed), then one
+          // release add.
+          if (R == 0) {
+            bulk_wait_all();
+            asm volatile("fence.proxy.async.global;" ::: "memory");
+            red_release_gpu(stored, 1u);
+          }
+        } else {
+          const int others = cl - cf;
+          if (R == 0) {
+            const long long w0 = clock64();
+            while (ld_acquire_gpu(stored) < (unsigned)others) {
+              if (clock64() - w0 > a.wait_cycles) {
+                atomicOr(&bar.err, 1u);
+                break;
+              }
             }
+          }
+          named_sync(1, 128);
+          // The other partials: copied into the activation ring when this is
+          // the CTA's last segment (every stage consumed), in pieces of PT
+          // tokens; else read from global memory.
+          int PT = (int)((int64_t)kStages * kTileB / ((int64_t)others * BM * 4)) / 16 * 16;
+          if (PT > BN) PT = BN;
+          const bool use_ring = i == iend && PT >= 16;
+          const float* ringf = reinterpret_cast<const float*>(tileB);
+#pragma unroll 1
+          for (int p0 = 0; p0 < BN; p0 += (use_ring ? PT : BN)) {
+            const int pt = use_ring ? (BN - p0 < PT ? BN - p0 : PT) : BN;
+            if (use_ring) {
+              if (R == 0) {
+                // The partials were written by other CTAs.
+                asm volatile("fence.proxy.async.global;" ::: "memory");
+                mbar_expect_tx(&bar.red, (uint32_t)(others * pt * BM * 4));
+                int idx = 0;
+                for (int cc = cf; cc <= cl; ++cc) {
+                  if (cc == c) continue;
+                  const int sl = 2 * cc + (range_start(cc, I, G) >= it0 ? 0 : 1);
+                  bulk_g2s(tileB + (size_t)idx * pt * BM * 4, a.part + (size_t)sl * BN * BM + (size_t)p0 * BM,
+                           (uint32_t)(pt * BM * 4), &bar.red);
+                  ++idx;
+                }
+              }
+              mbar_wait(&bar.red, red_phase & 1, &bar.err, a.wait_cycles);
+              ++red_phase;
+            }
+#pragma unroll 1
+            for (int c0 = p0; c0 < p0 + pt; c0 += 16) {
+              uint32_t r[16];
+              tmem_ld16(dcol + (uint32_t)c0, r);
+              float acc[16];
+#pragma unroll
+              for (int qq = 0; qq < 16; ++qq) acc[qq] = 0.f;
+              int idx = 0;
+              for (int cc = cf; cc <= cl; ++cc) {
+                if (cc == c) {
+#pragma unroll
+                  for (int qq = 0; qq < 16; ++qq) acc[qq] += __uint_as_float(r[qq]);
+                  continue;
+                }
+                if (use_ring) {
+                  const float* src = ringf + ((size_t)idx * pt + (c0 - p0)) * BM + R;
+#pragma unroll
+                  for (int qq = 0; qq < 16; ++qq) acc[qq] += src[qq * BM];
+                } else {
+                  const int sl = 2 * cc + (range_start(cc, I, G) >= it0 ? 0 : 1);
+                  const float* src = a.part + ((size_t)sl * BN + c0) * BM + R;
+                  float pv[16];
+#pragma unroll
+                  for (int qq = 0; qq < 16; ++qq) pv[qq] = __ldcg(src + (size_t)qq * BM);
+#pragma unroll
+                  for (int qq = 0; qq < 16; ++qq) acc[qq] += pv[qq];
+                }
+                ++idx;
+              }
+#pragma unroll
+              for (int qq = 0; qq < 16; ++qq) acc[qq] *= rsc;
+              emit_out(acc, row0, row_base, tok0 + c0);
+            }
+            if (use_ring) named_sync(1, 128);  // the piece is read before the next copy overwrites it
+          }
+          asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&bar.dempty[d]);
+          if (R == 0) {
+            tickets[0] = 0u;  // ready for the next call
+            stored[0] = 0u;
           }
         }
       }
     }
-  }
-
-  if (KS > 1) {
-    // ---- split-K: partial tiles -> owning CTA through distributed shared
-    //      memory. recv[q][i][c ^ (i & 31)] holds CTA q's partial of row i
-    //      of this CTA's slice (XOR on the column keeps the row-wise reads of
-    //      the final sum free of bank conflicts).
-    constexpr int SLICE = BM / KS;
-    float* recv = reinterpret_cast<float*>(tileB);  // KS * SLICE * BN floats = STAGES * kTileB bytes
-    __syncwarp();
-    cluster_sync();  // every MMA of the cluster is done: the activation stages are free
-    if (warp >= 4) {
-      const int R = threadIdx.x - 128;
-      const int owner = R / SLICE, i = R - owner * SLICE;
-      const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
-      float* row = recv + (size_t)(ks * SLICE + i) * BN;
-#pragma unroll 1
-      for (int c0 = 0; c0 < BN; c0 += 16) {
-        uint32_t r[16];
-        tmem_ld16(tmem + lane_base + (uint32_t)c0, r);
-#pragma unroll
-        for (int q = 0; q < 16; ++q) st_cluster_f32(row + ((c0 + q) ^ (i & 31)), (uint32_t)owner, __uint_as_float(r[q]));
-      }
-    }
-    cluster_sync();  // all partials have landed
-    griddep_wait();  // the output may still be read by the previous kernel until it completes
-    for (int idx = threadIdx.x; idx < SLICE * BN; idx += kThreads) {
-      const int c = idx / SLICE, i = idx - c * SLICE;  // token column c, slice row i
-      const int64_t frow = f0 + ks * SLICE + i;
-      const int64_t tok = t0 + c;
-      if (frow >= tm.R || tok >= a.tokens) continue;
-      float v = 0.f;
-#pragma unroll
-      for (int q = 0; q < KS; ++q) v += recv[(size_t)(q * SLICE + i) * BN + (c ^ (i & 31))];
-      v *= __half2float(a.rowscale[frow]);
-      if (a.out_f32)
-        reinterpret_cast<float*>(a.out)[tok * a.ld_out + frow] = v;
-      else
-        reinterpret_cast<__half*>(a.out)[tok * a.ld_out + frow] = __float2half_rn(v);
-    }
+    if (R == 0) bulk_wait_all();  // every store has been performed before the CTA exits
   }
 
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
   __syncthreads();
   if (bar.err != 0 && threadIdx.x == 0) {
-    // A wait gave up: let TMA copies that may still be in flight land
-    // (bounded) before the CTA exits, and report it.
-    for (int s = 0; s < STAGES; ++s) mbar_wait(&bar.full_b[s], 0, &bar.err, a.wait_cycles);
+    // A wait gave up: let the copies that may still be in flight land
+    // (bounded: the last copy issued into each slot) before the CTA exits,
+    // and report it.
+    const int nb = (int)bar.issued_b, nw = (int)bar.issued_w;
+    for (int j = nb - kStages < 0 ? 0 : nb - kStages; j < nb; ++j)
+      mbar_wait(&bar.full[j % kStages], (j / kStages) & 1, &bar.err, a.wait_cycles);
+    for (int j = nw - kWSlots < 0 ? 0 : nw - kWSlots; j < nw; ++j)
+      mbar_wait(&bar.full_w[j % kWSlots], (j / kWSlots) & 1, &bar.err, a.wait_cycles);
     atomicOr(a.status, kStatusTimeout);
   }
   if (warp == 1) {
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(tmem_cols<BN>()) : "memory");
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
   }
 }
 
@@ -434,7 +796,7 @@ cudaError_t make_act_map(CUtensorMap* map, const __half* base, int64_t rows, int
   if (fn == nullptr) return cudaErrorNotSupported;
   cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
   cuuint64_t strides[1] = {(cuuint64_t)(ld * 2)};
-  cuuint32_t box[2] = {(cuuint32_t)BK, (cuuint32_t)bn};
+  cuuint32_t box[2] = {(cuuint32_t)BOX, (cuuint32_t)bn};
   cuuint32_t estr[2] = {1, 1};
   CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<__half*>(base), dims, strides, box, estr,
                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
@@ -442,63 +804,76 @@ cudaError_t make_act_map(CUtensorMap* map, const __half* base, int64_t rows, int
   return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
-template <bool GEMM1, int BN, int KS>
-cudaError_t launch_gemm_bn(const PrefillArgs& a, const __half* act, int64_t ld_act, cudaStream_t st) {
-  CUtensorMap map;
+// Token tile of a pass of T tokens.
+int prefill_bn(int64_t T) { return T <= 16 ? 16 : T <= 32 ? 32 : T <= 64 ? 64 : T <= 128 ? 128 : 256; }
+
+// Grid of one GEMM: with partial tiles, the SM count (fewer when a CTA would
+// get less than kMinStagesPerCta stages); without, one CTA per tile.
+int prefill_grid(const SignMatrix& sm, int64_t T, int num_sms, bool split) {
+  const int64_t bn = prefill_bn(T);
+  const int64_t tiles = (int64_t)sm.RB * ((T + bn - 1) / bn);
+  if (!split) return (int)tiles;
+  const int64_t bkk = bk_of((int)bn);
+  const int64_t iters = tiles * ((sm.C + bkk - 1) / bkk);
+  int64_t g = iters / min_stages_per_cta((int)bn);
+  if (g > num_sms) g = num_sms;
+  if (g < 1) g = 1;
+  return (int)g;
+}
+
+// Tensor map of the output [tokens][ld] (FP16 or FP32) with `rows` valid
+// columns: boxes of 128 columns x 16 tokens, no swizzle; stores past the
+// matrix are dropped.
+cudaError_t make_out_map(CUtensorMap* map, void* base, int64_t tokens, int64_t rows, int64_t ld, bool f32) {
+  PFN_cuTensorMapEncodeTiled_v12000 fn = encode_fn();
+  if (fn == nullptr) return cudaErrorNotSupported;
+  const int64_t es = f32 ? 4 : 2;
+  cuuint64_t dims[2] = {(cuuint64_t)rows, (cuuint64_t)tokens};
+  cuuint64_t strides[1] = {(cuuint64_t)(ld * es)};
+  cuuint32_t box[2] = {(cuuint32_t)BM, 16u};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(map, f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, base, dims, strides,
+                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                  CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+template <bool GEMM1, int BN>
+cudaError_t launch_gemm_bn(const PrefillArgs& a, const __half* act, int64_t ld_act, int grid, cudaStream_t st) {
+  CUtensorMap map, omap;
   cudaError_t e = make_act_map(&map, act, a.tokens, a.sm.C, ld_act, BN);
   if (e != cudaSuccess) return e;
-  auto kern = prefill_kernel<GEMM1, BN, KS>;
-  // A cluster's CTAs wait for each other while holding tensor memory, so no
-  // third CTA may share an SM with two of them (one that blocks in
-  // tcgen05.alloc would wait for a CTA that waits for it): with at least
-  // 80 KB of shared memory per CTA, at most two CTAs fit on an SM and their
-  // tensor memory (<= 256 columns each) always fits.
-  constexpr int smem = (KS > 1 && smem_bytes<BN>() < 80 * 1024) ? 80 * 1024 : smem_bytes<BN>();
+  std::memset(&omap, 0, sizeof(omap));
+  if (a.out_vec) {
+    e = make_out_map(&omap, a.out, a.tokens, a.sm.R, a.ld_out, a.out_f32 != 0);
+    if (e != cudaSuccess) return e;
+  }
+  auto kern = prefill_kernel<GEMM1, BN>;
+  constexpr int smem = smem_bytes<BN>();
   e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((unsigned)a.sm.RB, (unsigned)((a.tokens + BN - 1) / BN), (unsigned)KS);
+  cfg.gridDim = dim3((unsigned)grid, 1, 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = st;
-  cudaLaunchAttribute attr[2];
+  cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
-  attr[1].id = cudaLaunchAttributeClusterDimension;
-  attr[1].val.clusterDim.x = 1;
-  attr[1].val.clusterDim.y = 1;
-  attr[1].val.clusterDim.z = (unsigned)KS;
   cfg.attrs = attr;
-  cfg.numAttrs = KS > 1 ? 2 : 1;
-  return cudaLaunchKernelEx(&cfg, kern, map, a);
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, map, omap, a);
 }
 
-// Tiling of one GEMM: the smallest token tile of 64 / 128 / 256 that covers
-// the pass, made smaller while the grid would leave half the SMs idle; with
-// tiles of 64, short passes (few row blocks x token tiles) split K over a
-// cluster of 2, 4 or 8 CTAs (every CTA keeps at least two K-stages) while
-// the grid fits one CTA per SM, or two per SM for contractions of 256
-// K-stages or more (measured: 8192 x 28672 at 64 tokens 164 -> 108 us; the
-// same on shorter contractions lost, e.g. 4096^2 31 -> 40 us).
 template <bool GEMM1>
 cudaError_t launch_gemm(const PrefillArgs& a, const __half* act, int64_t ld_act, int num_sms, cudaStream_t st) {
-  const int64_t rb = a.sm.RB;
-  int bn = a.tokens > 128 ? 256 : a.tokens > 64 ? 128 : 64;
-  while (bn > 64 && rb * ((a.tokens + bn - 1) / bn) < num_sms / 2) bn /= 2;
-  if (bn == 256) return launch_gemm_bn<GEMM1, 256, 1>(a, act, ld_act, st);
-  if (bn == 128) return launch_gemm_bn<GEMM1, 128, 1>(a, act, ld_act, st);
-  const int64_t base = rb * ((a.tokens + 63) / 64);
-  const int nk = (int)((a.sm.C + BK - 1) / BK);
-  int ks = 1;
-  const int64_t room = nk >= 256 ? 2 * (int64_t)num_sms : (int64_t)num_sms;
-  while (ks < 8 && base * ks * 2 <= room && nk >= 4 * ks) ks *= 2;
-  // every CTA of the split needs at least one stage
-  while (ks > 1 && (ks - 1) * ((nk + ks - 1) / ks) >= nk) ks /= 2;
-  switch (ks) {
-    case 8: return launch_gemm_bn<GEMM1, 64, 8>(a, act, ld_act, st);
-    case 4: return launch_gemm_bn<GEMM1, 64, 4>(a, act, ld_act, st);
-    case 2: return launch_gemm_bn<GEMM1, 64, 2>(a, act, ld_act, st);
-    default: return launch_gemm_bn<GEMM1, 64, 1>(a, act, ld_act, st);
+  const int grid = prefill_grid(a.sm, a.tokens, num_sms, a.part != nullptr);
+  switch (prefill_bn(a.tokens)) {
+    case 16: return launch_gemm_bn<GEMM1, 16>(a, act, ld_act, grid, st);
+    case 32: return launch_gemm_bn<GEMM1, 32>(a, act, ld_act, grid, st);
+    case 64: return launch_gemm_bn<GEMM1, 64>(a, act, ld_act, grid, st);
+    case 128: return launch_gemm_bn<GEMM1, 128>(a, act, ld_act, grid, st);
+    default: return launch_gemm_bn<GEMM1, 256>(a, act, ld_act, grid, st);
   }
 }
 
@@ -506,8 +881,21 @@ cudaError_t launch_gemm(const PrefillArgs& a, const __half* act, int64_t ld_act,
 
 int64_t prefill_h_ld(const af1_layer& L) { return (L.r + 7) / 8 * 8; }
 
+int64_t prefill_part_bytes(const af1_layer& L, int64_t tokens) {
+  const int64_t T = tokens < kPrefillPassTokens ? tokens : kPrefillPassTokens;
+  return (int64_t)2 * L.num_sms * prefill_bn(T) * BM * 4;
+}
+
+int64_t prefill_count_bytes(const af1_layer& L, int64_t tokens) {
+  const int64_t T = tokens < kPrefillPassTokens ? tokens : kPrefillPassTokens;
+  const int64_t nt = (T + prefill_bn(T) - 1) / prefill_bn(T);
+  const int64_t rb = L.p1.RB > L.p2.RB ? L.p1.RB : L.p2.RB;
+  return rb * nt * 8;
+}
+
 cudaError_t launch_prefill(const af1_layer& L, const void* x, int64_t ldx, int64_t tokens, void* y, int64_t ldy,
-                           int y_dtype, uint8_t* h_buf, unsigned* status, cudaStream_t st) {
+                           int y_dtype, uint8_t* h_buf, float* part, unsigned* count, unsigned* status,
+                           cudaStream_t st) {
   const int64_t ldh = prefill_h_ld(L);
   const int ysize = y_dtype == 0 ? 2 : 4;
   for (int64_t t0 = 0; t0 < tokens; t0 += kPrefillPassTokens) {
@@ -521,21 +909,22 @@ cudaError_t launch_prefill(const af1_layer& L, const void* x, int64_t ldx, int64
     g1.out = h_buf;
     g1.ld_out = ldh;
     g1.out_f32 = 0;
+    g1.out_vec = ((uintptr_t)h_buf % 16 == 0 && (ldh * 2) % 16 == 0) ? 1 : 0;
+    g1.part = part;
+    g1.count = count;
     g1.status = status;
     g1.wait_cycles = wait_budget();
     cudaError_t e = launch_gemm<true>(g1, static_cast<const __half*>(x) + t0 * ldx, ldx, L.num_sms, st);
     if (e != cudaSuccess) return e;
-    PrefillArgs g2 = {};
+    PrefillArgs g2 = g1;
     g2.signs = reinterpret_cast<const uint32_t*>(L.signs2);
     g2.sm = L.p2;
-    g2.tokens = T;
     g2.colscale = nullptr;
     g2.rowscale = reinterpret_cast<const __half*>(L.a);
     g2.out = static_cast<uint8_t*>(y) + t0 * ldy * ysize;
     g2.ld_out = ldy;
     g2.out_f32 = y_dtype == 0 ? 0 : 1;
-    g2.status = status;
-    g2.wait_cycles = g1.wait_cycles;
+    g2.out_vec = ((uintptr_t)g2.out % 16 == 0 && (ldy * ysize) % 16 == 0) ? 1 : 0;
     e = launch_gemm<false>(g2, reinterpret_cast<const __half*>(h_buf), ldh, L.num_sms, st);
     if (e != cudaSuccess) return e;
   }
