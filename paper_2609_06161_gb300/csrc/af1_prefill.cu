@@ -17,7 +17,7 @@
 // another. Without room for the partials (the built-in-scratch entry) the
 // grid is one CTA per tile.
 //
-// Roles of the 12 warps of a CTA, over the CTA's stages in order:
+// Roles of the 18 warps of a CTA, over the CTA's stages in order:
 //   * warp 0, one thread: copies each stage's packed signs (128 rows x 2
 //     words: 1 KB contiguous in the row-block layout) and, for GEMM1, its 64
 //     column scales into a ring of 14 small slots (cp.async.bulk), up to 14
@@ -27,11 +27,11 @@
 //     (B) of the stage by TMA (cp.async.bulk.tensor, 128-byte swizzle, zero
 //     fill past the tokens / columns) into a ring of 8 stages (6 for BN =
 //     256);
-//   * warps 4-7 expand the signs into FP16 (+-b_j for GEMM1, +-1 for GEMM2:
+//   * warps 4-11 expand the signs into FP16 (+-b_j for GEMM1, +-1 for GEMM2:
 //     exact) and store them into a ring of A buffers (one per stage) in
-//     tensor memory
-//     (tcgen05.st; warp w writes rows 32 (w % 4) .. +31, one row per thread
-//     = tensor-memory lane; eight warps with half a stage each were slower);
+//     tensor memory (tcgen05.st; warp w writes rows 32 (w % 4) .. +31, one
+//     row per thread = tensor-memory lane, and half (w - 4) / 4 of the
+//     stage's columns);
 //     A in tensor memory leaves shared-memory bandwidth to B;
 //   * warp 1, one thread: four tcgen05.mma.kind::f16 per stage (K = 16,
 //     N = BN, A from tensor memory, B from shared memory) into an
@@ -41,12 +41,13 @@
 //     memory for A), and the MMAs of the next tile wait for its read-back.
 //     Measured: this one thread needs about 175 cycles per MMA whatever N,
 //     so N = 128 tiles ran at half the rate of N = 256;
-//   * warps 8-11 read an accumulator back (tcgen05.ld), apply the feature
-//     scale and stage 16 tokens at a time in shared memory, which one thread
-//     writes out with a TMA store (or a bulk copy for a partial tile) while
-//     the warps go on to the next 16 (stores from the warps themselves were
-//     latency-bound in the store queue, and the MMA waits for this read-back
-//     when a tile has one accumulator).
+//   * two groups of four warps (12-15; 16, 17, 2, 3) read an accumulator
+//     back (tcgen05.ld) in alternate 16-token chunks, apply the feature
+//     scale and stage each chunk in shared memory, which one thread of the
+//     group writes out with a TMA store (or a bulk copy for a partial tile)
+//     (stores from the warps themselves were latency-bound in the store
+//     queue, and the MMA waits for this read-back when a tile has one
+//     accumulator).
 // All mbarrier waits are bounded; a wait that gives up sets the status word.
 #include <cuda.h>
 #include <cudaTypedefs.h>
@@ -65,10 +66,12 @@ namespace {
 
 constexpr int BM = 128;      // features per tile (MMA M, tensor-memory lanes)
 constexpr int BOX = 64;      // K per activation box: one 128-byte swizzle row of FP16
-constexpr int kThreads = 512;
+constexpr int kThreads = 576;
 constexpr int kTmemCols = 512;  // accumulators (2 x BN, or 1 x 256) + one A buffer per stage
 constexpr int kExpandWarps = 8;  // warps 4..11
-constexpr int kEpiWarp0 = 12;    // warps 12..15
+constexpr int kEpiWarp0 = 12;    // epilogue group 0: warps 12..15; group 1: warps 16, 17, 2, 3
+constexpr int kEpiWarps = 8;
+__device__ __forceinline__ bool is_epi_warp(int w) { return w == 2 || w == 3 || w >= kEpiWarp0; }
 constexpr int kMaxStages = 8;
 constexpr int kMaxWSlots = 14;
 
@@ -228,8 +231,8 @@ __device__ __forceinline__ void bulk_s2g(void* dst, const void* src, uint32_t by
                : "memory");
 }
 __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
-// At most one group still reading its shared-memory source.
-__device__ __forceinline__ void bulk_wait_read1() { asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory"); }
+// No group still reading its shared-memory source.
+__device__ __forceinline__ void bulk_wait_read0() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
 // Every group complete (its writes performed).
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 __device__ __forceinline__ void tmem_ld16_nowait(uint32_t addr, uint32_t (&r)[16]) {
@@ -328,7 +331,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int d = 0; d < ND; ++d) {
       mbar_init(&bar.dfull[d], 1);
-      mbar_init(&bar.dempty[d], 4);
+      mbar_init(&bar.dempty[d], kEpiWarps);
     }
     mbar_init(&bar.red, 1);
     bar.err = 0;
@@ -543,23 +546,32 @@ __global__ void __launch_bounds__(kThreads, 1)
     // own expansion needs no input and would otherwise compete with this
     // one's for the SMs.
     griddep_launch_dependents();
-  } else if (warp >= kEpiWarp0) {
+  } else if (is_epi_warp(warp)) {
     // ---- epilogue: accumulator -> registers -> output or partial tile --------
+    // Two groups of four warps (one warp per tensor-memory lane quadrant
+    // each) take alternate 16-token chunks, so two read-back chains run at
+    // once (the MMA waits for this read-back when a tile has one
+    // accumulator). Group g stages its chunk in buffer g; its first thread
+    // writes it out.
     const int q = warp & 3;
+    const int g = (warp >= kEpiWarp0 && warp < kEpiWarp0 + 4) ? 0 : 1;
     const int R = q * 32 + lane;
+    const bool issuer = R == 0;                // the group's thread that writes chunks out
+    const bool leader = issuer && g == 0;      // takes tickets and counts partials
+    const int gbar = 1 + g;                    // named barrier of the group (128 threads)
+    constexpr int kBothBar = 3;                // named barrier of both groups (256 threads)
     const uint32_t lane_base = (uint32_t)(q * 32) << 16;
     const bool tma_out = a.out_vec != 0;  // else each warp stores its own rows
+    uint8_t* buf = estage + g * kEpiStageBytes;
     griddep_wait();  // the outputs (and partial tiles) may still be read by the previous kernel
     uint32_t red_phase = 0;  // completions of bar.red seen
-    int ebuf = 0;            // staging buffer of the next chunk
     // One 16-token chunk of the tile (this thread's row R, v[q] = token
-    // c0 + q), staged [token][row] and written by one thread: into the
-    // output (TMA store; rows and tokens past the matrix are not written)
-    // or, with part != nullptr, into a partial slot (bulk copy).
+    // c0 + q), staged [token][row] and written by the group's first thread:
+    // into the output (TMA store; rows and tokens past the matrix are not
+    // written) or, with part != nullptr, into a partial slot (bulk copy).
     auto emit = [&](const float (&v)[16], float* part, int c0, int64_t row_base, int64_t tok) {
-      uint8_t* buf = estage + ebuf * kEpiStageBytes;
-      if (R == 0) bulk_wait_read1();  // the store issued from this buffer two chunks ago has read it
-      named_sync(1, 128);
+      if (issuer) bulk_wait_read0();  // the group's previous store has read the buffer
+      named_sync(gbar, 128);
       if (part != nullptr || a.out_f32) {
         float* b = reinterpret_cast<float*>(buf);
 #pragma unroll
@@ -570,25 +582,24 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int qq = 0; qq < 16; ++qq) b[qq * BM + R] = __float2half_rn(v[qq]);
       }
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      named_sync(1, 128);
-      if (R == 0) {
+      named_sync(gbar, 128);
+      if (issuer) {
         if (part != nullptr)
           bulk_s2g(part + (size_t)c0 * BM, buf, 16 * BM * 4);
         else
           tma_store_2d(&out_map, buf, (int)row_base, (int)tok);
         bulk_commit();
       }
-      ebuf ^= 1;
     };
     auto emit_out = [&](const float (&v)[16], int64_t row0, int64_t row_base, int64_t tok) {
       if (tma_out) {
         emit(v, nullptr, 0, row_base, tok);
       } else if (a.out_f32) {
-        store_chunk<float>(v, reinterpret_cast<float*>(estage) + q * 512, reinterpret_cast<float*>(a.out), a.ld_out,
-                           row0, tm.R, tok, a.tokens, false, lane);
+        store_chunk<float>(v, reinterpret_cast<float*>(estage) + (g * 4 + q) * 512, reinterpret_cast<float*>(a.out),
+                           a.ld_out, row0, tm.R, tok, a.tokens, false, lane);
       } else {
-        store_chunk<__half>(v, reinterpret_cast<__half*>(estage) + q * 1024, reinterpret_cast<__half*>(a.out),
-                            a.ld_out, row0, tm.R, tok, a.tokens, false, lane);
+        store_chunk<__half>(v, reinterpret_cast<__half*>(estage) + (g * 4 + q) * 1024,
+                            reinterpret_cast<__half*>(a.out), a.ld_out, row0, tm.R, tok, a.tokens, false, lane);
       }
     };
     int64_t i = i0;
@@ -609,16 +620,16 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int64_t row_base = (int64_t)rb * BM;
       const int64_t row0 = row_base + q * 32;  // first row of this warp's quadrant
       if (ka == 0 && kb == nk) {
-        // A whole tile: scale and store; the next chunk's read-back is in
-        // flight while this one is staged.
+        // A whole tile: scale and store this group's chunks; the next
+        // chunk's read-back is in flight while this one is staged.
         uint32_t r[16];
-        tmem_ld16(dcol, r);
+        if (16 * g < BN) tmem_ld16(dcol + (uint32_t)(16 * g), r);
 #pragma unroll 1
-        for (int c0 = 0; c0 < BN; c0 += 16) {
+        for (int c0 = 16 * g; c0 < BN; c0 += 32) {
           float v[16];
 #pragma unroll
           for (int qq = 0; qq < 16; ++qq) v[qq] = __uint_as_float(r[qq]) * rsc;
-          if (c0 + 16 < BN) tmem_ld16_nowait(dcol + (uint32_t)(c0 + 16), r);
+          if (c0 + 32 < BN) tmem_ld16_nowait(dcol + (uint32_t)(c0 + 32), r);
           emit_out(v, row0, row_base, tok0 + c0);
           tmem_wait_ld();
         }
@@ -639,37 +650,38 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int cf = cta_of(it0, I, G), cl = cta_of(it0 + nk - 1, I, G);
         unsigned* tickets = a.count + 2 * (size_t)t;
         unsigned* stored = tickets + 1;
-        if (R == 0) bar.last = atom_add_acq_rel_gpu(tickets, 1u) == (unsigned)(cl - cf) ? 1u : 0u;
-        named_sync(1, 128);
+        if (leader) bar.last = atom_add_acq_rel_gpu(tickets, 1u) == (unsigned)(cl - cf) ? 1u : 0u;
+        named_sync(kBothBar, 256);
         const bool last = bar.last != 0;
-        named_sync(1, 128);  // bar.last is reused by the next shared tile
+        named_sync(kBothBar, 256);  // bar.last is reused by the next shared tile
         if (!last) {
           const int slot = 2 * c + (i0 >= it0 ? 0 : 1);
           float* P = a.part + (size_t)slot * BN * BM;
           uint32_t r[16];
-          tmem_ld16(dcol, r);
+          if (16 * g < BN) tmem_ld16(dcol + (uint32_t)(16 * g), r);
 #pragma unroll 1
-          for (int c0 = 0; c0 < BN; c0 += 16) {
+          for (int c0 = 16 * g; c0 < BN; c0 += 32) {
             float v[16];
 #pragma unroll
             for (int qq = 0; qq < 16; ++qq) v[qq] = __uint_as_float(r[qq]);
-            if (c0 + 16 < BN) tmem_ld16_nowait(dcol + (uint32_t)(c0 + 16), r);
+            if (c0 + 32 < BN) tmem_ld16_nowait(dcol + (uint32_t)(c0 + 32), r);
             emit(v, P, c0, 0, 0);
             tmem_wait_ld();
           }
           asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
           __syncwarp();
           if (lane == 0) mbar_arrive(&bar.dempty[d]);
-          // The partial's copies complete (their writes performed), then one
+          // Both groups' copies complete (their writes performed), then one
           // release add.
-          if (R == 0) {
+          if (issuer) {
             bulk_wait_all();
             asm volatile("fence.proxy.async.global;" ::: "memory");
-            red_release_gpu(stored, 1u);
           }
+          named_sync(kBothBar, 256);
+          if (leader) red_release_gpu(stored, 1u);
         } else {
           const int others = cl - cf;
-          if (R == 0) {
+          if (leader) {
             const long long w0 = clock64();
             while (ld_acquire_gpu(stored) < (unsigned)others) {
               if (clock64() - w0 > a.wait_cycles) {
@@ -678,19 +690,19 @@ __global__ void __launch_bounds__(kThreads, 1)
               }
             }
           }
-          named_sync(1, 128);
+          named_sync(kBothBar, 256);
           // The other partials: copied into the activation ring when this is
           // the CTA's last segment (every stage consumed), in pieces of PT
           // tokens; else read from global memory.
-          int PT = (int)((int64_t)kStages * kTileB / ((int64_t)others * BM * 4)) / 16 * 16;
+          int PT = (int)((int64_t)kStages * kTileB / ((int64_t)others * BM * 4)) / 32 * 32;
           if (PT > BN) PT = BN;
-          const bool use_ring = i == iend && PT >= 16;
+          const bool use_ring = i == iend && PT >= 32;
           const float* ringf = reinterpret_cast<const float*>(tileB);
 #pragma unroll 1
           for (int p0 = 0; p0 < BN; p0 += (use_ring ? PT : BN)) {
             const int pt = use_ring ? (BN - p0 < PT ? BN - p0 : PT) : BN;
             if (use_ring) {
-              if (R == 0) {
+              if (leader) {
                 // The partials were written by other CTAs.
                 asm volatile("fence.proxy.async.global;" ::: "memory");
                 mbar_expect_tx(&bar.red, (uint32_t)(others * pt * BM * 4));
@@ -707,7 +719,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               ++red_phase;
             }
 #pragma unroll 1
-            for (int c0 = p0; c0 < p0 + pt; c0 += 16) {
+            for (int c0 = p0 + 16 * g; c0 < p0 + pt; c0 += 32) {
               uint32_t r[16];
               tmem_ld16(dcol + (uint32_t)c0, r);
               float acc[16];
@@ -739,22 +751,23 @@ __global__ void __launch_bounds__(kThreads, 1)
               for (int qq = 0; qq < 16; ++qq) acc[qq] *= rsc;
               emit_out(acc, row0, row_base, tok0 + c0);
             }
-            if (use_ring) named_sync(1, 128);  // the piece is read before the next copy overwrites it
+            if (use_ring) named_sync(kBothBar, 256);  // the piece is read before the next copy overwrites it
           }
           asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
           __syncwarp();
           if (lane == 0) mbar_arrive(&bar.dempty[d]);
-          if (R == 0) {
+          if (leader) {
             tickets[0] = 0u;  // ready for the next call
             stored[0] = 0u;
           }
         }
       }
     }
-    if (R == 0) bulk_wait_all();  // every store has been performed before the CTA exits
+    if (issuer) bulk_wait_all();  // every store has been performed before the CTA exits
   }
 
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  __syncwarp();  // every lane of the warp arrives at the barrier (lanes of a role warp finish at different times)
   __syncthreads();
   if (bar.err != 0 && threadIdx.x == 0) {
     // A wait gave up: let the copies that may still be in flight land
