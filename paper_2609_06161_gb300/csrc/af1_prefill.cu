@@ -115,9 +115,6 @@ template <int BN>
 __host__ __device__ constexpr int wslots() {
   return BN == 256 ? 6 : 14;
 }
-// Stages of K per CTA below which the stream-K grid is made smaller (more
-// CTAs per tile means more partial tiles for its last contributor to sum).
-constexpr int min_stages_per_cta(int bn) { return bn == 256 ? 8 : bn <= 32 ? 8 : 16; }
 // At least 116 KB so that two CTAs never share an SM (each allocates all of
 // its tensor memory).
 // Epilogue staging: two buffers of one 16-token x 128-row chunk (FP32 at
@@ -694,9 +691,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           // The other partials: copied into the activation ring when this is
           // the CTA's last segment (every stage consumed), in pieces of PT
           // tokens; else read from global memory.
-          int PT = (int)((int64_t)kStages * kTileB / ((int64_t)others * BM * 4)) / 32 * 32;
+          int PT = (int)((int64_t)kStages * kTileB / ((int64_t)others * BM * 4)) / 16 * 16;
           if (PT > BN) PT = BN;
-          const bool use_ring = i == iend && PT >= 32;
+          const bool use_ring = i == iend && PT >= 16;
           const float* ringf = reinterpret_cast<const float*>(tileB);
 #pragma unroll 1
           for (int p0 = 0; p0 < BN; p0 += (use_ring ? PT : BN)) {
@@ -820,18 +817,37 @@ cudaError_t make_act_map(CUtensorMap* map, const __half* base, int64_t rows, int
 // Token tile of a pass of T tokens.
 int prefill_bn(int64_t T) { return T <= 16 ? 16 : T <= 32 ? 32 : T <= 64 ? 64 : T <= 128 ? 128 : 256; }
 
-// Grid of one GEMM: with partial tiles, the SM count (fewer when a CTA would
-// get less than kMinStagesPerCta stages); without, one CTA per tile.
+// Grid of one GEMM. Without room for partial tiles: one CTA per tile.
+// Otherwise the grid (at most one CTA per SM) that minimises a CTA's modelled
+// time: its stages, a fixed cost (pipeline fill, epilogue) and, when tiles
+// are shared, the summing CTA's read of the other parts (its slowest step:
+// about 20 bytes per cycle measured). Filling every SM regardless spread
+// the 8 row-block tiles of a 1024 x 8192 layer over 8 CTAs each and the
+// sums took longer than the stages (64 tokens: 26 -> 37 us).
 int prefill_grid(const SignMatrix& sm, int64_t T, int num_sms, bool split) {
   const int64_t bn = prefill_bn(T);
   const int64_t tiles = (int64_t)sm.RB * ((T + bn - 1) / bn);
   if (!split) return (int)tiles;
   const int64_t bkk = bk_of((int)bn);
-  const int64_t iters = tiles * ((sm.C + bkk - 1) / bkk);
-  int64_t g = iters / min_stages_per_cta((int)bn);
-  if (g > num_sms) g = num_sms;
-  if (g < 1) g = 1;
-  return (int)g;
+  const int64_t nk = (sm.C + bkk - 1) / bkk;
+  const int64_t iters = tiles * nk;
+  const double t_stage = (double)(bkk / 16) * 134.0 + 150.0;  // cycles: MMAs, barrier check, commit
+  const double t_fixed = 4000.0 + 45.0 * (double)bn;           // fill, epilogue of a tile
+  const double part_cycles = (double)bn * BM * 4 / 20.0;       // reading one partial tile
+  int64_t best_g = 1;
+  double best = 1e300;
+  for (int64_t g = 1; g <= num_sms && g <= iters; ++g) {
+    const int64_t per = (iters + g - 1) / g;  // stages of the busiest CTA
+    int64_t parts = 1;                        // CTAs sharing one tile (at most)
+    if (per % nk != 0 || (iters % g) != 0) parts = per >= nk ? 2 : (nk + per - 1) / per + 1;
+    const double cost =
+        (double)per * t_stage + t_fixed + (parts > 1 ? 3000.0 + (double)(parts - 1) * part_cycles : 0.0);
+    if (cost < best * 0.995) {  // prefer fewer CTAs on ties
+      best = cost;
+      best_g = g;
+    }
+  }
+  return (int)best_g;
 }
 
 // Tensor map of the output [tokens][ld] (FP16 or FP32) with `rows` valid
