@@ -142,7 +142,7 @@ struct PrefillArgs {
   int out_f32;
   int out_vec;             // out and ld_out allow 16-byte stores
   float* part;             // partial tiles: 2 slots per CTA of 128 rows x BN FP32 (nullptr: one tile per CTA)
-  unsigned* count;         // two counters per tile: tickets taken, partials stored (zero between calls)
+  unsigned* count;         // per tile: tickets taken, partials stored (zero between calls)
   unsigned* status;
   long long wait_cycles;  // budget of every bounded wait (clock64 cycles)
 };
@@ -158,7 +158,9 @@ struct __align__(8) PrefillBarriers {
   uint64_t red;                // partial tiles copied in for a reduction
   uint32_t tmem_addr;
   uint32_t err;
-  uint32_t last;               // epilogue: this CTA completes the shared tile
+  uint32_t last;               // epilogue: this CTA holds the last ticket of the shared tile
+  uint32_t npend;              // epilogue: a shared tile this CTA sums at the end of its range
+  uint32_t pend[2];
 };
 
 __device__ __forceinline__ void tmem_ld16(uint32_t addr, uint32_t (&r)[16]) {
@@ -334,6 +336,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     bar.err = 0;
     bar.issued_b = 0;
     bar.issued_w = 0;
+    bar.npend = 0;
     bar.last = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&act_map)) : "memory");
@@ -554,7 +557,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int g = (warp >= kEpiWarp0 && warp < kEpiWarp0 + 4) ? 0 : 1;
     const int R = q * 32 + lane;
     const bool issuer = R == 0;                // the group's thread that writes chunks out
-    const bool leader = issuer && g == 0;      // takes tickets and counts partials
+    const bool leader = issuer && g == 0;      // counts partials and copies parts in
     const int gbar = 1 + g;                    // named barrier of the group (128 threads)
     constexpr int kBothBar = 3;                // named barrier of both groups (256 threads)
     const uint32_t lane_base = (uint32_t)(q * 32) << 16;
@@ -599,6 +602,87 @@ __global__ void __launch_bounds__(kThreads, 1)
                             reinterpret_cast<__half*>(a.out), a.ld_out, row0, tm.R, tok, a.tokens, false, lane);
       }
     };
+    // Sum shared tile t: wait (bounded) for the stored parts, copy them into
+    // the activation ring PT tokens at a time, and add in contributor order;
+    // this CTA's own part comes from accumulator columns own_dcol, or from
+    // its slot when own_dcol is all ones.
+    auto sum_tile = [&](int t, uint32_t own_dcol) {
+      const int64_t it0 = (int64_t)t * nk;
+      const int cf = cta_of(it0, I, G), cl = cta_of(it0 + nk - 1, I, G);
+      const bool own_tmem = own_dcol != 0xFFFFFFFFu;
+      const int parts = cl - cf + 1;
+      const int copied = own_tmem ? parts - 1 : parts;  // parts read from the slots
+      unsigned* tickets = a.count + 2 * (size_t)t;
+      if (leader) {
+        const long long w0 = clock64();
+        while (ld_acquire_gpu(tickets + 1) < (unsigned)copied) {
+          if (clock64() - w0 > a.wait_cycles) {
+            atomicOr(&bar.err, 1u);
+            break;
+          }
+        }
+      }
+      named_sync(kBothBar, 256);
+      const int rb = t % RB, tok0 = (t / RB) * BN;
+      const int64_t frow = (int64_t)rb * BM + R;
+      const float rsc = frow < tm.R ? __half2float(a.rowscale[frow]) : 0.f;
+      const int64_t row_base = (int64_t)rb * BM;
+      const int64_t row0 = row_base + q * 32;
+      int PT = (int)((int64_t)kStages * kTileB / ((int64_t)copied * BM * 4)) / 16 * 16;
+      if (PT > BN) PT = BN;
+      if (PT < 16) {  // the host's grid keeps the parts within the ring; never taken
+        if (leader) atomicOr(&bar.err, 1u);
+        return;
+      }
+      const float* ringf = reinterpret_cast<const float*>(tileB);
+#pragma unroll 1
+      for (int p0 = 0; p0 < BN; p0 += PT) {
+        const int pt = BN - p0 < PT ? BN - p0 : PT;
+        if (leader) {
+          // The parts were written by other CTAs (and perhaps this one).
+          asm volatile("fence.proxy.async.global;" ::: "memory");
+          mbar_expect_tx(&bar.red, (uint32_t)(copied * pt * BM * 4));
+          int idx = 0;
+          for (int cc = cf; cc <= cl; ++cc) {
+            if (own_tmem && cc == c) continue;
+            const int sl = 2 * cc + (range_start(cc, I, G) >= it0 ? 0 : 1);
+            bulk_g2s(tileB + (size_t)idx * pt * BM * 4, a.part + (size_t)sl * BN * BM + (size_t)p0 * BM,
+                     (uint32_t)(pt * BM * 4), &bar.red);
+            ++idx;
+          }
+        }
+        mbar_wait(&bar.red, red_phase & 1, &bar.err, a.wait_cycles);
+        ++red_phase;
+#pragma unroll 1
+        for (int c0 = p0 + 16 * g; c0 < p0 + pt; c0 += 32) {
+          uint32_t r[16];
+          if (own_tmem) tmem_ld16(own_dcol + (uint32_t)c0, r);
+          float acc[16];
+#pragma unroll
+          for (int qq = 0; qq < 16; ++qq) acc[qq] = 0.f;
+          int idx = 0;
+          for (int cc = cf; cc <= cl; ++cc) {
+            if (own_tmem && cc == c) {
+#pragma unroll
+              for (int qq = 0; qq < 16; ++qq) acc[qq] += __uint_as_float(r[qq]);
+              continue;
+            }
+            const float* src = ringf + ((size_t)idx * pt + (c0 - p0)) * BM + R;
+#pragma unroll
+            for (int qq = 0; qq < 16; ++qq) acc[qq] += src[qq * BM];
+            ++idx;
+          }
+#pragma unroll
+          for (int qq = 0; qq < 16; ++qq) acc[qq] *= rsc;
+          emit_out(acc, row0, row_base, tok0 + c0);
+        }
+        named_sync(kBothBar, 256);  // the piece is read before the next copy overwrites it
+      }
+      if (leader) {
+        tickets[0] = 0u;  // ready for the next call
+        tickets[1] = 0u;
+      }
+    };
     int64_t i = i0;
     const int64_t iend = i0 + n;
     for (int u = 0; i < iend; ++u) {
@@ -635,25 +719,30 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) mbar_arrive(&bar.dempty[d]);
       } else {
         // Part of a shared tile (CTAs cf .. cl contribute). Each takes a
-        // ticket when its accumulator is final; the last ticket sums the
-        // tile, the others store their partial into their slot (0 for the
-        // segment the CTA's range starts with, 1 for the one it ends with;
-        // [token][row] over the tile's 128 rows) and count it as stored. The
-        // summing CTA keeps its own part in tensor memory and waits (bounded)
-        // only for CTAs that hold a ticket, i.e. that are resident and only
-        // storing. Sums run in contributor order, so the result does not
-        // depend on which CTA sums.
+        // ticket when its accumulator is final (acquire-release add). The
+        // last ticket sums the tile: at once when this is the CTA's last
+        // segment (its activation ring is then idle; its own part stays in
+        // tensor memory), else at the end of its range. Every other part is
+        // stored into its CTA's slot (0 for the segment the CTA's range starts
+        // with, 1 for the one it ends with; [token][row] over the tile's 128
+        // rows) and counted as stored (release add). The summing CTA waits
+        // (bounded) only for parts of CTAs that hold a ticket, i.e. that are
+        // resident and only storing.
         const int64_t it0 = (int64_t)t * nk;
         const int cf = cta_of(it0, I, G), cl = cta_of(it0 + nk - 1, I, G);
         unsigned* tickets = a.count + 2 * (size_t)t;
-        unsigned* stored = tickets + 1;
         if (leader) bar.last = atom_add_acq_rel_gpu(tickets, 1u) == (unsigned)(cl - cf) ? 1u : 0u;
         named_sync(kBothBar, 256);
         const bool last = bar.last != 0;
         named_sync(kBothBar, 256);  // bar.last is reused by the next shared tile
-        if (!last) {
+        if (last && i == iend) {
+          sum_tile(t, dcol);
+          asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&bar.dempty[d]);
+        } else {
           const int slot = 2 * c + (i0 >= it0 ? 0 : 1);
-          float* P = a.part + (size_t)slot * BN * BM;
+          float* Pp = a.part + (size_t)slot * BN * BM;
           uint32_t r[16];
           if (16 * g < BN) tmem_ld16(dcol + (uint32_t)(16 * g), r);
 #pragma unroll 1
@@ -662,7 +751,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int qq = 0; qq < 16; ++qq) v[qq] = __uint_as_float(r[qq]);
             if (c0 + 32 < BN) tmem_ld16_nowait(dcol + (uint32_t)(c0 + 32), r);
-            emit(v, P, c0, 0, 0);
+            emit(v, Pp, c0, 0, 0);
             tmem_wait_ld();
           }
           asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -675,91 +764,18 @@ __global__ void __launch_bounds__(kThreads, 1)
             asm volatile("fence.proxy.async.global;" ::: "memory");
           }
           named_sync(kBothBar, 256);
-          if (leader) red_release_gpu(stored, 1u);
-        } else {
-          const int others = cl - cf;
           if (leader) {
-            const long long w0 = clock64();
-            while (ld_acquire_gpu(stored) < (unsigned)others) {
-              if (clock64() - w0 > a.wait_cycles) {
-                atomicOr(&bar.err, 1u);
-                break;
-              }
-            }
-          }
-          named_sync(kBothBar, 256);
-          // The other partials: copied into the activation ring when this is
-          // the CTA's last segment (every stage consumed), in pieces of PT
-          // tokens; else read from global memory.
-          int PT = (int)((int64_t)kStages * kTileB / ((int64_t)others * BM * 4)) / 16 * 16;
-          if (PT > BN) PT = BN;
-          const bool use_ring = i == iend && PT >= 16;
-          const float* ringf = reinterpret_cast<const float*>(tileB);
-#pragma unroll 1
-          for (int p0 = 0; p0 < BN; p0 += (use_ring ? PT : BN)) {
-            const int pt = use_ring ? (BN - p0 < PT ? BN - p0 : PT) : BN;
-            if (use_ring) {
-              if (leader) {
-                // The partials were written by other CTAs.
-                asm volatile("fence.proxy.async.global;" ::: "memory");
-                mbar_expect_tx(&bar.red, (uint32_t)(others * pt * BM * 4));
-                int idx = 0;
-                for (int cc = cf; cc <= cl; ++cc) {
-                  if (cc == c) continue;
-                  const int sl = 2 * cc + (range_start(cc, I, G) >= it0 ? 0 : 1);
-                  bulk_g2s(tileB + (size_t)idx * pt * BM * 4, a.part + (size_t)sl * BN * BM + (size_t)p0 * BM,
-                           (uint32_t)(pt * BM * 4), &bar.red);
-                  ++idx;
-                }
-              }
-              mbar_wait(&bar.red, red_phase & 1, &bar.err, a.wait_cycles);
-              ++red_phase;
-            }
-#pragma unroll 1
-            for (int c0 = p0 + 16 * g; c0 < p0 + pt; c0 += 32) {
-              uint32_t r[16];
-              tmem_ld16(dcol + (uint32_t)c0, r);
-              float acc[16];
-#pragma unroll
-              for (int qq = 0; qq < 16; ++qq) acc[qq] = 0.f;
-              int idx = 0;
-              for (int cc = cf; cc <= cl; ++cc) {
-                if (cc == c) {
-#pragma unroll
-                  for (int qq = 0; qq < 16; ++qq) acc[qq] += __uint_as_float(r[qq]);
-                  continue;
-                }
-                if (use_ring) {
-                  const float* src = ringf + ((size_t)idx * pt + (c0 - p0)) * BM + R;
-#pragma unroll
-                  for (int qq = 0; qq < 16; ++qq) acc[qq] += src[qq * BM];
-                } else {
-                  const int sl = 2 * cc + (range_start(cc, I, G) >= it0 ? 0 : 1);
-                  const float* src = a.part + ((size_t)sl * BN + c0) * BM + R;
-                  float pv[16];
-#pragma unroll
-                  for (int qq = 0; qq < 16; ++qq) pv[qq] = __ldcg(src + (size_t)qq * BM);
-#pragma unroll
-                  for (int qq = 0; qq < 16; ++qq) acc[qq] += pv[qq];
-                }
-                ++idx;
-              }
-#pragma unroll
-              for (int qq = 0; qq < 16; ++qq) acc[qq] *= rsc;
-              emit_out(acc, row0, row_base, tok0 + c0);
-            }
-            if (use_ring) named_sync(kBothBar, 256);  // the piece is read before the next copy overwrites it
-          }
-          asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&bar.dempty[d]);
-          if (leader) {
-            tickets[0] = 0u;  // ready for the next call
-            stored[0] = 0u;
+            red_release_gpu(tickets + 1, 1u);
+            if (last) bar.pend[bar.npend++] = (uint32_t)t;
           }
         }
       }
     }
+    // A shared tile whose last ticket this CTA took before its last segment:
+    // every part (its own too) is in the slots now that the ring is idle.
+    named_sync(kBothBar, 256);
+    const int npend = (int)bar.npend;
+    for (int pi = 0; pi < npend; ++pi) sum_tile((int)bar.pend[pi], 0xFFFFFFFFu);
     if (issuer) bulk_wait_all();  // every store has been performed before the CTA exits
   }
 
@@ -834,12 +850,16 @@ int prefill_grid(const SignMatrix& sm, int64_t T, int num_sms, bool split) {
   const double t_stage = (double)(bkk / 16) * 134.0 + 150.0;  // cycles: MMAs, barrier check, commit
   const double t_fixed = 4000.0 + 45.0 * (double)bn;           // fill, epilogue of a tile
   const double part_cycles = (double)bn * BM * 4 / 20.0;       // reading one partial tile
+  // The summing CTA copies 16 tokens of every part into its activation ring.
+  const int64_t ring = (int64_t)(bn == 256 ? 3 : 8) * bn * bkk * 2;
+  const int64_t max_parts = ring / (16 * BM * 4);
   int64_t best_g = 1;
   double best = 1e300;
   for (int64_t g = 1; g <= num_sms && g <= iters; ++g) {
     const int64_t per = (iters + g - 1) / g;  // stages of the busiest CTA
     int64_t parts = 1;                        // CTAs sharing one tile (at most)
     if (per % nk != 0 || (iters % g) != 0) parts = per >= nk ? 2 : (nk + per - 1) / per + 1;
+    if (parts > max_parts) continue;
     const double cost =
         (double)per * t_stage + t_fixed + (parts > 1 ? 3000.0 + (double)(parts - 1) * part_cycles : 0.0);
     if (cost < best * 0.995) {  // prefer fewer CTAs on ties

@@ -339,8 +339,8 @@ def test_prefill_full_size_sampled_rows(P, m, n):
 
 @pytest.mark.parametrize("m,n,r,tokens", [(1024, 8192, 892, 64), (4096, 4096, 2028, 20), (1000, 700, 321, 33)])
 def test_prefill_short_pass_split_k(P, m, n, r, tokens):
-    """Short passes (few row blocks x token tiles) split K over a cluster of
-    2-8 CTAs and sum the partial tiles through distributed shared memory."""
+    """Short passes (few row blocks x token tiles): the persistent grid splits
+    K, so tiles are shared by several CTAs and summed from their partials."""
     d = synth.layer_words(8100 + m + tokens, m, n, r, tokens, outlier_frac=0.01)
     layer = words_layer(P, d, m, n, r, any_rank=r > O.rank_for_budget(m, n, 1))
     for out_dtype in (torch.float32, torch.float16):
@@ -348,6 +348,51 @@ def test_prefill_short_pass_split_k(P, m, n, r, tokens):
         rows = np.sort(synth.rng(6).choice(m, size=min(m, 128), replace=False))
         ref = O.forward_from_packed(d["Uw"], d["Vw"], d["a"], d["s"], d["b"], d["x"], m, n, r, rows=rows)
         assert O.rowwise_rel_err(y[:, rows], ref) <= TOL, out_dtype
+    layer.free()
+
+
+# Cases chosen (with the host's grid model) to cover each path of the
+# persistent prefill kernel: tiles of 32, 64, 128 and 256 tokens; tiles
+# shared by 2, 3, 4 and 8 CTAs, summed in 2-4 pieces of the activation ring;
+# two accumulators (tiles of <= 128 tokens) and one (256); both GEMMs
+# shared; ragged rows, columns and tokens; whole tiles only.
+STREAM_K_CASES = [
+    (1024, 8192, 910, 512),   # GEMM 1: 256-token tiles shared by 4 CTAs, 3 ring pieces
+    (700, 900, 333, 17),      # GEMM 1: 32-token tiles shared by 3 CTAs, 2 pieces
+    (4096, 4096, 2028, 100),  # both GEMMs: 128-token tiles shared by 4 CTAs
+    (1024, 4096, 800, 300),   # 256-token tiles shared by 2 CTAs, a ragged second token tile
+    (2048, 1536, 700, 64),    # 64-token tiles shared by 3 CTAs
+    (384, 5000, 300, 200),    # ragged K (5000), 3 CTAs per tile
+    (1024, 8192, 892, 64),    # 64-token tiles shared by 8 CTAs, 4 ring pieces
+    (512, 3000, 400, 130),    # whole tiles only
+    (3000, 512, 300, 129),    # whole tiles, ragged rows
+]
+
+
+@pytest.mark.parametrize("m,n,r,tokens", STREAM_K_CASES)
+def test_prefill_stream_k_paths(P, m, n, r, tokens):
+    d = synth.layer_words(8300 + m + n + tokens, m, n, r, tokens, outlier_frac=0.01)
+    layer = words_layer(P, d, m, n, r, any_rank=True)
+    rows = np.sort(synth.rng(7).choice(m, size=min(m, 160), replace=False))
+    ref = O.forward_from_packed(d["Uw"], d["Vw"], d["a"], d["s"], d["b"], d["x"], m, n, r, rows=rows)
+    for out_dtype in (torch.float32, torch.float16):
+        y = run_gpu(layer, d["x"], n, out_dtype)
+        assert O.rowwise_rel_err(y[:, rows], ref) <= TOL, out_dtype
+    layer.free()
+
+
+@pytest.mark.parametrize("m,n,r,tokens", [(1024, 8192, 910, 512), (700, 900, 333, 17), (4096, 4096, 2028, 100),
+                                          (1024, 8192, 892, 64)])
+def test_prefill_stream_k_integer_bit_exact_and_deterministic(P, m, n, r, tokens):
+    # Shared tiles are summed in contributor order whichever CTA counts last:
+    # with integer inputs every partial and sum is exact (bit-for-bit with
+    # the oracle), and repeated calls give identical bits.
+    d = synth.integer_layer(4242 + m + tokens, m, n, r, tokens)
+    layer = signs_layer(P, d, any_rank=True)
+    y0 = run_gpu(layer, d["x"], n, torch.float32)
+    np.testing.assert_array_equal(y0, oracle_from_signs(d, n))
+    for _ in range(2):
+        np.testing.assert_array_equal(run_gpu(layer, d["x"], n, torch.float32), y0)
     layer.free()
 
 
