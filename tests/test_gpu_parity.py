@@ -396,6 +396,20 @@ def test_prefill_stream_k_integer_bit_exact_and_deterministic(P, m, n, r, tokens
     layer.free()
 
 
+def test_prefill_two_passes(P):
+    """More than 2048 tokens: passes of 2048 (tiles of 256) and a tail pass of
+    52 (tiles of 64), the second writing at a token offset."""
+    m, n, r, tokens = 1024, 1536, 600, 2100
+    d = synth.layer_words(8500, m, n, r, tokens, outlier_frac=0.01)
+    layer = words_layer(P, d, m, n, r, any_rank=True)
+    rows = np.sort(synth.rng(8).choice(m, size=128, replace=False))
+    ref = O.forward_from_packed(d["Uw"], d["Vw"], d["a"], d["s"], d["b"], d["x"], m, n, r, rows=rows)
+    for out_dtype in (torch.float32, torch.float16):
+        y = run_gpu(layer, d["x"], n, out_dtype)
+        assert O.rowwise_rel_err(y[:, rows], ref) <= TOL, out_dtype
+    layer.free()
+
+
 @pytest.mark.parametrize("m,n,r,tokens", [(128, 2048, 128, 64), (256, 1024, 256, 17)])
 def test_prefill_split_k_integer_bit_exact(P, m, n, r, tokens):
     # The split-K partials are summed in a fixed order; with integer inputs
