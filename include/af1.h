@@ -318,7 +318,10 @@ AF1_API int af1_static_status(void* stream);
 
 /* Synchronize `stream` and report the status word the kernels keep in a
  * workspace: AF1_OK, or AF1_ERR_TIMEOUT if a bounded device-side wait gave
- * up since the workspace was last cleared (the word is then reset to 0). */
+ * up since the workspace was last cleared (the word is then reset to 0).
+ * After AF1_ERR_TIMEOUT the outputs of the calls since the last check are
+ * undefined and other bookkeeping words (the prefill's per-tile counters)
+ * may be left non-zero: zero-fill the whole workspace before reusing it. */
 AF1_API int af1_workspace_status(void* workspace, void* stream);
 
 /* Budget of every bounded device-side wait (mbarrier phases, dependency
