@@ -45,6 +45,9 @@ DECODE_TRAFFIC_B1_PER_LAYER = 28145408
 # step's algorithmic bytes (ncu, profiles/lut_kernel_llama3_8b_hisa_b1.md);
 # a full step's traffic is this ratio times its algorithmic bytes.
 DECODE_TRAFFIC_RATIO_HISA_B1 = 170377216 / 164560648
+# The same on the grouped schedule (q|k|v and gate|up as one multi-layer call
+# each): ncu, profiles/lut_kernel_llama3_8b_hisa_b1_group.md.
+DECODE_TRAFFIC_RATIO_HISA_B1_GROUP = 169385216 / 164560648
 TC_DECODE = False  # set from --tc-decode
 
 
@@ -62,11 +65,13 @@ def parse():
                    help="decode: config 1 (1-16 tokens); prefill: config 2 (2048 tokens, tensor cores)")
     p.add_argument("--tokens", type=int, default=2048, help="prefill tokens per call")
     p.add_argument("--no-graph", action="store_true", help="eager launches instead of a CUDA graph (for profilers)")
-    p.add_argument("--schedule", choices=["dag", "serial", "group", "step"], default="dag",
+    p.add_argument("--schedule", choices=["dag", "serial", "group", "step"], default=None,
                    help="dag: a decoder layer's independent linears (q/k/v, gate/up) on parallel streams; "
                         "serial: all 7 linears chained on one stream; group: q|k|v and gate|up as one "
                         "af1_linear_forward_multi call each (shared input), one stream; step: the whole step "
-                        "as one persistent launch (af1_step_run) with the DAG's level order")
+                        "as one persistent launch (af1_step_run) with the DAG's level order. Default: group for "
+                        "decode passes of 1-2 tokens, dag otherwise (the faster of the two measured on GB300: "
+                        "1 token 1.32 vs 1.43 ms per step, 16 tokens 6.39 vs 5.30)")
     p.add_argument("--ranks", choices=["hisa", "uniform"], default="hisa",
                    help="decode stack ranks: hisa = 1.0-BPW rank x U(0.7, 1.3), renormalised to 1.0 BPW over the "
                         "stack (the default workload); uniform = every matrix at its 1.0-BPW rank")
@@ -79,7 +84,10 @@ def parse():
                         "measurement and profiling, e.g. with --no-graph under ncu)")
     p.add_argument("--tc-decode", action="store_true",
                    help="create layers with AF1_FLAG_TC_DECODE (tensor-core decode kernel instead of lookup tables)")
-    return p.parse_args()
+    a = p.parse_args()
+    if a.schedule is None:
+        a.schedule = "group" if (a.workload == "decode" and a.batch <= 2) else "dag"
+    return a
 
 
 def workload_ranks(args, rank_fn=None, bits_fn=None):
@@ -502,6 +510,18 @@ def step_launches(objs, b, schedule):
     return total
 
 
+def group_step(P, views, stream, ws, ws_multi):
+    """One decode step over views = [(layer, x, y)] * 7 per decoder layer with
+    q|k|v and gate|up each as one af1_linear_forward_multi call (the decoder's
+    shared inputs), all on one stream."""
+    for li in range(len(views) // 7):
+        q, k, v, o, gate, up, down = views[7 * li:7 * li + 7]
+        P.forward_multi([q[0], k[0], v[0]], q[1], [q[2], k[2], v[2]], ws_multi, stream=stream)
+        o[0].forward_into(o[1], o[2], ws, stream=stream)
+        P.forward_multi([gate[0], up[0]], gate[1], [gate[2], up[2]], ws_multi, stream=stream)
+        down[0].forward_into(down[1], down[2], ws, stream=stream)
+
+
 def dag_step(torch, views, stream, side, ws, ws_side):
     """One decode step over views = [(layer, x, y)] * 7 per decoder layer on
     the decoder's dependency DAG: per layer q | k | v in parallel, then o, then
@@ -642,11 +662,22 @@ def stack_other_ranks(P, torch, peaks, stream, steps, args):
     side = [torch.cuda.Stream(), torch.cuda.Stream()]
     ws_side = [torch.zeros_like(ws), torch.zeros_like(ws)]
     views = list(zip(layers, xs, ys))
-    ms_dag = time_graph(torch, lambda: dag_step(torch, views, stream, side, ws, ws_side), stream,
-                        max(5, min(steps, 20)))
+    group = args.schedule == "group"
+    if group:
+        ws_multi = torch.zeros(max(max(P.workspace_bytes_multi([layers[7 * li + j] for j in (0, 1, 2)], 1),
+                                       P.workspace_bytes_multi([layers[7 * li + j] for j in (4, 5)], 1))
+                                   for li in range(LAYERS)), dtype=torch.uint8, device="cuda")
+
+        def run():
+            group_step(P, views, stream, ws, ws_multi)
+    else:
+        def run():
+            dag_step(torch, views, stream, side, ws, ws_side)
+    ms_dag = time_graph(torch, run, stream, max(5, min(steps, 20)))
     alg = sum(algorithmic_bytes(m, n, r, 1) for (m, n), r in zip(mn, ranks))
     bits = sum(P.storage_bits(m, n, r) for (m, n), r in zip(mn, ranks))
-    out = {"workload": f"32 x 7 LLaMA-3-8B linears, {other} ranks, 1 token, decoder DAG, CUDA graph",
+    out = {"workload": f"32 x 7 LLaMA-3-8B linears, {other} ranks, 1 token, "
+                       f"{'q|k|v and gate|up as grouped calls, one stream' if group else 'decoder DAG'}, CUDA graph",
            "ranks": other, "ms_per_token": ms_dag, "tokens_per_s": 1e3 / ms_dag,
            "us_per_linear": ms_dag * 1e3 / len(mn), "bpw": bits / sum(m * n for (m, n) in mn),
            "rank_min": min(ranks), "rank_max": max(ranks), "achieved_gbs": alg / (ms_dag * 1e-3) / 1e9,
@@ -772,12 +803,7 @@ def main():
     def step_group():
         # q, k, v read one input and gate, up another (the decoder's shared
         # activations): one multi-layer call each.
-        for li in range(len(views) // 7):
-            q, k, v, o, gate, up, down = views[7 * li:7 * li + 7]
-            P.forward_multi([q[0], k[0], v[0]], q[1], [q[2], k[2], v[2]], ws_multi, stream=stream)
-            o[0].forward_into(o[1], o[2], ws, stream=stream)
-            P.forward_multi([gate[0], up[0]], gate[1], [gate[2], up[2]], ws_multi, stream=stream)
-            down[0].forward_into(down[1], down[2], ws, stream=stream)
+        group_step(P, views, stream, ws, ws_multi)
 
     def make_graph(fn):
         with torch.cuda.stream(stream):
@@ -944,7 +970,12 @@ def main():
             if b == 1 and not TC_DECODE and args.schedule == "dag":
                 traffic = (DECODE_TRAFFIC_B1_PER_LAYER * args.layers if args.ranks == "uniform"
                            else int(round(DECODE_TRAFFIC_RATIO_HISA_B1 * alg)))
+            elif (b == 1 and not TC_DECODE and args.schedule == "group" and args.ranks == "hisa"
+                  and DECODE_TRAFFIC_RATIO_HISA_B1_GROUP is not None):
+                traffic = int(round(DECODE_TRAFFIC_RATIO_HISA_B1_GROUP * alg))
             kname = ("af1_step_run (one persistent step_kernel launch per step)" if args.schedule == "step" else
+                     "af1_linear_forward_multi / af1_linear_forward (two lookup-table kernels per call, "
+                     "lut_kernel<1|2>)" if args.schedule == "group" else
                      "af1_linear_forward (two lookup-table kernels per call, lut_kernel<1|2>, stream_kernel<1|2> "
                      "for the largest matrices)")
             roof = {"bound": "hbm", "kernel": kname,

@@ -307,10 +307,52 @@ int plan_one(const SignMatrix& sm, int T, int sms, int max_smem, int* cpc_out, i
 
 }  // namespace
 
+// Several problems in one launch: the cluster size that keeps every CTA of
+// the group resident (one wave), preferably with at least two CTAs per SM
+// (the lookups need them to hide their latency: one CTA per SM made the
+// gate | up first phase 5 -> 6 us), and minimises the busiest SM's load,
+// ceil(CTAs / SMs) x (chunks per CTA + 2, the fixed cost of a CTA in chunk
+// units); 0 if no size fits one wave. (Each problem's own split, as for one
+// problem, made the gate | up launch of a LLaMA-3-8B layer 672 CTAs for 608
+// resident slots: two waves, 12 us for its second phase.)
+int plan_group_ks(const SignMatrix* sm, int count, int T, int sms, int max_smem) {
+  const int Tg = T < kGroupTokens ? T : kGroupTokens;
+  const int groups = (T + kGroupTokens - 1) / kGroupTokens;
+  const int64_t per_sm_smem = (int64_t)max_smem + 1024;  // the SM's shared memory (a CTA may take all but 1 KB)
+  int best_ks = 0;
+  int64_t best = 0;
+  bool best_two = false;  // the best so far has at least two CTAs per SM
+  for (int ks = 1; ks <= kMaxKS; ++ks) {
+    int64_t ctas = 0;
+    int cpc_max = 0, need = 0;
+    bool ok = true;
+    for (int i = 0; i < count; ++i) {
+      const int cpc = (sm[i].NCH + ks - 1) / ks;
+      if (cpc > kMaxCPC) ok = false;
+      const int nd = lut_smem(cpc, ks, Tg, pairs_for(Tg)).total;
+      if (nd > need) need = nd;
+      if (cpc > cpc_max) cpc_max = cpc;
+      ctas += (int64_t)sm[i].RB * groups * ks;
+    }
+    if (!ok || need > max_smem) continue;
+    int64_t resident = per_sm_smem / need;
+    if (resident > 4) resident = 4;  // __launch_bounds__(256, 4)
+    if (ctas > resident * sms) continue;
+    const int64_t load = ((ctas + sms - 1) / sms) * (cpc_max + 2);
+    const bool two = ctas >= 2 * (int64_t)sms;
+    if (best_ks == 0 || (two && !best_two) || (two == best_two && load < best)) {
+      best = load;
+      best_ks = ks;
+      best_two = two;
+    }
+  }
+  return best_ks;
+}
+
 // One problem: its own split. Several (layers sharing their input, one
-// launch): the largest of their splits' cluster sizes for all, each problem
-// cutting its columns into that many slices (the last CTAs of a problem with
-// fewer chunks get none).
+// launch): the cluster size of plan_group_ks, or failing that the largest of
+// their own splits' cluster sizes; each problem cuts its columns into that
+// many slices (the last CTAs of a problem with fewer chunks get none).
 LutPlan plan_lut(const SignMatrix* sm, int count, int T, int num_sms, int max_smem) {
   LutPlan p;
   if (count < 1 || count > kMaxGroup || T < 1 || T > kMaxPassTokens) return p;
@@ -323,6 +365,10 @@ LutPlan plan_lut(const SignMatrix* sm, int count, int T, int num_sms, int max_sm
     const int k = plan_one(sm[i], T, sms, max_smem, &cpc, &smem);
     if (k == 0) return p;
     if (k > KS) KS = k;
+  }
+  if (count > 1) {
+    const int g = plan_group_ks(sm, count, T, sms, max_smem);
+    if (g > 0) KS = g;
   }
   int smem = 0;
   for (int i = 0; i < count; ++i) {
