@@ -288,7 +288,7 @@ __device__ __forceinline__ int64_t range_start(int c, int64_t I, int G) { return
 template <bool GEMM1, int BN>
 __global__ void __launch_bounds__(kThreads, 1)
     prefill_kernel(const __grid_constant__ CUtensorMap act_map, const __grid_constant__ CUtensorMap out_map,
-                   const PrefillArgs a) {
+                   const __grid_constant__ CUtensorMap out_map32, const PrefillArgs a) {
   constexpr int BK = bk<BN>();
   constexpr int kTileB = tile_b_bytes<BN>();
   constexpr int kBoxBytes = BN * BOX * 2;
@@ -700,7 +700,41 @@ __global__ void __launch_bounds__(kThreads, 1)
       const float rsc = frow < tm.R ? __half2float(a.rowscale[frow]) : 0.f;
       const int64_t row_base = (int64_t)rb * BM;
       const int64_t row0 = row_base + q * 32;  // first row of this warp's quadrant
-      if (ka == 0 && kb == nk) {
+      if (ka == 0 && kb == nk && tma_out && !a.out_f32 && BN >= 32) {
+        // A whole tile with FP16 output: 32-token chunks (alternating between
+        // the groups), staged as two 16-token halves and written by one TMA
+        // store (half the barriers, waits and store issues per token of
+        // 16-token chunks); the next half's read-back is in flight while one
+        // is staged.
+        __half* hb = reinterpret_cast<__half*>(buf);
+        uint32_t r[16];
+        if (32 * g < BN) tmem_ld16(dcol + (uint32_t)(32 * g), r);
+#pragma unroll 1
+        for (int c0 = 32 * g; c0 < BN; c0 += 64) {
+          if (issuer) bulk_wait_read0();  // the group's previous store has read the buffer
+          named_sync(gbar, 128);
+#pragma unroll 1
+          for (int h = 0; h < 2; ++h) {
+            float v[16];
+#pragma unroll
+            for (int qq = 0; qq < 16; ++qq) v[qq] = __uint_as_float(r[qq]) * rsc;
+            const int next = h == 0 ? c0 + 16 : c0 + 64;
+            if (next < BN) tmem_ld16_nowait(dcol + (uint32_t)next, r);
+#pragma unroll
+            for (int qq = 0; qq < 16; ++qq) hb[(16 * h + qq) * BM + R] = __float2half_rn(v[qq]);
+            if (next < BN) tmem_wait_ld();
+          }
+          asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+          named_sync(gbar, 128);
+          if (issuer) {
+            tma_store_2d(&out_map32, buf, (int)row_base, (int)(tok0 + c0));
+            bulk_commit();
+          }
+        }
+        asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bar.dempty[d]);
+      } else if (ka == 0 && kb == nk) {
         // A whole tile: scale and store this group's chunks; the next
         // chunk's read-back is in flight while this one is staged.
         uint32_t r[16];
@@ -871,15 +905,16 @@ int prefill_grid(const SignMatrix& sm, int64_t T, int num_sms, bool split) {
 }
 
 // Tensor map of the output [tokens][ld] (FP16 or FP32) with `rows` valid
-// columns: boxes of 128 columns x 16 tokens, no swizzle; stores past the
+// columns: boxes of 128 columns x box_tokens tokens, no swizzle; stores past the
 // matrix are dropped.
-cudaError_t make_out_map(CUtensorMap* map, void* base, int64_t tokens, int64_t rows, int64_t ld, bool f32) {
+cudaError_t make_out_map(CUtensorMap* map, void* base, int64_t tokens, int64_t rows, int64_t ld, bool f32,
+                         int box_tokens) {
   PFN_cuTensorMapEncodeTiled_v12000 fn = encode_fn();
   if (fn == nullptr) return cudaErrorNotSupported;
   const int64_t es = f32 ? 4 : 2;
   cuuint64_t dims[2] = {(cuuint64_t)rows, (cuuint64_t)tokens};
   cuuint64_t strides[1] = {(cuuint64_t)(ld * es)};
-  cuuint32_t box[2] = {(cuuint32_t)BM, 16u};
+  cuuint32_t box[2] = {(cuuint32_t)BM, (cuuint32_t)box_tokens};
   cuuint32_t estr[2] = {1, 1};
   CUresult r = fn(map, f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, base, dims, strides,
                   box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
@@ -889,12 +924,14 @@ cudaError_t make_out_map(CUtensorMap* map, void* base, int64_t tokens, int64_t r
 
 template <bool GEMM1, int BN>
 cudaError_t launch_gemm_bn(const PrefillArgs& a, const __half* act, int64_t ld_act, int grid, cudaStream_t st) {
-  CUtensorMap map, omap;
+  CUtensorMap map, omap, omap32;
   cudaError_t e = make_act_map(&map, act, a.tokens, a.sm.C, ld_act, BN);
   if (e != cudaSuccess) return e;
   std::memset(&omap, 0, sizeof(omap));
+  std::memset(&omap32, 0, sizeof(omap32));
   if (a.out_vec) {
-    e = make_out_map(&omap, a.out, a.tokens, a.sm.R, a.ld_out, a.out_f32 != 0);
+    e = make_out_map(&omap, a.out, a.tokens, a.sm.R, a.ld_out, a.out_f32 != 0, 16);
+    if (e == cudaSuccess && !a.out_f32) e = make_out_map(&omap32, a.out, a.tokens, a.sm.R, a.ld_out, false, 32);
     if (e != cudaSuccess) return e;
   }
   auto kern = prefill_kernel<GEMM1, BN>;
@@ -911,7 +948,7 @@ cudaError_t launch_gemm_bn(const PrefillArgs& a, const __half* act, int64_t ld_a
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, kern, map, omap, a);
+  return cudaLaunchKernelEx(&cfg, kern, map, omap, omap32, a);
 }
 
 template <bool GEMM1>
