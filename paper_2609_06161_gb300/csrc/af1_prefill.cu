@@ -6,49 +6,52 @@
 //   GEMM2: y[t][i] = a_i * sum_k U[i][k] * H[t][k]          (U, m x r)
 //
 // Output tiles are 128 features x BN tokens (BN = 16, 32, 64, 128 or 256),
-// with K cut into stages of 64. The kernel is persistent and stream-K: the grid
-// (at most one CTA per SM) splits the (tile, K-stage) iterations into equal
-// contiguous ranges, so a CTA runs a few whole tiles plus, at either end of
-// its range, part of a tile shared with its neighbour. A shared tile's
-// contributors store FP32 partial tiles in the workspace and count
-// themselves on the tile's counter; the last to arrive sums the partials in
-// a fixed order (so results do not depend on timing), applies the feature
-// scale, stores the output and clears the counter. No CTA waits for
-// another. Without room for the partials (the built-in-scratch entry) the
-// grid is one CTA per tile.
+// with K cut into stages of 128 (BN = 256) or 64. The kernel is persistent
+// and stream-K: the grid (at most one CTA per SM, chosen on the host by a
+// cost model) splits the (tile, K-stage) iterations into equal contiguous
+// ranges, so a CTA runs some whole tiles plus, at either end of its range,
+// part of a tile shared with its neighbours. A shared tile's contributors
+// take tickets when their part is final; all but the last store FP32
+// partial tiles in the workspace, and the last sums the parts in a fixed
+// contributor order (results do not depend on timing), applies the feature
+// scale and stores the output (see sum_tile). No CTA waits for another that
+// may not be running. Without room for the partials (the built-in-scratch
+// entry) the grid is one CTA per tile.
 //
 // Roles of the 18 warps of a CTA, over the CTA's stages in order:
-//   * warp 0, one thread: copies each stage's packed signs (128 rows x 2
-//     words: 1 KB contiguous in the row-block layout) and, for GEMM1, its 64
-//     column scales into a ring of 14 small slots (cp.async.bulk), up to 14
-//     stages ahead and independent of the MMA (with the signs loaded by the
-//     expanders one stage ahead, each stage waited about 1,500 cycles on the
-//     load against 600 of MMA work); then the BN x 64 FP16 activation tile
-//     (B) of the stage by TMA (cp.async.bulk.tensor, 128-byte swizzle, zero
-//     fill past the tokens / columns) into a ring of 8 stages (6 for BN =
-//     256);
+//   * warp 0, one thread: copies each stage's packed signs (the row block's
+//     words of the stage, 1-2 KB contiguous in the row-block layout) and,
+//     for GEMM1, its column scales into a ring of small slots
+//     (cp.async.bulk), 6-14 stages ahead and independent of the MMA (with
+//     the signs loaded by the expanders one stage ahead, each stage waited
+//     about 1,500 cycles on the load); then the stage's FP16 activation
+//     tile(s) (B, BN x 64 per box) by TMA (cp.async.bulk.tensor, 128-byte
+//     swizzle, zero fill past the tokens / columns) into a ring of 3 stages
+//     of 64 KB (BN = 256) or 8;
 //   * warps 4-11 expand the signs into FP16 (+-b_j for GEMM1, +-1 for GEMM2:
 //     exact) and store them into a ring of A buffers (one per stage) in
 //     tensor memory (tcgen05.st; warp w writes rows 32 (w % 4) .. +31, one
 //     row per thread = tensor-memory lane, and half (w - 4) / 4 of the
-//     stage's columns);
-//     A in tensor memory leaves shared-memory bandwidth to B;
-//   * warp 1, one thread: four tcgen05.mma.kind::f16 per stage (K = 16,
+//     stage's columns); A in tensor memory leaves shared-memory bandwidth to
+//     B;
+//   * warp 1, one thread: the stage's tcgen05.mma.kind::f16 (K = 16 each,
 //     N = BN, A from tensor memory, B from shared memory) into an
-//     accumulator (D, FP32, BN columns). Tiles of up to 128 tokens alternate
-//     between two accumulators, so the epilogue of one tile overlaps the
-//     MMAs of the next; tiles of 256 have one (two would leave no tensor
-//     memory for A), and the MMAs of the next tile wait for its read-back.
-//     Measured: this one thread needs about 175 cycles per MMA whatever N,
-//     so N = 128 tiles ran at half the rate of N = 256;
+//     accumulator (D, FP32, BN columns), after one wait on the stage's
+//     barrier (completed by the activation copy and the 8 expander warps),
+//     then one commit. Measured: this thread needs 134 cycles per MMA, N =
+//     128 or 256 alike, plus 77 per commit and 67 per barrier check, and the
+//     tensor pipe idles meanwhile; hence stages of 128 and tiles of 256.
+//     Tiles of up to 128 tokens alternate between two accumulators, so the
+//     epilogue of one tile overlaps the MMAs of the next; tiles of 256 have
+//     one (two would leave no tensor memory for A), and the MMAs of the next
+//     tile wait for its read-back;
 //   * two groups of four warps (12-15; 16, 17, 2, 3) read an accumulator
-//     back (tcgen05.ld) in alternate 16-token chunks, apply the feature
-//     scale and stage each chunk in shared memory, which one thread of the
-//     group writes out with a TMA store (or a bulk copy for a partial tile)
-//     (stores from the warps themselves were latency-bound in the store
-//     queue, and the MMA waits for this read-back when a tile has one
-//     accumulator).
-// All mbarrier waits are bounded; a wait that gives up sets the status word.
+//     back (tcgen05.ld) in alternate chunks (32 tokens for FP16 outputs, 16
+//     for FP32 ones and partial tiles), apply the feature scale and stage
+//     each chunk in shared memory, which one thread of the group writes out
+//     with a TMA store (or a bulk copy for a partial tile) (stores from the
+//     warps themselves were latency-bound in the store queue).
+// All waits are bounded; a wait that gives up sets the status word.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_fp16.h>
