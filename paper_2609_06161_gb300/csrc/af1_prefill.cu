@@ -118,21 +118,46 @@ template <int BN>
 __host__ __device__ constexpr int wslots() {
   return BN == 256 ? 6 : 14;
 }
-// At least 116 KB so that two CTAs never share an SM (each allocates all of
-// its tensor memory).
 // Epilogue staging: two buffers of one 16-token x 128-row chunk (FP32 at
 // most), [token][row].
 constexpr int kEpiStageBytes = 16 * 128 * 4;
+constexpr int kSmemCap = 227 * 1024;  // opt-in shared memory of a CTA
 template <int BN>
-__host__ __device__ constexpr int smem_used() {
+__host__ __device__ constexpr int smem_base() {
   return stages<BN>() * tile_b_bytes<BN>() + wslots<BN>() * wslot_bytes<BN>() + 2 * kEpiStageBytes +
          1024 /* barriers */ + 1024 /* base alignment */;
 }
+// Extra landing space right after the activation ring, for the parts of a
+// shared tile that a CTA sums (the ring alone holds 16 tokens of at most 2-4
+// parts for tiles of 16-32 tokens, and pieces of 16 tokens each paid a
+// round trip): what the CTA's shared memory has left, for tiles of up to
+// 128 tokens. The whole CTA takes the SM anyway (it allocates all of its
+// tensor memory).
+template <int BN>
+__host__ __device__ constexpr int land_bytes() {
+  return BN == 256 ? 0 : (kSmemCap - smem_base<BN>()) / 1024 * 1024;
+}
+// Bytes a summing CTA can copy parts into: the activation ring and the land.
+template <int BN>
+__host__ __device__ constexpr int landing_bytes() {
+  return stages<BN>() * tile_b_bytes<BN>() + land_bytes<BN>();
+}
 template <int BN>
 __host__ __device__ constexpr int smem_bytes() {
-  return smem_used<BN>() < 116 * 1024 ? 116 * 1024 : smem_used<BN>();
+  return smem_base<BN>() + land_bytes<BN>();
 }
-static_assert(smem_used<256>() <= 227 * 1024, "shared memory");
+static_assert(smem_bytes<256>() <= kSmemCap, "shared memory");
+static_assert(smem_bytes<16>() <= kSmemCap && smem_bytes<128>() <= kSmemCap, "shared memory");
+// Host side: landing bytes for a tile width of bn tokens.
+inline int64_t landing_bytes_of(int bn) {
+  switch (bn) {
+    case 16: return landing_bytes<16>();
+    case 32: return landing_bytes<32>();
+    case 64: return landing_bytes<64>();
+    case 128: return landing_bytes<128>();
+    default: return landing_bytes<256>();
+  }
+}
 
 struct PrefillArgs {
   const uint32_t* signs;  // packed signs, af1_layout.h row-block layout
@@ -306,8 +331,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   extern __shared__ uint8_t smem_raw[];
   // 1024-byte alignment for the swizzled operand tiles.
   uint8_t* smem = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-  uint8_t* tileB = smem;
-  uint8_t* wring = smem + kStages * kTileB;
+  uint8_t* tileB = smem;  // activation ring, then the landing space of sum_tile
+  uint8_t* wring = smem + kStages * kTileB + land_bytes<BN>();
   uint8_t* estage = wring + kWSlots * kWSlotBytes;
   PrefillBarriers& bar = *reinterpret_cast<PrefillBarriers*>(estage + 2 * kEpiStageBytes);
 
@@ -631,7 +656,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const float rsc = frow < tm.R ? __half2float(a.rowscale[frow]) : 0.f;
       const int64_t row_base = (int64_t)rb * BM;
       const int64_t row0 = row_base + q * 32;
-      int PT = (int)((int64_t)kStages * kTileB / ((int64_t)copied * BM * 4)) / 16 * 16;
+      int PT = (int)((int64_t)landing_bytes<BN>() / ((int64_t)copied * BM * 4)) / 16 * 16;
       if (PT > BN) PT = BN;
       if (PT < 16) {  // the host's grid keeps the parts within the ring; never taken
         if (leader) atomicOr(&bar.err, 1u);
@@ -888,7 +913,7 @@ int prefill_grid(const SignMatrix& sm, int64_t T, int num_sms, bool split) {
   const double t_fixed = 4000.0 + 45.0 * (double)bn;           // fill, epilogue of a tile
   const double part_cycles = (double)bn * BM * 4 / 20.0;       // reading one partial tile
   // The summing CTA copies 16 tokens of every part into its activation ring.
-  const int64_t ring = (int64_t)(bn == 256 ? 3 : 8) * bn * bkk * 2;
+  const int64_t ring = landing_bytes_of((int)bn);
   const int64_t max_parts = ring / (16 * BM * 4);
   int64_t best_g = 1;
   double best = 1e300;
