@@ -105,6 +105,83 @@ def test_multi_llama_qkv_full_size(P):
         L.free()
 
 
+@pytest.mark.parametrize("specs", [[(200, 77), (100, 40), (100, 40)], [(300, 120), (64, 30)],
+                                   [(256, 200), (129, 60), (64, 33), (1000, 321)]])
+@pytest.mark.parametrize("tokens", [18, 40, 64, 129, 300])
+def test_multi_prefill_matches_oracle(P, specs, tokens):
+    """Passes longer than 16 tokens: each layer runs the stream-K prefill
+    GEMMs from its own workspace slice, all reporting to the first slice's
+    status word (ragged ranks and row counts per layer)."""
+    n = 700
+    ds, layers, x = _group(P, 140 + tokens + len(specs), n, specs, tokens)
+    ys = _run(P, layers, x, n, tokens)
+    for d, y in zip(ds, ys):
+        err = O.rowwise_rel_err(y, oracle_from_signs(d, n))
+        assert err <= TOL, err
+    for L in layers:
+        L.free()
+
+
+@pytest.mark.parametrize("tokens", [17, 100, 257])
+def test_multi_prefill_integer_bit_exact_fp16_out(P, tokens):
+    """Integer-valued layers through the multi-layer call at prefill sizes
+    (every sum exact in FP32, H exact in FP16), FP16 outputs (the 32-token
+    TMA-store chunks), twice: equal bits each time, and equal to the
+    oracle's value rounded to FP16 (|y| stays far below the FP16 range)."""
+    n = 512
+    ds, layers, x = _group(P, 170 + tokens, n, [(300, 200), (130, 100), (64, 40)], tokens, integer=True)
+    y1 = _run(P, layers, x, n, tokens, out_dtype=torch.float16)
+    y2 = _run(P, layers, x, n, tokens, out_dtype=torch.float16)
+    for d, a, b in zip(ds, y1, y2):
+        np.testing.assert_array_equal(a, b)
+        ref = oracle_from_signs(d, n)
+        assert np.abs(ref).max() < 60000
+        np.testing.assert_array_equal(a, ref.astype(np.float16).astype(np.float64))
+    for L in layers:
+        L.free()
+
+
+@pytest.mark.parametrize("tokens", [64, 2048, 2100])
+def test_multi_prefill_matches_single_calls(P, tokens):
+    """The multi-layer call agrees with each layer's own call (up to the
+    rounding of H to FP16 should the stream-K split differ), including a
+    second pass of tokens, and sampled tokens match the oracle."""
+    n = 1024
+    specs = [(1024, 400), (256, 160), (256, 160)]
+    ds, layers, x = _group(P, 190 + tokens, n, specs, tokens)
+    ys = _run(P, layers, x, n, tokens)
+    xt = f16(x).reshape(tokens, n)
+    toks = np.sort(synth.rng(tokens).choice(tokens, size=min(tokens, 64), replace=False))
+    xs = np.asarray(x).reshape(tokens, n)[toks]
+    for L, y, d in zip(layers, ys, ds):
+        y_one = L.forward(xt, out_dtype=torch.float32).double().cpu().numpy()
+        assert O.rowwise_rel_err(y, y_one) <= 1e-3
+        ref = oracle_from_signs(dict(d, x=xs), n)
+        assert O.rowwise_rel_err(y[toks], ref) <= TOL
+    for L in layers:
+        L.free()
+
+
+def test_multi_llama_qkv_prefill_full_size(P):
+    """q, k, v of a LLaMA-3-8B-shaped layer at their 1.0-BPW ranks over a
+    2048-token pass: sampled rows and tokens against the oracle."""
+    n, tokens = 4096, 2048
+    specs = [(4096, O.rank_for_budget(4096, n, 1)), (1024, O.rank_for_budget(1024, n, 1)),
+             (1024, O.rank_for_budget(1024, n, 1))]
+    ds = [synth.layer_words(320 + i, m, n, r, tokens) for i, (m, r) in enumerate(specs)]
+    from tests.af1_cases import words_layer
+    layers = [words_layer(P, d, m, n, r) for d, (m, r) in zip(ds, specs)]
+    ys = _run(P, layers, ds[0]["x"], n, tokens)
+    toks = np.sort(synth.rng(7).choice(tokens, size=24, replace=False))
+    xs = np.asarray(ds[0]["x"]).reshape(tokens, n)[toks].reshape(-1)
+    for d, (m, r), y in zip(ds, specs, ys):
+        rows = np.sort(synth.rng(m).choice(m, size=96, replace=False))
+        ref = O.forward_from_packed(d["Uw"], d["Vw"], d["a"], d["s"], d["b"], xs, m, n, r, rows=rows)
+        assert O.rowwise_rel_err(y[toks][:, rows], ref) <= TOL
+    for L in layers:
+        L.free()
+
+
 def test_multi_errors(P):
     d1 = synth.layer_signs(95, 64, 96, 20, 1)
     d2 = synth.layer_signs(96, 64, 128, 20, 1)
