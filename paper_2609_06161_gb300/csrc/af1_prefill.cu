@@ -455,12 +455,21 @@ __global__ void __launch_bounds__(kThreads, 1)
         const bool seg_end = j == n - 1 || k == nk - 1;
         // MMA kk: K 16 kk .. + 15 of the stage = tensor-memory columns 8 kk ..
         // of its A buffer and, of its activation tile, box kk / 4, 32-byte
-        // step kk % 4 of the swizzled rows.
+        // step kk % 4 of the swizzled rows. The stage's operand addresses are
+        // all formed before its first MMA (the empty asm pins them there):
+        // this thread's issue sets the tensor pipe's pace, and address
+        // arithmetic between two MMAs is a gap in it.
+        constexpr int kMma = BK / 16;
+        uint64_t bdesc[kMma];
+        uint32_t aaddr[kMma];
 #pragma unroll
-        for (int kk = 0; kk < BK / 16 - 1; ++kk) {
-          mma_f16_ts<BN>(d_tmem, tmem + (uint32_t)(ND * BN + s * kACols + kk * 8),
-                         smem_desc(b0 + s * kTileB + (kk / 4) * kBoxBytes + (kk % 4) * 32), !(first && kk == 0));
+        for (int kk = 0; kk < kMma; ++kk) {
+          bdesc[kk] = smem_desc(b0 + s * kTileB + (kk / 4) * kBoxBytes + (kk % 4) * 32);
+          aaddr[kk] = tmem + (uint32_t)(ND * BN + s * kACols + kk * 8);
+          asm volatile("" : "+l"(bdesc[kk]), "+r"(aaddr[kk]));
         }
+#pragma unroll
+        for (int kk = 0; kk < kMma - 1; ++kk) mma_f16_ts<BN>(d_tmem, aaddr[kk], bdesc[kk], !(first && kk == 0));
         // Stage j + 1: its accumulator must be free (with one accumulator
         // that needs this segment's epilogue, so it waits after the commit).
         const bool ahead = j + 1 < n && !(seg_end && ND == 1);
@@ -469,9 +478,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_wait(&bar.dempty[(u + 1) % ND], (((u + 1) / ND) & 1) ^ 1, &bar.err, a.wait_cycles);
           wait_stage(j + 1);
         }
-        constexpr int kl = BK / 16 - 1;
-        mma_f16_ts<BN>(d_tmem, tmem + (uint32_t)(ND * BN + s * kACols + kl * 8),
-                       smem_desc(b0 + s * kTileB + (kl / 4) * kBoxBytes + (kl % 4) * 32), true);
+        mma_f16_ts<BN>(d_tmem, aaddr[kMma - 1], bdesc[kMma - 1], true);
         mma_commit(&bar.empty[s]);
         if (seg_end) mma_commit(&bar.dfull[u % ND]);
         if (j + 1 < n) {
