@@ -48,7 +48,7 @@ DECODE_TRAFFIC_RATIO_HISA_B1 = 170377216 / 164560648
 # The same on the grouped schedule (q|k|v and gate|up as one multi-layer call
 # each): ncu, profiles/lut_kernel_llama3_8b_hisa_b1_group.md.
 DECODE_TRAFFIC_RATIO_HISA_B1_GROUP = 169385216 / 164560648
-TC_DECODE = False  # set from --tc-decode
+DECODE_KERNEL = "auto"  # set from --decode-kernel / --tc-decode
 
 
 def parse():
@@ -83,7 +83,12 @@ def parse():
                         "--steps calls rotating over copies larger than L2; prints one JSON line (per-shape "
                         "measurement and profiling, e.g. with --no-graph under ncu)")
     p.add_argument("--tc-decode", action="store_true",
-                   help="create layers with AF1_FLAG_TC_DECODE (tensor-core decode kernel instead of lookup tables)")
+                   help="create layers with AF1_FLAG_TC_DECODE (the e4m3 tensor-core decode kernel); "
+                        "same as --decode-kernel tc")
+    p.add_argument("--decode-kernel", choices=["auto", "lut", "mma", "tc"], default="auto",
+                   help="decode kernel of the layers: auto (the library's dispatch: lookup tables below 4 tokens, "
+                        "16-bit-operand tensor cores from 4), lut (AF1_FLAG_LUT_DECODE), mma (AF1_FLAG_MMA_DECODE), "
+                        "tc (AF1_FLAG_TC_DECODE)")
     a = p.parse_args()
     if a.schedule is None:
         a.schedule = "group" if (a.workload == "decode" and a.batch <= 2) else "dag"
@@ -275,6 +280,17 @@ SCHEDULES = {"dag": "q|k|v and gate|up on parallel streams (decoder dependency D
              "step": "the whole step as one persistent launch (af1_step_run) in the decoder's level order"}
 
 
+DECODE_KERNEL_NAMES = {"lut": "lookup tables on the CUDA cores",
+                       "mma": "tcgen05 kind::f16 tensor cores (+-b_j FP16 / +-1 BF16 signs)",
+                       "tc": "tcgen05 kind::f8f6f4 tensor cores (e4m3 signs and activation terms)"}
+
+
+def decode_kernel_name(b):
+    if DECODE_KERNEL != "auto":
+        return DECODE_KERNEL_NAMES[DECODE_KERNEL] + " (layer flag)"
+    return DECODE_KERNEL_NAMES[decode_kernel_of(b)] + " (default dispatch)"
+
+
 def config_dict(args):
     if args.workload == "prefill":
         return {"workload": (f"LLaMA-3-8B-shaped AF1 linears (q,k,v,o,gate,up,down at 1.0-BPW ranks) x {args.layers} "
@@ -291,8 +307,7 @@ def config_dict(args):
                          f"/ down 4096x14336), {ranks}, x {args.layers} layers, decode batch {args.batch}, "
                          + SCHEDULES[args.schedule] + ("" if args.no_graph else ", CUDA graph")),
             "batch": args.batch, "layers": args.layers, "linears_per_step": 7 * args.layers, "ranks": args.ranks,
-            "decode_kernel": ("tensor cores (AF1_FLAG_TC_DECODE)" if args.tc_decode
-                              else "lookup tables on the CUDA cores (default)"),
+            "decode_kernel": decode_kernel_name(args.batch),
             "l2": "inputs larger than L2 (packed weights per step >> 129 MB), no flush"}
 
 
@@ -352,6 +367,12 @@ class Clocks:
 # The AF1 arm
 # ---------------------------------------------------------------------------
 
+def decode_flags():
+    """Layer-constructor keywords of the decode kernel chosen on the command line."""
+    return {"tc_decode": DECODE_KERNEL == "tc", "mma_decode": DECODE_KERNEL == "mma",
+            "lut_decode": DECODE_KERNEL == "lut"}
+
+
 def build_layers(P, torch, layers, batch, rank, outlier_frac=0.0, ranks=None):
     """7 linears per layer with seeded synthetic words; ranks: one per linear
     (default: every matrix's 1.0-BPW rank)."""
@@ -365,7 +386,7 @@ def build_layers(P, torch, layers, batch, rank, outlier_frac=0.0, ranks=None):
             f16 = lambda bits: torch.from_numpy(np.ascontiguousarray(bits).view(np.float16)).cuda()
             Uw = torch.from_numpy(d["Uw"].view(np.int32)).cuda()
             Vw = torch.from_numpy(d["Vw"].view(np.int32)).cuda()
-            layer = P.Layer.from_words(Uw, Vw, f16(d["a"]), f16(d["s"]), f16(d["b"]), m, n, r, tc_decode=TC_DECODE,
+            layer = P.Layer.from_words(Uw, Vw, f16(d["a"]), f16(d["s"]), f16(d["b"]), m, n, r, **decode_flags(),
                                        any_rank=ranks is not None)
             del Uw, Vw
             x = f16(d["x"]).reshape(batch, n)
@@ -389,7 +410,7 @@ def device_layer(P, torch, m, n, r, seed, any_rank=False):
     rs = synth.rng(seed)
     f16 = lambda bits: torch.from_numpy(np.ascontiguousarray(bits).view(np.float16)).cuda()
     a, s_, b = f16(synth.scales_f16(rs, m)), f16(synth.scales_f16(rs, r)), f16(synth.scales_f16(rs, n))
-    layer = P.Layer.from_words(Uw, Vw, a, s_, b, m, n, r, any_rank=any_rank, tc_decode=TC_DECODE)
+    layer = P.Layer.from_words(Uw, Vw, a, s_, b, m, n, r, any_rank=any_rank, **decode_flags())
     del Uw, Vw
     return layer
 
@@ -464,7 +485,7 @@ def sweep(P, torch, peaks, stream):
                  "speedup_vs_dense_bf16": us_dense / us}
             if b <= 16:
                 alg = algorithmic_bytes(m, n, r, b)
-                e.update({"path": "decode", "bound": "hbm", "algorithmic_bytes": alg,
+                e.update({"path": "decode", "kernel": decode_kernel_of(b), "bound": "hbm", "algorithmic_bytes": alg,
                           "achieved_gbs": alg / (us * 1e-6) / 1e9, "frac": alg / (us * 1e-6) / 1e9 / hbm})
             else:
                 fl = 2 * b * r * (m + n)
@@ -479,17 +500,32 @@ def sweep(P, torch, peaks, stream):
     return out
 
 
-TC_MIN_TOKENS, TC_MIN_SIGNS = 8, 16 << 20  # the library's rule for the prepared tensor-core decode
+# The library's default dispatch: passes of more than 4 tokens run on the
+# 16-bit-operand tensor-core kernel, passes of 1-4 tokens on the lookup tables.
+LUT_MAX_TOKENS = 4
+
+
+def decode_kernel_of(b):
+    """The kernel family the phases of a decode call of b tokens run on, per
+    the library's dispatch and the layers' decode-kernel flag."""
+    if DECODE_KERNEL != "auto":
+        return DECODE_KERNEL
+    return "mma" if b > LUT_MAX_TOKENS else "lut"
 
 
 def phase_launches(m, n, r, b):
-    """Kernel launches of one decode call (b <= 16 tokens) per the library's
-    dispatch: a phase on the lookup-table kernel is one launch, a phase on the
-    tensor-core kernel with a prepared B operand is two (prep + decode)."""
-    if TC_DECODE:
-        return sum(2 if b > 4 else 1 for _ in (0, 1))
-    wide = b >= TC_MIN_TOKENS
-    return sum(2 if wide and R * C >= TC_MIN_SIGNS else 1 for (R, C) in ((r, n), (m, r)))
+    """Kernel launches of one decode call (b <= 16 tokens): one per phase,
+    plus a B-operand preparation launch per phase when the e4m3 tensor-core
+    kernel runs a pass of more than 4 tokens."""
+    if decode_kernel_of(b) == "tc":
+        return 4 if b > 4 else 2
+    return 2
+
+
+def grouped_call(lay, grp, b):
+    """A multi-layer call runs as one launch per phase when every phase of
+    every layer of the group takes the lookup-table kernel."""
+    return decode_kernel_of(b) == "lut"
 
 
 def step_launches(objs, b, schedule):
@@ -500,7 +536,7 @@ def step_launches(objs, b, schedule):
         calls = [phase_launches(m, n, r, b) for (_nm, m, n, r, _L, _x) in lay]
         if schedule == "group":
             for grp in ((0, 1, 2), (4, 5)):
-                if all(calls[i] == 2 for i in grp):  # every phase on the lookup-table kernel: one launch per phase
+                if grouped_call(lay, grp, b):  # every phase on the lookup-table kernel: one launch per phase
                     total += 2
                 else:
                     total += sum(calls[i] for i in grp)
@@ -739,9 +775,9 @@ def prefill_extra(P, torch, peaks, stream, steps):
 
 
 def main():
-    global TC_DECODE
+    global DECODE_KERNEL
     args = parse()
-    TC_DECODE = args.tc_decode
+    DECODE_KERNEL = "tc" if args.tc_decode else args.decode_kernel
     b = resolve_workload(args)
     if args.impl == "reference":
         run_reference(args, b)
@@ -967,10 +1003,10 @@ def main():
             # at one token, from the ncu capture summarised in
             # profiles/lut_kernel_llama3_8b_b1.md, times 32 layers.
             traffic = None
-            if b == 1 and not TC_DECODE and args.schedule == "dag":
+            if b == 1 and decode_kernel_of(b) == "lut" and args.schedule == "dag":
                 traffic = (DECODE_TRAFFIC_B1_PER_LAYER * args.layers if args.ranks == "uniform"
                            else int(round(DECODE_TRAFFIC_RATIO_HISA_B1 * alg)))
-            elif (b == 1 and not TC_DECODE and args.schedule == "group" and args.ranks == "hisa"
+            elif (b == 1 and decode_kernel_of(b) == "lut" and args.schedule == "group" and args.ranks == "hisa"
                   and DECODE_TRAFFIC_RATIO_HISA_B1_GROUP is not None):
                 traffic = int(round(DECODE_TRAFFIC_RATIO_HISA_B1_GROUP * alg))
             kname = ("af1_step_run (one persistent step_kernel launch per step)" if args.schedule == "step" else

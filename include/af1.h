@@ -92,6 +92,17 @@ extern "C" {
    clustered kernel (matrices whose clustered split needs more than one wave
    of CTAs). Results agree within the library's tolerance. */
 #define AF1_FLAG_STREAM_DECODE 8
+/* Run every decode pass (1..16 tokens) on the tensor-core kernel with 16-bit
+   operands (tcgen05 MMAs on exact +-b_j FP16 or +-1 BF16 sign values, the
+   activations as FP16 and the rank intermediate as three BF16 terms that
+   hold its FP32 value exactly). Without a decode flag the library takes this
+   kernel for passes of more than 4 tokens and the lookup-table kernels for
+   passes of 1 to 4 tokens. Results agree within the library's tolerance. */
+#define AF1_FLAG_MMA_DECODE 16
+/* Run every decode pass (1..16 tokens) on the CUDA-core lookup-table kernels
+   (clustered or streaming), never on a tensor-core kernel. At most one of
+   AF1_FLAG_TC_DECODE, AF1_FLAG_MMA_DECODE and AF1_FLAG_LUT_DECODE may be set. */
+#define AF1_FLAG_LUT_DECODE 32
 
 typedef struct af1_layer_desc {
   int64_t m;       /* d_out: rows of W_hat, length of a, length of y rows */

@@ -39,16 +39,20 @@ AF1_FLAG_ANY_RANK = 1
 AF1_FLAG_TC_DECODE = 2
 AF1_FLAG_BF16_SCALES = 4
 AF1_FLAG_STREAM_DECODE = 8
+AF1_FLAG_MMA_DECODE = 16
+AF1_FLAG_LUT_DECODE = 32
 
 
-def _flags(any_rank: bool, tc_decode: bool, scales=(), stream_decode: bool = False) -> int:
+def _flags(any_rank: bool, tc_decode: bool, scales=(), stream_decode: bool = False, mma_decode: bool = False,
+           lut_decode: bool = False) -> int:
     """Layer flags; BF16 scale tensors select AF1_FLAG_BF16_SCALES."""
     dts = {t.dtype for t in scales}
     if len(dts) > 1 or not dts <= {torch.float16, torch.bfloat16}:
         raise ValueError("a, s and b must all be float16 or all bfloat16")
     bf16 = dts == {torch.bfloat16}
     return ((AF1_FLAG_ANY_RANK if any_rank else 0) | (AF1_FLAG_TC_DECODE if tc_decode else 0)
-            | (AF1_FLAG_BF16_SCALES if bf16 else 0) | (AF1_FLAG_STREAM_DECODE if stream_decode else 0))
+            | (AF1_FLAG_BF16_SCALES if bf16 else 0) | (AF1_FLAG_STREAM_DECODE if stream_decode else 0)
+            | (AF1_FLAG_MMA_DECODE if mma_decode else 0) | (AF1_FLAG_LUT_DECODE if lut_decode else 0))
 _ERR_NAMES = {
     -1: "AF1_ERR_INVALID_ARG", -2: "AF1_ERR_BAD_POINTER", -3: "AF1_ERR_MISALIGNED",
     -4: "AF1_ERR_OVER_BUDGET", -5: "AF1_ERR_INVALID_SIGN", -6: "AF1_ERR_CUDA",
@@ -231,13 +235,16 @@ class Layer:
     @classmethod
     def from_signs(cls, U: torch.Tensor, V: torch.Tensor, a: torch.Tensor, s: torch.Tensor,
                    b: torch.Tensor, any_rank: bool = False, return_words: bool = False, stream=None,
-                   tc_decode: bool = False, stream_decode: bool = False):
+                   tc_decode: bool = False, stream_decode: bool = False, mma_decode: bool = False,
+                   lut_decode: bool = False):
         """U: int8 (m, r), V: int8 (n, r) of +-1; a, s, b: float16 vectors. All on
         the current CUDA device. With return_words, also returns the canonical
         packed words (Uw: (m, W(r)), Vw: (r, W(n)) as int32 tensors). tc_decode
-        selects the tensor-core decode kernel (AF1_FLAG_TC_DECODE), stream_decode
-        the streaming CUDA-core kernel for 1- and 2-token passes
-        (AF1_FLAG_STREAM_DECODE)."""
+        selects the e4m3 tensor-core decode kernel (AF1_FLAG_TC_DECODE),
+        mma_decode the 16-bit-operand tensor-core decode kernel for every pass
+        (AF1_FLAG_MMA_DECODE), lut_decode the lookup-table kernels for every
+        pass (AF1_FLAG_LUT_DECODE), stream_decode the streaming CUDA-core kernel
+        for 1- and 2-token passes (AF1_FLAG_STREAM_DECODE)."""
         m, r = U.shape
         n = V.shape[0]
         if V.shape[1] != r:
@@ -248,7 +255,7 @@ class Layer:
         if return_words:
             Uw = torch.empty((m, words_per_row(r)), dtype=torch.int32, device=U.device)
             Vw = torch.empty((r, words_per_row(n)), dtype=torch.int32, device=U.device)
-        d = _Desc(m, n, r, _flags(any_rank, tc_decode, (a, s, b), stream_decode), 0)
+        d = _Desc(m, n, r, _flags(any_rank, tc_decode, (a, s, b), stream_decode, mma_decode, lut_decode), 0)
         h = _vp()
         _check(_lib.af1_pack_layer(ctypes.byref(d), _ptr(U), _ptr(V), _ptr(a), _ptr(s), _ptr(b),
                                    _ptr(Uw), _ptr(Vw), _stream_handle(stream), ctypes.byref(h)))
@@ -258,11 +265,12 @@ class Layer:
     @classmethod
     def from_words(cls, Uw: torch.Tensor, Vw: torch.Tensor, a: torch.Tensor, s: torch.Tensor,
                    b: torch.Tensor, m: int, n: int, r: int, any_rank: bool = False, stream=None,
-                   tc_decode: bool = False, stream_decode: bool = False):
+                   tc_decode: bool = False, stream_decode: bool = False, mma_decode: bool = False,
+                   lut_decode: bool = False):
         """Uw: (m, W(r)), Vw: (r, W(n)) canonical packed words (int32/uint32)."""
         Uw, Vw = Uw.contiguous(), Vw.contiguous()
         a, s, b = a.contiguous(), s.contiguous(), b.contiguous()
-        d = _Desc(m, n, r, _flags(any_rank, tc_decode, (a, s, b), stream_decode), 0)
+        d = _Desc(m, n, r, _flags(any_rank, tc_decode, (a, s, b), stream_decode, mma_decode, lut_decode), 0)
         h = _vp()
         _check(_lib.af1_load_packed_layer(ctypes.byref(d), _ptr(Uw), _ptr(Vw), _ptr(a), _ptr(s), _ptr(b),
                                           _stream_handle(stream), ctypes.byref(h)))

@@ -71,8 +71,14 @@ int check_desc(const af1_layer_desc* d) {
   if (d->m > ((int64_t)1 << 30) || d->n > af1::kMaxCols || d->r > af1::kMaxCols)
     return fail(AF1_ERR_INVALID_ARG, "m must be <= 2^30 and n, r <= " + std::to_string(af1::kMaxCols));
   if (d->reserved != 0 || (d->flags & ~(AF1_FLAG_ANY_RANK | AF1_FLAG_TC_DECODE | AF1_FLAG_BF16_SCALES |
-                                                AF1_FLAG_STREAM_DECODE)) != 0)
+                                                AF1_FLAG_STREAM_DECODE | AF1_FLAG_MMA_DECODE |
+                                                AF1_FLAG_LUT_DECODE)) != 0)
     return fail(AF1_ERR_INVALID_ARG, "unknown flags or non-zero reserved field");
+  {
+    const int kernel_flags = d->flags & (AF1_FLAG_TC_DECODE | AF1_FLAG_MMA_DECODE | AF1_FLAG_LUT_DECODE);
+    if ((kernel_flags & (kernel_flags - 1)) != 0)
+      return fail(AF1_ERR_INVALID_ARG, "at most one of AF1_FLAG_TC_DECODE, AF1_FLAG_MMA_DECODE, AF1_FLAG_LUT_DECODE");
+  }
   if (!(d->flags & AF1_FLAG_ANY_RANK)) {
     int64_t rmax = 0;
     int rc = rank_rule(d->m, d->n, 1, 1, &rmax);

@@ -44,6 +44,7 @@
 // the largest magnitude in [128, 256), and split into 4 e4m3 terms
 // (z' ~ t1 + t2 + t3 + t4, about 16 significant bits) that occupy 4 of the N
 // rows of B. Products are exact and the MMA accumulates in FP32.
+#include <cuda_bf16.h>
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -689,6 +690,383 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const DecodeArgs a)
 }
 
 // ---------------------------------------------------------------------------
+// Decode kernel with 16-bit MMA operands (tcgen05.mma kind::f16), passes of
+// up to 16 tokens. The signs become exact 16-bit A values in tensor memory:
+//   phase 1: A = +-b_j (FP16; the column scale carries the sign), B = x
+//            (FP16, N = 16 rows, row t = token t), so D = sum_j +-b_j x_j;
+//   phase 2: A = +-1 (BF16), B = s' split exactly into three BF16 terms
+//            s' = hi + mid + lo (N = 16/32/48 rows, term q of token t in row
+//            3 t + q): BF16 keeps FP32's exponent range, and 8 + 8 + 8
+//            significant bits hold FP32's 24, so no scaling is needed.
+// Every product is exact and the MMA accumulates in FP32: the result is the
+// FP32 signed sum the lookup-table kernels form, summed in another order.
+// Against the e4m3 kernel above there is no activation split, no power-of-
+// two scale and no sign correction, and the B operand is a copy (phase 1) or
+// a three-way split (phase 2) that the CTA builds itself, so no preparation
+// kernel runs. A chunk of A takes 64 tensor-memory columns (two values per
+// column), twice the e4m3 chunk. The CTA structure is the e4m3 kernel's:
+// bulk copies of the signs first, warps 0-3 expand, warps 4-7 build B and
+// issue the MMAs (K = 16 each) into NACC accumulators, warps 0-3 read them
+// back and push the partial sums to the cluster CTA that owns each row.
+// ---------------------------------------------------------------------------
+
+__host__ __device__ constexpr int hnacc_for(int N) { return N == 16 ? 4 : 2; }
+__host__ __device__ constexpr int hnbuf_for(int N) { return (kTmemCols - hnacc_for(N) * N) / 64; }
+// B rows of a pass of T tokens: one per token (phase 1), three (phase 2).
+__host__ __device__ constexpr int hdecode_n(int phase, int T) { return phase == 1 ? 16 : (3 * T + 15) / 16 * 16; }
+
+struct __align__(8) HDecodeHeader {
+  uint64_t wfull[kMaxCPC];  // packed chunk c has landed (chunk 0: with the column scales)
+  uint64_t afull[4];        // A buffer holds its chunk (128 expander arrivals)
+  uint64_t aempty[4];       // the MMAs that read an A buffer are done (NACC commits)
+  uint64_t ddone;           // all MMAs done (NACC commits)
+  uint32_t tmem_base, err;
+};
+
+struct HDecodeSmem {
+  int bt, w, cs, recv, rs, hdr, total;  // byte offsets from the 1024-aligned base
+};
+
+__host__ __device__ inline HDecodeSmem hdecode_smem(int N, int CPC, int KS, int T) {
+  HDecodeSmem p;
+  int off = 0;
+  p.bt = off;
+  off += 2 * N * 128 * CPC;  // B: K half h of chunk c at (2 c + h) N 128, 1024-aligned
+  p.w = off;
+  off += kChunkBytes * CPC;
+  p.cs = off;
+  off += CPC * kChunkCols * 2;  // phase 1: the column scales of the CTA's chunks
+  p.recv = off;
+  off = align128(off + KS * T * slice_rows(KS) * 4);
+  p.rs = off;
+  off = align128(off + slice_rows(KS) * 4);
+  p.hdr = off;
+  off = align128(off + (int)sizeof(HDecodeHeader));
+  p.total = off + 1024;  // slack for aligning the base to 1024 bytes
+  return p;
+}
+
+// D (FP32) [+]= A (tensor memory) x B (shared memory)^T, kind::f16, M = 128,
+// K = 16, N rows of B; A and B both FP16, or both BF16.
+template <int N, bool BF16>
+__device__ __forceinline__ void mma_h(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, bool accumulate) {
+  constexpr uint32_t fmt = BF16 ? 1u : 0u;
+  constexpr uint32_t idesc =
+      (1u << 4) | (fmt << 7) | (fmt << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(kBlockRows >> 4) << 24);
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate ? 1u : 0u)
+      : "memory");
+}
+
+// Sign bits p of bytes 1 and 3 of `pair_bytes` -> the sign bits (15, 31) of
+// a 16-bit pair: bit 1 keeps v, bit 0 negates it.
+__device__ __forceinline__ uint32_t sign_pair(uint32_t pair_bytes, int p, uint32_t v) {
+  return v ^ (~(pair_bytes << (7 - p)) & 0x80008000u);
+}
+
+// Word w of a row -> 16 tensor-memory columns of 16-bit A values in K order:
+// column 4 jj + u holds columns 8 jj + 2 u, + 1 of the word. Column 4 p + e
+// of the word is bit 8 e + p (af1_layout.h); v[jj] holds the magnitudes of
+// columns 8 jj .. 8 jj + 7 as four pairs.
+__device__ __forceinline__ void expand_word_h(uint32_t w, const uint4 (&v)[4], uint32_t* s) {
+  const uint32_t b01 = __byte_perm(w, 0u, 0x1404);  // bytes 0, 1 (e = 0, 1) -> bytes 1, 3
+  const uint32_t b23 = __byte_perm(w, 0u, 0x3424);  // bytes 2, 3 (e = 2, 3) -> bytes 1, 3
+#pragma unroll
+  for (int jj = 0; jj < 4; ++jj) {
+    const int p = 2 * jj;
+    s[4 * jj + 0] = sign_pair(b01, p, v[jj].x);
+    s[4 * jj + 1] = sign_pair(b23, p, v[jj].y);
+    s[4 * jj + 2] = sign_pair(b01, p + 1, v[jj].z);
+    s[4 * jj + 3] = sign_pair(b23, p + 1, v[jj].w);
+  }
+}
+
+__device__ __forceinline__ void tmem_st16p(uint32_t addr, const uint32_t* r) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(
+          addr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), "r"(r[9]),
+      "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
+      : "memory");
+}
+
+// Three BF16 terms of v (hi + mid + lo == v exactly for finite FP32 v).
+__device__ __forceinline__ void bf16_split3(float v, uint16_t* t3) {
+  const __nv_bfloat16 hi = __float2bfloat16_rn(v);
+  const float r1 = v - __bfloat162float(hi);
+  const __nv_bfloat16 mid = __float2bfloat16_rn(r1);
+  const __nv_bfloat16 lo = __float2bfloat16_rn(r1 - __bfloat162float(mid));
+  t3[0] = __bfloat16_as_ushort(hi);
+  t3[1] = __bfloat16_as_ushort(mid);
+  t3[2] = __bfloat16_as_ushort(lo);
+}
+
+// The B operand of the CTA's K slice (chunks of columns from k0, kv valid
+// columns), built by 128 threads (bt = 0..127): 16-byte units of 8 columns,
+// row n of K half h of chunk c at Bt + (2 c + h) N 128 + n 128, unit j at
+// (j ^ (n & 7)) 16 (128-byte swizzle, K-major). Columns >= kv are zero.
+template <int PHASE, int N>
+__device__ __forceinline__ void build_b_h(const DecodeArgs& a, int T, int nch, int64_t k0, int kv, int bt,
+                                          uint8_t* Bt) {
+  const int nu = nch * (kChunkCols / 8);  // 8-column units per token
+  for (int i = bt; i < T * nu; i += 128) {
+    const int t = i / nu, u = i - t * nu;
+    const int kl = 8 * u;
+    const int c = u >> 4, hh = (u >> 3) & 1, j = u & 7;
+    uint8_t* half_base = Bt + (2 * c + hh) * (N * 128);
+    if (PHASE == 1) {
+      uint4 v = make_uint4(0u, 0u, 0u, 0u);
+      const __half* p = a.x + (int64_t)t * a.ldx + k0 + kl;
+      if (kl + 7 < kv) {
+        v = __ldcg(reinterpret_cast<const uint4*>(p));
+      } else {
+        uint16_t e[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) e[q] = kl + q < kv ? __half_as_ushort(__ldcg(p + q)) : (uint16_t)0;
+        v = make_uint4(e[0] | (uint32_t)e[1] << 16, e[2] | (uint32_t)e[3] << 16, e[4] | (uint32_t)e[5] << 16,
+                       e[6] | (uint32_t)e[7] << 16);
+      }
+      *reinterpret_cast<uint4*>(half_base + t * 128 + ((j ^ (t & 7)) << 4)) = v;
+    } else {
+      float f[8];
+      const float* p = a.zin + (int64_t)t * a.ldz + k0 + kl;
+      if (kl + 7 < kv) {
+        const float4 z0 = __ldcg(reinterpret_cast<const float4*>(p));
+        const float4 z1 = __ldcg(reinterpret_cast<const float4*>(p + 4));
+        f[0] = z0.x; f[1] = z0.y; f[2] = z0.z; f[3] = z0.w;
+        f[4] = z1.x; f[5] = z1.y; f[6] = z1.z; f[7] = z1.w;
+      } else {
+#pragma unroll
+        for (int q = 0; q < 8; ++q) f[q] = kl + q < kv ? __ldcg(p + q) : 0.f;
+      }
+      uint16_t e[3][8];
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        uint16_t t3[3];
+        bf16_split3(f[q], t3);
+        e[0][q] = t3[0];
+        e[1][q] = t3[1];
+        e[2][q] = t3[2];
+      }
+#pragma unroll
+      for (int term = 0; term < 3; ++term) {
+        const int n = 3 * t + term;
+        const uint4 v = make_uint4(e[term][0] | (uint32_t)e[term][1] << 16, e[term][2] | (uint32_t)e[term][3] << 16,
+                                   e[term][4] | (uint32_t)e[term][5] << 16, e[term][6] | (uint32_t)e[term][7] << 16);
+        *reinterpret_cast<uint4*>(half_base + n * 128 + ((j ^ (n & 7)) << 4)) = v;
+      }
+    }
+  }
+}
+
+template <int PHASE, int N>
+__global__ void __launch_bounds__(kThreads, 1) hdecode_kernel(const DecodeArgs a) {
+  constexpr int NACC = hnacc_for(N);
+  constexpr int NBUF = hnbuf_for(N);
+  constexpr int DCOL = NBUF * 64;  // first accumulator column
+  constexpr bool BF16 = PHASE == 2;
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  const int T = a.tokens;
+  const int KS = a.KS;
+  const HDecodeSmem sp = hdecode_smem(N, a.CPC, KS, T);
+  uint8_t* Bt = smem + sp.bt;
+  const uint32_t* W = reinterpret_cast<const uint32_t*>(smem + sp.w);
+  const uint8_t* cs = smem + sp.cs;
+  float* recv = reinterpret_cast<float*>(smem + sp.recv);
+  float* rs = reinterpret_cast<float*>(smem + sp.rs);
+  HDecodeHeader& h = *reinterpret_cast<HDecodeHeader*>(smem + sp.hdr);
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int rb = blockIdx.x, ks = blockIdx.y;
+  const int nch_total = a.sm.NCH;
+  const int c0 = ks * a.CPC;
+  const int nch = min(a.CPC, nch_total - c0);  // >= 1 by construction of KS
+  const int64_t row0 = (int64_t)rb * kBlockRows;
+  const int64_t k0 = (int64_t)c0 * kChunkCols;
+  const int kv = (int)min((int64_t)nch * kChunkCols, a.sm.C - k0);  // valid columns of this CTA
+  const int slice = slice_rows(KS);
+  const int my0 = ks * slice;  // first block row this CTA finalises
+
+  cluster_arrive_relaxed();  // matched by cluster_wait before the first remote store
+
+  if (tid == 128) {
+    for (int c = 0; c < nch; ++c) mbar_init(&h.wfull[c], 1);
+    for (int b = 0; b < NBUF; ++b) {
+      mbar_init(&h.afull[b], 128);
+      mbar_init(&h.aempty[b], NACC);
+    }
+    mbar_init(&h.ddone, NACC);
+    h.err = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    // Packed chunks of this CTA (contiguous 2 KB blocks of row block rb) and,
+    // for phase 1, the column scales of its chunks (the layer's b is
+    // zero-padded to whole chunks), which land with chunk 0.
+    const uint8_t* src = a.signs + ((int64_t)rb * nch_total + c0) * kChunkBytes;
+    for (int c = 0; c < nch; ++c) {
+      const uint32_t extra = (PHASE == 1 && c == 0) ? (uint32_t)(nch * kChunkCols * 2) : 0u;
+      mbar_expect_tx(&h.wfull[c], kChunkBytes + extra);
+      bulk_g2s(smem + sp.w + c * kChunkBytes, src + (int64_t)c * kChunkBytes, kChunkBytes, &h.wfull[c]);
+      if (extra != 0) bulk_g2s(smem + sp.cs, a.colscale + k0, extra, &h.wfull[0]);
+    }
+  }
+  __syncwarp();
+  if (warp == 4) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&h.tmem_base)),
+                 "r"((uint32_t)kTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  // Row scales of the rows this CTA finalises (layer constants).
+  for (int i = tid; i < slice; i += kThreads) {
+    const int64_t row = row0 + my0 + i;
+    rs[i] = (my0 + i < kBlockRows && row < a.sm.R) ? __half2float(a.rowscale[row]) : 0.f;
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = h.tmem_base;
+
+  if (warp < 4) {
+    // ---- A: expand packed chunks into the tensor-memory ring --------------
+    const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+    bool ok = true;
+    for (int c = 0; c < nch && ok; ++c) {
+      const int b = c % NBUF, use = c / NBUF;
+      if (use >= 1) {
+        ok = mbar_wait(&h.aempty[b], (use - 1) & 1, &h.err, a.wait_cycles);
+        tc_fence_after();
+      }
+      if (ok) ok = mbar_wait(&h.wfull[c], 0, &h.err, a.wait_cycles);
+      if (!ok) break;
+      const uint32_t* wc = W + c * (kChunkBytes / 4);
+      const uint32_t addr = tmem + lane_base + (uint32_t)(b * 64);
+#pragma unroll
+      for (int kw = 0; kw < kChunkWords; ++kw) {
+        uint4 v[4];
+#pragma unroll
+        for (int jj = 0; jj < 4; ++jj) {
+          if (PHASE == 1)
+            v[jj] = *reinterpret_cast<const uint4*>(cs + (c * kChunkCols + 32 * kw + 8 * jj) * 2);
+          else
+            v[jj] = make_uint4(0x3F803F80u, 0x3F803F80u, 0x3F803F80u, 0x3F803F80u);  // BF16 pairs of 1
+        }
+        uint32_t r[16];
+        expand_word_h(wc[kw * kBlockRows + tid], v, r);
+        tmem_st16p(addr + (uint32_t)(16 * kw), r);
+      }
+      asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+      tc_fence_before();
+      mbar_arrive(&h.afull[b]);
+    }
+  } else {
+    // ---- B: activations -> the swizzled B tile; then the MMAs -------------
+    const int bt = tid - 128;
+    griddep_wait();  // activations are written by the previous kernel
+    build_b_h<PHASE, N>(a, T, nch, k0, kv, bt, Bt);
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // B is read by the tensor cores
+    builders_sync();
+    const int ia = warp - 4;
+    if (lane == 0 && ia < NACC) {
+      // ---- MMA issue: chunk c, K step kk (16 columns) by issuer kk % NACC --
+      const uint32_t b0 = smem_u32(Bt);
+      bool ok = true;
+      for (int c = 0; c < nch && ok; ++c) {
+        const int b = c % NBUF, use = c / NBUF;
+        ok = mbar_wait(&h.afull[b], use & 1, &h.err, a.wait_cycles);
+        if (!ok) break;
+        tc_fence_after();
+#pragma unroll
+        for (int kk = ia; kk < 8; kk += NACC) {
+          mma_h<N, BF16>(tmem + (uint32_t)(DCOL + ia * N), tmem + (uint32_t)(b * 64 + kk * 8),
+                         smem_desc(b0 + (uint32_t)((2 * c + (kk >> 2)) * N * 128 + (kk & 3) * 32)),
+                         c > 0 || kk >= NACC);
+        }
+        mma_commit(&h.aempty[b]);
+      }
+      mma_commit(&h.ddone);
+    }
+    __syncwarp();
+  }
+
+  griddep_launch_dependents();
+  // ---- epilogue: accumulators -> per-row partial sums -> owner CTA ----------
+  griddep_wait();  // outputs may still be read by the previous kernel until it completes
+  cluster_wait();  // every CTA of the cluster has started
+  if (warp < 4) {
+    const bool ok = mbar_wait(&h.ddone, 0, &h.err, a.wait_cycles);
+    tc_fence_after();
+    const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+    const int i = tid;  // block row
+    const int owner = i / slice;
+    float acc[N];
+#pragma unroll
+    for (int j = 0; j < N; ++j) acc[j] = 0.f;
+#pragma unroll
+    for (int d = 0; d < NACC; ++d) {
+#pragma unroll
+      for (int cb = 0; cb < N / 16; ++cb) {
+        uint32_t r[16];
+        tmem_ld16(tmem + lane_base + (uint32_t)(DCOL + d * N + cb * 16), r);
+        asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+        for (int j = 0; j < 16; ++j) acc[cb * 16 + j] += __uint_as_float(r[j]);
+      }
+    }
+    if (ok) {
+      constexpr int TMAX = PHASE == 1 ? N : N / 3;  // tokens the B rows hold
+#pragma unroll
+      for (int t = 0; t < TMAX; ++t) {
+        if (t < T) {
+          const float p = PHASE == 1 ? acc[t] : (acc[3 * t] + acc[3 * t + 1]) + acc[3 * t + 2];
+          st_cluster_f32(recv + ((ks * T + t) * slice + (i - owner * slice)), (uint32_t)owner, p);
+        }
+      }
+    }
+  }
+  // All partials of the cluster have landed in their owners' buffers.
+  cluster_sync();
+  const int cnt = min(slice, kBlockRows - my0);
+  for (int idx = tid; idx < T * cnt; idx += kThreads) {
+    const int t = idx / cnt;
+    const int i = idx - t * cnt;
+    const int64_t row = row0 + my0 + i;
+    if (row >= a.sm.R) continue;
+    float v = 0.f;
+    for (int q = 0; q < KS; ++q) v += recv[(q * T + t) * slice + i];
+    const float out = v * rs[i];
+    if (PHASE == 1) {
+      a.sout[(int64_t)t * a.lds + row] = out;
+    } else if (a.ydtype == 0) {
+      reinterpret_cast<__half*>(a.y)[(int64_t)t * a.ldy + row] = __float2half_rn(out);
+    } else {
+      reinterpret_cast<float*>(a.y)[(int64_t)t * a.ldy + row] = out;
+    }
+  }
+
+  // ---- teardown ---------------------------------------------------------------
+  tc_fence_before();
+  __syncthreads();
+  if (tid == 128 && h.err != 0) {
+    // Something timed out: let the bulk copies drain (bounded) so that none
+    // lands after the CTA has exited, and report it.
+    for (int c = 0; c < nch; ++c) mbar_wait(&h.wfull[c], 0, &h.err, a.wait_cycles);
+    atomicOr(a.status, kStatusTimeout);
+  }
+  if (warp == 4) {
+    tc_fence_after();
+    if (lane == 0) mbar_wait(&h.ddone, 0, &h.err, a.wait_cycles);  // no MMA may still read tensor memory
+    __syncwarp();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"((uint32_t)kTmemCols)
+                 : "memory");
+  }
+}
+
+// ---------------------------------------------------------------------------
 // Prep kernel: the B operand of every K slice of a pass, built once per slice
 // instead of once per row block (the split of a pass of T tokens into 4T
 // e4m3 terms costs about 40 instructions per value and grows with T, while
@@ -773,14 +1151,6 @@ struct DecodePlan {
 
 int n_for_tokens(int T) { return T <= 4 ? 16 : T <= 8 ? 32 : 64; }
 
-// Passes of at least kTcMinTokens tokens over a sign matrix of at least
-// kTcMinSigns signs use the tensor-core kernel with a prepared B operand when
-// the workspace holds it (measured at 8 and 16 tokens: faster from about
-// 30 M signs per phase, e.g. 8192x28672 at 8 tokens 170 -> 96 us, 14336x4096
-// at 16 tokens 57.8 -> 50.2 us; slower on 4096^2, 33.7 vs 22.2 us at 16).
-constexpr int kTcMinTokens = 8;
-constexpr int64_t kTcMinSigns = 16 << 20;
-
 constexpr int kTwoPerSmSmem = 110 * 1024;  // at or below this, two CTAs share an SM
 
 // Split of one sign matrix for a pass of T tokens: about one CTA per SM
@@ -857,6 +1227,62 @@ DecodePlan plan_decode(int phase, const SignMatrix& sm, int T, int num_sms, int 
   return p;
 }
 
+
+// Split of one sign matrix for the 16-bit-operand kernel: the same rules as
+// plan_decode (about one CTA per SM, KS <= 16, a finer split where it lets
+// two CTAs share an SM and lowers waves x chunks per CTA, then K split
+// further while a CTA streams more chunks than its A ring holds), with that
+// kernel's shared memory and ring depth.
+DecodePlan plan_hdecode(int phase, const SignMatrix& sm, int T, int num_sms, int max_smem) {
+  DecodePlan p;
+  p.N = hdecode_n(phase, T);
+  const int sms = num_sms > 0 ? num_sms : kDefaultSms;
+  const int nbuf = hnbuf_for(p.N);
+  int ks = sms / (sm.RB > 0 ? sm.RB : 1);
+  if (ks < 1) ks = 1;
+  if (ks > kMaxKS) ks = kMaxKS;
+  if (ks > sm.NCH) ks = sm.NCH;
+  auto waves = [&](int KS, int need) {
+    const int64_t slots = (int64_t)sms * (need <= kTwoPerSmSmem ? 2 : 1);
+    return ((int64_t)sm.RB * KS + slots - 1) / slots;
+  };
+  for (; ks <= kMaxKS; ++ks) {
+    const int cpc = (sm.NCH + ks - 1) / ks;
+    if (cpc > kMaxCPC) continue;
+    const int KS = (sm.NCH + cpc - 1) / cpc;
+    const int need = hdecode_smem(p.N, cpc, KS, T).total;
+    if (need > max_smem) continue;
+    p.KS = KS;
+    p.CPC = cpc;
+    p.smem = need < kMinSmem ? kMinSmem : need;
+    p.ok = true;
+    if (need > kTwoPerSmSmem) {
+      for (int k2 = ks + 1; k2 <= kMaxKS && k2 <= sm.NCH; ++k2) {
+        const int c2 = (sm.NCH + k2 - 1) / k2;
+        const int K2 = (sm.NCH + c2 - 1) / c2;
+        const int n2 = hdecode_smem(p.N, c2, K2, T).total;
+        if (n2 <= kTwoPerSmSmem && waves(K2, n2) * c2 < waves(p.KS, p.smem) * p.CPC) {
+          p.KS = K2;
+          p.CPC = c2;
+          p.smem = n2 < kMinSmem ? kMinSmem : n2;
+        }
+      }
+    }
+    while (p.CPC > nbuf && p.KS * 2 <= 8 && (int64_t)sm.RB * p.KS * 2 <= 2 * sms) {
+      const int k2 = p.KS * 2;
+      const int c2 = (sm.NCH + k2 - 1) / k2;
+      const int K2 = (sm.NCH + c2 - 1) / c2;
+      const int n2 = hdecode_smem(p.N, c2, K2, T).total;
+      if (n2 > max_smem) break;
+      p.KS = K2;
+      p.CPC = c2;
+      p.smem = n2 < kMinSmem ? kMinSmem : n2;
+    }
+    return p;
+  }
+  return p;
+}
+
 template <int PHASE, int N>
 cudaError_t launch_prep(const DecodeArgs& a, const DecodePlan& p, cudaStream_t st) {
   auto kern = bprep_kernel<PHASE, N>;
@@ -917,6 +1343,47 @@ cudaError_t launch_decode(DecodeArgs a, const DecodePlan& p, cudaStream_t st) {
     case 16: return launch_decode_n<PHASE, 16, false>(a, p, st);
     case 32: return prep ? launch_decode_n<PHASE, 32, true>(a, p, st) : launch_decode_n<PHASE, 32, false>(a, p, st);
     default: return prep ? launch_decode_n<PHASE, 64, true>(a, p, st) : launch_decode_n<PHASE, 64, false>(a, p, st);
+  }
+}
+
+template <int PHASE, int N>
+cudaError_t launch_hdecode_n(const DecodeArgs& a, const DecodePlan& p, cudaStream_t st) {
+  auto kern = hdecode_kernel<PHASE, N>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, p.smem);
+  if (e != cudaSuccess) return e;
+  if (p.KS > 8) {
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    if (e != cudaSuccess) return e;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)a.sm.RB, (unsigned)p.KS, 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = (size_t)p.smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = 1;
+  attr[1].val.clusterDim.y = (unsigned)p.KS;
+  attr[1].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  return cudaLaunchKernelEx(&cfg, kern, a);
+}
+
+template <int PHASE>
+cudaError_t launch_hdecode(DecodeArgs a, const DecodePlan& p, cudaStream_t st) {
+  a.KS = p.KS;
+  a.CPC = p.CPC;
+  if constexpr (PHASE == 1) {
+    return launch_hdecode_n<1, 16>(a, p, st);
+  } else {
+    switch (p.N) {
+      case 16: return launch_hdecode_n<2, 16>(a, p, st);
+      case 32: return launch_hdecode_n<2, 32>(a, p, st);
+      default: return launch_hdecode_n<2, 48>(a, p, st);
+    }
   }
 }
 
@@ -994,22 +1461,39 @@ Workspace plan_workspace(const af1_layer& L, int64_t tokens, bool prep, bool swi
 
 namespace {
 
-// Kernel of one phase of a decode pass of T tokens: the tensor-core kernel
-// (tc), the streaming CUDA-core kernel (stream.ok) or the clustered one
-// (lut.ok); tc also when neither CUDA-core kernel has a plan.
+// Kernel of one phase of a decode pass of T tokens: the e4m3 tensor-core
+// kernel (tc, AF1_FLAG_TC_DECODE), the 16-bit-operand tensor-core kernel
+// (mma), the streaming CUDA-core kernel (stream.ok) or the clustered one
+// (lut.ok); mma also when neither CUDA-core kernel has a plan.
 struct PhaseChoice {
   bool tc = false;
+  bool mma = false;
   LutPlan lut;
   StreamPlan stream;
 };
 
+// Passes of more than kLutMaxTokens tokens take the 16-bit-operand
+// tensor-core kernel by default. The lookup tables' work grows with the
+// tokens (a table read per 4 signs per token pair, and from 5 tokens on a
+// second token group of CTAs that reads every sign tile again), the MMAs'
+// hardly does, but expanding signs into tensor memory costs more per sign
+// than a lookup. Measured on the 32-layer HiSA-rank stack (decoder DAG, ms
+// per step, lookup tables vs MMA): 4 tokens 2.56 vs 2.91, 6 tokens 3.96 vs
+// 3.23, 8 tokens 4.05 vs 3.40. (Per call in isolation the MMA kernel already
+// wins at 4 tokens on matrices of 8 Mi signs and more, e.g. 14336x4096 21.5
+// vs 19.9 us, but loses inside the stack, where it shares the SMs with the
+// sibling linears' kernels.)
+constexpr int kLutMaxTokens = 4;
+
 PhaseChoice choose_phase(const af1_layer& L, int phase, const SignMatrix& m, int T, const Workspace& W) {
+  (void)W;
   PhaseChoice c;
-  // The tensor-core kernel when the layer asks for it, or for wide passes
-  // over matrices large enough for it (with a prepared B operand) to be the
-  // faster one.
-  if ((L.flags & AF1_FLAG_TC_DECODE) != 0 || (W.bbuf != 0 && T >= kTcMinTokens && m.R * m.C >= kTcMinSigns)) {
+  if ((L.flags & AF1_FLAG_TC_DECODE) != 0) {
     c.tc = true;
+    return c;
+  }
+  if ((L.flags & AF1_FLAG_MMA_DECODE) != 0 || ((L.flags & AF1_FLAG_LUT_DECODE) == 0 && T > kLutMaxTokens)) {
+    c.mma = true;
     return c;
   }
   c.lut = plan_lut(&m, 1, T, L.num_sms, L.max_smem);
@@ -1029,7 +1513,7 @@ PhaseChoice choose_phase(const af1_layer& L, int phase, const SignMatrix& m, int
     }
     if (want) c.stream = plan_stream(phase, m, T, L.num_sms, L.max_smem);
   }
-  if (!c.stream.ok && !c.lut.ok) c.tc = true;
+  if (!c.stream.ok && !c.lut.ok) c.mma = true;
   return c;
 }
 
@@ -1065,15 +1549,22 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
   // Widest pass whose plans fit (16 tokens normally; fewer only for very
   // long contractions).
   int pass = kMaxPassTokens;
-  DecodePlan p1, p2;
+  bool fits = false;
   for (;;) {
     const int T = (int)(tokens < pass ? tokens : pass);
-    p1 = plan_decode(1, L.p1, T, L.num_sms, L.max_smem, false);
-    p2 = plan_decode(2, L.p2, T, L.num_sms, L.max_smem, false);
-    if ((p1.ok && p2.ok) || pass <= 4) break;
+    fits = plan_decode(1, L.p1, T, L.num_sms, L.max_smem, false).ok &&
+           plan_decode(2, L.p2, T, L.num_sms, L.max_smem, false).ok;
+    if (fits) {
+      // The 16-bit-operand kernel's B tiles grow with the pass (3 T rows in
+      // phase 2): its plans must fit too where it would run.
+      const PhaseChoice c1 = choose_phase(L, 1, L.p1, T, W), c2 = choose_phase(L, 2, L.p2, T, W);
+      if (c1.mma && !plan_hdecode(1, L.p1, T, L.num_sms, L.max_smem).ok) fits = false;
+      if (c2.mma && !plan_hdecode(2, L.p2, T, L.num_sms, L.max_smem).ok) fits = false;
+    }
+    if (fits || pass <= 4) break;
     pass /= 2;
   }
-  if (!p1.ok || !p2.ok) return cudaErrorInvalidConfiguration;
+  if (!fits) return cudaErrorInvalidConfiguration;
   for (int64_t t0 = 0; t0 < tokens; t0 += pass) {
     const int T = (int)((tokens - t0) < pass ? (tokens - t0) : pass);
     PhaseChoice c1 = choose_phase(L, 1, L.p1, T, W), c2 = choose_phase(L, 2, L.p2, T, W);
@@ -1081,12 +1572,15 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
     // LLaMA-70B 28672 x 8192 matrix at one token: 22.5 -> 18.7 us per call;
     // the converse, a streamed first phase pulling the second along, was
     // slower on 8192 x 28672: 21.7 -> 24.1 us).
-    if (!c1.tc && !c1.stream.ok && c2.stream.ok) c1.stream = plan_stream(1, L.p1, T, L.num_sms, L.max_smem);
+    if (!c1.tc && !c1.mma && !c1.stream.ok && c2.stream.ok)
+      c1.stream = plan_stream(1, L.p1, T, L.num_sms, L.max_smem);
     DecodePlan q1, q2;
     const bool prep = W.bbuf != 0 && n_for_tokens(T) > 16;  // launch_decode prepares B then
     if (c1.tc) q1 = plan_decode(1, L.p1, T, L.num_sms, L.max_smem, prep);
     if (c2.tc) q2 = plan_decode(2, L.p2, T, L.num_sms, L.max_smem, prep);
-    if ((c1.tc && !q1.ok) || (c2.tc && !q2.ok)) return cudaErrorInvalidConfiguration;
+    if (c1.mma) q1 = plan_hdecode(1, L.p1, T, L.num_sms, L.max_smem);
+    if (c2.mma) q2 = plan_hdecode(2, L.p2, T, L.num_sms, L.max_smem);
+    if (((c1.tc || c1.mma) && !q1.ok) || ((c2.tc || c2.mma) && !q2.ok)) return cudaErrorInvalidConfiguration;
 
     DecodeArgs a1 = {};
     a1.signs = L.signs1;
@@ -1106,7 +1600,7 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
     // SwiGLU input: the CUDA-core kernels form h while staging; the
     // tensor-core kernel reads it from the workspace.
     const __half* u1 = x2 != nullptr ? ux + t0 * ldx : nullptr;
-    if (u1 != nullptr && c1.tc) {
+    if (u1 != nullptr && (c1.tc || c1.mma)) {
       e = launch_swiglu(a1.x, u1, ldx, T, L.n, hx, ldh, st);
       if (e != cudaSuccess) return e;
       a1.x = hx;
@@ -1114,6 +1608,8 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
     }
     if (c1.tc) {
       e = launch_decode<1>(a1, q1, st);
+    } else if (c1.mma) {
+      e = launch_hdecode<1>(a1, q1, st);
     } else if (c1.stream.ok) {
       LutProblem q = lut_problem(a1);
       q.x2 = u1;
@@ -1139,7 +1635,8 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
     a2.wait_cycles = a1.wait_cycles;
     a2.bbuf = a1.bbuf;
     a2.bstats = a1.bstats;
-    e = c2.tc         ? launch_decode<2>(a2, q2, st)
+    e = c2.tc          ? launch_decode<2>(a2, q2, st)
+        : c2.mma       ? launch_hdecode<2>(a2, q2, st)
         : c2.stream.ok ? launch_stream(2, lut_problem(a2), T, y_dtype, c2.stream, stat, st)
                        : launch_lut(2, lut_args(a2), c2.lut, st);
     if (e != cudaSuccess) return e;
@@ -1169,7 +1666,7 @@ cudaError_t launch_forward_multi(const af1_layer* const* Ls, int count, const vo
     const af1_layer& L = *Ls[i];
     const Workspace W = plan_workspace(L, tokens, prep);
     const PhaseChoice c1 = choose_phase(L, 1, L.p1, T, W), c2 = choose_phase(L, 2, L.p2, T, W);
-    if (c1.tc || c2.tc || c1.stream.ok || c2.stream.ok) group = false;
+    if (c1.tc || c2.tc || c1.mma || c2.mma || c1.stream.ok || c2.stream.ok) group = false;
     m1[i] = L.p1;
     m2[i] = L.p2;
   }

@@ -1,11 +1,14 @@
-"""Both decode kernels against the FP64 oracle, through the C ABI.
+"""The decode kernels against the FP64 oracle, through the C ABI.
 
-Decode passes (1..16 tokens) run on the CUDA-core lookup-table kernel by
-default; AF1_FLAG_TC_DECODE selects the tensor-core kernel. These cases cover
-the tensor-core kernel explicitly and the lookup-table kernel at its plan's
-edges: clusters whose last CTA finalises a short or empty slice of rows
-(14 and 15 CTAs per cluster), token groups with a ragged last group, and the
-longest contraction the library accepts (32768 columns).
+Decode passes (1..16 tokens) run on the CUDA-core lookup-table kernels up to
+4 tokens and on the 16-bit-operand tensor-core kernel from 5 tokens on (by
+default; test_gpu_mma_decode.py covers that kernel); AF1_FLAG_TC_DECODE
+selects the e4m3 tensor-core kernel and AF1_FLAG_LUT_DECODE the lookup-table
+kernels at every width. These cases cover the e4m3 kernel explicitly and the
+lookup-table kernel at its plan's edges: clusters whose last CTA finalises a
+short or empty slice of rows (14 and 15 CTAs per cluster), token groups with
+a ragged last group, and the longest contraction the library accepts (32768
+columns).
 """
 import numpy as np
 import pytest
@@ -66,7 +69,7 @@ def test_tensor_core_decode_full_size_sampled_rows(P, m, n, tokens):
 @pytest.mark.parametrize("tokens", [1, 4, 6, 13])
 def test_lookup_decode_cluster_slices(P, m, n, r, tokens):
     d = synth.layer_signs(3 * m + n + tokens, m, n, r, tokens)
-    layer = signs_layer(P, d)
+    layer = signs_layer(P, d, lut_decode=True)
     y = run_gpu(layer, d["x"], n, torch.float32)
     err = O.rowwise_rel_err(y, oracle_from_signs(d, n))
     assert err <= TOL, err
@@ -74,12 +77,13 @@ def test_lookup_decode_cluster_slices(P, m, n, r, tokens):
 
 
 @pytest.mark.parametrize("tokens", [1, 5, 16])
-@pytest.mark.parametrize("tc_decode", [False, True])
-def test_longest_contraction(P, tokens, tc_decode):
+@pytest.mark.parametrize("kernel", ["default", "tc", "lut", "mma"])
+def test_longest_contraction(P, tokens, kernel):
     m, n = 256, 32768
     r = O.rank_for_budget(m, n, 1)
     d = synth.layer_words(5 + tokens, m, n, r, tokens)
-    layer = words_layer(P, d, m, n, r, tc_decode=tc_decode)
+    layer = words_layer(P, d, m, n, r, tc_decode=kernel == "tc", lut_decode=kernel == "lut",
+                        mma_decode=kernel == "mma")
     y = run_gpu(layer, d["x"], n)
     ref = O.forward_from_packed(d["Uw"], d["Vw"], d["a"], d["s"], d["b"], d["x"], m, n, r)
     assert O.rowwise_rel_err(y, ref) <= TOL
