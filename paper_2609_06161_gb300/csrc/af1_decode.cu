@@ -806,56 +806,82 @@ __device__ __forceinline__ void bf16_split3(float v, uint16_t* t3) {
 // The B operand of the CTA's K slice (chunks of columns from k0, kv valid
 // columns), built by 128 threads (bt = 0..127): 16-byte units of 8 columns,
 // row n of K half h of chunk c at Bt + (2 c + h) N 128 + n 128, unit j at
-// (j ^ (n & 7)) 16 (128-byte swizzle, K-major). Columns >= kv are zero.
+// (j ^ (n & 7)) 16 (128-byte swizzle, K-major). Columns >= kv are zero. The
+// activations come from L2 (written by the previous kernel): each thread
+// issues the loads of UB units before it converts and stores any, so a CTA
+// waits for about T nu / (128 UB) round trips instead of T nu / 128.
+template <int PHASE>
+__device__ __forceinline__ void load_unit_h(const DecodeArgs& a, int t, int kl, int64_t k0, int kv, uint4 (&raw)[2]) {
+  if (PHASE == 1) {
+    const __half* p = a.x + (int64_t)t * a.ldx + k0 + kl;
+    if (kl + 7 < kv) {
+      raw[0] = __ldcg(reinterpret_cast<const uint4*>(p));
+    } else {
+      uint16_t e[8];
+#pragma unroll
+      for (int q = 0; q < 8; ++q) e[q] = kl + q < kv ? __half_as_ushort(__ldcg(p + q)) : (uint16_t)0;
+      raw[0] = make_uint4(e[0] | (uint32_t)e[1] << 16, e[2] | (uint32_t)e[3] << 16, e[4] | (uint32_t)e[5] << 16,
+                          e[6] | (uint32_t)e[7] << 16);
+    }
+  } else {
+    const float* p = a.zin + (int64_t)t * a.ldz + k0 + kl;
+    if (kl + 7 < kv) {
+      raw[0] = __ldcg(reinterpret_cast<const uint4*>(p));
+      raw[1] = __ldcg(reinterpret_cast<const uint4*>(p + 4));
+    } else {
+      uint32_t f[8];
+#pragma unroll
+      for (int q = 0; q < 8; ++q) f[q] = kl + q < kv ? __float_as_uint(__ldcg(p + q)) : 0u;
+      raw[0] = make_uint4(f[0], f[1], f[2], f[3]);
+      raw[1] = make_uint4(f[4], f[5], f[6], f[7]);
+    }
+  }
+}
+
 template <int PHASE, int N>
 __device__ __forceinline__ void build_b_h(const DecodeArgs& a, int T, int nch, int64_t k0, int kv, int bt,
                                           uint8_t* Bt) {
+  constexpr int UB = 4;
   const int nu = nch * (kChunkCols / 8);  // 8-column units per token
-  for (int i = bt; i < T * nu; i += 128) {
-    const int t = i / nu, u = i - t * nu;
-    const int kl = 8 * u;
-    const int c = u >> 4, hh = (u >> 3) & 1, j = u & 7;
-    uint8_t* half_base = Bt + (2 * c + hh) * (N * 128);
-    if (PHASE == 1) {
-      uint4 v = make_uint4(0u, 0u, 0u, 0u);
-      const __half* p = a.x + (int64_t)t * a.ldx + k0 + kl;
-      if (kl + 7 < kv) {
-        v = __ldcg(reinterpret_cast<const uint4*>(p));
+  const int total = T * nu;
+  for (int i0 = bt; i0 < total; i0 += UB * 128) {
+    uint4 raw[UB][2];
+#pragma unroll
+    for (int u = 0; u < UB; ++u) {
+      const int i = i0 + u * 128;
+      if (i < total) {
+        const int t = i / nu;
+        load_unit_h<PHASE>(a, t, 8 * (i - t * nu), k0, kv, raw[u]);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < UB; ++u) {
+      const int i = i0 + u * 128;
+      if (i >= total) break;
+      const int t = i / nu, uu = i - t * nu;
+      const int c = uu >> 4, hh = (uu >> 3) & 1, j = uu & 7;
+      uint8_t* half_base = Bt + (2 * c + hh) * (N * 128);
+      if (PHASE == 1) {
+        *reinterpret_cast<uint4*>(half_base + t * 128 + ((j ^ (t & 7)) << 4)) = raw[u][0];
       } else {
-        uint16_t e[8];
+        const uint32_t fw[8] = {raw[u][0].x, raw[u][0].y, raw[u][0].z, raw[u][0].w,
+                                raw[u][1].x, raw[u][1].y, raw[u][1].z, raw[u][1].w};
+        uint16_t e[3][8];
 #pragma unroll
-        for (int q = 0; q < 8; ++q) e[q] = kl + q < kv ? __half_as_ushort(__ldcg(p + q)) : (uint16_t)0;
-        v = make_uint4(e[0] | (uint32_t)e[1] << 16, e[2] | (uint32_t)e[3] << 16, e[4] | (uint32_t)e[5] << 16,
-                       e[6] | (uint32_t)e[7] << 16);
-      }
-      *reinterpret_cast<uint4*>(half_base + t * 128 + ((j ^ (t & 7)) << 4)) = v;
-    } else {
-      float f[8];
-      const float* p = a.zin + (int64_t)t * a.ldz + k0 + kl;
-      if (kl + 7 < kv) {
-        const float4 z0 = __ldcg(reinterpret_cast<const float4*>(p));
-        const float4 z1 = __ldcg(reinterpret_cast<const float4*>(p + 4));
-        f[0] = z0.x; f[1] = z0.y; f[2] = z0.z; f[3] = z0.w;
-        f[4] = z1.x; f[5] = z1.y; f[6] = z1.z; f[7] = z1.w;
-      } else {
+        for (int q = 0; q < 8; ++q) {
+          uint16_t t3[3];
+          bf16_split3(__uint_as_float(fw[q]), t3);
+          e[0][q] = t3[0];
+          e[1][q] = t3[1];
+          e[2][q] = t3[2];
+        }
 #pragma unroll
-        for (int q = 0; q < 8; ++q) f[q] = kl + q < kv ? __ldcg(p + q) : 0.f;
-      }
-      uint16_t e[3][8];
-#pragma unroll
-      for (int q = 0; q < 8; ++q) {
-        uint16_t t3[3];
-        bf16_split3(f[q], t3);
-        e[0][q] = t3[0];
-        e[1][q] = t3[1];
-        e[2][q] = t3[2];
-      }
-#pragma unroll
-      for (int term = 0; term < 3; ++term) {
-        const int n = 3 * t + term;
-        const uint4 v = make_uint4(e[term][0] | (uint32_t)e[term][1] << 16, e[term][2] | (uint32_t)e[term][3] << 16,
-                                   e[term][4] | (uint32_t)e[term][5] << 16, e[term][6] | (uint32_t)e[term][7] << 16);
-        *reinterpret_cast<uint4*>(half_base + n * 128 + ((j ^ (n & 7)) << 4)) = v;
+        for (int term = 0; term < 3; ++term) {
+          const int n = 3 * t + term;
+          const uint4 v = make_uint4(e[term][0] | (uint32_t)e[term][1] << 16, e[term][2] | (uint32_t)e[term][3] << 16,
+                                     e[term][4] | (uint32_t)e[term][5] << 16, e[term][6] | (uint32_t)e[term][7] << 16);
+          *reinterpret_cast<uint4*>(half_base + n * 128 + ((j ^ (n & 7)) << 4)) = v;
+        }
       }
     }
   }
