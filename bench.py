@@ -1009,7 +1009,12 @@ def main():
             elif (b == 1 and decode_kernel_of(b) == "lut" and args.schedule == "group" and args.ranks == "hisa"
                   and DECODE_TRAFFIC_RATIO_HISA_B1_GROUP is not None):
                 traffic = int(round(DECODE_TRAFFIC_RATIO_HISA_B1_GROUP * alg))
+            fam = decode_kernel_of(b)
             kname = ("af1_step_run (one persistent step_kernel launch per step)" if args.schedule == "step" else
+                     "af1_linear_forward (two 16-bit-operand tensor-core kernels per call, hdecode_kernel<1|2>)"
+                     if fam == "mma" else
+                     "af1_linear_forward (two e4m3 tensor-core kernels per call, decode_kernel<1|2>, with "
+                     "bprep_kernel for passes of more than 4 tokens)" if fam == "tc" else
                      "af1_linear_forward_multi / af1_linear_forward (two lookup-table kernels per call, "
                      "lut_kernel<1|2>)" if args.schedule == "group" else
                      "af1_linear_forward (two lookup-table kernels per call, lut_kernel<1|2>, stream_kernel<1|2> "
