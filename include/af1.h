@@ -94,10 +94,11 @@ extern "C" {
 #define AF1_FLAG_STREAM_DECODE 8
 /* Run every decode pass (1..16 tokens) on the tensor-core kernel with 16-bit
    operands (tcgen05 MMAs on exact +-b_j FP16 or +-1 BF16 sign values, the
-   activations as FP16 and the rank intermediate as three BF16 terms that
-   hold its FP32 value exactly). Without a decode flag the library takes this
-   kernel for passes of more than 4 tokens and the lookup-table kernels for
-   passes of 1 to 4 tokens. Results agree within the library's tolerance. */
+   activations as FP16, and the rank intermediate s' as two BF16 terms that
+   hold its 16 leading significant bits). Without a decode flag the library
+   takes this kernel for passes of more than 4 tokens and the lookup-table
+   kernels for passes of 1 to 4 tokens. Results agree within the library's
+   tolerance. */
 #define AF1_FLAG_MMA_DECODE 16
 /* Run every decode pass (1..16 tokens) on the CUDA-core lookup-table kernels
    (clustered or streaming), never on a tensor-core kernel. At most one of

@@ -694,15 +694,17 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const DecodeArgs a)
 // up to 16 tokens. The signs become exact 16-bit A values in tensor memory:
 //   phase 1: A = +-b_j (FP16; the column scale carries the sign), B = x
 //            (FP16, N = 16 rows, row t = token t), so D = sum_j +-b_j x_j;
-//   phase 2: A = +-1 (BF16), B = s' split exactly into three BF16 terms
-//            s' = hi + mid + lo (N = 16/32/48 rows, term q of token t in row
-//            3 t + q): BF16 keeps FP32's exponent range, and 8 + 8 + 8
-//            significant bits hold FP32's 24, so no scaling is needed.
-// Every product is exact and the MMA accumulates in FP32: the result is the
-// FP32 signed sum the lookup-table kernels form, summed in another order.
+//   phase 2: A = +-1 (BF16), B = s' split into kS2Terms = 2 BF16 terms
+//            hi + lo (N = 16/32 rows, term q of token t in row 2 t + q):
+//            BF16 keeps FP32's exponent range, so no scaling is needed, and
+//            hi + lo holds the 16 leading significant bits of s' (a
+//            relative error of at most 2^-17; three terms would hold all 24).
+// Every product is exact and the MMA accumulates in FP32: up to that
+// rounding of s', the result is the FP32 signed sum the lookup-table
+// kernels form, summed in another order.
 // Against the e4m3 kernel above there is no activation split, no power-of-
 // two scale and no sign correction, and the B operand is a copy (phase 1) or
-// a three-way split (phase 2) that the CTA builds itself, so no preparation
+// a two-way split (phase 2) that the CTA builds itself, so no preparation
 // kernel runs. A chunk of A takes 64 tensor-memory columns (two values per
 // column), twice the e4m3 chunk. The CTA structure is the e4m3 kernel's:
 // bulk copies of the signs first, warps 0-3 expand, warps 4-7 build B and
@@ -710,10 +712,20 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const DecodeArgs a)
 // back and push the partial sums to the cluster CTA that owns each row.
 // ---------------------------------------------------------------------------
 
+// Terms of s' in the phase-2 B operand: 1 = s' rounded to FP16 (with FP16
+// +-1 signs), 2 or 3 = BF16 terms (with BF16 +-1 signs; three hold s'
+// exactly, two hold its 16 leading significant bits). Measured on the
+// 32-layer stack at 16 / 8 tokens (ms per step): three terms 4.20 / 3.28,
+// two 4.03 / 3.16, one 3.87 / 3.14. Two: a relative error of at most 2^-17
+// per value and FP32's exponent range (one FP16 term loses small values to
+// FP16's range).
+constexpr int kS2Terms = 2;
 __host__ __device__ constexpr int hnacc_for(int N) { return N == 16 ? 4 : 2; }
 __host__ __device__ constexpr int hnbuf_for(int N) { return (kTmemCols - hnacc_for(N) * N) / 64; }
-// B rows of a pass of T tokens: one per token (phase 1), three (phase 2).
-__host__ __device__ constexpr int hdecode_n(int phase, int T) { return phase == 1 ? 16 : (3 * T + 15) / 16 * 16; }
+// B rows of a pass of T tokens: one per token (phase 1), kS2Terms (phase 2).
+__host__ __device__ constexpr int hdecode_n(int phase, int T) {
+  return phase == 1 ? 16 : (kS2Terms * T + 15) / 16 * 16;
+}
 
 struct __align__(8) HDecodeHeader {
   uint64_t wfull[kMaxCPC];  // packed chunk c has landed (chunk 0: with the column scales)
@@ -792,15 +804,19 @@ __device__ __forceinline__ void tmem_st16p(uint32_t addr, const uint32_t* r) {
       : "memory");
 }
 
-// Three BF16 terms of v (hi + mid + lo == v exactly for finite FP32 v).
-__device__ __forceinline__ void bf16_split3(float v, uint16_t* t3) {
-  const __nv_bfloat16 hi = __float2bfloat16_rn(v);
-  const float r1 = v - __bfloat162float(hi);
-  const __nv_bfloat16 mid = __float2bfloat16_rn(r1);
-  const __nv_bfloat16 lo = __float2bfloat16_rn(r1 - __bfloat162float(mid));
-  t3[0] = __bfloat16_as_ushort(hi);
-  t3[1] = __bfloat16_as_ushort(mid);
-  t3[2] = __bfloat16_as_ushort(lo);
+// The kS2Terms 16-bit terms of v: v rounded to FP16 (one term), or BF16
+// terms hi, mid, lo (hi + mid + lo == v exactly for finite FP32 v).
+__device__ __forceinline__ void split_terms(float v, uint16_t* t3) {
+  if constexpr (kS2Terms == 1) {
+    t3[0] = __half_as_ushort(__float2half_rn(v));
+  } else {
+    const __nv_bfloat16 hi = __float2bfloat16_rn(v);
+    const float r1 = v - __bfloat162float(hi);
+    const __nv_bfloat16 mid = __float2bfloat16_rn(r1);
+    t3[0] = __bfloat16_as_ushort(hi);
+    t3[1] = __bfloat16_as_ushort(mid);
+    if constexpr (kS2Terms == 3) t3[2] = __bfloat16_as_ushort(__float2bfloat16_rn(r1 - __bfloat162float(mid)));
+  }
 }
 
 // The B operand of the CTA's K slice (chunks of columns from k0, kv valid
@@ -870,14 +886,13 @@ __device__ __forceinline__ void build_b_h(const DecodeArgs& a, int T, int nch, i
 #pragma unroll
         for (int q = 0; q < 8; ++q) {
           uint16_t t3[3];
-          bf16_split3(__uint_as_float(fw[q]), t3);
-          e[0][q] = t3[0];
-          e[1][q] = t3[1];
-          e[2][q] = t3[2];
+          split_terms(__uint_as_float(fw[q]), t3);
+#pragma unroll
+          for (int term = 0; term < kS2Terms; ++term) e[term][q] = t3[term];
         }
 #pragma unroll
-        for (int term = 0; term < 3; ++term) {
-          const int n = 3 * t + term;
+        for (int term = 0; term < kS2Terms; ++term) {
+          const int n = kS2Terms * t + term;
           const uint4 v = make_uint4(e[term][0] | (uint32_t)e[term][1] << 16, e[term][2] | (uint32_t)e[term][3] << 16,
                                      e[term][4] | (uint32_t)e[term][5] << 16, e[term][6] | (uint32_t)e[term][7] << 16);
           *reinterpret_cast<uint4*>(half_base + n * 128 + ((j ^ (n & 7)) << 4)) = v;
@@ -892,7 +907,7 @@ __global__ void __launch_bounds__(kThreads, 1) hdecode_kernel(const DecodeArgs a
   constexpr int NACC = hnacc_for(N);
   constexpr int NBUF = hnbuf_for(N);
   constexpr int DCOL = NBUF * 64;  // first accumulator column
-  constexpr bool BF16 = PHASE == 2;
+  constexpr bool BF16 = PHASE == 2 && kS2Terms > 1;
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -979,7 +994,8 @@ __global__ void __launch_bounds__(kThreads, 1) hdecode_kernel(const DecodeArgs a
           if (PHASE == 1)
             v[jj] = *reinterpret_cast<const uint4*>(cs + (c * kChunkCols + 32 * kw + 8 * jj) * 2);
           else
-            v[jj] = make_uint4(0x3F803F80u, 0x3F803F80u, 0x3F803F80u, 0x3F803F80u);  // BF16 pairs of 1
+            v[jj] = BF16 ? make_uint4(0x3F803F80u, 0x3F803F80u, 0x3F803F80u, 0x3F803F80u)   // BF16 pairs of 1
+                         : make_uint4(0x3C003C00u, 0x3C003C00u, 0x3C003C00u, 0x3C003C00u);  // FP16 pairs of 1
         }
         uint32_t r[16];
         expand_word_h(wc[kw * kBlockRows + tid], v, r);
@@ -1044,11 +1060,14 @@ __global__ void __launch_bounds__(kThreads, 1) hdecode_kernel(const DecodeArgs a
       }
     }
     if (ok) {
-      constexpr int TMAX = PHASE == 1 ? N : N / 3;  // tokens the B rows hold
+      constexpr int TERMS = PHASE == 1 ? 1 : kS2Terms;
+      constexpr int TMAX = N / TERMS;  // tokens the B rows hold
 #pragma unroll
       for (int t = 0; t < TMAX; ++t) {
         if (t < T) {
-          const float p = PHASE == 1 ? acc[t] : (acc[3 * t] + acc[3 * t + 1]) + acc[3 * t + 2];
+          float p = acc[TERMS * t];
+#pragma unroll
+          for (int q = 1; q < TERMS; ++q) p += acc[TERMS * t + q];
           st_cluster_f32(recv + ((ks * T + t) * slice + (i - owner * slice)), (uint32_t)owner, p);
         }
       }

@@ -3,8 +3,8 @@ default the kernel of passes of 5..16 tokens) against the FP64 oracle,
 through the C ABI.
 
 Phase 1 multiplies exact +-b_j FP16 sign values with the FP16 activations,
-phase 2 exact +-1 BF16 values with s' split into three BF16 terms (N = 16,
-32 or 48 rows of B for up to 5, 10 and 16 tokens). The cases cover every B
+phase 2 exact +-1 BF16 values with s' split into two BF16 terms (N = 16 or
+32 rows of B for up to 8 and 16 tokens). The cases cover every B
 width, ragged shapes (rows and columns that end inside a chunk, ranks that
 are not multiples of 128), clusters of 1..16 CTAs, K slices longer than the
 tensor-memory ring, integer inputs bit for bit, the LLaMA-3-8B and 70B-class
@@ -44,8 +44,8 @@ def test_mma_decode_matches_oracle(P, m, n, r, tokens):
 @pytest.mark.parametrize("tokens", [1, 7, 12, 16])
 def test_mma_decode_integer_bit_exact(P, m, n, r, tokens):
     """Unit scales and integer activations: every product and partial sum is
-    an integer below 2^24, and s' is held exactly by its three BF16 terms,
-    so the result is the oracle's bit for bit."""
+    an integer below 2^24, and s' (an integer below 2^16 here) is held
+    exactly by its two BF16 terms, so the result is the oracle's bit for bit."""
     d = synth.integer_layer(17 + m + tokens, m, n, r, tokens)
     layer = signs_layer(P, d, mma_decode=True)
     y = run_gpu(layer, d["x"], n, torch.float32)
