@@ -181,9 +181,9 @@ FULL_70B = [(8192, 8192), (1024, 8192), (28672, 8192), (8192, 28672)]
 @pytest.mark.parametrize("tokens", [8, 64, 512])
 def test_full_size_70b_sampled_rows(P, m, n, tokens):
     """The 70B-class shapes of the decode/prefill crossover sweep at their
-    full size: 8 tokens (decode; the prepared tensor-core operand on the large
-    matrices) and 64 / 512 tokens (prefill; split K over a cluster at 64,
-    including the long-K split of the 8192 x 28672 first GEMM)."""
+    full size: 8 tokens (decode on the 16-bit-operand tensor-core kernel)
+    and 64 / 512 tokens (prefill, including the long-K split of the
+    8192 x 28672 first GEMM)."""
     r = O.rank_for_budget(m, n, 1)
     d = synth.layer_words(3000 + m // 1024 + n // 1024 + tokens, m, n, r, tokens)
     layer = words_layer(P, d, m, n, r)
@@ -216,12 +216,15 @@ def test_workspace_shared_across_layers_and_calls(P):
     lb.free()
 
 
-def test_cuda_graph_replay(P):
+@pytest.mark.parametrize("tokens", [2, 12])
+def test_cuda_graph_replay(P, tokens):
+    """A forward call captured in a CUDA graph and replayed: the lookup-table
+    kernels (2 tokens) and the 16-bit-operand tensor-core kernel (12)."""
     m, n, r = 1024, 4096, 800
-    d = synth.layer_signs(31, m, n, r, 2)
+    d = synth.layer_signs(31 + tokens, m, n, r, tokens)
     layer = signs_layer(P, d)
-    x = f16(d["x"]).reshape(2, n)
-    y = torch.empty((2, m), dtype=torch.float32, device="cuda")
+    x = f16(d["x"]).reshape(tokens, n)
+    y = torch.empty((tokens, m), dtype=torch.float32, device="cuda")
     ws = layer.make_workspace()
     s = torch.cuda.Stream()
     with torch.cuda.stream(s):
