@@ -80,6 +80,10 @@ cudaError_t launch_swiglu(const __half* g, const __half* u, int64_t ldx, int64_t
 // default is about 1 s at the GB300's 2 GHz clock.
 constexpr long long kDefaultWaitCycles = 2000000000ll;
 long long wait_budget();
+// Whether the lookup-table kernels' second phase lets its dependent launch
+// only after its lookups (af1_set_launch_order(AF1_LAUNCH_LATE);
+// process-wide).
+bool late_launch();
 // Set the calling thread's af1_last_error() message; returns `code`.
 int set_error(int code, const std::string& msg);
 
@@ -111,6 +115,7 @@ struct LutArgs {
   int KS;            // set by the launcher: CTAs per cluster, common to all problems
   unsigned* status;
   long long wait_cycles;  // budget of every bounded wait (clock64 cycles)
+  int late_trigger;       // phase 2: let the dependent launch after the lookups, not after the input
   LutProblem prob[kMaxGroup];
 };
 struct LutPlan {

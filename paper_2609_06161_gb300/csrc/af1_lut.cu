@@ -153,9 +153,13 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const __grid_constant_
   // CTAs copy their U words from HBM while this kernel computes (they hold
   // no input of another call). Measured against launching it after the
   // lookups (below): config-1 stack 6.33 -> 6.22 us per linear on the DAG
-  // schedule, 6.42 -> 6.13 grouped, 8.62 -> 8.42 serial; letting phase 2's
-  // own dependents launch this early too lost on the DAG (6.43).
-  if (PHASE == 1) griddep_launch_dependents();
+  // schedule, 6.42 -> 6.13 grouped, 8.62 -> 8.42 serial. Phase 2 does the
+  // same unless the caller asked for the late order (AF1_LAUNCH_LATE): early
+  // wins on one stream (32-layer HiSA-rank step at one token, grouped calls:
+  // 1.323 -> 1.277 ms), late on the decoder DAG over three streams (1.480
+  // -> 1.437 ms), where the next kernel's waiting CTAs would hold SM slots
+  // that the sibling streams' kernels need.
+  if (PHASE == 1 || !a.late_trigger) griddep_launch_dependents();
   stage_activations<PHASE, kThreads, SWIGLU>(pb, xg, x2g, zg, T, nch, k0, zs, zrow, tid);
   if (tid < slice) rs[tid] = rs_own;
   __syncthreads();
@@ -178,12 +182,12 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const __grid_constant_
     }
   }
 
-  // Phase 2 lets the next kernel launch only now: its CTAs would otherwise
-  // hold SM slots (waiting for this kernel) that sibling kernels on other
-  // streams need, and its sign copies still get the reduction's time as a
-  // head start (measured: config-1 stack 7.40 -> 6.53 us per linear on the
-  // DAG schedule, trigger at the start vs here).
-  if (PHASE == 2) griddep_launch_dependents();
+  // The late order: phase 2 lets the next kernel launch only now, so its
+  // CTAs do not hold SM slots (waiting for this kernel) that sibling kernels
+  // on other streams need, and its sign copies still get the reduction's
+  // time as a head start (measured: config-1 stack 7.40 -> 6.53 us per
+  // linear on the DAG schedule, trigger at the start vs here).
+  if (PHASE == 2 && a.late_trigger) griddep_launch_dependents();
   // ---- partial sums -> owner CTA of each row -> final sums -------------------
   cluster_wait();  // every CTA of the cluster has started
   {

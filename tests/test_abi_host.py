@@ -114,3 +114,19 @@ def test_host_validation_errors():
                                   None) == -1
     lib.af1_free(None)  # NULL-safe
     assert P.version().startswith("af1-gb300")
+
+
+def test_launch_order_setting():
+    _ensure_built()
+    import paper_2609_06161_gb300 as P
+    assert P.get_launch_order() == P.AF1_LAUNCH_EARLY  # the default
+    try:
+        P.set_launch_order(P.AF1_LAUNCH_LATE)
+        assert P.get_launch_order() == P.AF1_LAUNCH_LATE
+        with pytest.raises(P.AF1Error) as e:
+            P.set_launch_order(2)
+        assert e.value.code == -1
+        assert P.get_launch_order() == P.AF1_LAUNCH_LATE  # unchanged by the rejected call
+    finally:
+        P.set_launch_order(P.AF1_LAUNCH_EARLY)
+    assert P.get_launch_order() == P.AF1_LAUNCH_EARLY
