@@ -307,8 +307,8 @@ def config_dict(args):
                          f"/ down 4096x14336), {ranks}, x {args.layers} layers, decode batch {args.batch}, "
                          + SCHEDULES[args.schedule] + ("" if args.no_graph else ", CUDA graph")),
             "batch": args.batch, "layers": args.layers, "linears_per_step": 7 * args.layers, "ranks": args.ranks,
-            "launch_order": ("late (af1_set_launch_order: the DAG's parallel streams)" if args.schedule == "dag"
-                             else "early (af1_set_launch_order: one stream)"),
+            "stream_layout": ("AF1_MANY_STREAMS (af1_set_stream_layout: the DAG's parallel streams)"
+                              if args.schedule == "dag" else "AF1_ONE_STREAM (af1_set_stream_layout)"),
             "decode_kernel": decode_kernel_name(args.batch),
             "l2": "inputs larger than L2 (packed weights per step >> 129 MB), no flush"}
 
@@ -445,10 +445,10 @@ def sweep(P, torch, peaks, stream):
     and 512 tokens (prefill path, tensor roofline); each against dense BF16
     torch.matmul of the same shape. Calls rotate over copies of the layer
     totalling at least twice the L2, so every call streams its weights from
-    HBM. Single calls on one stream: the early launch order."""
+    HBM. Single calls on one stream: the one-stream layout."""
     import math
     import synth
-    P.set_launch_order(P.AF1_LAUNCH_EARLY)
+    P.set_stream_layout(P.AF1_ONE_STREAM)
     hbm = peaks.get("hbm_gbs", 6800.0)
     tpk = peaks.get("bf16_tflops_sustained", 1700.0)
     plan = [("q/o", 4096, 4096, (1, 4, 16)), ("k/v", 1024, 4096, (1, 4, 16)),
@@ -636,8 +636,8 @@ def mlp_swiglu(P, torch, stream, steps):
     the down projection of h = FP16(SiLU(gate) * up). Fused: the down call
     forms h itself (af1_linear_forward_swiglu); unfused: h by torch
     elementwise ops, then af1_linear_forward. 32 blocks rotate (weights far
-    larger than L2); CUDA graph; the late launch order (two streams)."""
-    P.set_launch_order(P.AF1_LAUNCH_LATE)
+    larger than L2); CUDA graph; the many-streams layout (two streams)."""
+    P.set_stream_layout(P.AF1_MANY_STREAMS)
     blocks = 32
     rank = P.rank_for_budget
     mk = lambda m, n, seed: device_layer(P, torch, m, n, rank(m, n), seed)
@@ -684,10 +684,10 @@ def mlp_swiglu(P, torch, stream, steps):
             "unfused": "h by torch elementwise ops (FP32 SiLU and product, FP16 store), then af1_linear_forward"}
 
 
-def launch_order_for(P, schedule):
-    """AF1_LAUNCH_LATE for the decoder DAG (parallel streams), AF1_LAUNCH_EARLY
+def stream_layout_for(P, schedule):
+    """AF1_MANY_STREAMS for the decoder DAG (parallel streams), AF1_ONE_STREAM
     for the one-stream schedules."""
-    return P.AF1_LAUNCH_LATE if schedule == "dag" else P.AF1_LAUNCH_EARLY
+    return P.AF1_MANY_STREAMS if schedule == "dag" else P.AF1_ONE_STREAM
 
 
 def stack_other_ranks(P, torch, peaks, stream, steps, args):
@@ -719,7 +719,7 @@ def stack_other_ranks(P, torch, peaks, stream, steps, args):
     else:
         def run():
             dag_step(torch, views, stream, side, ws, ws_side)
-    P.set_launch_order(launch_order_for(P, args.schedule))
+    P.set_stream_layout(stream_layout_for(P, args.schedule))
     ms_dag = time_graph(torch, run, stream, max(5, min(steps, 20)))
     alg = sum(algorithmic_bytes(m, n, r, 1) for (m, n), r in zip(mn, ranks))
     bits = sum(P.storage_bits(m, n, r) for (m, n), r in zip(mn, ranks))
@@ -853,9 +853,9 @@ def main():
         group_step(P, views, stream, ws, ws_multi)
 
     def make_graph(fn, name):
-        # The lookup-table kernels' launch order suits the schedule: late on
-        # the DAG's parallel streams, early on one stream (af1_set_launch_order).
-        P.set_launch_order(launch_order_for(P, name))
+        # The library's stream layout suits the schedule: several streams for
+        # the DAG, one stream otherwise (af1_set_stream_layout).
+        P.set_stream_layout(stream_layout_for(P, name))
         with torch.cuda.stream(stream):
             fn()
         torch.cuda.synchronize()

@@ -345,24 +345,29 @@ AF1_API int af1_workspace_status(void* workspace, void* stream);
 AF1_API int af1_set_wait_cycles(int64_t cycles);
 AF1_API int64_t af1_get_wait_cycles(void);
 
-/* When the second kernel of a decode call on the lookup-table kernels
- * (passes of 1 to 4 tokens) lets the next kernel of its stream launch
- * (programmatic dependent launch; the next kernel's CTAs then fetch their
- * sign words and wait for this kernel's outputs):
- *   AF1_LAUNCH_EARLY (default): as soon as it has read its input. Best when
- *     the caller runs its layers on one stream (measured on a 32-layer
- *     decode step at one token: 1.323 -> 1.277 ms).
- *   AF1_LAUNCH_LATE: after its lookups, which keeps SM slots free for
- *     kernels on other streams. Best when several streams run layers at
- *     once (the same step on the decoder's dependency DAG over three
- *     streams: 1.480 -> 1.437 ms).
- * Results are identical either way. Process-wide, for launches after the
- * call on any thread; a launch captured in a CUDA graph keeps the order it
- * was captured with. Errors: INVALID_ARG (another value). */
-#define AF1_LAUNCH_EARLY 0
-#define AF1_LAUNCH_LATE 1
-AF1_API int af1_set_launch_order(int order);
-AF1_API int af1_get_launch_order(void);
+/* How the caller runs its layers' calls, which the lookup-table decode
+ * kernels (passes of 1 to 4 tokens) adapt to:
+ *   AF1_ONE_STREAM (default): one call after another on one stream. The
+ *     second kernel of a call lets the next kernel of the stream launch
+ *     (programmatic dependent launch) as soon as it has read its input, so
+ *     the next kernel's CTAs fetch their sign words meanwhile, and a single
+ *     call spreads each phase over about three CTAs per SM.
+ *   AF1_MANY_STREAMS: several streams run layers at once (e.g. q | k | v of
+ *     a decoder layer on three streams). The next kernel launches only after
+ *     the lookups, and a call takes about two CTAs per SM, which leaves SM
+ *     slots to the kernels of the other streams.
+ * Measured on a 32-layer decode step at one token: grouped calls on one
+ * stream 1.323 ms (many-stream settings) -> 1.249 ms (one-stream settings);
+ * the decoder's dependency DAG over three streams 1.478 -> 1.436 ms the
+ * other way round. Both give results within the library's tolerance (the
+ * K split of a call, and so the order of its FP32 sums, can differ).
+ * Process-wide, for calls made after this one on any thread; a launch
+ * captured in a CUDA graph keeps the setting it was captured with.
+ * Errors: INVALID_ARG (another value). */
+#define AF1_ONE_STREAM 0
+#define AF1_MANY_STREAMS 1
+AF1_API int af1_set_stream_layout(int layout);
+AF1_API int af1_get_stream_layout(void);
 
 /* ---- A decode step as one launch ---------------------------------------------
  * Many linears (e.g. the 7 of each decoder layer of a model) in dependent

@@ -127,10 +127,10 @@ _lib.af1_set_wait_cycles.argtypes = [_i64]
 _lib.af1_set_wait_cycles.restype = ctypes.c_int
 _lib.af1_get_wait_cycles.argtypes = []
 _lib.af1_get_wait_cycles.restype = _i64
-_lib.af1_set_launch_order.argtypes = [ctypes.c_int]
-_lib.af1_set_launch_order.restype = ctypes.c_int
-_lib.af1_get_launch_order.argtypes = []
-_lib.af1_get_launch_order.restype = ctypes.c_int
+_lib.af1_set_stream_layout.argtypes = [ctypes.c_int]
+_lib.af1_set_stream_layout.restype = ctypes.c_int
+_lib.af1_get_stream_layout.argtypes = []
+_lib.af1_get_stream_layout.restype = ctypes.c_int
 
 
 class _StepLinear(ctypes.Structure):
@@ -228,19 +228,20 @@ def get_wait_cycles() -> int:
     return int(_lib.af1_get_wait_cycles())
 
 
-AF1_LAUNCH_EARLY = 0
-AF1_LAUNCH_LATE = 1
+AF1_ONE_STREAM = 0
+AF1_MANY_STREAMS = 1
 
 
-def set_launch_order(order: int) -> None:
-    """AF1_LAUNCH_EARLY (default; best on one stream) or AF1_LAUNCH_LATE (best
-    when several streams run layers at once): when the lookup-table decode
-    kernels let the next kernel of their stream launch (af1_set_launch_order)."""
-    _check(_lib.af1_set_launch_order(int(order)))
+def set_stream_layout(layout: int) -> None:
+    """AF1_ONE_STREAM (default: calls one after another on one stream) or
+    AF1_MANY_STREAMS (several streams run layers at once); the lookup-table
+    decode kernels adapt their launch order and CTA count to it
+    (af1_set_stream_layout)."""
+    _check(_lib.af1_set_stream_layout(int(layout)))
 
 
-def get_launch_order() -> int:
-    return int(_lib.af1_get_launch_order())
+def get_stream_layout() -> int:
+    return int(_lib.af1_get_stream_layout())
 
 
 class Layer:

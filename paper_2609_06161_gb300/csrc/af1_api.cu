@@ -182,14 +182,14 @@ int check_scales(const uint16_t* a, const uint16_t* s, const uint16_t* b, int de
 
 namespace {
 std::atomic<long long> g_wait_cycles{af1::kDefaultWaitCycles};
-std::atomic<int> g_launch_order{AF1_LAUNCH_EARLY};
+std::atomic<int> g_stream_layout{AF1_ONE_STREAM};
 }  // namespace
 
 namespace af1 {
 // Record a failure in the calling thread's af1_last_error() message.
 int set_error(int code, const std::string& msg) { return fail(code, msg); }
 long long wait_budget() { return g_wait_cycles.load(std::memory_order_relaxed); }
-bool late_launch() { return g_launch_order.load(std::memory_order_relaxed) == AF1_LAUNCH_LATE; }
+bool many_streams() { return g_stream_layout.load(std::memory_order_relaxed) == AF1_MANY_STREAMS; }
 }  // namespace af1
 
 extern "C" {
@@ -611,15 +611,15 @@ int af1_set_wait_cycles(int64_t cycles) {
 
 int64_t af1_get_wait_cycles(void) { return g_wait_cycles.load(std::memory_order_relaxed); }
 
-int af1_set_launch_order(int order) {
-  if (order != AF1_LAUNCH_EARLY && order != AF1_LAUNCH_LATE)
-    return fail(AF1_ERR_INVALID_ARG, "order must be AF1_LAUNCH_EARLY or AF1_LAUNCH_LATE");
-  g_launch_order.store(order, std::memory_order_relaxed);
+int af1_set_stream_layout(int layout) {
+  if (layout != AF1_ONE_STREAM && layout != AF1_MANY_STREAMS)
+    return fail(AF1_ERR_INVALID_ARG, "layout must be AF1_ONE_STREAM or AF1_MANY_STREAMS");
+  g_stream_layout.store(layout, std::memory_order_relaxed);
   g_err.clear();
   return AF1_OK;
 }
 
-int af1_get_launch_order(void) { return g_launch_order.load(std::memory_order_relaxed); }
+int af1_get_stream_layout(void) { return g_stream_layout.load(std::memory_order_relaxed); }
 
 void af1_free(af1_layer* layer) { destroy_layer(layer); }
 

@@ -1458,7 +1458,7 @@ LutArgs lut_args(const DecodeArgs& d) {
   a.ydtype = d.ydtype;
   a.status = d.status;
   a.wait_cycles = d.wait_cycles;
-  a.late_trigger = late_launch() ? 1 : 0;
+  a.late_trigger = many_streams() ? 1 : 0;
   a.prob[0] = lut_problem(d);
   return a;
 }
@@ -1738,7 +1738,7 @@ cudaError_t launch_forward_multi(const af1_layer* const* Ls, int count, const vo
   a1.ydtype = a2.ydtype = y_dtype;
   a1.status = a2.status = status;
   a1.wait_cycles = a2.wait_cycles = wait_budget();
-  a1.late_trigger = a2.late_trigger = late_launch() ? 1 : 0;
+  a1.late_trigger = a2.late_trigger = many_streams() ? 1 : 0;
   for (int i = 0; i < count; ++i) {
     const af1_layer& L = *Ls[i];
     const Workspace W = plan_workspace(L, tokens, prep);

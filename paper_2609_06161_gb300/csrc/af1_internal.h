@@ -80,10 +80,10 @@ cudaError_t launch_swiglu(const __half* g, const __half* u, int64_t ldx, int64_t
 // default is about 1 s at the GB300's 2 GHz clock.
 constexpr long long kDefaultWaitCycles = 2000000000ll;
 long long wait_budget();
-// Whether the lookup-table kernels' second phase lets its dependent launch
-// only after its lookups (af1_set_launch_order(AF1_LAUNCH_LATE);
-// process-wide).
-bool late_launch();
+// Whether the caller runs layers on several streams at once
+// (af1_set_stream_layout(AF1_MANY_STREAMS); process-wide): the lookup-table
+// kernels then let their dependents launch late and take fewer CTAs.
+bool many_streams();
 // Set the calling thread's af1_last_error() message; returns `code`.
 int set_error(int code, const std::string& msg);
 

@@ -154,7 +154,7 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const __grid_constant_
   // no input of another call). Measured against launching it after the
   // lookups (below): config-1 stack 6.33 -> 6.22 us per linear on the DAG
   // schedule, 6.42 -> 6.13 grouped, 8.62 -> 8.42 serial. Phase 2 does the
-  // same unless the caller asked for the late order (AF1_LAUNCH_LATE): early
+  // same unless the caller runs several streams (AF1_MANY_STREAMS): early
   // wins on one stream (32-layer HiSA-rank step at one token, grouped calls:
   // 1.323 -> 1.277 ms), late on the decoder DAG over three streams (1.480
   // -> 1.437 ms), where the next kernel's waiting CTAs would hold SM slots
@@ -281,16 +281,21 @@ cudaError_t launch_np(const LutArgs& a, const LutPlan& p, cudaStream_t st) {
 namespace {
 
 // Split of one sign matrix for a pass of T <= 16 tokens, run as ceil(T / 4)
-// token groups of CTAs: about two CTAs per SM (row blocks x KS x groups ~
-// 2 SMs, KS <= 16 CTAs per cluster), CTAs small enough that three fit on an
-// SM, and at most kMaxCPC chunks each. Returns KS (0: no plan), *cpc and
-// *smem.
+// token groups of CTAs: about three CTAs per SM when the caller runs one
+// stream, two when it runs several (row blocks x KS x groups ~ 3 or 2 SMs,
+// KS <= 16 CTAs per cluster), CTAs small enough that three fit on an SM,
+// and at most kMaxCPC chunks each. Returns KS (0: no plan), *cpc and *smem.
+// Measured on the 32-layer HiSA-rank step at one token (ms per step, two /
+// three / four CTAs per SM): one stream, one call per layer 1.850 / 1.747 /
+// 1.745, grouped calls (q | k | v and gate | up keep their own one-wave
+// split) 1.278 / 1.249 / 1.442; the DAG over three streams 1.436 / 1.478.
 int plan_one(const SignMatrix& sm, int T, int sms, int max_smem, int* cpc_out, int* smem_out) {
   const int Tg = T < kGroupTokens ? T : kGroupTokens;
   const int groups = (T + kGroupTokens - 1) / kGroupTokens;
   const int cap = max_smem / 3 < 72 * 1024 ? max_smem / 3 : 72 * 1024;
   const int64_t tiles = (int64_t)sm.RB * groups;
-  int ks = (int)((2 * sms + tiles - 1) / tiles);
+  const int per_sm = many_streams() ? 2 : 3;
+  int ks = (int)((per_sm * sms + tiles - 1) / tiles);
   if (ks > kMaxKS) ks = kMaxKS;
   if (ks > sm.NCH) ks = sm.NCH;
   if (ks < 1) ks = 1;

@@ -116,17 +116,17 @@ def test_host_validation_errors():
     assert P.version().startswith("af1-gb300")
 
 
-def test_launch_order_setting():
+def test_stream_layout_setting():
     _ensure_built()
     import paper_2609_06161_gb300 as P
-    assert P.get_launch_order() == P.AF1_LAUNCH_EARLY  # the default
+    assert P.get_stream_layout() == P.AF1_ONE_STREAM  # the default
     try:
-        P.set_launch_order(P.AF1_LAUNCH_LATE)
-        assert P.get_launch_order() == P.AF1_LAUNCH_LATE
+        P.set_stream_layout(P.AF1_MANY_STREAMS)
+        assert P.get_stream_layout() == P.AF1_MANY_STREAMS
         with pytest.raises(P.AF1Error) as e:
-            P.set_launch_order(2)
+            P.set_stream_layout(2)
         assert e.value.code == -1
-        assert P.get_launch_order() == P.AF1_LAUNCH_LATE  # unchanged by the rejected call
+        assert P.get_stream_layout() == P.AF1_MANY_STREAMS  # unchanged by the rejected call
     finally:
-        P.set_launch_order(P.AF1_LAUNCH_EARLY)
-    assert P.get_launch_order() == P.AF1_LAUNCH_EARLY
+        P.set_stream_layout(P.AF1_ONE_STREAM)
+    assert P.get_stream_layout() == P.AF1_ONE_STREAM
