@@ -47,7 +47,7 @@ DECODE_TRAFFIC_B1_PER_LAYER = 28145408
 DECODE_TRAFFIC_RATIO_HISA_B1 = 170377216 / 164560648
 # The same on the grouped schedule (q|k|v and gate|up as one multi-layer call
 # each): ncu, profiles/lut_kernel_llama3_8b_hisa_b1_group.md.
-DECODE_TRAFFIC_RATIO_HISA_B1_GROUP = 169385216 / 164560648
+DECODE_TRAFFIC_RATIO_HISA_B1_GROUP = 169402880 / 164560648
 DECODE_KERNEL = "auto"  # set from --decode-kernel / --tc-decode
 
 
