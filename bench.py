@@ -492,7 +492,8 @@ def sweep(P, torch, peaks, stream):
                           "achieved_gbs": alg / (us * 1e-6) / 1e9, "frac": alg / (us * 1e-6) / 1e9 / hbm})
             else:
                 fl = 2 * b * r * (m + n)
-                e.update({"path": "prefill", "bound": "tensor", "flops": fl,
+                e.update({"path": "one 16-bit-operand decode pass" if mid_pass_of(m, n, r, b) else "prefill",
+                          "bound": "tensor", "flops": fl,
                           "achieved_tflops": fl / (us * 1e-6) / 1e12, "frac": fl / (us * 1e-6) / 1e12 / tpk})
             out.append(e)
             del ws, x, y, xb
@@ -514,6 +515,16 @@ def decode_kernel_of(b):
     if DECODE_KERNEL != "auto":
         return DECODE_KERNEL
     return "mma" if b > LUT_MAX_TOKENS else "lut"
+
+
+def mid_pass_of(m, n, r, b):
+    """Whether a call of 17..64 tokens runs as one pass of the 16-bit-operand
+    decode kernel instead of the prefill kernel (the library's rule: up to 24
+    tokens below 70 M signs, up to 64 below 20 M; no LUT or e4m3 flag)."""
+    if DECODE_KERNEL in ("lut", "tc") or not 16 < b <= 64:
+        return False
+    signs = r * (m + n)
+    return (b <= 24 and signs <= 70_000_000) or signs <= 20_000_000
 
 
 def phase_launches(m, n, r, b):

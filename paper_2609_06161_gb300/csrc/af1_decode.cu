@@ -713,19 +713,22 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const DecodeArgs a)
 // ---------------------------------------------------------------------------
 
 // Terms of s' in the phase-2 B operand: 1 = s' rounded to FP16 (with FP16
-// +-1 signs), 2 or 3 = BF16 terms (with BF16 +-1 signs; three hold s'
-// exactly, two hold its 16 leading significant bits). Measured on the
-// 32-layer stack at 16 / 8 tokens (ms per step): three terms 4.20 / 3.28,
-// two 4.03 / 3.16, one 3.87 / 3.14. Two: a relative error of at most 2^-17
-// per value and FP32's exponent range (one FP16 term loses small values to
-// FP16's range).
+// +-1 signs), 2 = BF16 terms (with BF16 +-1 signs) that hold its 16 leading
+// significant bits. Measured on the 32-layer stack at 16 / 8 tokens (ms per
+// step): three BF16 terms (s' exactly) 4.20 / 3.28, two 4.03 / 3.16, one
+// 3.87 / 3.14. Two: a relative error of at most 2^-17 per value and FP32's
+// exponent range (one FP16 term loses small values to FP16's range; three
+// would need an epilogue that sums a token's terms across column blocks).
 constexpr int kS2Terms = 2;
-__host__ __device__ constexpr int hnacc_for(int N) { return N == 16 ? 4 : 2; }
+// Accumulators (one MMA issuer each) and A-ring depth for N rows of B,
+// within the CTA's 256 tensor-memory columns: N 16: 4 and 3; 32: 2 and 3;
+// 48 / 64: 2 and 2; 128: 1 and 2.
+__host__ __device__ constexpr int hnacc_for(int N) { return N == 16 ? 4 : N <= 64 ? 2 : 1; }
 __host__ __device__ constexpr int hnbuf_for(int N) { return (kTmemCols - hnacc_for(N) * N) / 64; }
-// B rows of a pass of T tokens: one per token (phase 1), kS2Terms (phase 2).
-__host__ __device__ constexpr int hdecode_n(int phase, int T) {
-  return phase == 1 ? 16 : (kS2Terms * T + 15) / 16 * 16;
-}
+// B rows of a pass of T tokens (up to kMidMaxTokens): T rows (phase 1) or
+// kS2Terms T rows (phase 2), rounded up to 16, 32, 64 or 128.
+__host__ __device__ constexpr int hround_n(int rows) { return rows <= 16 ? 16 : rows <= 32 ? 32 : rows <= 64 ? 64 : 128; }
+__host__ __device__ constexpr int hdecode_n(int phase, int T) { return hround_n(phase == 1 ? T : kS2Terms * T); }
 
 struct __align__(8) HDecodeHeader {
   uint64_t wfull[kMaxCPC];  // packed chunk c has landed (chunk 0: with the column scales)
@@ -804,18 +807,16 @@ __device__ __forceinline__ void tmem_st16p(uint32_t addr, const uint32_t* r) {
       : "memory");
 }
 
-// The kS2Terms 16-bit terms of v: v rounded to FP16 (one term), or BF16
-// terms hi, mid, lo (hi + mid + lo == v exactly for finite FP32 v).
+// The kS2Terms 16-bit terms of v: v rounded to FP16 (one term), or the BF16
+// terms hi and lo (v - hi is exact in FP32; lo is it rounded to BF16).
 __device__ __forceinline__ void split_terms(float v, uint16_t* t3) {
   if constexpr (kS2Terms == 1) {
     t3[0] = __half_as_ushort(__float2half_rn(v));
   } else {
     const __nv_bfloat16 hi = __float2bfloat16_rn(v);
     const float r1 = v - __bfloat162float(hi);
-    const __nv_bfloat16 mid = __float2bfloat16_rn(r1);
     t3[0] = __bfloat16_as_ushort(hi);
-    t3[1] = __bfloat16_as_ushort(mid);
-    if constexpr (kS2Terms == 3) t3[2] = __bfloat16_as_ushort(__float2bfloat16_rn(r1 - __bfloat162float(mid)));
+    t3[1] = __bfloat16_as_ushort(__float2bfloat16_rn(r1));
   }
 }
 
@@ -1045,30 +1046,35 @@ __global__ void __launch_bounds__(kThreads, 1) hdecode_kernel(const DecodeArgs a
     const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
     const int i = tid;  // block row
     const int owner = i / slice;
-    float acc[N];
+    // One block of 16 accumulator columns at a time (the accumulators summed
+    // in a fixed order), then the tokens whose terms lie in the block.
+    constexpr int TERMS = PHASE == 1 ? 1 : kS2Terms;
+    static_assert(16 % TERMS == 0, "a token's terms must lie in one block of 16 columns");
+    constexpr int TPB = 16 / TERMS;  // tokens per block
 #pragma unroll
-    for (int j = 0; j < N; ++j) acc[j] = 0.f;
+    for (int cb = 0; cb < N / 16; ++cb) {
+      if (cb * TPB >= T) break;
+      float acc[16];
 #pragma unroll
-    for (int d = 0; d < NACC; ++d) {
+      for (int j = 0; j < 16; ++j) acc[j] = 0.f;
 #pragma unroll
-      for (int cb = 0; cb < N / 16; ++cb) {
+      for (int d = 0; d < NACC; ++d) {
         uint32_t r[16];
         tmem_ld16(tmem + lane_base + (uint32_t)(DCOL + d * N + cb * 16), r);
         asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 #pragma unroll
-        for (int j = 0; j < 16; ++j) acc[cb * 16 + j] += __uint_as_float(r[j]);
+        for (int j = 0; j < 16; ++j) acc[j] += __uint_as_float(r[j]);
       }
-    }
-    if (ok) {
-      constexpr int TERMS = PHASE == 1 ? 1 : kS2Terms;
-      constexpr int TMAX = N / TERMS;  // tokens the B rows hold
+      if (ok) {
 #pragma unroll
-      for (int t = 0; t < TMAX; ++t) {
-        if (t < T) {
-          float p = acc[TERMS * t];
+        for (int tl = 0; tl < TPB; ++tl) {
+          const int t = cb * TPB + tl;
+          if (t < T) {
+            float p = acc[TERMS * tl];
 #pragma unroll
-          for (int q = 1; q < TERMS; ++q) p += acc[TERMS * t + q];
-          st_cluster_f32(recv + ((ks * T + t) * slice + (i - owner * slice)), (uint32_t)owner, p);
+            for (int q = 1; q < TERMS; ++q) p += acc[TERMS * tl + q];
+            st_cluster_f32(recv + ((ks * T + t) * slice + (i - owner * slice)), (uint32_t)owner, p);
+          }
         }
       }
     }
@@ -1421,14 +1427,13 @@ template <int PHASE>
 cudaError_t launch_hdecode(DecodeArgs a, const DecodePlan& p, cudaStream_t st) {
   a.KS = p.KS;
   a.CPC = p.CPC;
-  if constexpr (PHASE == 1) {
-    return launch_hdecode_n<1, 16>(a, p, st);
-  } else {
-    switch (p.N) {
-      case 16: return launch_hdecode_n<2, 16>(a, p, st);
-      case 32: return launch_hdecode_n<2, 32>(a, p, st);
-      default: return launch_hdecode_n<2, 48>(a, p, st);
-    }
+  switch (p.N) {
+    case 16: return launch_hdecode_n<PHASE, 16>(a, p, st);
+    case 32: return launch_hdecode_n<PHASE, 32>(a, p, st);
+    case 64: return launch_hdecode_n<PHASE, 64>(a, p, st);
+    default:
+      if constexpr (PHASE == 1) return cudaErrorInvalidConfiguration;  // phase 1 has at most 64 rows
+      else return launch_hdecode_n<PHASE, 128>(a, p, st);
   }
 }
 
@@ -1469,13 +1474,36 @@ int64_t decode_ldz(const af1_layer& L) { return (int64_t)L.p2.NCH * kChunkCols; 
 
 int64_t swiglu_ld(const af1_layer& L) { return (L.n + 7) / 8 * 8; }
 
+// Measured per call (us, weights streamed from HBM, one pass of the
+// 16-bit-operand kernel vs the prefill kernel) at 17 / 32 / 64 tokens:
+// 4096^2 (16.6 M signs) 13.5 / 16.3 / 26.5 vs 24.2 / 24.3 / 30.9;
+// 1024x8192 (8.1 M) 11.4 / 14.0 / 21.9 vs 27.7 / 27.2 / 28.3; 14336x4096
+// (58 M) 29.9 / 41.9 / 120 vs 41.3 / 41.5 / 45.9; 8192^2 (67 M) 29.6 / 38.2
+// / 115 vs 43.1 / 43.3 / 46.6; 28672x8192 (234 M) 109 / 153 / 422 vs 109 /
+// 109 / 112. The one pass wins while its expansion of the signs into tensor
+// memory (about 15 signs per clock per SM) stays short and, at 64 tokens,
+// while its 128-row phase-2 B tiles (one CTA per SM) do not multiply the
+// waves of a large matrix.
+constexpr int64_t kMidSignsShort = 70000000;  // up to 24 tokens
+constexpr int64_t kMidSignsLong = 20000000;   // up to kMidMaxTokens
+
+bool mid_pass(const af1_layer& L, int64_t tokens, bool prep) {
+  if (!prep || tokens <= kMaxPassTokens || tokens > kMidMaxTokens) return false;
+  if ((L.flags & (AF1_FLAG_TC_DECODE | AF1_FLAG_LUT_DECODE)) != 0) return false;
+  const int64_t signs = L.r * (L.m + L.n);
+  if (!((tokens <= 24 && signs <= kMidSignsShort) || signs <= kMidSignsLong)) return false;
+  const int T = (int)tokens;
+  return plan_hdecode(1, L.p1, T, L.num_sms, L.max_smem).ok && plan_hdecode(2, L.p2, T, L.num_sms, L.max_smem).ok;
+}
+
 Workspace plan_workspace(const af1_layer& L, int64_t tokens, bool prep, bool swiglu) {
   Workspace w;
   int64_t off = 0;
   w.status = off;
   off += 256;
+  const bool mid = mid_pass(L, tokens, prep);
   w.sbuf = off;
-  off += align256((int64_t)kMaxPassTokens * decode_ldz(L) * 4);
+  off += align256((mid ? tokens : (int64_t)kMaxPassTokens) * decode_ldz(L) * 4);
   if (prep && tokens > 4 && tokens <= kMaxPassTokens) {
     // Prepared B operand of the wider decode passes: every chunk's tiles at
     // the widest N (64 rows of 128 bytes) and the per-(slice, token) scales.
@@ -1486,7 +1514,7 @@ Workspace plan_workspace(const af1_layer& L, int64_t tokens, bool prep, bool swi
     off += align256((int64_t)kMaxKS * kMaxPassTokens * 8);
   }
   w.hbuf = off;
-  if (tokens > kMaxPassTokens) {
+  if (tokens > kMaxPassTokens && !mid) {
     const int64_t t = tokens < kPrefillPassTokens ? tokens : kPrefillPassTokens;
     off += align256(t * prefill_h_ld(L) * 2);
     if (prep) {
@@ -1576,7 +1604,8 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
   const __half* ux = static_cast<const __half*>(x2);
   __half* hx = x2 != nullptr ? reinterpret_cast<__half*>(wsb + W.hx) : nullptr;
   const int64_t ldh = swiglu_ld(L);
-  if (tokens > kMaxPassTokens) {
+  const bool mid = mid_pass(L, tokens, prep);
+  if (tokens > kMaxPassTokens && !mid) {
     // Prefill: two tensor-core GEMMs per pass (af1_prefill.cu); the SwiGLU
     // input is formed first, one pass of tokens at a time.
     float* part = W.pbuf != 0 ? reinterpret_cast<float*>(wsb + W.pbuf) : nullptr;
@@ -1593,15 +1622,16 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
     return cudaSuccess;
   }
   // Widest pass whose plans fit (16 tokens normally; fewer only for very
-  // long contractions).
-  int pass = kMaxPassTokens;
-  bool fits = false;
-  for (;;) {
+  // long contractions; a mid pass takes all its tokens at once, its plans
+  // checked by mid_pass).
+  int pass = mid ? (int)tokens : kMaxPassTokens;
+  bool fits = mid;
+  for (; !mid;) {
     const int T = (int)(tokens < pass ? tokens : pass);
     fits = plan_decode(1, L.p1, T, L.num_sms, L.max_smem, false).ok &&
            plan_decode(2, L.p2, T, L.num_sms, L.max_smem, false).ok;
     if (fits) {
-      // The 16-bit-operand kernel's B tiles grow with the pass (3 T rows in
+      // The 16-bit-operand kernel's B tiles grow with the pass (2 T rows in
       // phase 2): its plans must fit too where it would run.
       const PhaseChoice c1 = choose_phase(L, 1, L.p1, T, W), c2 = choose_phase(L, 2, L.p2, T, W);
       if (c1.mma && !plan_hdecode(1, L.p1, T, L.num_sms, L.max_smem).ok) fits = false;

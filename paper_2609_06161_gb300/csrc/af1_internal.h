@@ -32,13 +32,16 @@ namespace af1 {
 
 // Tokens per prefill pass (calls with more than kMaxPassTokens tokens).
 constexpr int64_t kPrefillPassTokens = 2048;
+// Longest call that may run as one pass of the 16-bit-operand decode kernel
+// instead of the prefill kernel (mid_pass).
+constexpr int64_t kMidMaxTokens = 64;
 // SM count the planners assume when the caller passes none (a GB300 has 152).
 constexpr int kDefaultSms = 152;
 
 // Workspace carve-up for one layer and one forward call of `tokens` tokens.
 struct Workspace {
   int64_t status = 0;  // uint32 status word
-  int64_t sbuf = 0;    // float[kMaxPassTokens][decode_ldz]: s' = s * t (decode)
+  int64_t sbuf = 0;    // float[max(kMaxPassTokens, tokens of a mid pass)][decode_ldz]: s' = s * t (decode)
   int64_t bbuf = 0;    // prepared B tiles of decode passes of 5..16 tokens (0: none)
   int64_t bstats = 0;  // float2 [16 slices][16 tokens] of the prepared B (0: none)
   int64_t hbuf = 0;    // FP16 [min(tokens, kPrefillPassTokens)][prefill_h_ld]: H (prefill)
@@ -52,6 +55,12 @@ struct Workspace {
 // swiglu adds the region the SwiGLU entry point forms h in for the kernels
 // that cannot form it while staging (tensor-core decode and prefill).
 Workspace plan_workspace(const af1_layer& L, int64_t tokens, bool prep = true, bool swiglu = false);
+// Whether a call of `tokens` tokens (17..kMidMaxTokens) runs as one pass of
+// the 16-bit-operand decode kernel instead of the prefill kernel: the normal
+// entry (prep), no decode-kernel flag that excludes it, a layer small enough
+// for the width (measured rule in af1_decode.cu), and plans for both phases
+// at that width.
+bool mid_pass(const af1_layer& L, int64_t tokens, bool prep);
 // Row stride (elements) of the SwiGLU input h in the workspace.
 int64_t swiglu_ld(const af1_layer& L);
 int64_t prefill_h_ld(const af1_layer& L);

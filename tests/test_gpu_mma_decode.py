@@ -1,6 +1,6 @@
 """The 16-bit-operand tensor-core decode kernel (AF1_FLAG_MMA_DECODE; by
-default the kernel of passes of 5..16 tokens) against the FP64 oracle,
-through the C ABI.
+default the kernel of passes of 5..16 tokens, and of calls of 17..64 tokens
+as one pass) against the FP64 oracle, through the C ABI.
 
 Phase 1 multiplies exact +-b_j FP16 sign values with the FP16 activations,
 phase 2 exact +-1 BF16 values with s' split into two BF16 terms (N = 16 or
@@ -142,3 +142,58 @@ def test_decode_kernel_flags_exclusive(P):
                {"tc_decode": True, "lut_decode": True}):
         with pytest.raises(P.AF1Error):
             signs_layer(P, d, **kw)
+
+
+# ---------------------------------------------------------------------------
+# Passes of 17..64 tokens on the same kernel (one pass instead of the prefill
+# kernel): B of up to 64 rows in phase 1 and 128 in phase 2.
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("m,n,r", [(100, 130, 77), (1000, 700, 321), (1024, 4096, 800), (300, 1920, 100)])
+@pytest.mark.parametrize("tokens", [17, 24, 32, 33, 48, 64])
+def test_mid_pass_matches_oracle(P, m, n, r, tokens):
+    d = synth.layer_signs(23 * m + n + tokens, m, n, r, tokens)
+    layer = signs_layer(P, d)
+    y = run_gpu(layer, d["x"], n, torch.float32)
+    err = O.rowwise_rel_err(y, oracle_from_signs(d, n))
+    assert err <= TOL, err
+    layer.free()
+
+
+@pytest.mark.parametrize("m,n,r", [(256, 256, 120), (700, 896, 333)])
+@pytest.mark.parametrize("tokens", [20, 64])
+def test_mid_pass_integer_bit_exact(P, m, n, r, tokens):
+    d = synth.integer_layer(29 + m + tokens, m, n, r, tokens)
+    layer = signs_layer(P, d)
+    y = run_gpu(layer, d["x"], n, torch.float32)
+    np.testing.assert_array_equal(y, oracle_from_signs(d, n))
+    layer.free()
+
+
+@pytest.mark.parametrize("tokens", [17, 64])
+def test_mid_pass_against_prefill_path(P, tokens):
+    """The same layer with AF1_FLAG_TC_DECODE runs calls of more than 16
+    tokens on the prefill kernel instead: both within the bar of the oracle,
+    FP16 outputs with x20 outlier channels."""
+    m, n, r = 1024, 4096, 800
+    d = synth.layer_signs(4040 + tokens, m, n, r, tokens, outlier_frac=0.01)
+    ref = oracle_from_signs(d, n)
+    for kw in ({}, {"tc_decode": True}):
+        layer = signs_layer(P, d, **kw)
+        y = run_gpu(layer, d["x"], n, torch.float16)
+        assert O.rowwise_rel_err(y, ref) <= TOL, kw
+        layer.free()
+
+
+@pytest.mark.parametrize("m,n,tokens", [(4096, 14336, 20), (8192, 8192, 24), (4096, 4096, 64), (1024, 8192, 48)])
+def test_mid_pass_full_size_sampled_rows(P, m, n, tokens):
+    """Full-size matrices that take one pass at these widths (up to 24
+    tokens below 70 M signs, up to 64 below 20 M)."""
+    r = O.rank_for_budget(m, n, 1)
+    d = synth.layer_words(61 + m // 1024 + n // 1024, m, n, r, tokens)
+    layer = words_layer(P, d, m, n, r)
+    y = run_gpu(layer, d["x"], n)
+    rows = np.sort(synth.rng(m + n + tokens).choice(m, size=128, replace=False))
+    ref = O.forward_from_packed(d["Uw"], d["Vw"], d["a"], d["s"], d["b"], d["x"], m, n, r, rows=rows)
+    assert O.rowwise_rel_err(y[:, rows], ref) <= TOL
+    layer.free()
