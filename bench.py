@@ -519,12 +519,12 @@ def decode_kernel_of(b):
 
 def mid_pass_of(m, n, r, b):
     """Whether a call of 17..64 tokens runs as one pass of the 16-bit-operand
-    decode kernel instead of the prefill kernel (the library's rule: up to 24
+    decode kernel instead of the prefill kernel (the library's rule: up to 32
     tokens below 70 M signs, up to 64 below 20 M; no LUT or e4m3 flag)."""
     if DECODE_KERNEL in ("lut", "tc") or not 16 < b <= 64:
         return False
     signs = r * (m + n)
-    return (b <= 24 and signs <= 70_000_000) or signs <= 20_000_000
+    return (b <= 32 and signs <= 70_000_000) or signs <= 20_000_000
 
 
 def phase_launches(m, n, r, b):

@@ -720,15 +720,22 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const DecodeArgs a)
 // exponent range (one FP16 term loses small values to FP16's range; three
 // would need an epilogue that sums a token's terms across column blocks).
 constexpr int kS2Terms = 2;
+// Calls of 17..kMidMaxTokens tokens run as one pass (mid_pass) with s' as
+// ONE FP16 term, the rounding their prefill path makes of its H (reading
+// R11): two BF16 terms make phase 2's B 128 rows at 64 tokens (32 KB per
+// chunk, one CTA per SM). Measured at 32 / 64 tokens (us, two terms -> one):
+// 14336x4096 41.9 -> 39.2 / 120 -> 113, 4096x14336 47.4 -> 40.2 / 133 ->
+// 131, 8192^2 38.2 -> 33.3 / 115 -> 79.9.
+__host__ __device__ constexpr int s2_terms(int T) { return T <= kMaxPassTokens ? kS2Terms : 1; }
 // Accumulators (one MMA issuer each) and A-ring depth for N rows of B,
 // within the CTA's 256 tensor-memory columns: N 16: 4 and 3; 32: 2 and 3;
 // 48 / 64: 2 and 2; 128: 1 and 2.
 __host__ __device__ constexpr int hnacc_for(int N) { return N == 16 ? 4 : N <= 64 ? 2 : 1; }
 __host__ __device__ constexpr int hnbuf_for(int N) { return (kTmemCols - hnacc_for(N) * N) / 64; }
 // B rows of a pass of T tokens (up to kMidMaxTokens): T rows (phase 1) or
-// kS2Terms T rows (phase 2), rounded up to 16, 32, 64 or 128.
-__host__ __device__ constexpr int hround_n(int rows) { return rows <= 16 ? 16 : rows <= 32 ? 32 : rows <= 64 ? 64 : 128; }
-__host__ __device__ constexpr int hdecode_n(int phase, int T) { return hround_n(phase == 1 ? T : kS2Terms * T); }
+// s2_terms(T) T rows (phase 2), rounded up to 16, 32 or 64.
+__host__ __device__ constexpr int hround_n(int rows) { return rows <= 16 ? 16 : rows <= 32 ? 32 : 64; }
+__host__ __device__ constexpr int hdecode_n(int phase, int T) { return hround_n(phase == 1 ? T : s2_terms(T) * T); }
 
 struct __align__(8) HDecodeHeader {
   uint64_t wfull[kMaxCPC];  // packed chunk c has landed (chunk 0: with the column scales)
@@ -807,10 +814,11 @@ __device__ __forceinline__ void tmem_st16p(uint32_t addr, const uint32_t* r) {
       : "memory");
 }
 
-// The kS2Terms 16-bit terms of v: v rounded to FP16 (one term), or the BF16
+// The TERMS 16-bit terms of v: v rounded to FP16 (one term), or the BF16
 // terms hi and lo (v - hi is exact in FP32; lo is it rounded to BF16).
+template <int TERMS>
 __device__ __forceinline__ void split_terms(float v, uint16_t* t3) {
-  if constexpr (kS2Terms == 1) {
+  if constexpr (TERMS == 1) {
     t3[0] = __half_as_ushort(__float2half_rn(v));
   } else {
     const __nv_bfloat16 hi = __float2bfloat16_rn(v);
@@ -855,7 +863,7 @@ __device__ __forceinline__ void load_unit_h(const DecodeArgs& a, int t, int kl, 
   }
 }
 
-template <int PHASE, int N>
+template <int PHASE, int N, int TERMS>
 __device__ __forceinline__ void build_b_h(const DecodeArgs& a, int T, int nch, int64_t k0, int kv, int bt,
                                           uint8_t* Bt) {
   constexpr int UB = 4;
@@ -887,13 +895,13 @@ __device__ __forceinline__ void build_b_h(const DecodeArgs& a, int T, int nch, i
 #pragma unroll
         for (int q = 0; q < 8; ++q) {
           uint16_t t3[3];
-          split_terms(__uint_as_float(fw[q]), t3);
+          split_terms<TERMS>(__uint_as_float(fw[q]), t3);
 #pragma unroll
-          for (int term = 0; term < kS2Terms; ++term) e[term][q] = t3[term];
+          for (int term = 0; term < TERMS; ++term) e[term][q] = t3[term];
         }
 #pragma unroll
-        for (int term = 0; term < kS2Terms; ++term) {
-          const int n = kS2Terms * t + term;
+        for (int term = 0; term < TERMS; ++term) {
+          const int n = TERMS * t + term;
           const uint4 v = make_uint4(e[term][0] | (uint32_t)e[term][1] << 16, e[term][2] | (uint32_t)e[term][3] << 16,
                                      e[term][4] | (uint32_t)e[term][5] << 16, e[term][6] | (uint32_t)e[term][7] << 16);
           *reinterpret_cast<uint4*>(half_base + n * 128 + ((j ^ (n & 7)) << 4)) = v;
@@ -903,12 +911,13 @@ __device__ __forceinline__ void build_b_h(const DecodeArgs& a, int T, int nch, i
   }
 }
 
-template <int PHASE, int N>
+// TERMS: terms of s' per token in phase 2's B (1: FP16, 2: BF16).
+template <int PHASE, int N, int TERMS>
 __global__ void __launch_bounds__(kThreads, 1) hdecode_kernel(const DecodeArgs a) {
   constexpr int NACC = hnacc_for(N);
   constexpr int NBUF = hnbuf_for(N);
   constexpr int DCOL = NBUF * 64;  // first accumulator column
-  constexpr bool BF16 = PHASE == 2 && kS2Terms > 1;
+  constexpr bool BF16 = PHASE == 2 && TERMS > 1;
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -1010,7 +1019,7 @@ __global__ void __launch_bounds__(kThreads, 1) hdecode_kernel(const DecodeArgs a
     // ---- B: activations -> the swizzled B tile; then the MMAs -------------
     const int bt = tid - 128;
     griddep_wait();  // activations are written by the previous kernel
-    build_b_h<PHASE, N>(a, T, nch, k0, kv, bt, Bt);
+    build_b_h<PHASE, N, TERMS>(a, T, nch, k0, kv, bt, Bt);
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // B is read by the tensor cores
     builders_sync();
     const int ia = warp - 4;
@@ -1048,9 +1057,9 @@ __global__ void __launch_bounds__(kThreads, 1) hdecode_kernel(const DecodeArgs a
     const int owner = i / slice;
     // One block of 16 accumulator columns at a time (the accumulators summed
     // in a fixed order), then the tokens whose terms lie in the block.
-    constexpr int TERMS = PHASE == 1 ? 1 : kS2Terms;
-    static_assert(16 % TERMS == 0, "a token's terms must lie in one block of 16 columns");
-    constexpr int TPB = 16 / TERMS;  // tokens per block
+    constexpr int NT = PHASE == 1 ? 1 : TERMS;  // B rows per token
+    static_assert(16 % NT == 0, "a token's terms must lie in one block of 16 columns");
+    constexpr int TPB = 16 / NT;  // tokens per block
 #pragma unroll
     for (int cb = 0; cb < N / 16; ++cb) {
       if (cb * TPB >= T) break;
@@ -1070,9 +1079,9 @@ __global__ void __launch_bounds__(kThreads, 1) hdecode_kernel(const DecodeArgs a
         for (int tl = 0; tl < TPB; ++tl) {
           const int t = cb * TPB + tl;
           if (t < T) {
-            float p = acc[TERMS * tl];
+            float p = acc[NT * tl];
 #pragma unroll
-            for (int q = 1; q < TERMS; ++q) p += acc[TERMS * tl + q];
+            for (int q = 1; q < NT; ++q) p += acc[NT * tl + q];
             st_cluster_f32(recv + ((ks * T + t) * slice + (i - owner * slice)), (uint32_t)owner, p);
           }
         }
@@ -1397,9 +1406,9 @@ cudaError_t launch_decode(DecodeArgs a, const DecodePlan& p, cudaStream_t st) {
   }
 }
 
-template <int PHASE, int N>
+template <int PHASE, int N, int TERMS>
 cudaError_t launch_hdecode_n(const DecodeArgs& a, const DecodePlan& p, cudaStream_t st) {
-  auto kern = hdecode_kernel<PHASE, N>;
+  auto kern = hdecode_kernel<PHASE, N, TERMS>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, p.smem);
   if (e != cudaSuccess) return e;
   if (p.KS > 8) {
@@ -1427,14 +1436,19 @@ template <int PHASE>
 cudaError_t launch_hdecode(DecodeArgs a, const DecodePlan& p, cudaStream_t st) {
   a.KS = p.KS;
   a.CPC = p.CPC;
-  switch (p.N) {
-    case 16: return launch_hdecode_n<PHASE, 16>(a, p, st);
-    case 32: return launch_hdecode_n<PHASE, 32>(a, p, st);
-    case 64: return launch_hdecode_n<PHASE, 64>(a, p, st);
-    default:
-      if constexpr (PHASE == 1) return cudaErrorInvalidConfiguration;  // phase 1 has at most 64 rows
-      else return launch_hdecode_n<PHASE, 128>(a, p, st);
+  if (PHASE == 1 || s2_terms(a.tokens) == 1) {
+    switch (p.N) {
+      case 16: return launch_hdecode_n<PHASE, 16, 1>(a, p, st);
+      case 32: return launch_hdecode_n<PHASE, 32, 1>(a, p, st);
+      default: return launch_hdecode_n<PHASE, 64, 1>(a, p, st);
+    }
   }
+  if constexpr (PHASE == 2) {
+    static_assert(kS2Terms == 2, "passes of up to 16 tokens: two BF16 terms, 16 or 32 rows");
+    if (p.N == 16) return launch_hdecode_n<2, 16, 2>(a, p, st);
+    return launch_hdecode_n<2, 32, 2>(a, p, st);
+  }
+  return cudaErrorInvalidConfiguration;
 }
 
 int64_t align256(int64_t v) { return (v + 255) / 256 * 256; }
@@ -1476,22 +1490,24 @@ int64_t swiglu_ld(const af1_layer& L) { return (L.n + 7) / 8 * 8; }
 
 // Measured per call (us, weights streamed from HBM, one pass of the
 // 16-bit-operand kernel vs the prefill kernel) at 17 / 32 / 64 tokens:
-// 4096^2 (16.6 M signs) 13.5 / 16.3 / 26.5 vs 24.2 / 24.3 / 30.9;
-// 1024x8192 (8.1 M) 11.4 / 14.0 / 21.9 vs 27.7 / 27.2 / 28.3; 14336x4096
-// (58 M) 29.9 / 41.9 / 120 vs 41.3 / 41.5 / 45.9; 8192^2 (67 M) 29.6 / 38.2
-// / 115 vs 43.1 / 43.3 / 46.6; 28672x8192 (234 M) 109 / 153 / 422 vs 109 /
-// 109 / 112. The one pass wins while its expansion of the signs into tensor
-// memory (about 15 signs per clock per SM) stays short and, at 64 tokens,
-// while its 128-row phase-2 B tiles (one CTA per SM) do not multiply the
-// waves of a large matrix.
-constexpr int64_t kMidSignsShort = 70000000;  // up to 24 tokens
+// 4096^2 (16.6 M signs) 13.2 / 15.7 / 25.2 vs 24.2 / 24.3 / 30.9;
+// 1024x8192 (8.1 M) 11.3 / 13.8 / 21.6 vs 27.7 / 27.2 / 28.3; 14336x4096
+// (58 M) 28.4 / 39.2 / 113 vs 41.3 / 41.5 / 45.9; 4096x14336 (58 M) 30.4 /
+// 40.2 / 131 vs 42.9 / 43.0 / 47.7; 8192^2 (67 M) 25.3 / 33.3 / 79.9 vs
+// 43.1 / 43.3 / 46.6; 28672x8192 (234 M) 103 / 142 / 298 vs 109 / 109 /
+// 112; 8192x28672 (234 M) 171 / 227 vs 116 / 116. The one pass wins while
+// its expansion of the signs into tensor memory (about 15 signs per clock
+// per SM) stays short and, at 64 tokens, on small layers only (its 64-row
+// tiles and 64-token epilogue multiply a larger matrix's waves; eight
+// activation loads in flight per builder instead of four: 2 %).
+constexpr int64_t kMidSignsShort = 70000000;  // up to 32 tokens
 constexpr int64_t kMidSignsLong = 20000000;   // up to kMidMaxTokens
 
 bool mid_pass(const af1_layer& L, int64_t tokens, bool prep) {
   if (!prep || tokens <= kMaxPassTokens || tokens > kMidMaxTokens) return false;
   if ((L.flags & (AF1_FLAG_TC_DECODE | AF1_FLAG_LUT_DECODE)) != 0) return false;
   const int64_t signs = L.r * (L.m + L.n);
-  if (!((tokens <= 24 && signs <= kMidSignsShort) || signs <= kMidSignsLong)) return false;
+  if (!((tokens <= 32 && signs <= kMidSignsShort) || signs <= kMidSignsLong)) return false;
   const int T = (int)tokens;
   return plan_hdecode(1, L.p1, T, L.num_sms, L.max_smem).ok && plan_hdecode(2, L.p2, T, L.num_sms, L.max_smem).ok;
 }

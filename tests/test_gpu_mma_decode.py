@@ -185,9 +185,9 @@ def test_mid_pass_against_prefill_path(P, tokens):
         layer.free()
 
 
-@pytest.mark.parametrize("m,n,tokens", [(4096, 14336, 20), (8192, 8192, 24), (4096, 4096, 64), (1024, 8192, 48)])
+@pytest.mark.parametrize("m,n,tokens", [(4096, 14336, 20), (8192, 8192, 32), (4096, 4096, 64), (1024, 8192, 48)])
 def test_mid_pass_full_size_sampled_rows(P, m, n, tokens):
-    """Full-size matrices that take one pass at these widths (up to 24
+    """Full-size matrices that take one pass at these widths (up to 32
     tokens below 70 M signs, up to 64 below 20 M)."""
     r = O.rank_for_budget(m, n, 1)
     d = synth.layer_words(61 + m // 1024 + n // 1024, m, n, r, tokens)
