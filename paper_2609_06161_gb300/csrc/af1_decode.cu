@@ -691,20 +691,24 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const DecodeArgs a)
 
 // ---------------------------------------------------------------------------
 // Decode kernel with 16-bit MMA operands (tcgen05.mma kind::f16), passes of
-// up to 16 tokens. The signs become exact 16-bit A values in tensor memory:
+// up to 16 tokens, and calls of 17..64 tokens on small layers as one pass
+// (mid_pass). The signs become exact 16-bit A values in tensor memory:
 //   phase 1: A = +-b_j (FP16; the column scale carries the sign), B = x
-//            (FP16, N = 16 rows, row t = token t), so D = sum_j +-b_j x_j;
-//   phase 2: A = +-1 (BF16), B = s' split into kS2Terms = 2 BF16 terms
-//            hi + lo (N = 16/32 rows, term q of token t in row 2 t + q):
-//            BF16 keeps FP32's exponent range, so no scaling is needed, and
-//            hi + lo holds the 16 leading significant bits of s' (a
-//            relative error of at most 2^-17; three terms would hold all 24).
+//            (FP16, N = 16/32/64 rows, row t = token t), so
+//            D = sum_j +-b_j x_j;
+//   phase 2, up to 16 tokens: A = +-1 (BF16), B = s' split into
+//            kS2Terms = 2 BF16 terms hi + lo (N = 16/32 rows, term q of
+//            token t in row 2 t + q): BF16 keeps FP32's exponent range, so
+//            no scaling is needed, and hi + lo holds the 16 leading
+//            significant bits of s' (a relative error of at most 2^-17);
+//   phase 2, one pass of 17..64 tokens: A = +-1 (FP16), B = s' rounded to
+//            FP16 (N = 32/64 rows), as the prefill path rounds its H.
 // Every product is exact and the MMA accumulates in FP32: up to that
 // rounding of s', the result is the FP32 signed sum the lookup-table
 // kernels form, summed in another order.
 // Against the e4m3 kernel above there is no activation split, no power-of-
 // two scale and no sign correction, and the B operand is a copy (phase 1) or
-// a two-way split (phase 2) that the CTA builds itself, so no preparation
+// a split (phase 2) that the CTA builds itself, so no preparation
 // kernel runs. A chunk of A takes 64 tensor-memory columns (two values per
 // column), twice the e4m3 chunk. The CTA structure is the e4m3 kernel's:
 // bulk copies of the signs first, warps 0-3 expand, warps 4-7 build B and

@@ -182,11 +182,12 @@ __global__ void __launch_bounds__(kThreads, 4) lut_kernel(const __grid_constant_
     }
   }
 
-  // The late order: phase 2 lets the next kernel launch only now, so its
-  // CTAs do not hold SM slots (waiting for this kernel) that sibling kernels
-  // on other streams need, and its sign copies still get the reduction's
-  // time as a head start (measured: config-1 stack 7.40 -> 6.53 us per
-  // linear on the DAG schedule, trigger at the start vs here).
+  // With several streams (AF1_MANY_STREAMS): phase 2 lets the next kernel
+  // launch only now, so its CTAs do not hold SM slots (waiting for this
+  // kernel) that sibling kernels on other streams need, and its sign copies
+  // still get the reduction's time as a head start (measured: config-1
+  // stack 7.40 -> 6.53 us per linear on the DAG schedule, trigger at the
+  // start vs here).
   if (PHASE == 2 && a.late_trigger) griddep_launch_dependents();
   // ---- partial sums -> owner CTA of each row -> final sums -------------------
   cluster_wait();  // every CTA of the cluster has started
