@@ -97,8 +97,11 @@ extern "C" {
    activations as FP16, and the rank intermediate s' as two BF16 terms that
    hold its 16 leading significant bits). Without a decode flag the library
    takes this kernel for passes of more than 4 tokens and the lookup-table
-   kernels for passes of 1 to 4 tokens. Results agree within the library's
-   tolerance. */
+   kernels for passes of 1 to 4 tokens; calls of 17 to 64 tokens on small
+   layers (up to 32 tokens below 70 M signs r (m + n), up to 64 below 20 M)
+   run as one pass of it, with s' rounded to FP16 as the prefill kernel
+   rounds its intermediate, unless AF1_FLAG_TC_DECODE or AF1_FLAG_LUT_DECODE
+   is set. Results agree within the library's tolerance. */
 #define AF1_FLAG_MMA_DECODE 16
 /* Run every decode pass (1..16 tokens) on the CUDA-core lookup-table kernels
    (clustered or streaming), never on a tensor-core kernel. At most one of
