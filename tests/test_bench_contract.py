@@ -94,3 +94,27 @@ def test_job_time_is_the_slowest_rank():
     for rank, t, v in got:
         assert t == 15.0
         assert v == pytest.approx(4 * 2 * 3 / 15.0)
+
+
+def test_kernel_bookkeeping_follows_the_dispatch(monkeypatch):
+    """The bench names each call's kernel and counts launches from the
+    library's dispatch rules: lookup tables up to 4 tokens, the 16-bit-operand
+    kernel from 5 to 16, one pass of it for 17-64 tokens on small layers (up
+    to 32 tokens below 70 M signs, up to 64 below 20 M), the prefill kernel
+    otherwise; layer flags override."""
+    sys.path.insert(0, ROOT)
+    import bench
+    monkeypatch.setattr(bench, "DECODE_KERNEL", "auto")
+    assert [bench.decode_kernel_of(b) for b in (1, 2, 4, 5, 8, 16)] == ["lut"] * 3 + ["mma"] * 3
+    assert bench.mid_pass_of(4096, 4096, 2028, 17) and bench.mid_pass_of(4096, 4096, 2028, 64)
+    assert bench.mid_pass_of(8192, 8192, 4076, 32) and not bench.mid_pass_of(8192, 8192, 4076, 33)
+    assert not bench.mid_pass_of(28672, 8192, 6352, 17)
+    assert not bench.mid_pass_of(4096, 4096, 2028, 16) and not bench.mid_pass_of(4096, 4096, 2028, 65)
+    assert bench.phase_launches(4096, 4096, 2028, 16) == 2
+    for forced in ("lut", "tc"):
+        monkeypatch.setattr(bench, "DECODE_KERNEL", forced)
+        assert not bench.mid_pass_of(4096, 4096, 2028, 17)
+        assert bench.decode_kernel_of(1) == forced
+    assert bench.phase_launches(4096, 4096, 2028, 8) == 4  # e4m3 kernel: a preparation launch per phase
+    monkeypatch.setattr(bench, "DECODE_KERNEL", "mma")
+    assert bench.decode_kernel_of(1) == "mma" and bench.mid_pass_of(4096, 4096, 2028, 20)
