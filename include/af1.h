@@ -108,6 +108,22 @@ extern "C" {
    AF1_FLAG_TC_DECODE, AF1_FLAG_MMA_DECODE and AF1_FLAG_LUT_DECODE may be set. */
 #define AF1_FLAG_LUT_DECODE 32
 
+/* The launch plan of one phase of the 16-bit-operand tensor-core decode
+ * kernel (AF1_FLAG_MMA_DECODE; by default passes of 5 to 16 tokens and
+ * one-pass calls of 17 to 64), computed on the host alone (no GPU needed):
+ * an R x C sign matrix (phase 1: r x n; phase 2: m x r) times `tokens`
+ * vectors (1..64) on a GPU with num_sms SMs and max_smem bytes of opt-in
+ * shared memory per block. out[0..9] = {rows N of the B operand,
+ * accumulators (one MMA issuer each), A-ring depth in 128-column chunks,
+ * tensor-memory columns used (of the 256 a CTA allocates), CTAs per cluster
+ * along K, 128-column chunks per CTA, dynamic shared memory per CTA in
+ * bytes, grid x (row blocks of 128), grid y (CTAs per cluster), 1 if a plan
+ * exists else 0}. Errors: INVALID_ARG (phase not 1 or 2, R or C outside
+ * 1..2^30 / 1..32768, tokens outside 1..64, num_sms < 1, max_smem < 1,
+ * out NULL). */
+AF1_API int af1_mma_plan_dry(int phase, int64_t R, int64_t C, int64_t tokens, int num_sms, int max_smem,
+                             int32_t* out);
+
 typedef struct af1_layer_desc {
   int64_t m;       /* d_out: rows of W_hat, length of a, length of y rows */
   int64_t n;       /* d_in: columns of W_hat, length of b and of x rows   */

@@ -127,6 +127,9 @@ _lib.af1_set_wait_cycles.argtypes = [_i64]
 _lib.af1_set_wait_cycles.restype = ctypes.c_int
 _lib.af1_get_wait_cycles.argtypes = []
 _lib.af1_get_wait_cycles.restype = _i64
+_lib.af1_mma_plan_dry.argtypes = [ctypes.c_int, _i64, _i64, _i64, ctypes.c_int, ctypes.c_int,
+                                  ctypes.POINTER(ctypes.c_int32)]
+_lib.af1_mma_plan_dry.restype = ctypes.c_int
 _lib.af1_set_stream_layout.argtypes = [ctypes.c_int]
 _lib.af1_set_stream_layout.restype = ctypes.c_int
 _lib.af1_get_stream_layout.argtypes = []
@@ -226,6 +229,16 @@ def set_wait_cycles(cycles: int) -> None:
 
 def get_wait_cycles() -> int:
     return int(_lib.af1_get_wait_cycles())
+
+
+def mma_plan_dry(phase: int, R: int, C: int, tokens: int, num_sms: int = 152, max_smem: int = 232448) -> dict:
+    """The 16-bit-operand decode kernel's launch plan for one phase (an R x C
+    sign matrix times `tokens` vectors), computed on the host
+    (af1_mma_plan_dry); no GPU needed."""
+    out = (ctypes.c_int32 * 10)()
+    _check(_lib.af1_mma_plan_dry(int(phase), int(R), int(C), int(tokens), int(num_sms), int(max_smem), out))
+    keys = ("rows", "accumulators", "ring", "tmem_cols", "ks", "cpc", "smem", "grid_x", "grid_y", "ok")
+    return dict(zip(keys, list(out)))
 
 
 AF1_ONE_STREAM = 0

@@ -1741,6 +1741,24 @@ cudaError_t launch_forward(const af1_layer& L, const void* x, int64_t ldx, int64
 }
 
 
+}  // namespace af1
+
+extern "C" int af1_mma_plan_dry(int phase, int64_t R, int64_t C, int64_t tokens, int num_sms, int max_smem,
+                                int32_t* out) {
+  using namespace af1;
+  if (out == nullptr || (phase != 1 && phase != 2) || R < 1 || R > ((int64_t)1 << 30) || C < 1 || C > kMaxCols ||
+      tokens < 1 || tokens > kMidMaxTokens || num_sms < 1 || max_smem < 1)
+    return set_error(AF1_ERR_INVALID_ARG, "af1_mma_plan_dry: argument out of range");
+  const SignMatrix sm = make_sign_matrix(R, C);
+  const DecodePlan p = plan_hdecode(phase, sm, (int)tokens, num_sms, max_smem);
+  const int nacc = hnacc_for(p.N), nbuf = hnbuf_for(p.N);
+  const int32_t v[10] = {p.N, nacc, nbuf, nacc * p.N + nbuf * 64, p.KS, p.CPC, p.smem, sm.RB, p.KS, p.ok ? 1 : 0};
+  for (int i = 0; i < 10; ++i) out[i] = v[i];
+  return AF1_OK;
+}
+
+namespace af1 {
+
 int64_t multi_workspace_offset(const af1_layer* const* Ls, int i, int64_t tokens, bool prep) {
   int64_t off = 0;
   for (int j = 0; j < i; ++j) off += align256(plan_workspace(*Ls[j], tokens, prep).total);
